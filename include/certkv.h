@@ -1,0 +1,192 @@
+/*
+ * certkv.h — C ABI of the CertKV exact-budget KV-cache compressor and of
+ * decode attention over the packed cache it produces, for NVIDIA GB300
+ * (sm_103a).
+ *
+ * The method is the one of "Beyond Sparse Weights: When Is Attention
+ * Compressible?", §4 (CertKV: value-aware compression under exact budgets),
+ * Eq. (certkv-curve), Algorithm 1 and the appendix "CertKV: implementation and
+ * exact-budget protocol".  Once per (sequence, layer), after prefill:
+ *
+ *   a1/a2  score   observation-window softmax mass per cached token and KV head
+ *                  (the SnapKV observation-window scorer the paper keeps
+ *                  unchanged), normalised to a_j = (s_j)_+ / sum_i (s_i)_+;
+ *   a3     order   per-head stable order by a descending, ties by lower index;
+ *   a4     curve   suffix moments m_h(b), W_h(b), Q_h(b) over the evicted
+ *                  ranks and the centred-dispersion curve
+ *                  c_h(b) = sqrt((m_h(b) Q_h(b) - ||W_h(b)||^2)_+), b = 0..n-1;
+ *   a5     budget  B_real = B_live - H, b_min = max{1, floor(alpha B_real / H)},
+ *                  T-step Lagrangian bisection on a shared multiplier, then
+ *                  best-marginal repair until sum_h b_h = B_real;
+ *   a6     select  the top-b_h real tokens of each head;
+ *   a7     tail    one synthetic pair per head: the mass-weighted key and value
+ *                  centroids (k*, v*) of the evicted suffix;
+ *   a8     pack    a ragged bf16 cache holding exactly B_live live slots per
+ *                  (sequence, layer): b_h real slots + 1 tail slot per head.
+ *   a9     decode  softmax attention over the b_h + 1 slots of each head
+ *                  (the "plain slot" of the paper's ablation table).
+ *
+ * Conventions shared by every entry point
+ *   - Pointers named in the argument lists are DEVICE pointers unless a
+ *     comment says otherwise.  The caller owns every buffer: the library never
+ *     allocates or frees memory.
+ *   - All work is enqueued on the caller's stream `stream` (a cudaStream_t
+ *     passed as void*; NULL = the legacy default stream) and the calls return
+ *     without synchronising.  Arguments are validated on the host before any
+ *     launch; a call that returns non-zero has enqueued nothing.
+ *   - Tensors are dense, row-major, with these layouts (B = batch, L = layers,
+ *     Hq query heads, H = hkv KV heads, G = Hq / H, n context, d head dim,
+ *     w observation window):
+ *         K, V   bf16  [B][L][H][n][d]
+ *         Q_obs  bf16  [B][L][Hq][w][d]   the last w prefill queries
+ *         q      bf16  [B][L][Hq][d]      one decode query per head
+ *     Query head qh reads KV head qh / G.  Observation row t of a query head
+ *     sits at absolute position n - w + t and sees keys j <= n - w + t.
+ *   - A "unit" is one (sequence, layer, KV head): u = (b * L + l) * H + h.
+ *   - Device-side problems (non-finite scores, an evicted suffix with zero
+ *     mass) are recorded in a status word inside the workspace; read it with
+ *     certkv_read_status().  No kernel traps.
+ *   - Supported sizes: d = 128; 1 <= H <= 32; G = Hq / H an integer with
+ *     1 <= G <= 16; 1 <= w < n; n <= 2^24; B * L * H <= 2^24.
+ */
+#ifndef CERTKV_H
+#define CERTKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- return codes -------------------------------------------------------- */
+#define CERTKV_OK          0
+#define CERTKV_EINVAL      1  /* bad shape, pointer or parameter                 */
+#define CERTKV_EBUDGET     2  /* budget infeasible: B_live < 2H or B_live > H*n  */
+#define CERTKV_EWORKSPACE  3  /* workspace missing, misaligned or too small      */
+#define CERTKV_ECAPACITY   4  /* packed-cache capacity below B * L * B_live      */
+#define CERTKV_ECUDA       5  /* a CUDA runtime call failed                      */
+
+/* bits of the device status word returned by certkv_read_status() */
+#define CERTKV_STATUS_NONFINITE   1u  /* a score or curve value was NaN/Inf     */
+#define CERTKV_STATUS_ZERO_TAIL   2u  /* an evicted suffix had zero mass: its
+                                         tail slot is the uniform mean instead */
+
+/* ---- problem description ------------------------------------------------- */
+typedef struct {
+  int32_t batch;   /* B  sequences                                   */
+  int32_t layers;  /* L  layers compressed in this call              */
+  int32_t hq;      /* Hq query heads                                 */
+  int32_t hkv;     /* H  KV heads                                    */
+  int32_t n;       /* context length (cached tokens per KV head)     */
+  int32_t d;       /* head dimension (128)                           */
+  int32_t w;       /* observation window (last w prefill queries)    */
+} certkv_shape;
+
+/* Statistic used for the allocation curve (paper: one-factor ablations). */
+#define CERTKV_STAT_CENTERED    0  /* c = sqrt((m Q - ||W||^2)_+)  (default, Eq. certkv-curve) */
+#define CERTKV_STAT_UNCENTERED  1  /* c = sqrt(m Q)                                             */
+#define CERTKV_STAT_TAIL_MASS   2  /* c = m                                                     */
+
+typedef struct {
+  float   scale;          /* softmax scale for <q,k>; 0 selects 1/sqrt(d)            */
+  int32_t pool_kernel;    /* observation-score average-pool width, odd >= 1; 5 default;
+                             zero padding, divided by the width, window keys excluded  */
+  int32_t protect_window; /* 1 (default): the w window keys get the head's maximum
+                             pooled score; 0: their own mean causal probability       */
+  int32_t alpha_num;      /* safeguard alpha = alpha_num / alpha_den (default 1 / 5), */
+  int32_t alpha_den;      /*   0 <= alpha <= 1, exact rational                        */
+  int32_t bisect_steps;   /* T, number of bisection steps (default 40), 0..200        */
+  int32_t statistic;      /* CERTKV_STAT_* (default CERTKV_STAT_CENTERED)             */
+  int32_t tail_slot;      /* 1 (default): one synthetic tail slot per head is charged
+                             to the budget; 0: no slot, the slot goes to a real token */
+} certkv_params;
+
+/* Ragged packed cache.  Segment u (one per unit) holds real_counts[u] real
+ * slots in ascending original position followed, when params.tail_slot = 1,
+ * by the tail slot; offsets[u] is its first slot.  Each (sequence, layer)
+ * owns exactly B_live consecutive slots: offsets[(b*L+l)*H] = (b*L+l)*B_live. */
+typedef struct {
+  void*    k;               /* bf16 [capacity_slots][d]                          */
+  void*    v;               /* bf16 [capacity_slots][d]                          */
+  int64_t* offsets;         /* [B*L*H + 1] first slot of each segment            */
+  int32_t* real_counts;     /* [B*L*H] b_h, real slots per segment               */
+  int32_t* positions;       /* [capacity_slots] original token index; -1 = tail  */
+  int64_t  capacity_slots;  /* slots available in k, v and positions             */
+  float*   tail_f32;        /* optional (NULL = skip) [B*L*H][2][d]: k*, v* in fp32
+                               before rounding to bf16                            */
+  double*  tail_mass;       /* optional (NULL = skip) [B*L*H]: m_h(b_h)          */
+} certkv_packed;
+
+/* Fill `p` with the defaults listed above.  Host call. */
+void certkv_default_params(certkv_params* p);
+
+/* Live-slot budget of the paper's exact-budget protocol for a kept fraction
+ * keep_num / keep_den: H * floor(n * keep_num / keep_den), computed in exact
+ * integer arithmetic (the paper writes B_live = H floor(n (1 - r)) for an
+ * evicted fraction r).  Returns -1 for invalid arguments.  Host call. */
+int64_t certkv_live_budget(int32_t n, int32_t hkv, int64_t keep_num, int64_t keep_den);
+
+/* Workspace bytes needed by certkv_compress / certkv_compress_scored /
+ * certkv_score / certkv_curves for this shape (an upper bound for all four),
+ * and by certkv_decode_attn.  0 if the shape or parameters are invalid. */
+size_t certkv_workspace_bytes(const certkv_shape* shape, const certkv_params* params);
+size_t certkv_decode_workspace_bytes(const certkv_shape* shape);
+
+/* a1-a2: observation-window scores.  a_out: fp32 [B*L*H][n], each row a
+ * probability vector (a_j >= 0, sum 1) — §4 and the implementation appendix
+ * ("we normalize directly, rather than re-softmaxing").  K: bf16 as above;
+ * Q_obs: bf16 [B][L][Hq][w][d]. */
+int certkv_score(const certkv_shape* shape, const void* K, const void* Q_obs,
+                 const certkv_params* params, float* a_out,
+                 void* workspace, size_t workspace_bytes, void* stream);
+
+/* a3-a4: per-unit order and allocation curve, exposed for inspection.
+ * a: fp32 [B*L*H][n] scores (e.g. from certkv_score); V bf16 as above.
+ * perm_out: int32 [B*L*H][n], perm_out[u][r] = token at rank r (rank 0 =
+ * highest score, ties by lower index).  c_out: fp64 [B*L*H][n],
+ * c_out[u][b] = c_h(b) for the evicted suffix of ranks b..n-1 (Algorithm 1,
+ * suffix-scan and curve lines). */
+int certkv_curves(const certkv_shape* shape, const void* V, const float* a,
+                  const certkv_params* params, int32_t* perm_out, double* c_out,
+                  void* workspace, size_t workspace_bytes, void* stream);
+
+/* a3-a8 from given scores `a` (fp32 [B*L*H][n], e.g. from certkv_score):
+ * order, curves, exact-budget allocation, selection, tail slot and packing.
+ * budget_live = B_live, live slots per (sequence, layer); it must satisfy
+ * 2H <= B_live <= H*n when tail_slot = 1 and H <= B_live <= H*n when
+ * tail_slot = 0 (else CERTKV_EBUDGET). */
+int certkv_compress_scored(const certkv_shape* shape, const void* K, const void* V,
+                           const float* a, int64_t budget_live,
+                           const certkv_params* params, certkv_packed* out,
+                           void* workspace, size_t workspace_bytes, void* stream);
+
+/* a1-a8: the whole compression pass (Algorithm 1 with the observation-window
+ * scorer in front).  Same contract as certkv_compress_scored. */
+int certkv_compress(const certkv_shape* shape, const void* K, const void* V,
+                    const void* Q_obs, int64_t budget_live,
+                    const certkv_params* params, certkv_packed* out,
+                    void* workspace, size_t workspace_bytes, void* stream);
+
+/* a9: decode attention over the packed cache: for every query head qh of
+ * unit u = (b, l, qh / G), out[b][l][qh] = sum_s softmax_s(scale <q, k_s>) v_s
+ * over the real_counts[u] (+ 1 tail) slots of segment u.  q, out: bf16
+ * [B][L][Hq][d].  `packed` must come from certkv_compress* with the same
+ * shape and tail_slot; scale 0 selects 1/sqrt(d). */
+int certkv_decode_attn(const certkv_shape* shape, const void* q,
+                       const certkv_packed* packed, float scale, int32_t tail_slot,
+                       void* out, void* workspace, size_t workspace_bytes,
+                       void* stream);
+
+/* Synchronise `stream`, then return the device status word (CERTKV_STATUS_*
+ * bits, 0 = clean) that the last compress call on `workspace` left, or -1 if
+ * a CUDA call failed.  Host pointer args: none. */
+int certkv_read_status(const void* workspace, void* stream);
+
+/* Static description of a return code. */
+const char* certkv_strerror(int code);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CERTKV_H */

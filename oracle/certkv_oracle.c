@@ -1,0 +1,510 @@
+/*
+ * certkv_oracle.c — TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, float64 CPU restatement of the CertKV compression pass and of
+ * decode attention over its packed cache, written from "Beyond Sparse Weights:
+ * When Is Attention Compressible?" (§4, Eq. (certkv-curve), Algorithm 1 and the
+ * appendix "CertKV: implementation and exact-budget protocol").  It exists to
+ * check the CUDA library against; only the tests, the package's smoke check and
+ * the benchmark's CPU-baseline leg may load it.  It shares no code, header or
+ * table with the CUDA library.
+ *
+ * Every step is written in the paper's order with naive loops; the only library
+ * primitive is qsort (the per-head sort).  Inputs are the raw bf16 bytes the
+ * GPU consumed, widened exactly to float64.  Readings of points where the paper
+ * is silent are marked READING and listed in the design notes:
+ *   R-A1 scorer constants (mean over the G*w observation rows; causal mask in
+ *        the window; average pool of width `pool`, zero padding, divided by the
+ *        width, over non-window keys only; window keys get the unit's maximum
+ *        pooled score);
+ *   R-A2 ties in the order are broken by the lower token index;
+ *   R-A3 b counts kept tokens, the evicted suffix E(b) is ranks b..n-1;
+ *   R-A5/A6 B_live is given as an integer, alpha as an exact rational;
+ *   R-A7 lambda_hi = 2 max over every b in [0, n-1] and every head + 1;
+ *   R-A8 argmin ties go to the smallest b;
+ *   R-A9 repair adds one token to the head with the smallest marginal
+ *        c(b+1) - c(b) (lowest head index on ties), or, for a surplus, removes
+ *        one from the head with the smallest c(b-1) - c(b);
+ *   R-A10 the tail slot stores the centroids k* = sum a k / m, v* = sum a v / m;
+ *   R-A11 if m == 0 in floating point the slot is the uniform tail mean;
+ *   R-A12 the tail slot enters decode as a plain key/value pair (no logit bias).
+ *
+ * Build: cc -O2 -ffp-contract=off -fPIC -shared (no fused multiply-add, so that
+ * x86 and Arm builds round identically).
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ---------------------------------------------------------------- bf16 ---- */
+
+static double bf16_to_f64(uint16_t h) {
+  uint32_t u = (uint32_t)h << 16;
+  float f;
+  memcpy(&f, &u, sizeof f);
+  return (double)f;
+}
+
+/* Round a double to the nearest bf16, ties to even, in one rounding step. */
+uint16_t oracle_f64_to_bf16(double x) {
+  uint16_t sign = signbit(x) ? 0x8000u : 0u;
+  double ax = fabs(x);
+  if (isnan(x)) return (uint16_t)(sign | 0x7FC0u);
+  if (isinf(x)) return (uint16_t)(sign | 0x7F80u);
+  if (ax == 0.0) return sign;
+  const double min_normal = ldexp(1.0, -126);
+  if (ax < min_normal) {
+    /* subnormal bf16: quantum 2^-133 */
+    double r = nearbyint(ldexp(ax, 133)); /* default rounding: to nearest even */
+    return (uint16_t)(sign | (uint16_t)r); /* r == 128 encodes the min normal */
+  }
+  int e;
+  double f = frexp(ax, &e);          /* ax = f * 2^e, f in [0.5, 1) */
+  double r = nearbyint(ldexp(f, 8)); /* 8 significant bits: r in [128, 256] */
+  if (r == 256.0) { r = 128.0; e += 1; }
+  int biased = e - 1 + 127;          /* value = (r/128) * 2^(e-1) */
+  if (biased >= 255) return (uint16_t)(sign | 0x7F80u);
+  return (uint16_t)(sign | (uint16_t)(biased << 7) | (uint16_t)((int)r - 128));
+}
+
+/* ------------------------------------------------------------- scoring ---- */
+
+/*
+ * Observation-window scores of one unit (a1-a2; §4 "SnapKV's observation-window
+ * score", implementation appendix: a_j = (s_j)_+ / sum_i (s_i)_+).
+ *   K  [n][d]  keys of KV head h;  Qg [G][w][d] observation queries of the G
+ *   query heads that read h.  Writes a[n] (float64).  Returns 0.
+ */
+int oracle_scores(const uint16_t* K, const uint16_t* Qg, int n, int d, int w, int G,
+                  double scale, int pool, int protect, double* a) {
+  const int R = G * w;
+  const int nw = n - w; /* keys outside the observation window */
+  double* s = (double*)calloc((size_t)n, sizeof(double));
+  double* logit = (double*)malloc((size_t)n * sizeof(double));
+  double* qrow = (double*)malloc((size_t)d * sizeof(double));
+  double* st = (double*)malloc((size_t)n * sizeof(double));
+  if (!s || !logit || !qrow || !st) { free(s); free(logit); free(qrow); free(st); return -1; }
+
+  for (int g = 0; g < G; ++g) {
+    for (int t = 0; t < w; ++t) {
+      const uint16_t* q = Qg + ((size_t)g * w + t) * d;
+      for (int i = 0; i < d; ++i) qrow[i] = bf16_to_f64(q[i]);
+      const int visible = nw + t + 1; /* causal: row at position n-w+t sees j <= n-w+t */
+      double mx = -INFINITY;
+      for (int j = 0; j < visible; ++j) {
+        const uint16_t* k = K + (size_t)j * d;
+        double dot = 0.0;
+        for (int i = 0; i < d; ++i) dot += qrow[i] * bf16_to_f64(k[i]);
+        logit[j] = scale * dot;
+        if (logit[j] > mx) mx = logit[j];
+      }
+      double sum = 0.0;
+      for (int j = 0; j < visible; ++j) sum += exp(logit[j] - mx);
+      const double lse = mx + log(sum);
+      for (int j = 0; j < visible; ++j) s[j] += exp(logit[j] - lse);
+    }
+  }
+  for (int j = 0; j < n; ++j) s[j] /= (double)R; /* mean over the R observation rows */
+
+  /* average pool over the non-window keys, zero padding, divided by the width */
+  const int half = pool / 2;
+  double smax = -INFINITY;
+  for (int j = 0; j < nw; ++j) {
+    double acc = 0.0;
+    for (int i = j - half; i <= j + half; ++i)
+      if (i >= 0 && i < nw) acc += s[i];
+    st[j] = acc / (double)pool;
+    if (st[j] > smax) smax = st[j];
+  }
+  for (int j = nw; j < n; ++j) st[j] = protect ? smax : s[j];
+
+  double total = 0.0;
+  for (int j = 0; j < n; ++j) total += (st[j] > 0.0 ? st[j] : 0.0);
+  for (int j = 0; j < n; ++j) a[j] = (st[j] > 0.0 ? st[j] : 0.0) / total;
+
+  free(s); free(logit); free(qrow); free(st);
+  return 0;
+}
+
+/* ------------------------------------------------------------- order ----- */
+
+typedef struct { double a; int32_t j; } scored_t;
+
+static int cmp_desc_then_index(const void* x, const void* y) {
+  const scored_t* p = (const scored_t*)x;
+  const scored_t* q = (const scored_t*)y;
+  if (p->a > q->a) return -1;
+  if (p->a < q->a) return 1;
+  return (p->j < q->j) ? -1 : (p->j > q->j);
+}
+
+/* a3: perm[r] = token at rank r, scores descending, ties by lower index. */
+void oracle_order(const double* a, int n, int32_t* perm) {
+  scored_t* tmp = (scored_t*)malloc((size_t)n * sizeof(scored_t));
+  for (int j = 0; j < n; ++j) { tmp[j].a = a[j]; tmp[j].j = j; }
+  qsort(tmp, (size_t)n, sizeof(scored_t), cmp_desc_then_index);
+  for (int r = 0; r < n; ++r) perm[r] = tmp[r].j;
+  free(tmp);
+}
+
+/* ------------------------------------------------------------- curves ---- */
+
+/*
+ * a4: allocation curve of one unit (implementation appendix: suffix moments
+ * m(b) = sum a_j, W(b) = sum a_j v_j, Q(b) = sum a_j ||v_j||^2 over the evicted
+ * ranks b..n-1, and c(b)^2 = (m(b) Q(b) - ||W(b)||^2)_+ ; Eq. (certkv-curve)).
+ * statistic 0: centred, 1: sqrt(m Q) (uncentred ablation), 2: m (tail mass).
+ */
+void oracle_curve(const double* a, const uint16_t* V, const int32_t* perm, int n, int d,
+                  int statistic, double* c) {
+  double* W = (double*)calloc((size_t)d, sizeof(double));
+  double m = 0.0, Q = 0.0;
+  for (int b = n - 1; b >= 0; --b) {
+    const int j = perm[b];
+    const double aj = a[j];
+    const uint16_t* v = V + (size_t)j * d;
+    double vv = 0.0;
+    for (int i = 0; i < d; ++i) {
+      const double x = bf16_to_f64(v[i]);
+      W[i] += aj * x;
+      vv += x * x;
+    }
+    m += aj;
+    Q += aj * vv;
+    if (statistic == 2) { c[b] = m; continue; }
+    if (statistic == 1) { c[b] = sqrt(m * Q); continue; }
+    double ww = 0.0;
+    for (int i = 0; i < d; ++i) ww += W[i] * W[i];
+    const double c2 = m * Q - ww;
+    c[b] = sqrt(c2 > 0.0 ? c2 : 0.0);
+  }
+  free(W);
+}
+
+/* ---------------------------------------------------------- allocation ---- */
+
+/* b_min of the exact-budget protocol: max{1, floor(alpha * B_real / H)}. */
+int64_t oracle_b_min(int64_t B_real, int H, int64_t alpha_num, int64_t alpha_den) {
+  int64_t v = (alpha_num * B_real) / (alpha_den * (int64_t)H);
+  return v < 1 ? 1 : v;
+}
+
+/* smallest argmin over b in [lo, hi] of c[b] + lambda * b */
+static int argmin_penalised(const double* c, int lo, int hi, double lambda) {
+  int best_b = lo;
+  double best = c[lo] + lambda * (double)lo;
+  for (int b = lo + 1; b <= hi; ++b) {
+    const double f = c[b] + lambda * (double)b;
+    if (f < best) { best = f; best_b = b; }
+  }
+  return best_b;
+}
+
+/*
+ * a5: split B_real real-token slots across H heads (Algorithm 1: b_min,
+ * lambda bisection for T steps, b_h = b_h(lambda_hi), then one-token repair).
+ * curves[h] points at c_h(0..n-1).  B_real is the real-token budget (B_live - H
+ * when one tail slot per head is charged).  Writes b[H]; *repairs = number of
+ * one-token repairs.  Returns 0, or 2 if the budget is infeasible.
+ */
+int oracle_allocate(const double* const* curves, int H, int n, int64_t B_real,
+                    int64_t alpha_num, int64_t alpha_den, int T, int32_t* b,
+                    int64_t* repairs) {
+  const int64_t bmin = oracle_b_min(B_real, H, alpha_num, alpha_den);
+  if (B_real < (int64_t)H * bmin || B_real > (int64_t)H * (n - 1)) return 2;
+  const int lo_b = (int)bmin, hi_b = n - 1;
+
+  double cmax = 0.0;
+  for (int h = 0; h < H; ++h)
+    for (int bb = 0; bb < n; ++bb)
+      if (curves[h][bb] > cmax) cmax = curves[h][bb];
+  double lam_lo = 0.0, lam_hi = 2.0 * cmax + 1.0;
+
+  for (int t = 0; t < T; ++t) {
+    const double lam = (lam_lo + lam_hi) / 2.0;
+    int64_t total = 0;
+    for (int h = 0; h < H; ++h) total += argmin_penalised(curves[h], lo_b, hi_b, lam);
+    if (total > B_real) lam_lo = lam; else lam_hi = lam;
+  }
+  int64_t total = 0;
+  for (int h = 0; h < H; ++h) {
+    b[h] = argmin_penalised(curves[h], lo_b, hi_b, lam_hi);
+    total += b[h];
+  }
+  int64_t steps = 0;
+  while (total < B_real) { /* best-marginal repair: add one token */
+    int best_h = -1;
+    double best = INFINITY;
+    for (int h = 0; h < H; ++h) {
+      if (b[h] >= hi_b) continue;
+      const double delta = curves[h][b[h] + 1] - curves[h][b[h]];
+      if (best_h < 0 || delta < best) { best = delta; best_h = h; }
+    }
+    b[best_h] += 1; total += 1; steps += 1;
+  }
+  while (total > B_real) { /* surplus (not reachable from lambda_hi): remove one */
+    int best_h = -1;
+    double best = INFINITY;
+    for (int h = 0; h < H; ++h) {
+      if (b[h] <= lo_b) continue;
+      const double delta = curves[h][b[h] - 1] - curves[h][b[h]];
+      if (best_h < 0 || delta < best) { best = delta; best_h = h; }
+    }
+    b[best_h] -= 1; total -= 1; steps += 1;
+  }
+  if (repairs) *repairs = steps;
+  return 0;
+}
+
+/* --------------------------------------------------- selection and tail ---- */
+
+static int cmp_int32(const void* x, const void* y) {
+  const int32_t p = *(const int32_t*)x, q = *(const int32_t*)y;
+  return (p > q) - (p < q);
+}
+
+/* a6: kept set = ranks 0..b-1, emitted in ascending token position. */
+void oracle_select(const int32_t* perm, int b, int32_t* kept) {
+  memcpy(kept, perm, (size_t)b * sizeof(int32_t));
+  qsort(kept, (size_t)b, sizeof(int32_t), cmp_int32);
+}
+
+/*
+ * a7: synthetic tail pair over the evicted ranks b..n-1 (§4: r_j = a_j / m,
+ * (k*, v*) = E_{j~r}[(k_j, v_j)]).  Writes kstar[d], vstar[d]; returns m, and
+ * sets *zero_mass when m == 0 (then the uniform tail mean is stored).
+ */
+double oracle_tail(const double* a, const uint16_t* K, const uint16_t* V,
+                   const int32_t* perm, int n, int d, int b, double* kstar,
+                   double* vstar, int* zero_mass) {
+  double m = 0.0;
+  for (int i = 0; i < d; ++i) { kstar[i] = 0.0; vstar[i] = 0.0; }
+  for (int r = b; r < n; ++r) {
+    const int j = perm[r];
+    m += a[j];
+    for (int i = 0; i < d; ++i) {
+      kstar[i] += a[j] * bf16_to_f64(K[(size_t)j * d + i]);
+      vstar[i] += a[j] * bf16_to_f64(V[(size_t)j * d + i]);
+    }
+  }
+  *zero_mass = 0;
+  if (m > 0.0) {
+    for (int i = 0; i < d; ++i) { kstar[i] /= m; vstar[i] /= m; }
+  } else {
+    *zero_mass = 1;
+    for (int i = 0; i < d; ++i) { kstar[i] = 0.0; vstar[i] = 0.0; }
+    for (int r = b; r < n; ++r) {
+      const int j = perm[r];
+      for (int i = 0; i < d; ++i) {
+        kstar[i] += bf16_to_f64(K[(size_t)j * d + i]);
+        vstar[i] += bf16_to_f64(V[(size_t)j * d + i]);
+      }
+    }
+    for (int i = 0; i < d; ++i) { kstar[i] /= (double)(n - b); vstar[i] /= (double)(n - b); }
+  }
+  return m;
+}
+
+/* -------------------------------------------------------- whole pass ----- */
+
+typedef struct {
+  int B, L, Hq, H, n, d, w;
+  double scale;
+  int pool, protect, alpha_num, alpha_den, T, statistic, tail_slot;
+  int64_t B_live;
+} oracle_cfg;
+
+typedef struct {
+  const oracle_cfg* cfg;
+  const uint16_t *K, *V, *Q;
+  const float* a_in;       /* optional: scores to start from (conditioned mode) */
+  double* a;               /* [units][n] */
+  int32_t* perm;           /* [units][n] */
+  double* c;               /* [units][n] */
+  int32_t* counts;         /* [units] */
+  double* tail;            /* [units][2][d] */
+  double* tail_mass;       /* [units] */
+  int64_t* repairs;        /* [B*L] */
+  int* status;             /* [units] */
+  int phase;
+  int next;                /* work counter */
+  pthread_mutex_t lock;
+} job_t;
+
+static int take(job_t* jb, int limit) {
+  pthread_mutex_lock(&jb->lock);
+  int i = jb->next < limit ? jb->next++ : -1;
+  pthread_mutex_unlock(&jb->lock);
+  return i;
+}
+
+static void* worker(void* arg) {
+  job_t* jb = (job_t*)arg;
+  const oracle_cfg* g = jb->cfg;
+  const int units = g->B * g->L * g->H;
+  const int G = g->Hq / g->H;
+  const size_t n = (size_t)g->n, d = (size_t)g->d;
+  if (jb->phase == 0) { /* scores, order and curve per unit */
+    for (int u; (u = take(jb, units)) >= 0;) {
+      const int bl = u / g->H, h = u % g->H;
+      double* a = jb->a + (size_t)u * n;
+      if (jb->a_in) {
+        for (size_t j = 0; j < n; ++j) a[j] = (double)jb->a_in[(size_t)u * n + j];
+      } else {
+        const uint16_t* Qg = jb->Q + ((size_t)bl * g->Hq + (size_t)h * G) * g->w * d;
+        oracle_scores(jb->K + (size_t)u * n * d, Qg, g->n, g->d, g->w, G, g->scale,
+                      g->pool, g->protect, a);
+      }
+      oracle_order(a, g->n, jb->perm + (size_t)u * n);
+      oracle_curve(a, jb->V + (size_t)u * n * d, jb->perm + (size_t)u * n, g->n, g->d,
+                   g->statistic, jb->c + (size_t)u * n);
+    }
+  } else if (jb->phase == 1) { /* allocation per (sequence, layer) */
+    for (int bl; (bl = take(jb, g->B * g->L)) >= 0;) {
+      const double* curves[64];
+      for (int h = 0; h < g->H; ++h) curves[h] = jb->c + ((size_t)bl * g->H + h) * n;
+      const int64_t B_real = g->B_live - (g->tail_slot ? g->H : 0);
+      int rc = oracle_allocate(curves, g->H, g->n, B_real, g->alpha_num, g->alpha_den,
+                               g->T, jb->counts + (size_t)bl * g->H, jb->repairs + bl);
+      for (int h = 0; h < g->H; ++h) jb->status[bl * g->H + h] = rc;
+    }
+  } else { /* tail per unit */
+    for (int u; (u = take(jb, units)) >= 0;) {
+      if (!g->tail_slot) { jb->tail_mass[u] = 0.0; continue; }
+      int zero = 0;
+      jb->tail_mass[u] = oracle_tail(jb->a + (size_t)u * n, jb->K + (size_t)u * n * d,
+                                     jb->V + (size_t)u * n * d, jb->perm + (size_t)u * n,
+                                     g->n, g->d, jb->counts[u],
+                                     jb->tail + (size_t)u * 2 * d,
+                                     jb->tail + (size_t)u * 2 * d + d, &zero);
+      if (zero) jb->status[u] |= 0x100;
+    }
+  }
+  return NULL;
+}
+
+static void run_phase(job_t* jb, int phase, int threads) {
+  jb->phase = phase;
+  jb->next = 0;
+  if (threads <= 1) { worker(jb); return; }
+  pthread_t* tid = (pthread_t*)malloc((size_t)threads * sizeof(pthread_t));
+  for (int i = 0; i < threads; ++i) pthread_create(&tid[i], NULL, worker, jb);
+  for (int i = 0; i < threads; ++i) pthread_join(tid[i], NULL);
+  free(tid);
+}
+
+/*
+ * The whole compression pass over B*L*H units plus the packed cache, in the
+ * library's packed layout.  cfg_i holds {B, L, Hq, H, n, d, w, pool, protect,
+ * alpha_num, alpha_den, T, statistic, tail_slot}; scale and B_live separately.
+ * a_in (fp32 [units][n]) may be NULL; when given, scoring is skipped and the
+ * pass starts from these scores (conditioned mode).  Outputs (all required):
+ *   a [units][n], perm [units][n], c [units][n], counts [units],
+ *   offsets [units+1], positions [B*L*B_live], pk, pv bf16 [B*L*B_live][d],
+ *   tail [units][2][d] (k*, v* before rounding), tail_mass [units],
+ *   repairs [B*L].
+ * Returns 0, 2 (infeasible budget) or 0x100 bit set if some tail had zero mass.
+ */
+int oracle_compress(const int32_t* cfg_i, double scale, int64_t B_live,
+                    const uint16_t* K, const uint16_t* V, const uint16_t* Q,
+                    const float* a_in, int threads,
+                    double* a, int32_t* perm, double* c, int32_t* counts,
+                    int64_t* offsets, int32_t* positions, uint16_t* pk, uint16_t* pv,
+                    double* tail, double* tail_mass, int64_t* repairs) {
+  oracle_cfg g;
+  g.B = cfg_i[0]; g.L = cfg_i[1]; g.Hq = cfg_i[2]; g.H = cfg_i[3]; g.n = cfg_i[4];
+  g.d = cfg_i[5]; g.w = cfg_i[6]; g.pool = cfg_i[7]; g.protect = cfg_i[8];
+  g.alpha_num = cfg_i[9]; g.alpha_den = cfg_i[10]; g.T = cfg_i[11];
+  g.statistic = cfg_i[12]; g.tail_slot = cfg_i[13];
+  g.scale = scale; g.B_live = B_live;
+  if (g.H > 64) return 1;
+  const int units = g.B * g.L * g.H;
+  const size_t n = (size_t)g.n, d = (size_t)g.d;
+
+  job_t jb;
+  memset(&jb, 0, sizeof jb);
+  jb.cfg = &g; jb.K = K; jb.V = V; jb.Q = Q; jb.a_in = a_in;
+  jb.a = a; jb.perm = perm; jb.c = c; jb.counts = counts; jb.tail = tail;
+  jb.tail_mass = tail_mass; jb.repairs = repairs;
+  jb.status = (int*)calloc((size_t)units, sizeof(int));
+  pthread_mutex_init(&jb.lock, NULL);
+
+  run_phase(&jb, 0, threads);
+  run_phase(&jb, 1, threads);
+  int rc = 0;
+  for (int u = 0; u < units; ++u) if (jb.status[u] == 2) rc = 2;
+  if (rc == 0) run_phase(&jb, 2, threads);
+  for (int u = 0; u < units && rc == 0; ++u) if (jb.status[u] & 0x100) rc = 0x100;
+  pthread_mutex_destroy(&jb.lock);
+  free(jb.status);
+  if (rc == 2) return rc;
+
+  /* a8: pack.  Segment u: counts[u] real slots (ascending position) + tail slot. */
+  int32_t* kept = (int32_t*)malloc(n * sizeof(int32_t));
+  int64_t off = 0;
+  for (int u = 0; u < units; ++u) {
+    if (u % g.H == 0) off = (int64_t)(u / g.H) * g.B_live;
+    offsets[u] = off;
+    const int bu = counts[u];
+    oracle_select(perm + (size_t)u * n, bu, kept);
+    for (int s = 0; s < bu; ++s) {
+      const size_t src = ((size_t)u * n + (size_t)kept[s]) * d;
+      memcpy(pk + (size_t)(off + s) * d, K + src, d * sizeof(uint16_t));
+      memcpy(pv + (size_t)(off + s) * d, V + src, d * sizeof(uint16_t));
+      positions[off + s] = kept[s];
+    }
+    off += bu;
+    if (g.tail_slot) {
+      for (size_t i = 0; i < d; ++i) {
+        pk[(size_t)off * d + i] = oracle_f64_to_bf16(tail[(size_t)u * 2 * d + i]);
+        pv[(size_t)off * d + i] = oracle_f64_to_bf16(tail[(size_t)u * 2 * d + d + i]);
+      }
+      positions[off] = -1;
+      off += 1;
+    }
+  }
+  offsets[units] = (int64_t)g.B * g.L * g.B_live;
+  free(kept);
+  return rc;
+}
+
+/* ---------------------------------------------------------------- decode -- */
+
+/*
+ * a9: out[b][l][qh][:] = sum_s softmax_s(scale <q, k_s>) v_s over the slots of
+ * segment (b, l, qh / G), in float64 from the packed bf16 bytes.
+ */
+void oracle_decode(const int32_t* cfg_i, double scale, const uint16_t* q,
+                   const uint16_t* pk, const uint16_t* pv, const int64_t* offsets,
+                   const int32_t* counts, int tail_slot, double* out) {
+  const int B = cfg_i[0], L = cfg_i[1], Hq = cfg_i[2], H = cfg_i[3], d = cfg_i[5];
+  const int G = Hq / H;
+  for (int bl = 0; bl < B * L; ++bl) {
+    for (int qh = 0; qh < Hq; ++qh) {
+      const int u = bl * H + qh / G;
+      const int64_t off = offsets[u];
+      const int slots = counts[u] + (tail_slot ? 1 : 0);
+      const uint16_t* qv = q + ((size_t)bl * Hq + qh) * d;
+      double* o = out + ((size_t)bl * Hq + qh) * d;
+      double* lg = (double*)malloc((size_t)slots * sizeof(double));
+      double mx = -INFINITY;
+      for (int s = 0; s < slots; ++s) {
+        double dot = 0.0;
+        for (int i = 0; i < d; ++i)
+          dot += bf16_to_f64(qv[i]) * bf16_to_f64(pk[(size_t)(off + s) * d + i]);
+        lg[s] = scale * dot;
+        if (lg[s] > mx) mx = lg[s];
+      }
+      double z = 0.0;
+      for (int s = 0; s < slots; ++s) z += exp(lg[s] - mx);
+      for (int i = 0; i < d; ++i) o[i] = 0.0;
+      for (int s = 0; s < slots; ++s) {
+        const double p = exp(lg[s] - mx) / z;
+        for (int i = 0; i < d; ++i) o[i] += p * bf16_to_f64(pv[(size_t)(off + s) * d + i]);
+      }
+      free(lg);
+    }
+  }
+}
