@@ -1,0 +1,400 @@
+#!/usr/bin/env python3
+"""Benchmark of the CertKV hot path on GB300.
+
+One step = the whole compression pass over the workload (scores, order,
+curves, exact-budget allocation, selection, tail slots, packing; every layer
+and sequence in one call) followed by one decode-attention step over the packed
+cache.  Default workload: 32 layers, 32 query / 8 KV heads, d = 128, context
+131072, batch 1, window 64, budget 1/10 (Gaussian keys with Zipf-weighted
+planted keys).  Inputs (17 GB of K/V) are larger than L2, so no flush is
+needed between steps.
+
+Prints one JSON line.  `--impl reference` times the float64 CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "KV tokens compressed/sec and packed-decode GB/s; % of GB300 HBM roofline"
+UNIT = "KV tokens/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="C3")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            pk = json.load(f)
+        return dict(hbm=pk["hbm_gbs"], tensor=pk.get("bf16_tflops_sustained", pk["bf16_tflops"]),
+                    source="measured")
+    return dict(hbm=6800.0, tensor=1700.0, source="fallback")
+
+
+# ------------------------------------------------------------------ clocks --
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# -------------------------------------------------------------- roofline ----
+def kernel_work(wl, B_live, name):
+    """Algorithmic bytes and flops per launch of a kernel."""
+    U = wl.units
+    n, d, R = wl.n, wl.d, wl.G * wl.w
+    kbytes = U * n * d * 2
+    if name in ("score_pass1", "score_pass2"):
+        flops = 2.0 * R * d * n * U
+        # pass 1 streams K from HBM; pass 2 ideally re-reads it from L2
+        return dict(bytes=kbytes if name == "score_pass1" else 0, flops=flops)
+    if name == "curve_agg":
+        return dict(bytes=2 * kbytes, flops=0)       # K and V rows gathered by rank
+    if name == "curve_eval":
+        return dict(bytes=kbytes, flops=0)           # V rows gathered again
+    if name == "sort_scatter":
+        return dict(bytes=U * n * 16, flops=0)       # key + value in and out
+    if name == "copy_rows":
+        slots = wl.B * wl.L * (B_live - wl.H)
+        return dict(bytes=slots * d * 2 * 2 * 2, flops=0)
+    if name == "decode_split":
+        return dict(bytes=wl.B * wl.L * B_live * d * 2 * 2, flops=0)
+    return None
+
+
+def roofline_for(name, work, ms, peaks, traffic=None):
+    t = ms / 1e3
+    if work["flops"] and (work["bytes"] == 0 or
+                          work["flops"] / (peaks["tensor"] * 1e12) >
+                          work["bytes"] / (peaks["hbm"] * 1e9)):
+        ach = work["flops"] / t / 1e12
+        return {"kernel": name, "bound": "tensor", "achieved": round(ach, 2),
+                "peak": peaks["tensor"], "unit": "TFLOP/s", "frac": round(ach / peaks["tensor"], 4),
+                "traffic": traffic, "peak_source": peaks["source"] + " (sustained bf16)"}
+    ach = work["bytes"] / t / 1e9
+    return {"kernel": name, "bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm"],
+            "unit": "GB/s", "frac": round(ach / peaks["hbm"], 4), "traffic": traffic,
+            "peak_source": peaks["source"] + " (copy bandwidth)"}
+
+
+# ----------------------------------------------------------- oracle arms ----
+def oracle_sample(wl, layers, seed, B_live, threads=None):
+    """Run the float64 oracle on the given layers of sequence 0 (CPU inputs)."""
+    import oracle
+    from paper_2608_21541_gb300 import workloads as W
+    total = 0.0
+    for l in layers:
+        K, V, Q = W.draw_layer(wl, 0, l, seed=seed, device="cpu")
+        kb, vb, qb = (W.bf16_bits(x) for x in (K, V, Q))
+        t0 = time.perf_counter()
+        oracle.compress(kb.reshape(1, 1, *kb.shape), vb.reshape(1, 1, *vb.shape),
+                        qb.reshape(1, 1, *qb.shape), B=1, L=1, Hq=wl.Hq, H=wl.H, n=wl.n,
+                        d=wl.d, w=wl.w, B_live=B_live, threads=threads)
+        total += time.perf_counter() - t0
+    return total
+
+
+def run_reference(args, wl, rank):
+    if rank != 0:
+        return
+    threads = os.cpu_count() or 1
+    B_live = wl.B_live
+    times = []
+    for step in range(args.warmup + args.steps):
+        t = oracle_sample(wl, [step % wl.L], args.seed, B_live, threads)
+        if step >= args.warmup:
+            times.append(t)
+    sec = sum(times) / len(times)
+    value = wl.n / sec
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": config_dict(wl, B_live, "float64 CPU oracle, one layer of sequence 0 per step"),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": "one layer (8 KV heads x 131072 tokens) per step, layers "
+                                   "cycled, float64, all host threads"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_dict(wl, B_live, note=""):
+    d = {"workload": f"{wl.name}: {wl.description}", "model": "Llama-3-8B-shaped KV cache",
+         "global_batch": wl.B, "seq_len": wl.n, "layers": wl.L, "q_heads": wl.Hq,
+         "kv_heads": wl.H, "head_dim": wl.d, "obs_window": wl.w,
+         "budget": f"{wl.keep[0]}/{wl.keep[1]} (B_live={B_live} per layer incl. {wl.H} tail slots)",
+         "parallelism": "units (sequence, layer) sharded across ranks, no collective",
+         "l2": "inputs larger than L2 (no flush needed)"}
+    if note:
+        d["note"] = note
+    return d
+
+
+# --------------------------------------------------------------- our arm ----
+def run_ours(args, wl, rank, world):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_21541_gb300 import build as B
+    from paper_2608_21541_gb300 import certkv as ck
+    from paper_2608_21541_gb300 import workloads as W
+
+    B.build()
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    peaks = load_peaks()
+    B_live = wl.B_live
+    K, V, Q = W.draw(wl, seed=args.seed + rank, device=dev)
+    q = W.draw_decode_queries(wl, 0, seed=args.seed + rank, device=dev)
+    params = ck.certkv_default_params()
+    shape = ck.shape_of(K, Q)
+    ws = ck.workspace(ck.certkv_workspace_bytes(shape, params), dev)
+    dshape = ck.certkv_shape(wl.B, wl.L, wl.Hq, wl.H, 2, wl.d, 1)
+    dws = ck.workspace(ck.certkv_decode_workspace_bytes(dshape), dev)
+    packed = ck.Packed.empty(wl.B, wl.L, wl.H, wl.d, B_live, dev)
+    out = torch.empty_like(q)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        ck.certkv_compress(K, V, Q, B_live, params, out=packed, ws=ws, stream=stream)
+        ck.certkv_decode_attn(q, packed, hkv=wl.H, out=out, ws=dws, stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    status = ck.certkv_read_status(ws)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    clocks = ClockSampler(local)
+    ck.certkv_trace_enable(True)
+    ck.certkv_trace_report()  # clear
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    trace = ck.certkv_trace_report()
+    ck.certkv_trace_enable(False)
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    tokens = wl.B * wl.L * wl.n
+    value = world * tokens / (ms / 1e3)
+
+    # per-kernel shares and the dominant kernel's roofline
+    kernels = {}
+    launches = 0
+    total_ms = sum(v[1] for v in trace.values()) or 1.0
+    for name, (cnt, tms) in sorted(trace.items(), key=lambda kv: -kv[1][1]):
+        launches += cnt
+        kernels[name] = {"launches_per_step": cnt / args.steps,
+                         "ms_per_step": round(tms / args.steps, 4),
+                         "share": round(tms / total_ms, 4)}
+    roof_all = {}
+    for name in kernels:
+        work = kernel_work(wl, B_live, name)
+        if work:
+            per_launch_ms = trace[name][1] / trace[name][0]
+            launches_per_step = trace[name][0] / args.steps
+            w1 = {k: v / launches_per_step for k, v in work.items()}
+            roof_all[name] = roofline_for(name, w1, per_launch_ms, peaks)
+    dominant = next(iter(kernels))
+    roof = roof_all.get(dominant) or next(iter(roof_all.values()))
+
+    decode_ms = kernels.get("decode_split", {}).get("ms_per_step", 0) + \
+        kernels.get("decode_merge", {}).get("ms_per_step", 0)
+    decode_bytes = wl.B * wl.L * B_live * wl.d * 2 * 2
+    compress_ms = ms - decode_ms
+    roof_bytes = wl.B * wl.L * (wl.H * wl.n * wl.d * 2 * 2 + B_live * wl.d * 2 * 2)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": config_dict(wl, B_live),
+        "compress_ms": compress_ms,
+        "compress_hbm_roofline": {
+            "bytes": roof_bytes, "achieved_GBps": round(roof_bytes / (compress_ms / 1e3) / 1e9, 1),
+            "peak": peaks["hbm"], "frac": round(roof_bytes / (compress_ms / 1e3) / 1e9 /
+                                                peaks["hbm"], 4),
+            "definition": "K+V read + packed cache written, over the compression time"},
+        "decode_GBps": round(decode_bytes / (decode_ms / 1e3) / 1e9, 1) if decode_ms else None,
+        "roofline": roof, "kernels": kernels, "kernel_rooflines": roof_all,
+        "gpu_launches": launches, "device_status": status,
+        "clocks": clk,
+    }
+
+    if not args.no_e2e:
+        line["e2e"] = run_e2e(args, wl, K, V, Q, q, params, ws, dws, dev, stream, world, B_live)
+    del K, V, Q
+    torch.cuda.empty_cache()
+    if rank == 0 and world == 1 and not args.no_cpu:
+        threads = os.cpu_count() or 1
+        layers = [0, 1]
+        t = oracle_sample(wl, layers, args.seed, B_live, threads)
+        line["cpu_baseline"] = {"value": len(layers) * wl.n / t, "unit": UNIT, "cores": threads,
+                                "kind": "oracle",
+                                "sample": f"layers {layers} of sequence 0 (8 KV heads x "
+                                          f"{wl.n} tokens each), float64, all host threads"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, wl, K, V, Q, q, params, ws, dws, dev, stream, world, B_live):
+    """Same metric through the public API with host buffers: pinned host ->
+    device copies of the step's inputs, compress, decode, and the packed cache
+    and decode output copied back, all inside the timed region."""
+    import torch
+
+    from paper_2608_21541_gb300 import certkv as ck
+    hK = K.cpu().pin_memory()
+    hV = V.cpu().pin_memory()
+    hQ = Q.cpu().pin_memory()
+    hq = q.cpu().pin_memory()
+    dK, dV, dQ, dq = (torch.empty_like(x) for x in (K, V, Q, q))
+    packed = ck.Packed.empty(wl.B, wl.L, wl.H, wl.d, B_live, dev)
+    out = torch.empty_like(q)
+    host_out = dict(k=torch.empty(packed.k.shape, dtype=torch.bfloat16, pin_memory=True),
+                    v=torch.empty(packed.v.shape, dtype=torch.bfloat16, pin_memory=True),
+                    pos=torch.empty(packed.positions.shape, dtype=torch.int32, pin_memory=True),
+                    cnt=torch.empty(packed.real_counts.shape, dtype=torch.int32, pin_memory=True),
+                    off=torch.empty(packed.offsets.shape, dtype=torch.int64, pin_memory=True),
+                    out=torch.empty(q.shape, dtype=torch.bfloat16, pin_memory=True))
+
+    def step():
+        dK.copy_(hK, non_blocking=True)
+        dV.copy_(hV, non_blocking=True)
+        dQ.copy_(hQ, non_blocking=True)
+        dq.copy_(hq, non_blocking=True)
+        ck.certkv_compress(dK, dV, dQ, B_live, params, out=packed, ws=ws, stream=stream)
+        ck.certkv_decode_attn(dq, packed, hkv=wl.H, out=out, ws=dws, stream=stream)
+        host_out["k"].copy_(packed.k, non_blocking=True)
+        host_out["v"].copy_(packed.v, non_blocking=True)
+        host_out["pos"].copy_(packed.positions, non_blocking=True)
+        host_out["cnt"].copy_(packed.real_counts, non_blocking=True)
+        host_out["off"].copy_(packed.offsets, non_blocking=True)
+        host_out["out"].copy_(out, non_blocking=True)
+
+    step()
+    torch.cuda.synchronize()
+    steps = max(1, min(args.steps, 5))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    h2d = sum(x.numel() * x.element_size() for x in (hK, hV, hQ, hq))
+    d2h = sum(x.numel() * x.element_size() for x in host_out.values())
+    return {"value": world * wl.B * wl.L * wl.n / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
+            "steps": steps, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+
+def main():
+    args = parse()
+    from paper_2608_21541_gb300 import workloads as W
+    wl = W.WORKLOADS[args.config]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+    if args.impl == "reference":
+        run_reference(args, wl, rank)
+    else:
+        run_ours(args, wl, rank, world)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

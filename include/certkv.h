@@ -183,6 +183,17 @@ int certkv_decode_attn(const certkv_shape* shape, const void* q,
  * a CUDA call failed.  Host pointer args: none. */
 int certkv_read_status(const void* workspace, void* stream);
 
+/* Profiling aid, not part of the paper's method: when enabled (on = 1) every
+ * kernel launch of the library is bracketed by two CUDA events recorded on
+ * its stream (a pool of events is created once, by the first enable call on
+ * the current device); certkv_trace_report() synchronises, writes one line
+ * "name launches total_ms" per kernel into the host buffer `buf` (len bytes),
+ * clears the records and returns the bytes written, or -1 if the buffer is too
+ * small or a CUDA call failed.  certkv_trace_enable returns CERTKV_OK or
+ * CERTKV_ECUDA. */
+int certkv_trace_enable(int on);
+int certkv_trace_report(char* buf, size_t len);
+
 /* Static description of a return code. */
 const char* certkv_strerror(int code);
 

@@ -1,0 +1,337 @@
+// api.cu — the C ABI (include/certkv.h): host-side validation, workspace
+// carve-up and the launch sequence of each entry point.  Validation runs
+// before any launch; a call that returns an error has enqueued nothing.
+#include <math.h>
+#include <string.h>
+
+#include "../../include/certkv.h"
+#include "common.cuh"
+#include "internal.cuh"
+
+namespace certkv {
+
+namespace {
+
+size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+
+bool is_pow2_le16(int g) { return g == 1 || g == 2 || g == 4 || g == 8 || g == 16; }
+
+int check_shape(const certkv_shape* s) {
+  if (!s) return CERTKV_EINVAL;
+  if (s->batch < 1 || s->layers < 1 || s->hq < 1 || s->hkv < 1) return CERTKV_EINVAL;
+  if (s->d != kD) return CERTKV_EINVAL;
+  if (s->hkv > 32 || s->hq % s->hkv != 0) return CERTKV_EINVAL;
+  if (!is_pow2_le16(s->hq / s->hkv)) return CERTKV_EINVAL;
+  if (s->w < 1 || s->w >= s->n || s->n > (1 << 24)) return CERTKV_EINVAL;
+  const long long units = (long long)s->batch * s->layers * s->hkv;
+  if (units > (1LL << 24)) return CERTKV_EINVAL;
+  return CERTKV_OK;
+}
+
+int check_params(const certkv_params* q) {
+  if (!q) return CERTKV_EINVAL;
+  if (!(q->scale >= 0.0f) || !isfinite(q->scale)) return CERTKV_EINVAL;
+  if (q->pool_kernel < 1 || (q->pool_kernel & 1) == 0 || q->pool_kernel > 255) return CERTKV_EINVAL;
+  if (q->protect_window != 0 && q->protect_window != 1) return CERTKV_EINVAL;
+  if (q->alpha_den < 1 || q->alpha_num < 0 || q->alpha_num > q->alpha_den) return CERTKV_EINVAL;
+  if (q->bisect_steps < 0 || q->bisect_steps > 200) return CERTKV_EINVAL;
+  if (q->statistic < 0 || q->statistic > 2) return CERTKV_EINVAL;
+  if (q->tail_slot != 0 && q->tail_slot != 1) return CERTKV_EINVAL;
+  return CERTKV_OK;
+}
+
+// Fill the problem description; budget_live < 0 means "no budget needed".
+int make_prob(const certkv_shape* s, const certkv_params* q, int64_t budget_live, Prob* p) {
+  int rc = check_shape(s);
+  if (rc) return rc;
+  rc = check_params(q);
+  if (rc) return rc;
+  Prob& P = *p;
+  memset(&P, 0, sizeof P);
+  P.B = s->batch; P.L = s->layers; P.Hq = s->hq; P.H = s->hkv; P.n = s->n; P.d = s->d;
+  P.w = s->w; P.G = s->hq / s->hkv; P.R = P.G * P.w;
+  P.units = P.B * P.L * P.H;
+  P.bl = P.B * P.L;
+  P.scale = q->scale > 0.0f ? q->scale : (float)(1.0 / sqrt((double)s->d));
+  P.scale_log2 = P.scale * 1.4426950408889634f;
+  P.pool = q->pool_kernel; P.protect = q->protect_window;
+  P.alpha_num = q->alpha_num; P.alpha_den = q->alpha_den; P.T = q->bisect_steps;
+  P.statistic = q->statistic; P.tail_slot = q->tail_slot;
+  P.score_warps = (P.R + 15) / 16 < 16 ? (P.R + 15) / 16 : 16;
+  P.row_blocks = (P.R + 16 * P.score_warps - 1) / (16 * P.score_warps);
+  P.key_splits = (P.n + kScoreKeysPerCta - 1) / kScoreKeysPerCta;
+  P.sort_tiles = (P.n + kSortTile - 1) / kSortTile;
+  P.chunks = (P.n + kChunk - 1) / kChunk;
+  if (budget_live >= 0) {
+    const int64_t H = P.H;
+    const int64_t lo = P.tail_slot ? 2 * H : H;
+    if (budget_live < lo || budget_live > H * (int64_t)P.n) return CERTKV_EBUDGET;
+    P.B_live = budget_live;
+    P.B_real = budget_live - (P.tail_slot ? H : 0);
+    int64_t bmin = ((int64_t)P.alpha_num * P.B_real) / ((int64_t)P.alpha_den * H);
+    if (bmin < 1) bmin = 1;
+    if (P.B_real < H * bmin || P.B_real > H * (int64_t)(P.n - 1)) return CERTKV_EBUDGET;
+    P.b_min = (int)bmin;
+  } else {
+    P.b_min = 1;
+  }
+  P.hull_segs = (P.n - P.b_min + kHullSeg - 1) / kHullSeg;
+  return CERTKV_OK;
+}
+
+}  // namespace
+
+Layout make_layout(const Prob& p) {
+  Layout ly;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align256(off + bytes);
+    return o;
+  };
+  const size_t U = (size_t)p.units, n = (size_t)p.n;
+  ly.status = take(256);
+  ly.lse_part = take(U * p.R * p.key_splits * sizeof(float2));
+  ly.lse = take(U * p.R * sizeof(float));
+  ly.s_part = take(U * p.row_blocks * n * sizeof(float));
+  ly.s_tmp = take(U * n * sizeof(float));
+  ly.a = take(U * n * sizeof(float));
+  ly.keys0 = take(U * n * 4);
+  ly.keys1 = take(U * n * 4);
+  ly.vals0 = take(U * n * 4);
+  ly.vals1 = take(U * n * 4);
+  ly.hist = take(U * 256 * p.sort_tiles * 4);
+  ly.agg_mq = take(U * p.chunks * sizeof(float4));
+  ly.agg_v = take(U * p.chunks * kD * sizeof(float));
+  ly.agg_k = take(U * p.chunks * kD * sizeof(float));
+  ly.base_mq = take(U * p.chunks * sizeof(float4));
+  ly.base_v = take(U * p.chunks * kD * sizeof(float2));
+  ly.base_k = take(U * p.chunks * kD * sizeof(float2));
+  ly.curve = take(U * n * sizeof(float2));
+  ly.cmax = take(U * sizeof(unsigned long long));
+  ly.cand = take(U * n * sizeof(int32_t));
+  // the candidate counts are sized for the smallest b_min (1) so that one
+  // workspace size serves every budget of a shape
+  const size_t segs = (size_t)((p.n - 1 + kHullSeg - 1) / kHullSeg) + 1;
+  ly.ncand = take(U * segs * sizeof(int32_t));
+  ly.total = off;
+  return ly;
+}
+
+}  // namespace certkv
+
+namespace certkv_api {
+
+using namespace certkv;
+
+int cuda_ok(cudaError_t e) { return e == cudaSuccess ? CERTKV_OK : CERTKV_ECUDA; }
+
+bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
+
+// key-init for caller-given scores: keys0 = ~bits(a), vals0 = index; flags
+// negative or non-finite scores.
+__global__ void key_init_kernel(Prob p, const float* __restrict__ a, uint32_t* __restrict__ keys,
+                                int32_t* __restrict__ vals, uint32_t* status) {
+  const size_t total = (size_t)p.units * p.n;
+  bool bad = false;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const float x = a[i];
+    if (!(x >= 0.0f && x <= 3.0e38f)) bad = true;
+    keys[i] = score_key(x > 0.0f ? x : 0.0f);
+    vals[i] = (int32_t)(i % (size_t)p.n);
+  }
+  if (bad) raise_status(status, CERTKV_STATUS_NONFINITE);
+}
+
+int check_ws(const Prob& p, void* ws, size_t ws_bytes, Layout* ly) {
+  *ly = make_layout(p);
+  if (!ws || !aligned(ws, 256) || ws_bytes < ly->total) return CERTKV_EWORKSPACE;
+  return CERTKV_OK;
+}
+
+int check_packed(const Prob& p, const certkv_packed* out) {
+  if (!out || !out->k || !out->v || !out->offsets || !out->real_counts || !out->positions)
+    return CERTKV_EINVAL;
+  if (!aligned(out->k, 16) || !aligned(out->v, 16)) return CERTKV_EINVAL;
+  if (out->capacity_slots < (int64_t)p.bl * p.B_live) return CERTKV_ECAPACITY;
+  return CERTKV_OK;
+}
+
+int run_scored(const Prob& p, const Layout& ly, char* ws, const void* K, const void* V,
+               const float* a, certkv_packed* out, cudaStream_t st) {
+  launch_sort(p, ly, ws, a, st);
+  launch_curves(p, ly, ws, K, V, p.tail_slot != 0, st);
+  launch_allocate(p, ly, ws, out->real_counts, out->offsets, st);
+  launch_pack(p, ly, ws, K, V, a, out->k, out->v, out->offsets, out->real_counts, out->positions,
+              out->tail_f32, out->tail_mass, st);
+  return cuda_ok(cudaGetLastError());
+}
+
+}  // namespace certkv_api
+
+using namespace certkv;
+using namespace certkv_api;
+
+extern "C" {
+
+void certkv_default_params(certkv_params* p) {
+  if (!p) return;
+  p->scale = 0.0f;
+  p->pool_kernel = 5;
+  p->protect_window = 1;
+  p->alpha_num = 1;
+  p->alpha_den = 5;
+  p->bisect_steps = 40;
+  p->statistic = CERTKV_STAT_CENTERED;
+  p->tail_slot = 1;
+}
+
+int64_t certkv_live_budget(int32_t n, int32_t hkv, int64_t keep_num, int64_t keep_den) {
+  if (n < 1 || hkv < 1 || keep_num < 0 || keep_den < 1 || keep_num > keep_den) return -1;
+  return (int64_t)hkv * (((int64_t)n * keep_num) / keep_den);
+}
+
+size_t certkv_workspace_bytes(const certkv_shape* shape, const certkv_params* params) {
+  Prob p;
+  if (make_prob(shape, params, -1, &p)) return 0;
+  return make_layout(p).total;
+}
+
+size_t certkv_decode_workspace_bytes(const certkv_shape* shape) {
+  if (check_shape(shape)) return 0;
+  certkv_params q;
+  certkv_default_params(&q);
+  Prob p;
+  if (make_prob(shape, &q, -1, &p)) return 0;
+  return decode_workspace(p);
+}
+
+int certkv_score(const certkv_shape* shape, const void* K, const void* Q_obs,
+                 const certkv_params* params, float* a_out, void* workspace,
+                 size_t workspace_bytes, void* stream) {
+  Prob p;
+  int rc = make_prob(shape, params, -1, &p);
+  if (rc) return rc;
+  if (!K || !Q_obs || !a_out) return CERTKV_EINVAL;
+  Layout ly;
+  if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = reinterpret_cast<char*>(workspace);
+  if ((rc = cuda_ok(cudaMemsetAsync(ws + ly.status, 0, 256, st)))) return rc;
+  launch_score(p, ly, ws, K, Q_obs, a_out, st);
+  return cuda_ok(cudaGetLastError());
+}
+
+int certkv_curves(const certkv_shape* shape, const void* V, const float* a,
+                  const certkv_params* params, int32_t* perm_out, double* c_out, void* workspace,
+                  size_t workspace_bytes, void* stream) {
+  Prob p;
+  int rc = make_prob(shape, params, -1, &p);
+  if (rc) return rc;
+  if (!V || !a || (!perm_out && !c_out)) return CERTKV_EINVAL;
+  Layout ly;
+  if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = reinterpret_cast<char*>(workspace);
+  if ((rc = cuda_ok(cudaMemsetAsync(ws + ly.status, 0, 256, st)))) return rc;
+  {
+    TraceScope ts_("key_init", st);
+    key_init_kernel<<<1024, 256, 0, st>>>(p, a, reinterpret_cast<uint32_t*>(ws + ly.keys0),
+                                          reinterpret_cast<int32_t*>(ws + ly.vals0),
+                                          reinterpret_cast<uint32_t*>(ws + ly.status));
+  }
+  launch_sort(p, ly, ws, a, st);
+  launch_curves(p, ly, ws, V, V, false, st);
+  launch_export_curves(p, ly, ws, perm_out, c_out, st);
+  return cuda_ok(cudaGetLastError());
+}
+
+int certkv_compress_scored(const certkv_shape* shape, const void* K, const void* V,
+                           const float* a, int64_t budget_live, const certkv_params* params,
+                           certkv_packed* out, void* workspace, size_t workspace_bytes,
+                           void* stream) {
+  Prob p;
+  if (budget_live < 0) return CERTKV_EBUDGET;
+  int rc = make_prob(shape, params, budget_live, &p);
+  if (rc) return rc;
+  if (!K || !V || !a) return CERTKV_EINVAL;
+  if ((rc = check_packed(p, out))) return rc;
+  Layout ly;
+  if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = reinterpret_cast<char*>(workspace);
+  if ((rc = cuda_ok(cudaMemsetAsync(ws + ly.status, 0, 256, st)))) return rc;
+  {
+    TraceScope ts_("key_init", st);
+    key_init_kernel<<<1024, 256, 0, st>>>(p, a, reinterpret_cast<uint32_t*>(ws + ly.keys0),
+                                          reinterpret_cast<int32_t*>(ws + ly.vals0),
+                                          reinterpret_cast<uint32_t*>(ws + ly.status));
+  }
+  return run_scored(p, ly, ws, K, V, a, out, st);
+}
+
+int certkv_compress(const certkv_shape* shape, const void* K, const void* V, const void* Q_obs,
+                    int64_t budget_live, const certkv_params* params, certkv_packed* out,
+                    void* workspace, size_t workspace_bytes, void* stream) {
+  Prob p;
+  if (budget_live < 0) return CERTKV_EBUDGET;
+  int rc = make_prob(shape, params, budget_live, &p);
+  if (rc) return rc;
+  if (!K || !V || !Q_obs) return CERTKV_EINVAL;
+  if ((rc = check_packed(p, out))) return rc;
+  Layout ly;
+  if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = reinterpret_cast<char*>(workspace);
+  if ((rc = cuda_ok(cudaMemsetAsync(ws + ly.status, 0, 256, st)))) return rc;
+  float* a = reinterpret_cast<float*>(ws + ly.a);
+  launch_score(p, ly, ws, K, Q_obs, a, st);
+  return run_scored(p, ly, ws, K, V, a, out, st);
+}
+
+int certkv_decode_attn(const certkv_shape* shape, const void* q, const certkv_packed* packed,
+                       float scale, int32_t tail_slot, void* out, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+  int rc = check_shape(shape);
+  if (rc) return rc;
+  if (!q || !packed || !packed->k || !packed->v || !packed->offsets || !packed->real_counts || !out)
+    return CERTKV_EINVAL;
+  if (!aligned(packed->k, 16) || !aligned(packed->v, 16) || !aligned(q, 16)) return CERTKV_EINVAL;
+  if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
+  if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
+  certkv_params prm;
+  certkv_default_params(&prm);
+  Prob p;
+  if ((rc = make_prob(shape, &prm, -1, &p))) return rc;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < decode_workspace(p))
+    return CERTKV_EWORKSPACE;
+  const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  launch_decode(p, q, packed->k, packed->v, packed->offsets, packed->real_counts, tail_slot, sc,
+                out, reinterpret_cast<char*>(workspace), st);
+  return cuda_ok(cudaGetLastError());
+}
+
+int certkv_read_status(const void* workspace, void* stream) {
+  if (!workspace) return -1;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return -1;
+  uint32_t v = 0;
+  if (cudaMemcpy(&v, workspace, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
+  return (int)v;
+}
+
+const char* certkv_strerror(int code) {
+  switch (code) {
+    case CERTKV_OK: return "ok";
+    case CERTKV_EINVAL: return "invalid shape, pointer or parameter";
+    case CERTKV_EBUDGET: return "infeasible budget (need 2H <= B_live <= H*n with a tail slot)";
+    case CERTKV_EWORKSPACE: return "workspace missing, misaligned or too small";
+    case CERTKV_ECAPACITY: return "packed-cache capacity below B*L*B_live slots";
+    case CERTKV_ECUDA: return "CUDA runtime error";
+    default: return "unknown error";
+  }
+}
+
+}  // extern "C"

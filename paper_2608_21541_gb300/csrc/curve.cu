@@ -1,0 +1,323 @@
+// curve.cu — a4: suffix moments and the allocation curve of every unit.
+//
+// Implementation appendix (and Eq. certkv-curve): over the score-sorted axis,
+// for the evicted suffix E(b) = ranks b..n-1,
+//   m(b) = sum a_j,  W(b) = sum a_j v_j,  Q(b) = sum a_j ||v_j||^2,
+//   c(b)^2 = (m(b) Q(b) - ||W(b)||^2)_+ .
+// The ranks are cut into chunks of kChunk; one warp owns a chunk.
+//   agg     gathers V (and K, for the tail slot) in rank order and writes the
+//           chunk sums of a, a||v||^2 (double-float), a v and a k (fp32), and
+//           ||v||^2 per rank;
+//   prefix  suffix-sums the chunk sums over chunks in double-float;
+//   curve   walks each chunk from its last rank down, W(b) = W_base + P(b)
+//           with P the in-chunk partial, and evaluates
+//           c^2 = m Q - (||W_base||^2 + <2 W_base + P, P>) in double-float.
+// The scalar sums that dominate c^2 (m, Q, ||W_base||^2) are carried in
+// double-float so that c(b) agrees with a float64 evaluation to ~1e-13; the
+// small in-chunk vector terms stay in fp32.
+#include "common.cuh"
+#include "internal.cuh"
+
+namespace certkv {
+
+namespace {
+
+__device__ __forceinline__ void load_row4(const __nv_bfloat16* row, int lane, float (&x)[4]) {
+  uint2 raw = __ldg(reinterpret_cast<const uint2*>(row) + lane);
+  x[0] = bf16lo(raw.x);
+  x[1] = bf16hi(raw.x);
+  x[2] = bf16lo(raw.y);
+  x[3] = bf16hi(raw.y);
+}
+
+// lane t ends with sum over lanes of v[t]  (31 shuffles)
+__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      float keep = upper ? v[i + o] : v[i];
+      float send = upper ? v[i] : v[i + o];
+      v[i] = keep + __shfl_xor_sync(kFull, send, o);
+    }
+  }
+  return v[0];
+}
+
+}  // namespace
+
+// grid = (ceil(chunks / 4), units), block = 128 (one warp per chunk)
+__global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* __restrict__ keys,
+                                                        const int32_t* __restrict__ perm,
+                                                        const __nv_bfloat16* __restrict__ K,
+                                                        const __nv_bfloat16* __restrict__ V,
+                                                        bool need_k, float4* __restrict__ agg_mq,
+                                                        float* __restrict__ agg_v,
+                                                        float* __restrict__ agg_k,
+                                                        float* __restrict__ yrank) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int chunk = blockIdx.x * 4 + warp;
+  const int u = blockIdx.y;
+  if (chunk >= p.chunks) return;
+  const int n = p.n;
+  const int r0 = chunk * kChunk, r1 = min(n, r0 + kChunk);
+  const uint32_t* ku = keys + (size_t)u * n;
+  const int32_t* pu = perm + (size_t)u * n;
+  const __nv_bfloat16* Vu = V + (size_t)u * n * kD;
+  const __nv_bfloat16* Ku = K + (size_t)u * n * kD;
+
+  float sv[4] = {0.f, 0.f, 0.f, 0.f}, sk[4] = {0.f, 0.f, 0.f, 0.f};
+  DF m = df_make(0.f), q = df_make(0.f);
+  for (int rb = r0; rb < r1; rb += 32) {
+    const int r = rb + lane;
+    const bool ok = r < r1;
+    const float at = ok ? key_score(ku[r]) : 0.f;
+    const int jt = ok ? pu[r] : 0;
+    const int cnt = min(32, r1 - rb);
+    float yp[32];
+#pragma unroll
+    for (int s = 0; s < 32; ++s) {
+      yp[s] = 0.f;
+      if (s < cnt) {
+        const float as = __shfl_sync(kFull, at, s);
+        const int js = __shfl_sync(kFull, jt, s);
+        float v[4];
+        load_row4(Vu + (size_t)js * kD, lane, v);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          sv[i] = fmaf(as, v[i], sv[i]);
+          yp[s] = fmaf(v[i], v[i], yp[s]);
+        }
+        if (need_k) {
+          float k4[4];
+          load_row4(Ku + (size_t)js * kD, lane, k4);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) sk[i] = fmaf(as, k4[i], sk[i]);
+        }
+      }
+    }
+    const float yt = reduce_scatter32(yp, lane);
+    if (ok) yrank[(size_t)u * n + r] = yt;
+    DF dm = df_make(at);
+    DF dq = ok ? two_prod(at, yt) : df_make(0.f);
+    m = df_add(m, warp_sum_df(dm));
+    q = df_add(q, warp_sum_df(dq));
+  }
+  const size_t ci = (size_t)u * p.chunks + chunk;
+  reinterpret_cast<float4*>(agg_v + ci * kD)[lane] = make_float4(sv[0], sv[1], sv[2], sv[3]);
+  if (need_k)
+    reinterpret_cast<float4*>(agg_k + ci * kD)[lane] = make_float4(sk[0], sk[1], sk[2], sk[3]);
+  if (lane == 0) agg_mq[ci] = make_float4(m.hi, m.lo, q.hi, q.lo);
+}
+
+// grid = units, block = 128 (one thread per dimension): exclusive suffix sums
+// over chunks, in double-float.
+__global__ void __launch_bounds__(128) curve_prefix_kernel(Prob p, const float4* __restrict__ agg_mq,
+                                                           const float* __restrict__ agg_v,
+                                                           const float* __restrict__ agg_k,
+                                                           bool need_k, float4* __restrict__ base_mq,
+                                                           float2* __restrict__ base_v,
+                                                           float2* __restrict__ base_k) {
+  const int u = blockIdx.x, i = threadIdx.x;
+  const size_t c0 = (size_t)u * p.chunks;
+  DF rv = df_make(0.f), rk = df_make(0.f), rm = df_make(0.f), rq = df_make(0.f);
+  float nv = agg_v[(c0 + p.chunks - 1) * kD + i];
+  float nk = need_k ? agg_k[(c0 + p.chunks - 1) * kD + i] : 0.f;
+  float4 nmq = agg_mq[c0 + p.chunks - 1];
+  for (int c = p.chunks - 1; c >= 0; --c) {
+    const float cv = nv, ck = nk;
+    const float4 cmq = nmq;
+    if (c > 0) {  // prefetch the next (lower) chunk
+      nv = agg_v[(c0 + c - 1) * kD + i];
+      if (need_k) nk = agg_k[(c0 + c - 1) * kD + i];
+      nmq = agg_mq[c0 + c - 1];
+    }
+    base_v[(c0 + c) * kD + i] = make_float2(rv.hi, rv.lo);
+    if (need_k) base_k[(c0 + c) * kD + i] = make_float2(rk.hi, rk.lo);
+    if (i == 0) base_mq[c0 + c] = make_float4(rm.hi, rm.lo, rq.hi, rq.lo);
+    rv = df_add_f(rv, cv);
+    if (need_k) rk = df_add_f(rk, ck);
+    rm = df_add(rm, DF{cmq.x, cmq.y});
+    rq = df_add(rq, DF{cmq.z, cmq.w});
+  }
+}
+
+// grid = (ceil(chunks / 4), units), block = 128 (one warp per chunk)
+__global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t* __restrict__ keys,
+                                                         const int32_t* __restrict__ perm,
+                                                         const __nv_bfloat16* __restrict__ V,
+                                                         const float* __restrict__ yrank,
+                                                         const float4* __restrict__ base_mq,
+                                                         const float2* __restrict__ base_v,
+                                                         float2* __restrict__ curve,
+                                                         unsigned long long* __restrict__ cmax,
+                                                         uint32_t* status) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int chunk = blockIdx.x * 4 + warp;
+  const int u = blockIdx.y;
+  if (chunk >= p.chunks) return;
+  const int n = p.n;
+  const int r0 = chunk * kChunk, r1 = min(n, r0 + kChunk);
+  const uint32_t* ku = keys + (size_t)u * n;
+  const int32_t* pu = perm + (size_t)u * n;
+  const __nv_bfloat16* Vu = V + (size_t)u * n * kD;
+  const size_t ci = (size_t)u * p.chunks + chunk;
+
+  const float4 bmq = base_mq[ci];
+  const DF M0{bmq.x, bmq.y}, Q0{bmq.z, bmq.w};
+  float wb2x[4];
+  DF wb2 = df_make(0.f);
+  {
+    const float4* bv = reinterpret_cast<const float4*>(base_v + ci * kD) + lane * 2;
+    float4 x0 = bv[0], x1 = bv[1];
+    const float hi[4] = {x0.x, x0.z, x1.x, x1.z}, lo[4] = {x0.y, x0.w, x1.y, x1.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      wb2x[i] = 2.0f * hi[i];
+      DF sq = two_prod(hi[i], hi[i]);
+      sq = df_add_f(sq, 2.0f * hi[i] * lo[i]);
+      wb2 = df_add(wb2, sq);
+    }
+    wb2 = warp_sum_df(wb2);
+  }
+  float P[4] = {0.f, 0.f, 0.f, 0.f};
+  DF carry_m = df_make(0.f), carry_q = df_make(0.f);
+  unsigned long long best = 0ull;
+  bool bad = false;
+  const int nb = (r1 - r0 + 31) / 32;
+  for (int bi = nb - 1; bi >= 0; --bi) {
+    const int rb = r0 + bi * 32;
+    const int r = rb + lane;
+    const bool ok = r < r1;
+    const float at = ok ? key_score(ku[r]) : 0.f;
+    const int jt = ok ? pu[r] : 0;
+    const float yt = ok ? yrank[(size_t)u * n + r] : 0.f;
+    const int cnt = min(32, r1 - rb);
+    float xp[32];
+#pragma unroll
+    for (int s = 31; s >= 0; --s) {
+      const float as = __shfl_sync(kFull, at, s);
+      const int js = __shfl_sync(kFull, jt, s);
+      xp[s] = 0.f;
+      if (s < cnt) {
+        float v[4];
+        load_row4(Vu + (size_t)js * kD, lane, v);
+        float acc = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          P[i] = fmaf(as, v[i], P[i]);
+          acc = fmaf(wb2x[i] + P[i], P[i], acc);
+        }
+        xp[s] = acc;
+      }
+    }
+    const float xt = reduce_scatter32(xp, lane);
+    // in-batch inclusive suffix sums over lanes >= t
+    DF sm = df_make(at);
+    DF sq = ok ? two_prod(at, yt) : df_make(0.f);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      DF om{__shfl_down_sync(kFull, sm.hi, o), __shfl_down_sync(kFull, sm.lo, o)};
+      DF oq{__shfl_down_sync(kFull, sq.hi, o), __shfl_down_sync(kFull, sq.lo, o)};
+      if (lane + o < 32) {
+        sm = df_add(sm, om);
+        sq = df_add(sq, oq);
+      }
+    }
+    const DF Mt = df_add(M0, df_add(carry_m, sm));
+    const DF Qt = df_add(Q0, df_add(carry_q, sq));
+    DF c;
+    if (p.statistic == 2) {
+      c = Mt;
+    } else if (p.statistic == 1) {
+      c = df_sqrt(df_mul(Mt, Qt));
+    } else {
+      const DF W2 = df_add_f(wb2, xt);
+      c = df_sqrt(df_add(df_mul(Mt, Qt), df_neg(W2)));
+    }
+    if (ok) {
+      curve[(size_t)u * n + r] = make_float2(c.hi, c.lo);
+      if (!(c.hi <= 3.0e38f)) bad = true;
+      unsigned long long k = df_order_key(c);
+      best = k > best ? k : best;
+    }
+    carry_m = df_add(carry_m, shfl_df(sm, 0));
+    carry_q = df_add(carry_q, shfl_df(sq, 0));
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    unsigned long long other = __shfl_xor_sync(kFull, best, o);
+    best = other > best ? other : best;
+  }
+  if (lane == 0) atomicMax(cmax + u, best);
+  if (__any_sync(kFull, bad) && lane == 0) raise_status(status, 1u);
+}
+
+__global__ void cmax_clear_kernel(unsigned long long* cmax, int units) {
+  int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < units) cmax[i] = 0ull;
+}
+
+__global__ void export_curves_kernel(Prob p, const int32_t* __restrict__ perm,
+                                     const float2* __restrict__ curve, int32_t* __restrict__ perm_out,
+                                     double* __restrict__ c_out) {
+  const size_t total = (size_t)p.units * p.n;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (size_t)gridDim.x * blockDim.x) {
+    if (perm_out) perm_out[i] = perm[i];
+    if (c_out) {
+      float2 c = curve[i];
+      c_out[i] = (double)c.x + (double)c.y;
+    }
+  }
+}
+
+void launch_curves(const Prob& p, const Layout& ly, char* ws, const void* K, const void* V,
+                   bool need_k, cudaStream_t st) {
+  const uint32_t* keys = reinterpret_cast<const uint32_t*>(ws + ly.keys0);
+  const int32_t* perm = reinterpret_cast<const int32_t*>(ws + ly.vals0);
+  const __nv_bfloat16* Kb = reinterpret_cast<const __nv_bfloat16*>(K);
+  const __nv_bfloat16* Vb = reinterpret_cast<const __nv_bfloat16*>(V);
+  float4* agg_mq = reinterpret_cast<float4*>(ws + ly.agg_mq);
+  float* agg_v = reinterpret_cast<float*>(ws + ly.agg_v);
+  float* agg_k = reinterpret_cast<float*>(ws + ly.agg_k);
+  float* yrank = reinterpret_cast<float*>(ws + ly.s_tmp);  // pooled scores are dead by now
+  float4* base_mq = reinterpret_cast<float4*>(ws + ly.base_mq);
+  float2* base_v = reinterpret_cast<float2*>(ws + ly.base_v);
+  float2* base_k = reinterpret_cast<float2*>(ws + ly.base_k);
+  float2* curve = reinterpret_cast<float2*>(ws + ly.curve);
+  unsigned long long* cmax = reinterpret_cast<unsigned long long*>(ws + ly.cmax);
+  dim3 grid((p.chunks + 3) / 4, p.units);
+  {
+    TraceScope ts_("cmax_clear", st);
+    cmax_clear_kernel<<<(p.units + 255) / 256, 256, 0, st>>>(cmax, p.units);
+  }
+  {
+    TraceScope ts_("curve_agg", st);
+    curve_agg_kernel<<<grid, 128, 0, st>>>(p, keys, perm, Kb, Vb, need_k, agg_mq, agg_v, agg_k,
+                                           yrank);
+  }
+  {
+    TraceScope ts_("curve_prefix", st);
+    curve_prefix_kernel<<<p.units, 128, 0, st>>>(p, agg_mq, agg_v, agg_k, need_k, base_mq, base_v,
+                                                 base_k);
+  }
+  {
+    TraceScope ts_("curve_eval", st);
+    curve_eval_kernel<<<grid, 128, 0, st>>>(p, keys, perm, Vb, yrank, base_mq, base_v, curve, cmax,
+                                            reinterpret_cast<uint32_t*>(ws + ly.status));
+  }
+}
+
+void launch_export_curves(const Prob& p, const Layout& ly, char* ws, int32_t* perm_out,
+                          double* c_out, cudaStream_t st) {
+  {
+    TraceScope ts_("export_curves", st);
+    export_curves_kernel<<<1024, 256, 0, st>>>(p, reinterpret_cast<const int32_t*>(ws + ly.vals0),
+                                               reinterpret_cast<const float2*>(ws + ly.curve),
+                                               perm_out, c_out);
+  }
+}
+
+}  // namespace certkv

@@ -1,0 +1,215 @@
+// decode.cu — a9: decode attention over the packed cache.
+//
+// For each query head qh of unit u = (b, l, qh / G):
+//   out = sum_s softmax_s(scale <q, k_s>) v_s
+// over the real_counts[u] real slots plus the tail slot (the "plain slot" of
+// the paper's ablation table: the synthetic pair enters as an ordinary KV
+// entry).  Split-K: kDecodeSplits CTAs per unit each stream an interleaved
+// share of 32-slot tiles and keep online (max, sum, acc) for the G query
+// heads that share the unit, so every packed K/V byte is read once per step;
+// a merge kernel combines the splits in the log-sum-exp domain.
+#include "common.cuh"
+#include "internal.cuh"
+
+namespace certkv {
+
+struct DecodePart {  // one (unit, split, query head)
+  float m, l;
+};
+
+// grid = (units, kDecodeSplits), block = 128 (4 warps)
+template <int G>
+__global__ void __launch_bounds__(128) decode_split_kernel(Prob p, const __nv_bfloat16* __restrict__ q,
+                                                           const __nv_bfloat16* __restrict__ pk,
+                                                           const __nv_bfloat16* __restrict__ pv,
+                                                           const int64_t* __restrict__ offsets,
+                                                           const int32_t* __restrict__ counts,
+                                                           int tail_slot, float scale_log2,
+                                                           float2* __restrict__ part_ml,
+                                                           float* __restrict__ part_acc) {
+  __shared__ __align__(16) float qs[G][kD];
+  __shared__ float wm[4][G], wl[4][G];
+  __shared__ float wacc[4][G][kD];
+  const int u = blockIdx.x, split = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int bl = u / p.H, h = u - bl * p.H;
+  const __nv_bfloat16* qu = q + ((size_t)bl * p.Hq + (size_t)h * G) * kD;
+  for (int i = threadIdx.x; i < G * kD; i += blockDim.x)
+    (&qs[0][0])[i] = __bfloat162float(qu[i]) * scale_log2;
+  __syncthreads();
+
+  const int slots = counts[u] + tail_slot;
+  const int64_t off = offsets[u];
+  float m[G], l[G], acc[G][4];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    m[g] = -INFINITY;
+    l[g] = 0.f;
+    acc[g][0] = acc[g][1] = acc[g][2] = acc[g][3] = 0.f;
+  }
+  const int ntiles = (slots + 31) / 32;
+  for (int t = split * 4 + warp; t < ntiles; t += kDecodeSplits * 4) {
+    const int s = t * 32 + lane;
+    const bool ok = s < slots;
+    // scores: lane = slot
+    float x[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) x[g] = 0.f;
+    if (ok) {
+      const uint4* kr = reinterpret_cast<const uint4*>(pk + (size_t)(off + s) * kD);
+#pragma unroll 4
+      for (int c = 0; c < 16; ++c) {
+        const uint4 raw = __ldg(kr + c);
+        const float kf[8] = {bf16lo(raw.x), bf16hi(raw.x), bf16lo(raw.y), bf16hi(raw.y),
+                             bf16lo(raw.z), bf16hi(raw.z), bf16lo(raw.w), bf16hi(raw.w)};
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          const float4 q0 = *reinterpret_cast<const float4*>(&qs[g][c * 8]);
+          const float4 q1 = *reinterpret_cast<const float4*>(&qs[g][c * 8 + 4]);
+          x[g] = fmaf(q0.x, kf[0], x[g]);
+          x[g] = fmaf(q0.y, kf[1], x[g]);
+          x[g] = fmaf(q0.z, kf[2], x[g]);
+          x[g] = fmaf(q0.w, kf[3], x[g]);
+          x[g] = fmaf(q1.x, kf[4], x[g]);
+          x[g] = fmaf(q1.y, kf[5], x[g]);
+          x[g] = fmaf(q1.z, kf[6], x[g]);
+          x[g] = fmaf(q1.w, kf[7], x[g]);
+        }
+      }
+    } else {
+#pragma unroll
+      for (int g = 0; g < G; ++g) x[g] = -INFINITY;
+    }
+    float pr[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const float tm = warp_max(x[g]);
+      const float nm = fmaxf(m[g], tm);
+      const float corr = exp2f(m[g] - nm);
+      m[g] = nm;
+      l[g] *= corr;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc[g][i] *= corr;
+      pr[g] = ok ? exp2f(x[g] - nm) : 0.f;
+      l[g] += pr[g];
+    }
+    // values: lane = 4 dims
+    const int cnt = min(32, slots - t * 32);
+    for (int j = 0; j < cnt; ++j) {
+      const uint2 raw =
+          __ldg(reinterpret_cast<const uint2*>(pv + (size_t)(off + t * 32 + j) * kD) + lane);
+      const float v0 = bf16lo(raw.x), v1 = bf16hi(raw.x), v2 = bf16lo(raw.y), v3 = bf16hi(raw.y);
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const float pj = __shfl_sync(kFull, pr[g], j);
+        acc[g][0] = fmaf(pj, v0, acc[g][0]);
+        acc[g][1] = fmaf(pj, v1, acc[g][1]);
+        acc[g][2] = fmaf(pj, v2, acc[g][2]);
+        acc[g][3] = fmaf(pj, v3, acc[g][3]);
+      }
+    }
+  }
+  // combine the 4 warps
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    float lt = l[g];
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) lt += __shfl_xor_sync(kFull, lt, o);
+    if (lane == 0) {
+      wm[warp][g] = m[g];
+      wl[warp][g] = lt;
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) wacc[warp][g][lane * 4 + i] = acc[g][i];
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < G * kD; idx += blockDim.x) {
+    const int g = idx / kD, i = idx - g * kD;
+    float M = -INFINITY;
+#pragma unroll
+    for (int wi = 0; wi < 4; ++wi) M = fmaxf(M, wm[wi][g]);
+    float L = 0.f, A = 0.f;
+#pragma unroll
+    for (int wi = 0; wi < 4; ++wi) {
+      if (wm[wi][g] > -INFINITY) {
+        const float f = exp2f(wm[wi][g] - M);
+        L += wl[wi][g] * f;
+        A += wacc[wi][g][i] * f;
+      }
+    }
+    const size_t pi = ((size_t)u * kDecodeSplits + split) * G + g;
+    part_acc[pi * kD + i] = A;
+    if (i == 0) part_ml[pi] = make_float2(M, L);
+  }
+}
+
+// grid = units * G, block = 128: merge the splits of one query head.
+__global__ void __launch_bounds__(128) decode_merge_kernel(Prob p, int G,
+                                                           const float2* __restrict__ part_ml,
+                                                           const float* __restrict__ part_acc,
+                                                           __nv_bfloat16* __restrict__ out) {
+  const int ug = blockIdx.x;
+  const int u = ug / G, g = ug - u * G;
+  const int i = threadIdx.x;
+  float M = -INFINITY;
+  for (int s = 0; s < kDecodeSplits; ++s)
+    M = fmaxf(M, part_ml[((size_t)u * kDecodeSplits + s) * G + g].x);
+  float L = 0.f, A = 0.f;
+  for (int s = 0; s < kDecodeSplits; ++s) {
+    const size_t pi = ((size_t)u * kDecodeSplits + s) * G + g;
+    const float2 ml = part_ml[pi];
+    if (ml.x > -INFINITY) {
+      const float f = exp2f(ml.x - M);
+      L += ml.y * f;
+      A += part_acc[pi * kD + i] * f;
+    }
+  }
+  // query head index: (b, l, h*G + g) -> [B*L][Hq]
+  const int bl = u / p.H, h = u - bl * p.H;
+  out[((size_t)bl * p.Hq + (size_t)h * G + g) * kD + i] = __float2bfloat16_rn(A / L);
+}
+
+size_t decode_workspace(const Prob& p) {
+  const size_t parts = (size_t)p.units * kDecodeSplits * p.G;
+  return parts * sizeof(float2) + parts * kD * sizeof(float) + 512;
+}
+
+template <int G>
+static void launch_split(const Prob& p, const __nv_bfloat16* q, const __nv_bfloat16* pk,
+                         const __nv_bfloat16* pv, const int64_t* offsets, const int32_t* counts,
+                         int tail_slot, float sl2, float2* ml, float* acc, cudaStream_t st) {
+  {
+    TraceScope ts_("decode_split", st);
+    decode_split_kernel<G><<<dim3(p.units, kDecodeSplits), 128, 0, st>>>(p, q, pk, pv, offsets,
+                                                                         counts, tail_slot, sl2, ml,
+                                                                         acc);
+  }
+}
+
+void launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
+                   const int64_t* offsets, const int32_t* counts, int tail_slot, float scale,
+                   void* out, char* ws, cudaStream_t st) {
+  const size_t parts = (size_t)p.units * kDecodeSplits * p.G;
+  float2* ml = reinterpret_cast<float2*>(ws);
+  size_t acc_off = (parts * sizeof(float2) + 255) / 256 * 256;
+  float* acc = reinterpret_cast<float*>(ws + acc_off);
+  const float sl2 = scale * 1.4426950408889634f;
+  const __nv_bfloat16* qb = reinterpret_cast<const __nv_bfloat16*>(q);
+  const __nv_bfloat16* kb = reinterpret_cast<const __nv_bfloat16*>(pk);
+  const __nv_bfloat16* vb = reinterpret_cast<const __nv_bfloat16*>(pv);
+  switch (p.G) {
+    case 1: launch_split<1>(p, qb, kb, vb, offsets, counts, tail_slot, sl2, ml, acc, st); break;
+    case 2: launch_split<2>(p, qb, kb, vb, offsets, counts, tail_slot, sl2, ml, acc, st); break;
+    case 4: launch_split<4>(p, qb, kb, vb, offsets, counts, tail_slot, sl2, ml, acc, st); break;
+    case 8: launch_split<8>(p, qb, kb, vb, offsets, counts, tail_slot, sl2, ml, acc, st); break;
+    case 16: launch_split<16>(p, qb, kb, vb, offsets, counts, tail_slot, sl2, ml, acc, st); break;
+    default: return;
+  }
+  {
+    TraceScope ts_("decode_merge", st);
+    decode_merge_kernel<<<p.units * p.G, 128, 0, st>>>(p, p.G, ml, acc,
+                                                       reinterpret_cast<__nv_bfloat16*>(out));
+  }
+}
+
+}  // namespace certkv

@@ -1,0 +1,90 @@
+// internal.cuh — problem description and kernel launchers shared by the
+// translation units of the CertKV library.  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace certkv {
+
+// One compress/decode call, after host-side validation.
+struct Prob {
+  int B, L, Hq, H, n, d, w, G, R;  // R = G * w observation rows per KV head
+  int units;                       // B * L * H
+  int bl;                          // B * L
+  float scale;                     // softmax scale
+  float scale_log2;                // scale * log2(e)
+  int pool, protect;
+  int alpha_num, alpha_den, T, statistic, tail_slot;
+  int64_t B_live, B_real;
+  int b_min;
+  // derived launch geometry
+  int score_warps;  // warps per score CTA (16 rows each)
+  int row_blocks;   // ceil(R / (16 * score_warps))
+  int key_splits;   // ceil(n / kScoreKeysPerCta)
+  int sort_tiles;   // ceil(n / kSortTile)
+  int chunks;       // ceil(n / kChunk)
+  int hull_segs;    // ceil((n - b_min) / kHullSeg)
+};
+
+constexpr int kScoreKeysPerCta = 1024;
+constexpr int kScoreTileKeys = 64;
+
+// Workspace carve-up (byte offsets from the workspace base, 256-B aligned).
+struct Layout {
+  size_t status;     // uint32 status word (+ padding)
+  size_t lse_part;   // float2 [U][R][key_splits]
+  size_t lse;        // float  [U][R]   log2-domain LSE of each observation row
+  size_t s_part;     // float  [U][row_blocks][n]
+  size_t s_tmp;      // float  [U][n]   pooled scores
+  size_t a;          // float  [U][n]   scores (when the caller gives none)
+  size_t keys0, keys1, vals0, vals1;  // uint32/int32 [U][n]
+  size_t hist;       // uint32 [U][256][sort_tiles]
+  size_t agg_mq;     // float4 [U][chunks]  (m.hi, m.lo, q.hi, q.lo)
+  size_t agg_v;      // float  [U][chunks][d]
+  size_t agg_k;      // float  [U][chunks][d]
+  size_t base_mq;    // float4 [U][chunks]  suffix after the chunk
+  size_t base_v;     // float2 [U][chunks][d]
+  size_t base_k;     // float2 [U][chunks][d]
+  size_t curve;      // float2 [U][n]  c(b) as hi + lo
+  size_t cmax;       // uint64 [U]     order key of max_b c(b)
+  size_t cand;       // int32  [U][n]  allocator candidates
+  size_t ncand;      // int32  [U][hull_segs + 1]
+  size_t total;
+};
+
+Layout make_layout(const Prob& p);
+
+// ---- launchers (all asynchronous on `st`) --------------------------------
+void launch_score(const Prob& p, const Layout& ly, char* ws, const void* K, const void* Q,
+                  float* a_out, cudaStream_t st);
+void launch_sort(const Prob& p, const Layout& ly, char* ws, const float* a, cudaStream_t st);
+void launch_curves(const Prob& p, const Layout& ly, char* ws, const void* K, const void* V,
+                   bool need_k, cudaStream_t st);
+void launch_allocate(const Prob& p, const Layout& ly, char* ws, int32_t* counts,
+                     int64_t* offsets, cudaStream_t st);
+void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const void* V,
+                 const float* a, void* pk, void* pv, const int64_t* offsets,
+                 const int32_t* counts, int32_t* positions, float* tail_f32,
+                 double* tail_mass, cudaStream_t st);
+void launch_export_curves(const Prob& p, const Layout& ly, char* ws, int32_t* perm_out,
+                          double* c_out, cudaStream_t st);
+void launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
+                   const int64_t* offsets, const int32_t* counts, int tail_slot, float scale,
+                   void* out, char* ws, cudaStream_t st);
+size_t decode_workspace(const Prob& p);
+
+// ---- optional kernel timing (off by default) ------------------------------
+// When enabled with certkv_trace_enable(), every kernel launch is bracketed
+// by a pair of CUDA events recorded on the launching stream.
+void trace_begin(const char* name, cudaStream_t st);
+void trace_end(cudaStream_t st);
+
+struct TraceScope {
+  cudaStream_t st;
+  TraceScope(const char* name, cudaStream_t s) : st(s) { trace_begin(name, s); }
+  ~TraceScope() { trace_end(st); }
+};
+
+}  // namespace certkv

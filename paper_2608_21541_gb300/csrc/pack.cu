@@ -1,0 +1,202 @@
+// pack.cu — a6 select, a7 tail slot, a8 packed cache.
+//
+//   tail    (k*, v*) = sum_{E} a_j (k_j, v_j) / m over the evicted ranks
+//           b_h..n-1 (§4: the key and value centroids of the evicted suffix
+//           under r_j = a_j / m), from the chunk suffix sums plus the partial
+//           chunk, in double-float; rounded once to bf16 into the last slot.
+//   select  top-b_h real tokens = ranks 0..b_h-1; emitted in ascending
+//           position by comparing each token's sort key with the first
+//           evicted one (a threshold) and compacting in position order.
+//   copy    gathers the kept K and V rows bit-exactly into the packed cache.
+#include "common.cuh"
+#include "internal.cuh"
+
+namespace certkv {
+
+// grid = units, block = 128 (one thread per dimension)
+__global__ void __launch_bounds__(128) tail_kernel(
+    Prob p, const uint32_t* __restrict__ keys, const int32_t* __restrict__ perm,
+    const __nv_bfloat16* __restrict__ K, const __nv_bfloat16* __restrict__ V,
+    const float4* __restrict__ base_mq, const float2* __restrict__ base_v,
+    const float2* __restrict__ base_k, const int32_t* __restrict__ counts,
+    const int64_t* __restrict__ offsets, __nv_bfloat16* __restrict__ pk,
+    __nv_bfloat16* __restrict__ pv, int32_t* __restrict__ positions, float* __restrict__ tail_f32,
+    double* __restrict__ tail_mass, uint32_t* status) {
+  const int u = blockIdx.x, i = threadIdx.x;
+  const int n = p.n;
+  const int b = counts[u];
+  const uint32_t* ku = keys + (size_t)u * n;
+  const int32_t* pu = perm + (size_t)u * n;
+  const __nv_bfloat16* Ku = K + (size_t)u * n * kD;
+  const __nv_bfloat16* Vu = V + (size_t)u * n * kD;
+  const int kb = b / kChunk;
+  const int r_end = min(n, (kb + 1) * kChunk);
+  const size_t ci = (size_t)u * p.chunks + kb;
+  const float4 bmq = base_mq[ci];
+  DF m{bmq.x, bmq.y};
+  float2 t = base_v[ci * kD + i];
+  DF tv{t.x, t.y};
+  t = base_k[ci * kD + i];
+  DF tk{t.x, t.y};
+  for (int r = b; r < r_end; ++r) {
+    const float a = key_score(ku[r]);
+    const int j = pu[r];
+    const float v = __bfloat162float(Vu[(size_t)j * kD + i]);
+    const float k = __bfloat162float(Ku[(size_t)j * kD + i]);
+    m = df_add_f(m, a);
+    tv = df_add(tv, two_prod(a, v));
+    tk = df_add(tk, two_prod(a, k));
+  }
+  DF ks, vs;
+  if (m.hi > 0.0f) {
+    ks = df_div(tk, m);
+    vs = df_div(tv, m);
+  } else {  // zero tail mass in floating point: uniform mean of the tail
+    DF sk = df_make(0.f), sv = df_make(0.f);
+    for (int r = b; r < n; ++r) {
+      const int j = pu[r];
+      sv = df_add_f(sv, __bfloat162float(Vu[(size_t)j * kD + i]));
+      sk = df_add_f(sk, __bfloat162float(Ku[(size_t)j * kD + i]));
+    }
+    const DF cnt = df_make((float)(n - b));
+    ks = df_div(sk, cnt);
+    vs = df_div(sv, cnt);
+    if (i == 0) raise_status(status, 2u);
+  }
+  const int64_t slot = offsets[u] + b;
+  reinterpret_cast<uint16_t*>(pk)[slot * kD + i] = df_to_bf16(ks.hi, ks.lo);
+  reinterpret_cast<uint16_t*>(pv)[slot * kD + i] = df_to_bf16(vs.hi, vs.lo);
+  if (i == 0) positions[slot] = -1;
+  if (tail_f32) {
+    tail_f32[((size_t)u * 2 + 0) * kD + i] = ks.hi;
+    tail_f32[((size_t)u * 2 + 1) * kD + i] = vs.hi;
+  }
+  if (tail_mass && i == 0) tail_mass[u] = df_to_double(m);
+}
+
+// grid = units, block = 1024: positions of the kept tokens in ascending order.
+__global__ void __launch_bounds__(1024) select_kernel(Prob p, const float* __restrict__ a,
+                                                      const uint32_t* __restrict__ keys,
+                                                      const int32_t* __restrict__ perm,
+                                                      const int32_t* __restrict__ counts,
+                                                      const int64_t* __restrict__ offsets,
+                                                      int32_t* __restrict__ positions,
+                                                      uint32_t* status) {
+  __shared__ int warp_tot[32];
+  __shared__ int carry;
+  const int u = blockIdx.x;
+  const int n = p.n;
+  const int b = counts[u];
+  const uint32_t kt = keys[(size_t)u * n + b];  // first evicted rank
+  const int jt = perm[(size_t)u * n + b];
+  const float* au = a + (size_t)u * n;
+  int32_t* out = positions + offsets[u];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int kPer = 4;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base < n; base += blockDim.x * kPer) {
+    int j0 = base + threadIdx.x * kPer;
+    bool kept[kPer];
+    int cnt = 0;
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) {
+      int j = j0 + e;
+      bool k = false;
+      if (j < n) {
+        uint32_t kj = score_key(au[j]);
+        k = (kj < kt) || (kj == kt && j < jt);
+      }
+      kept[e] = k;
+      cnt += k;
+    }
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane == 31) warp_tot[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+      int t = lane < (int)(blockDim.x >> 5) ? warp_tot[lane] : 0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(kFull, t, o);
+        if (lane >= o) t += y;
+      }
+      warp_tot[lane] = t;
+    }
+    __syncthreads();
+    int pos = carry + (warp > 0 ? warp_tot[warp - 1] : 0) + incl - cnt;
+#pragma unroll
+    for (int e = 0; e < kPer; ++e)
+      if (kept[e]) {
+        if (pos < b) out[pos] = j0 + e;
+        ++pos;
+      }
+    __syncthreads();
+    if (threadIdx.x == 0) carry += warp_tot[(blockDim.x >> 5) - 1];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0 && carry != b) raise_status(status, 1u);
+}
+
+// grid = (units, rows_split), block = 256: copy kept rows (16 B per thread-step)
+__global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloat16* __restrict__ K,
+                                                        const __nv_bfloat16* __restrict__ V,
+                                                        const int32_t* __restrict__ counts,
+                                                        const int64_t* __restrict__ offsets,
+                                                        const int32_t* __restrict__ positions,
+                                                        __nv_bfloat16* __restrict__ pk,
+                                                        __nv_bfloat16* __restrict__ pv) {
+  const int u = blockIdx.x;
+  const int b = counts[u];
+  const int64_t off = offsets[u];
+  const uint4* Ku = reinterpret_cast<const uint4*>(K + (size_t)u * p.n * kD);
+  const uint4* Vu = reinterpret_cast<const uint4*>(V + (size_t)u * p.n * kD);
+  uint4* PK = reinterpret_cast<uint4*>(pk);
+  uint4* PV = reinterpret_cast<uint4*>(pv);
+  // 16 uint4 per row; 256 threads = 16 rows per step
+  const int sub = threadIdx.x & 15;
+  for (int row = blockIdx.y * 16 + (threadIdx.x >> 4); row < b; row += gridDim.y * 16) {
+    const int j = positions[off + row];
+    if (j < 0 || j >= p.n) continue;  // unreachable when the selection is consistent
+    PK[(size_t)(off + row) * 16 + sub] = __ldg(Ku + (size_t)j * 16 + sub);
+    PV[(size_t)(off + row) * 16 + sub] = __ldg(Vu + (size_t)j * 16 + sub);
+  }
+}
+
+void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const void* V,
+                 const float* a, void* pk, void* pv, const int64_t* offsets,
+                 const int32_t* counts, int32_t* positions, float* tail_f32,
+                 double* tail_mass, cudaStream_t st) {
+  const uint32_t* keys = reinterpret_cast<const uint32_t*>(ws + ly.keys0);
+  const int32_t* perm = reinterpret_cast<const int32_t*>(ws + ly.vals0);
+  const __nv_bfloat16* Kb = reinterpret_cast<const __nv_bfloat16*>(K);
+  const __nv_bfloat16* Vb = reinterpret_cast<const __nv_bfloat16*>(V);
+  __nv_bfloat16* PK = reinterpret_cast<__nv_bfloat16*>(pk);
+  __nv_bfloat16* PV = reinterpret_cast<__nv_bfloat16*>(pv);
+  uint32_t* status = reinterpret_cast<uint32_t*>(ws + ly.status);
+  {
+    TraceScope ts("select", st);
+    select_kernel<<<p.units, 1024, 0, st>>>(p, a, keys, perm, counts, offsets, positions, status);
+  }
+  int ysplit = (p.n + 15) / 16;
+  if (ysplit > 64) ysplit = 64;
+  {
+    TraceScope ts("copy_rows", st);
+    copy_rows_kernel<<<dim3(p.units, ysplit), 256, 0, st>>>(p, Kb, Vb, counts, offsets,
+                                                           positions, PK, PV);
+  }
+  if (p.tail_slot) {
+    TraceScope ts("tail", st);
+    tail_kernel<<<p.units, 128, 0, st>>>(
+        p, keys, perm, Kb, Vb, reinterpret_cast<const float4*>(ws + ly.base_mq),
+        reinterpret_cast<const float2*>(ws + ly.base_v),
+        reinterpret_cast<const float2*>(ws + ly.base_k), counts, offsets, PK, PV, positions,
+        tail_f32, tail_mass, status);
+  }
+}
+
+}  // namespace certkv

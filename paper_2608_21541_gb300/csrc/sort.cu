@@ -1,0 +1,175 @@
+// sort.cu — a3: per-unit stable order of the scores (descending, ties by
+// lower index; Algorithm 1 "sort by s_h descending").
+//
+// Segmented LSD radix sort over all units at once: 32-bit keys
+// (~bits(a), ascending = a descending), 8-bit digits, 4 passes.  Each pass is
+// histogram -> per-unit exclusive scan in (digit, tile) order -> stable
+// scatter.  The input of pass 0 is in index order, so stability yields the
+// lower-index tie-break.
+#include "common.cuh"
+#include "internal.cuh"
+
+namespace certkv {
+
+namespace {
+constexpr int kWarps = kSortThreads / 32;
+constexpr int kPerLane = kSortTile / kSortThreads;  // 16 keys per lane, striped per warp
+}  // namespace
+
+// grid = (tiles, units): per-tile digit histogram, stored [u][digit][tile].
+__global__ void __launch_bounds__(kSortThreads) radix_hist_kernel(const uint32_t* __restrict__ keys,
+                                                                  int n, int tiles, int shift,
+                                                                  uint32_t* __restrict__ hist) {
+  __shared__ uint32_t cnt[256];
+  const int tile = blockIdx.x, u = blockIdx.y;
+  cnt[threadIdx.x] = 0;
+  __syncthreads();
+  const uint32_t* ku = keys + (size_t)u * n;
+  const int base = tile * kSortTile;
+  for (int i = threadIdx.x; i < kSortTile; i += kSortThreads) {
+    int j = base + i;
+    if (j < n) atomicAdd(&cnt[(ku[j] >> shift) & 255u], 1u);
+  }
+  __syncthreads();
+  hist[((size_t)u * 256 + threadIdx.x) * tiles + tile] = cnt[threadIdx.x];
+}
+
+// grid = units: exclusive scan of the unit's 256 * tiles counters.
+__global__ void __launch_bounds__(1024) radix_scan_kernel(uint32_t* __restrict__ hist, int tiles) {
+  __shared__ uint32_t warp_tot[32];
+  __shared__ uint32_t carry;
+  uint32_t* h = hist + (size_t)blockIdx.x * 256 * tiles;
+  const int total = 256 * tiles;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base < total; base += blockDim.x) {
+    int i = base + threadIdx.x;
+    uint32_t v = i < total ? h[i] : 0u;
+    uint32_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      uint32_t y = __shfl_up_sync(kFull, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_tot[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+      uint32_t t = lane < (int)(blockDim.x >> 5) ? warp_tot[lane] : 0u;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        uint32_t y = __shfl_up_sync(kFull, t, o);
+        if (lane >= o) t += y;
+      }
+      warp_tot[lane] = t;  // inclusive
+    }
+    __syncthreads();
+    uint32_t excl = carry + (warp > 0 ? warp_tot[warp - 1] : 0u) + x - v;
+    if (i < total) h[i] = excl;
+    __syncthreads();
+    if (threadIdx.x == 0) carry += warp_tot[(blockDim.x >> 5) - 1];
+    __syncthreads();
+  }
+}
+
+// grid = (tiles, units): stable scatter of one tile.
+__global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
+    const uint32_t* __restrict__ kin, const int32_t* __restrict__ vin, uint32_t* __restrict__ kout,
+    int32_t* __restrict__ vout, int n, int tiles, int shift, const uint32_t* __restrict__ hist) {
+  __shared__ uint32_t wcnt[kWarps][256];
+  __shared__ uint32_t gbase[256];
+  const int tile = blockIdx.x, u = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < kWarps * 256; i += kSortThreads) (&wcnt[0][0])[i] = 0;
+  gbase[threadIdx.x] = hist[((size_t)u * 256 + threadIdx.x) * tiles + tile];
+  __syncthreads();
+
+  const uint32_t* ku = kin + (size_t)u * n;
+  const int32_t* vu = vin + (size_t)u * n;
+  const int wbase = tile * kSortTile + warp * (kSortTile / kWarps);
+  uint32_t key[kPerLane];
+  int32_t val[kPerLane];
+#pragma unroll
+  for (int i = 0; i < kPerLane; ++i) {
+    int j = wbase + i * 32 + lane;
+    bool ok = j < n;
+    key[i] = ok ? ku[j] : 0u;
+    val[i] = ok ? vu[j] : 0;
+  }
+  const uint32_t lt = (1u << lane) - 1u;
+  // 1. per-warp digit counts
+#pragma unroll
+  for (int i = 0; i < kPerLane; ++i) {
+    int j = wbase + i * 32 + lane;
+    bool ok = j < n;
+    uint32_t dgt = ok ? ((key[i] >> shift) & 255u) : 256u + lane;  // unique dummy digit
+    uint32_t peers = __match_any_sync(kFull, dgt);
+    if (ok && (peers & lt) == 0u) wcnt[warp][dgt] += __popc(peers);
+    __syncwarp();
+  }
+  __syncthreads();
+  // 2. exclusive scan across warps per digit
+  {
+    const int d = threadIdx.x;
+    uint32_t run = 0;
+#pragma unroll
+    for (int wi = 0; wi < kWarps; ++wi) {
+      uint32_t t = wcnt[wi][d];
+      wcnt[wi][d] = run;
+      run += t;
+    }
+  }
+  __syncthreads();
+  // 3. ranks and scatter, in element order
+  uint32_t* ko = kout + (size_t)u * n;
+  int32_t* vo = vout + (size_t)u * n;
+#pragma unroll
+  for (int i = 0; i < kPerLane; ++i) {
+    int j = wbase + i * 32 + lane;
+    bool ok = j < n;
+    uint32_t dgt = ok ? ((key[i] >> shift) & 255u) : 256u + lane;
+    uint32_t peers = __match_any_sync(kFull, dgt);
+    uint32_t before = 0;
+    if (ok) before = wcnt[warp][dgt];
+    __syncwarp();
+    if (ok) {
+      uint32_t pos = gbase[dgt] + before + __popc(peers & lt);
+      ko[pos] = key[i];
+      vo[pos] = val[i];
+      if ((peers & lt) == 0u) wcnt[warp][dgt] = before + __popc(peers);
+    }
+    __syncwarp();
+  }
+}
+
+void launch_sort(const Prob& p, const Layout& ly, char* ws, const float* /*a*/, cudaStream_t st) {
+  uint32_t* k0 = reinterpret_cast<uint32_t*>(ws + ly.keys0);
+  uint32_t* k1 = reinterpret_cast<uint32_t*>(ws + ly.keys1);
+  int32_t* v0 = reinterpret_cast<int32_t*>(ws + ly.vals0);
+  int32_t* v1 = reinterpret_cast<int32_t*>(ws + ly.vals1);
+  uint32_t* hist = reinterpret_cast<uint32_t*>(ws + ly.hist);
+  dim3 grid(p.sort_tiles, p.units);
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = pass * 8;
+    const uint32_t* kin = (pass & 1) ? k1 : k0;
+    const int32_t* vin = (pass & 1) ? v1 : v0;
+    uint32_t* kout = (pass & 1) ? k0 : k1;
+    int32_t* vout = (pass & 1) ? v0 : v1;
+    {
+      TraceScope ts_("sort_hist", st);
+      radix_hist_kernel<<<grid, kSortThreads, 0, st>>>(kin, p.n, p.sort_tiles, shift, hist);
+    }
+    {
+      TraceScope ts_("sort_scan", st);
+      radix_scan_kernel<<<p.units, 1024, 0, st>>>(hist, p.sort_tiles);
+    }
+    {
+      TraceScope ts_("sort_scatter", st);
+      radix_scatter_kernel<<<grid, kSortThreads, 0, st>>>(kin, vin, kout, vout, p.n, p.sort_tiles,
+                                                           shift, hist);
+    }
+  }
+  // after 4 passes the sorted keys / permutation are back in keys0 / vals0
+}
+
+}  // namespace certkv

@@ -1,0 +1,112 @@
+"""The C ABI library: it loads, exports every entry point the header declares,
+and rejects invalid shapes, budgets and workspaces on the host before any
+launch (CPU only; no compute call reaches a GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_21541_gb300 import build as B
+from paper_2608_21541_gb300 import certkv as ck
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include",
+                      "certkv.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return ck.load_library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(certkv_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_entry_points():
+    names = declared_functions()
+    assert set(names) == set(ck.EXPORTED), names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def shape(**kw):
+    s = dict(batch=1, layers=2, hq=32, hkv=8, n=4096, d=128, w=32)
+    s.update(kw)
+    return ck.certkv_shape(**s)
+
+
+def test_defaults_and_budget(lib):
+    p = ck.certkv_default_params()
+    assert (p.pool_kernel, p.protect_window, p.alpha_num, p.alpha_den, p.bisect_steps,
+            p.statistic, p.tail_slot) == (5, 1, 1, 5, 40, 0, 1)
+    assert ck.certkv_live_budget(4096, 8, 1, 10) == 8 * 409
+    assert ck.certkv_live_budget(65536, 8, 1, 10) == 8 * 6553
+    assert ck.certkv_live_budget(131072, 8, 1, 20) == 8 * 6553
+    assert ck.certkv_live_budget(4000, 1, 1, 10) == 400  # exact rational, no float floor
+    assert ck.certkv_live_budget(10, 1, 3, 2) == -1
+
+
+@pytest.mark.parametrize("bad", [dict(d=64), dict(hkv=33, hq=33), dict(hq=24, hkv=8),
+                                 dict(hq=12, hkv=4), dict(w=0), dict(w=4096), dict(n=(1 << 24) + 1),
+                                 dict(batch=0)])
+def test_invalid_shapes_have_no_workspace(lib, bad):
+    assert ck.certkv_workspace_bytes(shape(**bad)) == 0
+
+
+def test_workspace_size_grows_with_the_problem(lib):
+    a = ck.certkv_workspace_bytes(shape(n=4096))
+    b = ck.certkv_workspace_bytes(shape(n=8192))
+    assert 0 < a < b
+    assert ck.certkv_decode_workspace_bytes(shape()) > 0
+
+
+def _call_compress(lib, shp, budget, params=None, ws_bytes=None, ws_ptr=256, cap=None):
+    params = params or ck.certkv_default_params()
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
+    need = lib.certkv_workspace_bytes(ctypes.byref(shp), ctypes.byref(params))
+    packed = ck.certkv_packed(fake, fake, fake, fake, fake,
+                              cap if cap is not None else 1 << 40, None, None)
+    return lib.certkv_compress(ctypes.byref(shp), fake, fake, fake, budget, ctypes.byref(params),
+                               ctypes.byref(packed),
+                               ctypes.c_void_p(ws_ptr) if ws_ptr else None,
+                               need if ws_bytes is None else ws_bytes, None)
+
+
+def test_host_validation_errors(lib):
+    s = shape()
+    H, n = s.hkv, s.n
+    assert _call_compress(lib, shape(d=64), 2 * H) == ck.EINVAL
+    assert _call_compress(lib, s, 2 * H - 1) == ck.EBUDGET          # n_keep < 2
+    assert _call_compress(lib, s, H * n + 1) == ck.EBUDGET          # beyond H * n
+    assert _call_compress(lib, s, -5) == ck.EBUDGET
+    assert _call_compress(lib, s, 2 * H, ws_ptr=0) == ck.EWORKSPACE
+    assert _call_compress(lib, s, 2 * H, ws_ptr=257) == ck.EWORKSPACE  # misaligned
+    assert _call_compress(lib, s, 2 * H, ws_bytes=1024) == ck.EWORKSPACE
+    assert _call_compress(lib, s, 40 * H, cap=10) == ck.ECAPACITY
+    bad = ck.certkv_default_params(pool_kernel=4)
+    assert _call_compress(lib, s, 2 * H, params=bad) == ck.EINVAL
+    bad = ck.certkv_default_params(alpha_num=6, alpha_den=5)
+    assert _call_compress(lib, s, 2 * H, params=bad) == ck.EINVAL
+    bad = ck.certkv_default_params(statistic=3)
+    assert _call_compress(lib, s, 2 * H, params=bad) == ck.EINVAL
+    # without a tail slot the smallest budget is H
+    ns = ck.certkv_default_params(tail_slot=0)
+    assert _call_compress(lib, s, H - 1, params=ns) == ck.EBUDGET
+    assert ck.certkv_strerror(ck.EBUDGET).startswith("infeasible")
+
+
+def test_binding_refuses_a_missing_library(tmp_path):
+    saved = ck._lib
+    try:
+        ck._lib = None
+        with pytest.raises(RuntimeError, match="not found"):
+            ck.load_library(str(tmp_path / "missing.so"))
+    finally:
+        ck._lib = saved

@@ -1,0 +1,87 @@
+"""Full-size workloads, in the launch configuration the benchmark times (every
+layer and sequence in one call), checked against the oracle on sampled
+(sequence, layer) blocks: conditioned mode bit-exact, end-to-end scores within
+1e-4, decode within 2e-2, and the exact-budget equalities on every block."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import parity
+from paper_2608_21541_gb300 import certkv as ck
+from paper_2608_21541_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+def _layer_host(K, V, Q, b, l):
+    return (parity.bits(K[b:b + 1, l:l + 1]), parity.bits(V[b:b + 1, l:l + 1]),
+            parity.bits(Q[b:b + 1, l:l + 1]))
+
+
+def _check_blocks(wl, K, V, Q, a, packed, B_live, samples, e2e_scores=()):
+    got = parity.packed_np(packed)
+    H = wl.H
+    cnt = got["counts"].reshape(wl.B * wl.L, H)
+    assert (cnt.sum(1) == B_live - H).all(), "exact budget violated"
+    assert got["offsets"][-1] == wl.B * wl.L * B_live
+    a_host = a.view(wl.B, wl.L, H, wl.n)
+    for (b, l) in samples:
+        kb, vb, qb = _layer_host(K, V, Q, b, l)
+        a_bl = a_host[b, l].cpu().numpy()
+        kw = dict(B=1, L=1, Hq=wl.Hq, H=H, n=wl.n, d=wl.d, w=wl.w, B_live=B_live)
+        ref = oracle.compress(kb, vb, None, a_in=a_bl, **kw)
+        bl = b * wl.L + l
+        parity.check_conditioned(parity.slice_bl(got, bl, H, B_live), ref, H)
+        if (b, l) in e2e_scores:
+            full = oracle.compress(kb, vb, qb, **kw)
+            parity.check_scores(a_bl, full["a"])
+    return got
+
+
+def _run(wl, B_live, samples, e2e_scores=(), decode_steps=0, inputs=None):
+    K, V, Q = inputs if inputs is not None else W.draw(wl, device="cuda")
+    a = ck.certkv_score(K, Q)
+    packed = ck.certkv_compress(K, V, Q, B_live, with_tail=True)
+    torch.cuda.synchronize()
+    got = _check_blocks(wl, K, V, Q, a, packed, B_live, samples, e2e_scores)
+    for step in range(decode_steps):
+        q = W.draw_decode_queries(wl, step, device="cuda")
+        out = ck.certkv_decode_attn(q, packed, hkv=wl.H)
+        for (b, l) in samples:
+            bl = b * wl.L + l
+            sub = parity.slice_bl(got, bl, wl.H, B_live)
+            ref = oracle.decode(parity.bits(q[b:b + 1, l:l + 1]), sub["pk"], sub["pv"],
+                                sub["offsets"], sub["counts"], B=1, L=1, Hq=wl.Hq, H=wl.H,
+                                d=wl.d)
+            parity.check_decode(out[b:b + 1, l:l + 1], ref)
+    del a, packed
+    if inputs is None:
+        del K, V, Q
+    torch.cuda.empty_cache()
+
+
+def test_c2_full():
+    wl = W.WORKLOADS["C2"]
+    _run(wl, wl.B_live, samples=[(0, 0), (0, 13), (0, 31)], e2e_scores=[(0, 0)],
+         decode_steps=1)
+
+
+def test_c3_full():
+    wl = W.WORKLOADS["C3"]
+    _run(wl, wl.B_live, samples=[(0, 0), (0, 31)], e2e_scores=[(0, 0)], decode_steps=1)
+
+
+def test_c4_full_with_decode():
+    wl = W.WORKLOADS["C4"]
+    _run(wl, wl.B_live, samples=[(0, 0), (7, 31)], decode_steps=2)
+
+
+def test_c5_full_budget_sweep():
+    base = W.WORKLOADS["C5"]
+    inputs = W.draw(base, device="cuda")
+    for keep in base.keep_sweep:
+        wl = base.with_(keep=keep)
+        e2e = [(0, 0)] if keep == (1, 10) else []
+        _run(wl, wl.B_live, samples=[(0, 0), (0, 79)], e2e_scores=e2e, decode_steps=1,
+             inputs=inputs)
