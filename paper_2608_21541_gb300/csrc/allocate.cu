@@ -2,18 +2,22 @@
 // heads of every (sequence, layer) (Algorithm 1; implementation appendix).
 //
 // The paper's per-step argmin_b c_h(b) + lambda b over every b in
-// [b_min, n-1] is answered on a candidate subset that provably contains every
-// minimiser: the smallest minimiser of c(b) + lambda b for any lambda is a
-// vertex of the lower convex hull of the points (b, c(b)).  The candidates are
-//   hull_seg    per segment of kHullSeg points, a monotone-chain lower hull
-//               in fp32 that only drops a point when it lies above a chord by
-//               more than a rounding bound, so true hull vertices survive;
-//   hull_merge  the same tolerant chain over the concatenated survivors.
-// The bisection then evaluates c(b) + lambda b in float64 on the candidates
-// with the same expression and rounding as a direct scan (smallest b on
-// ties), so the result matches the algorithm as stated.  The best-marginal
-// repair walks one token at a time with the heads' upcoming curve values
-// staged in shared memory.
+// [b_min, n-1] is answered on a candidate subset that contains every
+// minimiser: the smallest minimiser of c(b) + lambda b, for any lambda, is a
+// vertex of the lower convex hull of the points (b, c(b)).  Candidates come
+// from two levels of filtering, both in parallel:
+//   hull_seg    one thread per segment of kHullSeg points;
+//   hull_group  one thread per group of kGroupSegs segments, over the
+//               segment survivors.
+// Each level shears its points by the chord of its range (the lower hull is
+// invariant under adding a linear function; the chord is computed in
+// double-float) so that fp32 only resolves the small residual, and runs a
+// monotone chain that drops a point only when it is above a chord by more
+// than the rounding of the test can explain.  True hull vertices therefore
+// always survive.
+// The bisection (T steps on the shared multiplier, smallest b on ties) and
+// the one-token best-marginal repair then run in double-float on the fp32
+// pipe; the multiplier itself is bisected in float64 as the paper states.
 #include <float.h>
 #include <limits.h>
 
@@ -24,20 +28,109 @@ namespace certkv {
 
 namespace {
 
-// Should middle point B be dropped from the lower hull, i.e. is it above the
-// chord from A to C by more than the fp32 rounding of this test can explain?
-__device__ __forceinline__ bool clearly_above(int xa, float ya, int xb, float yb, int xc, float yc) {
+__device__ __forceinline__ DF curve_df(const float2* c, int b) {
+  const float2 v = c[b];
+  return DF{v.x, v.y};
+}
+
+__device__ __forceinline__ bool df_less(DF x, DF y) {
+  return x.hi < y.hi || (x.hi == y.hi && x.lo < y.lo);
+}
+
+// Drop the middle point B of sheared values y only if it lies above the chord
+// A-C by more than the fp32 rounding of this test plus the error `dy` of the
+// sheared values can explain.
+__device__ __forceinline__ bool clearly_above(int xa, float ya, int xb, float yb, int xc, float yc,
+                                              float dy) {
   const float dx1 = (float)(xb - xa), dx2 = (float)(xc - xa);
-  const float dy1 = yb - ya, dy2 = yc - ya;
-  const float cross = dx1 * dy2 - dy1 * dx2;
+  const float cross = dx1 * (yc - ya) - (yb - ya) * dx2;
   const float ymax = fmaxf(fmaxf(fabsf(ya), fabsf(yb)), fabsf(yc));
-  const float eps = 16.0f * 5.9604645e-8f * ymax * (dx1 + dx2);  // 16 * 2^-24 * ...
+  const float eps = (dx1 + dx2) * (16.0f * 5.9604645e-8f * ymax + 8.0f * dy);
   return cross < -eps;
 }
 
-__device__ __forceinline__ double curve_at(const float2* c, int b) {
-  float2 v = c[b];
-  return (double)v.x + (double)v.y;
+// c(b) minus the chord through (b0, c0) with slope `slope`, in fp32, and a
+// bound on its error (2^-40 |c|, far above the double-float rounding).
+struct Shear {
+  const float2* cu;
+  int b0;
+  DF c0, slope;
+  __device__ __forceinline__ void at(int b, float& y, float& dy) const {
+    const DF cb = curve_df(cu, b);
+    const DF line = df_add(c0, df_mul_f(slope, (float)(b - b0)));
+    y = df_add(cb, df_neg(line)).hi;
+    dy = 9.094947e-13f * fmaxf(fabsf(cb.hi), fabsf(line.hi));
+  }
+};
+
+__device__ __forceinline__ Shear make_shear(const float2* cu, int b0, int b1) {
+  Shear s;
+  s.cu = cu;
+  s.b0 = b0;
+  s.c0 = curve_df(cu, b0);
+  const DF c1 = curve_df(cu, b1);
+  s.slope = (b1 > b0) ? df_div(df_add(c1, df_neg(s.c0)), df_make((float)(b1 - b0))) : df_make(0.f);
+  return s;
+}
+
+// Tolerant monotone chain over the points produced by `next(i)` for
+// i = 0..count-1 (in increasing b); the stack lives in `st` (it may alias the
+// input region as long as it never overtakes it).  Returns the stack size.
+template <typename Next>
+__device__ __forceinline__ int tolerant_chain(const Shear& sh, int count, Next next, int32_t* st) {
+  int top = 0;
+  int xa = 0, xb = 0;
+  float ya = 0.f, yb = 0.f, da = 0.f, db = 0.f;
+  for (int i = 0; i < count; ++i) {
+    const int b = next(i);
+    float y, dy;
+    sh.at(b, y, dy);
+    while (top >= 2 && clearly_above(xa, ya, xb, yb, b, y, fmaxf(fmaxf(da, db), dy))) {
+      --top;
+      xb = xa;
+      yb = ya;
+      db = da;
+      if (top >= 2) {
+        xa = st[top - 2];
+        sh.at(xa, ya, da);
+      }
+    }
+    st[top++] = b;
+    xa = xb;
+    ya = yb;
+    da = db;
+    xb = b;
+    yb = y;
+    db = dy;
+  }
+  return top;
+}
+
+// Candidate counts per unit: [hull_segs] segment counts, then [groups] group
+// counts (see Layout::ncand).
+__device__ __forceinline__ int groups_of(const Prob& p) {
+  return (p.hull_segs + kGroupSegs - 1) / kGroupSegs;
+}
+__device__ __forceinline__ size_t ncand_stride(const Prob& p) {
+  return (size_t)p.hull_segs + groups_of(p);
+}
+
+// warp-wide lexicographic argmin of (f, b)
+__device__ __forceinline__ void warp_argmin_df(DF& f, int& b) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    const DF of = shfl_xor_df(f, o);
+    const int ob = __shfl_xor_sync(kFull, b, o);
+    if (df_less(of, f) || (of.hi == f.hi && of.lo == f.lo && ob < b)) {
+      f = of;
+      b = ob;
+    }
+  }
+}
+
+__device__ __forceinline__ DF df_from_double(double x) {
+  const float hi = __double2float_rn(x);
+  return DF{hi, __double2float_rn(x - (double)hi)};
 }
 
 }  // namespace
@@ -51,88 +144,50 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   if (seg >= p.hull_segs) return;
   const int n = p.n;
   const float2* cu = curve + (size_t)u * n;
-  int32_t* st = cand + (size_t)u * n + (size_t)seg * kHullSeg;  // private stack
+  int32_t* st = cand + (size_t)u * n + (size_t)seg * kHullSeg;
   const int b0 = p.b_min + seg * kHullSeg;
   const int b1 = min(n, b0 + kHullSeg);
-  int top = 0;
-  int xa = 0, xb = 0;
-  float ya = 0.f, yb = 0.f;
-  for (int b = b0; b < b1; ++b) {
-    const float y = cu[b].x;
-    while (top >= 2 && clearly_above(xa, ya, xb, yb, b, y)) {
-      --top;
-      xb = xa;
-      yb = ya;
-      if (top >= 2) {
-        xa = st[top - 2];
-        ya = cu[xa].x;
-      }
-    }
-    st[top++] = b;
-    xa = xb;
-    ya = yb;
-    xb = b;
-    yb = y;
-  }
-  ncand[(size_t)u * (p.hull_segs + 1) + seg] = top;
+  const Shear sh = make_shear(cu, b0, b1 - 1);
+  const int top = tolerant_chain(sh, b1 - b0, [&](int i) { return b0 + i; }, st);
+  ncand[(size_t)u * ncand_stride(p) + seg] = top;
 }
 
-// grid = ceil(units / 128), one thread per unit: merge the segment survivors
-// in place into the front of the unit's candidate list.
-__global__ void __launch_bounds__(128) hull_merge_kernel(Prob p, const float2* __restrict__ curve,
+// grid = (ceil(groups / 128), units), one thread per group of segments.
+__global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* __restrict__ curve,
                                                          int32_t* __restrict__ cand,
                                                          int32_t* __restrict__ ncand) {
-  const int u = blockIdx.x * blockDim.x + threadIdx.x;
-  if (u >= p.units) return;
+  const int g = blockIdx.x * blockDim.x + threadIdx.x;
+  const int u = blockIdx.y;
+  if (g >= groups_of(p)) return;
   const int n = p.n;
   const float2* cu = curve + (size_t)u * n;
   int32_t* cl = cand + (size_t)u * n;
-  int32_t* nc = ncand + (size_t)u * (p.hull_segs + 1);
-  int top = 0;
-  int xa = 0, xb = 0;
-  float ya = 0.f, yb = 0.f;
-  for (int s = 0; s < p.hull_segs; ++s) {
-    const int cnt = nc[s];
-    const int32_t* src = cl + (size_t)s * kHullSeg;
-    for (int i = 0; i < cnt; ++i) {
-      const int b = src[i];
-      const float y = cu[b].x;
-      while (top >= 2 && clearly_above(xa, ya, xb, yb, b, y)) {
-        --top;
-        xb = xa;
-        yb = ya;
-        if (top >= 2) {
-          xa = cl[top - 2];
-          ya = cu[xa].x;
-        }
-      }
-      cl[top++] = b;
-      xa = xb;
-      ya = yb;
-      xb = b;
-      yb = y;
+  int32_t* nc = ncand + (size_t)u * ncand_stride(p);
+  const int s0 = g * kGroupSegs, s1 = min(p.hull_segs, s0 + kGroupSegs);
+  const int b0 = p.b_min + s0 * kHullSeg;
+  const int b1 = min(n, p.b_min + s1 * kHullSeg) - 1;
+  const Shear sh = make_shear(cu, b0, b1);
+  int total = 0;
+  for (int s = s0; s < s1; ++s) total += nc[s];
+  // walk the segment survivors in order; the output compacts to the group start
+  int s = s0, i = 0;
+  auto next = [&](int) {
+    while (i >= nc[s]) {
+      ++s;
+      i = 0;
     }
-  }
-  nc[p.hull_segs] = top;
+    return cl[(size_t)s * kHullSeg + i++];
+  };
+  const int top = tolerant_chain(sh, total, next, cl + (size_t)s0 * kHullSeg);
+  nc[p.hull_segs + g] = top;
 }
-
-namespace {
-// warp-wide lexicographic argmin of (f, b)
-__device__ __forceinline__ void warp_argmin(double& f, int& b) {
-#pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) {
-    double of = __shfl_xor_sync(kFull, f, o);
-    int ob = __shfl_xor_sync(kFull, b, o);
-    if (of < f || (of == f && ob < b)) {
-      f = of;
-      b = ob;
-    }
-  }
-}
-}  // namespace
 
 // grid = B*L, block = 256: bisection, repair, counts and offsets of one
-// (sequence, layer).
+// (sequence, layer).  Candidates are staged in shared memory when they fit;
+// the repair keeps a 64-value window of each head's upcoming curve values in
+// shared memory, refilled by the whole warp.
+constexpr int kCandCap = 16384;  // staged candidates: 128 KB of values + 64 KB of b (dynamic smem)
+
 __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2* __restrict__ curve,
                                                             const int32_t* __restrict__ cand,
                                                             const int32_t* __restrict__ ncand,
@@ -140,42 +195,80 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
                                                             int32_t* __restrict__ counts,
                                                             int64_t* __restrict__ offsets) {
   __shared__ int bsel[32];
+  __shared__ int coff[33];
   __shared__ double lam_sh[2];
-  __shared__ double win[32][64];
+  __shared__ float2 win[32][64];
+  extern __shared__ __align__(16) char dyn[];
+  float2* cy = reinterpret_cast<float2*>(dyn);
+  int32_t* cb_ = reinterpret_cast<int32_t*>(dyn + kCandCap * sizeof(float2));
   const int bl = blockIdx.x;
   const int H = p.H, n = p.n;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nwarps = blockDim.x >> 5;
   const int64_t B_real = p.B_real;
+  const int groups = groups_of(p);
+  const size_t stride = ncand_stride(p);
 
   if (threadIdx.x == 0) {
     double mx = 0.0;
+    int acc = 0;
     for (int h = 0; h < H; ++h) {
-      double v = df_to_double(df_from_order_key(cmax[(size_t)bl * H + h]));
+      const double v = df_to_double(df_from_order_key(cmax[(size_t)bl * H + h]));
       mx = v > mx ? v : mx;
+      coff[h] = acc;
+      const int32_t* nc = ncand + (size_t)(bl * H + h) * stride + p.hull_segs;
+      for (int g = 0; g < groups; ++g) acc += nc[g];
     }
+    coff[H] = acc;
     lam_sh[0] = 0.0;
     lam_sh[1] = __dadd_rn(__dmul_rn(2.0, mx), 1.0);
   }
   __syncthreads();
-
-  auto argmin_heads = [&](double lam) {
+  const bool staged = coff[H] <= kCandCap;
+  if (staged) {  // gather the group survivors of every head, in order
     for (int h = warp; h < H; h += nwarps) {
       const int u = bl * H + h;
-      const float2* cu = curve + (size_t)u * n;
+      const int32_t* nc = ncand + (size_t)u * stride + p.hull_segs;
       const int32_t* cl = cand + (size_t)u * n;
-      const int cnt = ncand[(size_t)u * (p.hull_segs + 1) + p.hull_segs];
-      double bf = INFINITY;
+      int acc = coff[h];
+      for (int g = 0; g < groups; ++g) {
+        const int cnt = nc[g];
+        for (int k = lane; k < cnt; k += 32) {
+          const int b = cl[(size_t)g * kGroupSegs * kHullSeg + k];
+          cb_[acc + k] = b;
+          cy[acc + k] = curve[(size_t)u * n + b];
+        }
+        acc += cnt;
+      }
+    }
+  }
+  __syncthreads();
+
+  auto argmin_heads = [&](double lam) {
+    const DF ld = df_from_double(lam);
+    for (int h = warp; h < H; h += nwarps) {
+      const int u = bl * H + h;
+      DF bf{INFINITY, 0.f};
       int bb = INT_MAX;
-      for (int k = lane; k < cnt; k += 32) {
-        const int b = cl[k];
-        const double f = __dadd_rn(curve_at(cu, b), __dmul_rn(lam, (double)b));
-        if (f < bf || (f == bf && b < bb)) {
+      auto consider = [&](int b, float2 c) {
+        const DF f = df_add(DF{c.x, c.y}, df_mul_f(ld, (float)b));
+        if (df_less(f, bf) || (f.hi == bf.hi && f.lo == bf.lo && b < bb)) {
           bf = f;
           bb = b;
         }
+      };
+      if (staged) {
+        for (int k = coff[h] + lane; k < coff[h + 1]; k += 32) consider(cb_[k], cy[k]);
+      } else {
+        const int32_t* nc = ncand + (size_t)u * stride + p.hull_segs;
+        const int32_t* cl = cand + (size_t)u * n;
+        for (int g = 0; g < groups; ++g)
+          for (int k = lane; k < nc[g]; k += 32) {
+            const int b = cl[(size_t)g * kGroupSegs * kHullSeg + k];
+            consider(b, curve[(size_t)u * n + b]);
+          }
       }
-      warp_argmin(bf, bb);
+      warp_argmin_df(bf, bb);
       if (lane == 0) bsel[h] = (bb == INT_MAX) ? p.b_min : bb;
     }
   };
@@ -201,46 +294,61 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
     const float2* cu = curve + (size_t)(bl * H + (live ? h : 0)) * n;
     int64_t tot = 0;
     for (int i = 0; i < H; ++i) tot += bsel[i];
+    const DF kNone{INFINITY, 0.f}, kBad{FLT_MAX, 0.f};
     // surplus (not reachable from lambda_hi, kept for robustness): remove one
     while (tot > B_real) {
-      double mg = INFINITY;
+      DF mg = kNone;
       if (live && b > p.b_min) {
-        double d = curve_at(cu, b - 1) - curve_at(cu, b);
-        mg = (d == d) ? d : DBL_MAX;
+        const DF d = df_add(curve_df(cu, b - 1), df_neg(curve_df(cu, b)));
+        mg = (d.hi == d.hi) ? d : kBad;
       }
       int who = lane;
-      warp_argmin(mg, who);
+      warp_argmin_df(mg, who);
       if (lane == who) --b;
       --tot;
     }
-    // best-marginal repair: add one token at a time
-    double cb = live ? curve_at(cu, b) : 0.0;
-    int wpos = 64;
+    // best-marginal repair: add one token at a time.  win[h][k] = c_h(base_h + k)
+    DF cur = live ? curve_df(cu, b) : df_make(0.f);
+    int base = b + 1;
+    for (int hh = 0; hh < H; ++hh) {
+      const int bh = __shfl_sync(kFull, b, hh);
+      const float2* ch = curve + (size_t)(bl * H + hh) * n;
+      for (int k = lane; k < 64; k += 32)
+        win[hh][k] = (bh + 1 + k < n) ? ch[bh + 1 + k] : make_float2(0.f, 0.f);
+    }
+    __syncwarp();
     while (tot < B_real) {
-      double mg = INFINITY;
+      DF mg = kNone;
       if (live && b < n - 1) {
-        if (wpos == 64) {
-          for (int k = 0; k < 64; ++k) win[h][k] = (b + 1 + k < n) ? curve_at(cu, b + 1 + k) : 0.0;
-          wpos = 0;
-        }
-        const double d = win[h][wpos] - cb;
-        mg = (d == d) ? d : DBL_MAX;
+        const float2 w = win[h][b + 1 - base];
+        const DF d = df_add(DF{w.x, w.y}, df_neg(cur));
+        mg = (d.hi == d.hi) ? d : kBad;
       }
       int who = lane;
-      warp_argmin(mg, who);
+      warp_argmin_df(mg, who);
+      const int nb = __shfl_sync(kFull, b, who) + 1;  // the winner's new count
+      const int wbase = __shfl_sync(kFull, base, who);
       if (lane == who) {
-        cb = win[h][wpos];
-        ++wpos;
-        ++b;
+        const float2 w = win[h][nb - base];
+        cur = DF{w.x, w.y};
+        b = nb;
       }
       ++tot;
+      if (nb + 1 - wbase >= 64 && nb < n - 1) {  // refill the winner's window
+        __syncwarp();
+        const float2* ch = curve + (size_t)(bl * H + who) * n;
+        for (int k = lane; k < 64; k += 32)
+          win[who][k] = (nb + 1 + k < n) ? ch[nb + 1 + k] : make_float2(0.f, 0.f);
+        if (lane == who) base = nb + 1;
+        __syncwarp();
+      }
     }
     // counts and offsets: segment = b_h real slots (+ 1 tail slot)
-    int seg = live ? b + p.tail_slot : 0;
+    const int seg = live ? b + p.tail_slot : 0;
     int incl = seg;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      int y = __shfl_up_sync(kFull, incl, o);
+      const int y = __shfl_up_sync(kFull, incl, o);
       if (lane >= o) incl += y;
     }
     if (live) {
@@ -256,18 +364,26 @@ void launch_allocate(const Prob& p, const Layout& ly, char* ws, int32_t* counts,
   const float2* curve = reinterpret_cast<const float2*>(ws + ly.curve);
   int32_t* cand = reinterpret_cast<int32_t*>(ws + ly.cand);
   int32_t* ncand = reinterpret_cast<int32_t*>(ws + ly.ncand);
-  dim3 g1((p.hull_segs + 127) / 128, p.units);
+  const int groups = (p.hull_segs + kGroupSegs - 1) / kGroupSegs;
   {
     TraceScope ts_("hull_seg", st);
-    hull_seg_kernel<<<g1, 128, 0, st>>>(p, curve, cand, ncand);
+    hull_seg_kernel<<<dim3((p.hull_segs + 127) / 128, p.units), 128, 0, st>>>(p, curve, cand,
+                                                                             ncand);
   }
   {
-    TraceScope ts_("hull_merge", st);
-    hull_merge_kernel<<<(p.units + 127) / 128, 128, 0, st>>>(p, curve, cand, ncand);
+    TraceScope ts_("hull_group", st);
+    hull_group_kernel<<<dim3((groups + 127) / 128, p.units), 128, 0, st>>>(p, curve, cand, ncand);
   }
   {
     TraceScope ts_("bisect_repair", st);
-    bisect_repair_kernel<<<p.bl, 256, 0, st>>>(
+    const size_t smem = kCandCap * (sizeof(float2) + sizeof(int32_t));
+    static bool attr = false;
+    if (!attr) {
+      cudaFuncSetAttribute(bisect_repair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem);
+      attr = true;
+    }
+    bisect_repair_kernel<<<p.bl, 256, smem, st>>>(
         p, curve, cand, ncand, reinterpret_cast<const unsigned long long*>(ws + ly.cmax), counts,
         offsets);
   }

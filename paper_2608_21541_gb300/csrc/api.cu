@@ -101,6 +101,7 @@ Layout make_layout(const Prob& p) {
   ly.vals0 = take(U * n * 4);
   ly.vals1 = take(U * n * 4);
   ly.hist = take(U * 256 * p.sort_tiles * 4);
+  ly.yrank = take(U * n * sizeof(float2));
   ly.agg_mq = take(U * p.chunks * sizeof(float4));
   ly.agg_v = take(U * p.chunks * kD * sizeof(float));
   ly.agg_k = take(U * p.chunks * kD * sizeof(float));
@@ -112,8 +113,9 @@ Layout make_layout(const Prob& p) {
   ly.cand = take(U * n * sizeof(int32_t));
   // the candidate counts are sized for the smallest b_min (1) so that one
   // workspace size serves every budget of a shape
-  const size_t segs = (size_t)((p.n - 1 + kHullSeg - 1) / kHullSeg) + 1;
-  ly.ncand = take(U * segs * sizeof(int32_t));
+  const size_t segs = (size_t)((p.n - 1 + kHullSeg - 1) / kHullSeg);
+  const size_t groups = (segs + kGroupSegs - 1) / kGroupSegs;
+  ly.ncand = take(U * (segs + groups) * sizeof(int32_t));
   ly.total = off;
   return ly;
 }

@@ -10,7 +10,8 @@ namespace certkv {
 
 constexpr int kD = 128;          // head dimension supported by the kernels
 constexpr int kChunk = 128;      // ranks per dispersion chunk (one warp)
-constexpr int kHullSeg = 1024;   // curve points per hull-filter thread
+constexpr int kHullSeg = 256;    // curve points per hull-filter thread
+constexpr int kGroupSegs = 16;   // hull-filter segments per group
 constexpr int kSortTile = 4096;  // keys per radix-sort tile
 constexpr int kSortThreads = 256;
 constexpr int kDecodeSplits = 16;

@@ -30,6 +30,21 @@ __device__ __forceinline__ void load_row4(const __nv_bfloat16* row, int lane, fl
   x[3] = bf16hi(raw.y);
 }
 
+// lane t ends with the double-float sum over lanes of v[t]  (62 shuffles)
+__device__ __forceinline__ DF reduce_scatter32_df(DF (&v)[32], int lane) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      DF keep = upper ? v[i + o] : v[i];
+      DF send = upper ? v[i] : v[i + o];
+      v[i] = df_add(keep, shfl_xor_df(send, o));
+    }
+  }
+  return v[0];
+}
+
 // lane t ends with sum over lanes of v[t]  (31 shuffles)
 __device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
 #pragma unroll
@@ -55,7 +70,7 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
                                                         bool need_k, float4* __restrict__ agg_mq,
                                                         float* __restrict__ agg_v,
                                                         float* __restrict__ agg_k,
-                                                        float* __restrict__ yrank) {
+                                                        float2* __restrict__ yrank) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int chunk = blockIdx.x * 4 + warp;
   const int u = blockIdx.y;
@@ -75,32 +90,40 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
     const float at = ok ? key_score(ku[r]) : 0.f;
     const int jt = ok ? pu[r] : 0;
     const int cnt = min(32, r1 - rb);
-    float yp[32];
+    DF yp[32];  // ||v||^2 partials: bf16 squares are exact in fp32, sums in double-float
 #pragma unroll
-    for (int s = 0; s < 32; ++s) {
-      yp[s] = 0.f;
-      if (s < cnt) {
-        const float as = __shfl_sync(kFull, at, s);
-        const int js = __shfl_sync(kFull, jt, s);
-        float v[4];
-        load_row4(Vu + (size_t)js * kD, lane, v);
+    for (int s0 = 0; s0 < 32; s0 += 8) {
+      // issue the 8 rows' loads first so that they are in flight together
+      uint2 vr[8], kr[8];
+      float as[8];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          sv[i] = fmaf(as, v[i], sv[i]);
-          yp[s] = fmaf(v[i], v[i], yp[s]);
-        }
-        if (need_k) {
-          float k4[4];
-          load_row4(Ku + (size_t)js * kD, lane, k4);
-#pragma unroll
-          for (int i = 0; i < 4; ++i) sk[i] = fmaf(as, k4[i], sk[i]);
+      for (int t = 0; t < 8; ++t) {
+        as[t] = __shfl_sync(kFull, at, s0 + t);
+        const int js = __shfl_sync(kFull, jt, s0 + t);
+        vr[t] = make_uint2(0u, 0u);
+        kr[t] = make_uint2(0u, 0u);
+        if (s0 + t < cnt) {
+          vr[t] = __ldg(reinterpret_cast<const uint2*>(Vu + (size_t)js * kD) + lane);
+          if (need_k) kr[t] = __ldg(reinterpret_cast<const uint2*>(Ku + (size_t)js * kD) + lane);
         }
       }
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        const float v[4] = {bf16lo(vr[t].x), bf16hi(vr[t].x), bf16lo(vr[t].y), bf16hi(vr[t].y)};
+        const float k4[4] = {bf16lo(kr[t].x), bf16hi(kr[t].x), bf16lo(kr[t].y), bf16hi(kr[t].y)};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          sv[i] = fmaf(as[t], v[i], sv[i]);
+          sk[i] = fmaf(as[t], k4[i], sk[i]);
+        }
+        DF y = two_sum(__fmul_rn(v[0], v[0]), __fmul_rn(v[1], v[1]));
+        yp[s0 + t] = df_add(y, two_sum(__fmul_rn(v[2], v[2]), __fmul_rn(v[3], v[3])));
+      }
     }
-    const float yt = reduce_scatter32(yp, lane);
-    if (ok) yrank[(size_t)u * n + r] = yt;
+    const DF yt = reduce_scatter32_df(yp, lane);
+    if (ok) yrank[(size_t)u * n + r] = make_float2(yt.hi, yt.lo);
     DF dm = df_make(at);
-    DF dq = ok ? two_prod(at, yt) : df_make(0.f);
+    DF dq = ok ? df_mul_f(yt, at) : df_make(0.f);
     m = df_add(m, warp_sum_df(dm));
     q = df_add(q, warp_sum_df(dq));
   }
@@ -147,7 +170,7 @@ __global__ void __launch_bounds__(128) curve_prefix_kernel(Prob p, const float4*
 __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t* __restrict__ keys,
                                                          const int32_t* __restrict__ perm,
                                                          const __nv_bfloat16* __restrict__ V,
-                                                         const float* __restrict__ yrank,
+                                                         const float2* __restrict__ yrank,
                                                          const float4* __restrict__ base_mq,
                                                          const float2* __restrict__ base_v,
                                                          float2* __restrict__ curve,
@@ -181,7 +204,11 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
     }
     wb2 = warp_sum_df(wb2);
   }
+  // The last chunk has W_base = 0 and a vanishing tail, so c(b)^2 there is a
+  // small difference of small terms: its partial sums run in double-float.
+  const bool exact = (chunk == p.chunks - 1);
   float P[4] = {0.f, 0.f, 0.f, 0.f};
+  DF Pd[4] = {df_make(0.f), df_make(0.f), df_make(0.f), df_make(0.f)};
   DF carry_m = df_make(0.f), carry_q = df_make(0.f);
   unsigned long long best = 0ull;
   bool bad = false;
@@ -192,30 +219,58 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
     const bool ok = r < r1;
     const float at = ok ? key_score(ku[r]) : 0.f;
     const int jt = ok ? pu[r] : 0;
-    const float yt = ok ? yrank[(size_t)u * n + r] : 0.f;
+    const float2 yv = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
     const int cnt = min(32, r1 - rb);
-    float xp[32];
+    DF xt;
+    if (!exact) {
+      float xp[32];
 #pragma unroll
-    for (int s = 31; s >= 0; --s) {
-      const float as = __shfl_sync(kFull, at, s);
-      const int js = __shfl_sync(kFull, jt, s);
-      xp[s] = 0.f;
-      if (s < cnt) {
-        float v[4];
-        load_row4(Vu + (size_t)js * kD, lane, v);
-        float acc = 0.f;
+      for (int s0 = 24; s0 >= 0; s0 -= 8) {
+        uint2 vr[8];
+        float as[8];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          P[i] = fmaf(as, v[i], P[i]);
-          acc = fmaf(wb2x[i] + P[i], P[i], acc);
+        for (int t = 7; t >= 0; --t) {  // loads first, highest rank of the group first
+          as[t] = __shfl_sync(kFull, at, s0 + t);
+          const int js = __shfl_sync(kFull, jt, s0 + t);
+          vr[t] = make_uint2(0u, 0u);
+          if (s0 + t < cnt) vr[t] = __ldg(reinterpret_cast<const uint2*>(Vu + (size_t)js * kD) + lane);
         }
-        xp[s] = acc;
+#pragma unroll
+        for (int t = 7; t >= 0; --t) {
+          const float v[4] = {bf16lo(vr[t].x), bf16hi(vr[t].x), bf16lo(vr[t].y), bf16hi(vr[t].y)};
+          float acc = 0.f;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            P[i] = fmaf(as[t], v[i], P[i]);
+            acc = fmaf(wb2x[i] + P[i], P[i], acc);
+          }
+          xp[s0 + t] = (s0 + t < cnt) ? acc : 0.f;
+        }
       }
+      xt = df_make(reduce_scatter32(xp, lane));
+    } else {
+      DF xp[32];
+      for (int s = 31; s >= 0; --s) {
+        const float as = __shfl_sync(kFull, at, s);
+        const int js = __shfl_sync(kFull, jt, s);
+        xp[s] = df_make(0.f);
+        if (s < cnt) {
+          float v[4];
+          load_row4(Vu + (size_t)js * kD, lane, v);
+          DF acc = df_make(0.f);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            Pd[i] = df_add(Pd[i], two_prod(as, v[i]));
+            acc = df_add(acc, df_mul(Pd[i], Pd[i]));
+          }
+          xp[s] = acc;
+        }
+      }
+      xt = reduce_scatter32_df(xp, lane);
     }
-    const float xt = reduce_scatter32(xp, lane);
     // in-batch inclusive suffix sums over lanes >= t
     DF sm = df_make(at);
-    DF sq = ok ? two_prod(at, yt) : df_make(0.f);
+    DF sq = ok ? df_mul_f(DF{yv.x, yv.y}, at) : df_make(0.f);
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       DF om{__shfl_down_sync(kFull, sm.hi, o), __shfl_down_sync(kFull, sm.lo, o)};
@@ -233,7 +288,7 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
     } else if (p.statistic == 1) {
       c = df_sqrt(df_mul(Mt, Qt));
     } else {
-      const DF W2 = df_add_f(wb2, xt);
+      const DF W2 = df_add(wb2, xt);
       c = df_sqrt(df_add(df_mul(Mt, Qt), df_neg(W2)));
     }
     if (ok) {
@@ -282,7 +337,7 @@ void launch_curves(const Prob& p, const Layout& ly, char* ws, const void* K, con
   float4* agg_mq = reinterpret_cast<float4*>(ws + ly.agg_mq);
   float* agg_v = reinterpret_cast<float*>(ws + ly.agg_v);
   float* agg_k = reinterpret_cast<float*>(ws + ly.agg_k);
-  float* yrank = reinterpret_cast<float*>(ws + ly.s_tmp);  // pooled scores are dead by now
+  float2* yrank = reinterpret_cast<float2*>(ws + ly.yrank);
   float4* base_mq = reinterpret_cast<float4*>(ws + ly.base_mq);
   float2* base_v = reinterpret_cast<float2*>(ws + ly.base_v);
   float2* base_k = reinterpret_cast<float2*>(ws + ly.base_k);

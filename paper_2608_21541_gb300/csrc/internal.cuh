@@ -41,6 +41,7 @@ struct Layout {
   size_t a;          // float  [U][n]   scores (when the caller gives none)
   size_t keys0, keys1, vals0, vals1;  // uint32/int32 [U][n]
   size_t hist;       // uint32 [U][256][sort_tiles]
+  size_t yrank;      // float2 [U][n]  ||v||^2 per rank, double-float
   size_t agg_mq;     // float4 [U][chunks]  (m.hi, m.lo, q.hi, q.lo)
   size_t agg_v;      // float  [U][chunks][d]
   size_t agg_k;      // float  [U][chunks][d]
@@ -50,7 +51,7 @@ struct Layout {
   size_t curve;      // float2 [U][n]  c(b) as hi + lo
   size_t cmax;       // uint64 [U]     order key of max_b c(b)
   size_t cand;       // int32  [U][n]  allocator candidates
-  size_t ncand;      // int32  [U][hull_segs + 1]
+  size_t ncand;      // int32  [U][hull_segs + groups] survivors per segment, per group
   size_t total;
 };
 

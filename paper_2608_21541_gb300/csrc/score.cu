@@ -215,12 +215,14 @@ __global__ void __launch_bounds__(512) score_pass_kernel(const __nv_bfloat16* __
       }
     }
     __syncthreads();  // tile buffer and column sums are complete
-    if (PASS2 && threadIdx.x < kScoreTileKeys) {
+    if (PASS2) {
       const float* cb = colsum + (t & 1) * warps * 64;
-      float s = 0.f;
-      for (int wi = 0; wi < warps; ++wi) s += cb[wi * 64 + threadIdx.x];
-      int j = j0 + threadIdx.x;
-      if (j < n) s_part[((size_t)u * p.row_blocks + rb) * n + j] = s;
+      for (int c = threadIdx.x; c < kScoreTileKeys; c += blockDim.x) {
+        float s = 0.f;
+        for (int wi = 0; wi < warps; ++wi) s += cb[wi * 64 + c];
+        const int j = j0 + c;
+        if (j < n) s_part[((size_t)u * p.row_blocks + rb) * n + j] = s;
+      }
     }
   }
 
@@ -300,8 +302,8 @@ __global__ void __launch_bounds__(1024) score_finalize_kernel(Prob p, const floa
   DF tot = df_make(0.f);
   for (int j = threadIdx.x; j < n; j += blockDim.x) {
     float v = (j < nw) ? sp[j] : (p.protect ? smax : au[j]);
+    if (!(fabsf(v) <= 3.0e38f)) raise_status(status, 1u);  // NaN or Inf
     v = v > 0.f ? v : 0.f;
-    if (!(v <= 3.0e38f)) raise_status(status, 1u);  // NaN or Inf
     if (j >= nw) sp[j] = v;
     tot = df_add_f(tot, v);
   }

@@ -9,7 +9,8 @@ Tolerances (stated once, used by every parity test):
     near-tie of the allocation objective (relative gap <= 1e-6 under the
     oracle's curves), and a kept set may differ only by tokens whose score
     lies within 1e-6 relative of the cut;
-  * decode outputs (bf16): 2e-2 maximum absolute error.
+  * decode outputs (bf16): 2e-2 maximum absolute error for |o| <= 1, and
+    2e-2 relative above (one bf16 quantum of |o| >= 8 already exceeds 2e-2).
 """
 from __future__ import annotations
 
@@ -125,6 +126,14 @@ def check_end_to_end(got: dict, ref: dict, a_gpu: np.ndarray, H: int):
 
 
 def check_decode(out, ref_out):
-    err = float(np.abs(out.float().cpu().numpy() - ref_out).max())
-    assert err <= DECODE_ATOL, f"decode max abs error {err:.3e}"
-    return err
+    """2e-2 absolute error for outputs of magnitude up to 1 and 2e-2 relative
+    above: a bf16 output of magnitude >= 8 is quantised in steps of 2^-4, so an
+    absolute bound cannot hold there for any implementation."""
+    got = out.float().cpu().numpy()
+    scale = np.maximum(1.0, np.abs(ref_out))
+    err = np.abs(got - ref_out) / scale
+    i = np.unravel_index(int(np.argmax(err)), err.shape)
+    worst = float(err[i])
+    assert worst <= DECODE_ATOL, (f"decode error {worst:.3e} at {i}: got {got[i]:.6g}, "
+                                  f"oracle {ref_out[i]:.6g}")
+    return worst
