@@ -40,6 +40,8 @@ def parse():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling only: compress this many layers instead of the workload's")
     return ap.parse_args()
 
 
@@ -145,6 +147,24 @@ def roofline_for(name, work, ms, peaks, traffic=None):
     return {"kernel": name, "bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm"],
             "unit": "GB/s", "frac": round(ach / peaks["hbm"], 4), "traffic": traffic,
             "peak_source": peaks["source"] + " (copy bandwidth)"}
+
+
+# ------------------------------------------------------------ multi-rank ----
+def max_over_ranks(value: float, world: int) -> float:
+    """The maximum of `value` over all ranks (the job's step time)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: int, world: int, ms: float) -> float:
+    """Whole-job throughput: every rank processes its own units (weak scaling)."""
+    return world * units_per_rank / (ms / 1e3)
 
 
 # ----------------------------------------------------------- oracle arms ----
@@ -258,13 +278,9 @@ def run_ours(args, wl, rank, world):
     clk = clocks.stop()
     trace = ck.certkv_trace_report()
     ck.certkv_trace_enable(False)
-    ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     tokens = wl.B * wl.L * wl.n
-    value = world * tokens / (ms / 1e3)
+    value = job_throughput(tokens, world, ms)
 
     # per-kernel shares and the dominant kernel's roofline
     kernels = {}
@@ -380,6 +396,8 @@ def main():
     args = parse()
     from paper_2608_21541_gb300 import workloads as W
     wl = W.WORKLOADS[args.config]
+    if args.layers:
+        wl = wl.with_(L=args.layers)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if world > 1:
