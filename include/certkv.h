@@ -66,6 +66,8 @@ extern "C" {
 #define CERTKV_EWORKSPACE  3  /* workspace missing, misaligned or too small      */
 #define CERTKV_ECAPACITY   4  /* packed-cache capacity below B * L * B_live      */
 #define CERTKV_ECUDA       5  /* a CUDA runtime call failed                      */
+#define CERTKV_ETOOLARGE   6  /* problem exceeds the fixed scratch of
+                                 certkv_decode_attn_noalloc                     */
 
 /* bits of the device status word returned by certkv_read_status() */
 #define CERTKV_STATUS_NONFINITE   1u  /* a score or curve value was NaN/Inf     */
@@ -177,6 +179,32 @@ int certkv_decode_attn(const certkv_shape* shape, const void* q,
                        const certkv_packed* packed, float scale, int32_t tail_slot,
                        void* out, void* workspace, size_t workspace_bytes,
                        void* stream);
+
+/* Decode attention that allocates nothing.  The paper has no counterpart: this
+ * entry point exists for callers that cannot hand the library a scratch
+ * buffer, for example a plugin that an inference server gives only its input
+ * and output tensors, or a per-token decode loop that must not call cudaMalloc
+ * because cudaMalloc can wait for the whole device and breaks a memory plan
+ * fixed at start-up.  It computes exactly what certkv_decode_attn computes
+ * (same kernels, same arguments minus the workspace); its split-K scratch is a
+ * fixed array of CERTKV_NOALLOC_SCRATCH_BYTES in the library's own device
+ * memory, present on every GPU that loads the library until the process exits.
+ *   - Limit: (B * L * H) * G * 16 partial records of 520 bytes must fit in the
+ *     array, i.e. (B * L * H) * G <= 2016 (one 32-layer, 8-KV-head, G = 4
+ *     sequence per call); larger calls return CERTKV_ETOOLARGE and enqueue
+ *     nothing.  Split a larger batch into several calls.
+ *   - The first call on each device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - Every call on a device shares the one array, and each call rewrites every
+ *     scratch record before reading it, so nothing has to start at zero; calls
+ *     that overlap on the GPU (different streams, threads or processes sharing
+ *     the context) race on the array: order them, e.g. on one stream.
+ *   - No cudaMalloc, cudaFree or allocating library routine is called.
+ * Returns CERTKV_OK, CERTKV_EINVAL, CERTKV_ETOOLARGE or CERTKV_ECUDA. */
+#define CERTKV_NOALLOC_SCRATCH_BYTES (16u << 20)
+int certkv_decode_attn_noalloc(const certkv_shape* shape, const void* q,
+                               const certkv_packed* packed, float scale, int32_t tail_slot,
+                               void* out, void* stream);
 
 /* Synchronise `stream`, then return the device status word (CERTKV_STATUS_*
  * bits, 0 = clean) that the last compress call on `workspace` left, or -1 if

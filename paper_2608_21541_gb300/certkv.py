@@ -18,7 +18,7 @@ import torch
 
 from . import build as _build
 
-OK, EINVAL, EBUDGET, EWORKSPACE, ECAPACITY, ECUDA = range(6)
+OK, EINVAL, EBUDGET, EWORKSPACE, ECAPACITY, ECUDA, ETOOLARGE = range(7)
 STATUS_NONFINITE = 1
 STATUS_ZERO_TAIL = 2
 STAT_CENTERED, STAT_UNCENTERED, STAT_TAIL_MASS = 0, 1, 2
@@ -48,7 +48,7 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_decode_workspace_bytes", "certkv_score", "certkv_curves",
             "certkv_compress_scored", "certkv_compress", "certkv_decode_attn",
             "certkv_read_status", "certkv_strerror", "certkv_trace_enable",
-            "certkv_trace_report")
+            "certkv_trace_report", "certkv_decode_attn_noalloc")
 
 _lock = threading.Lock()
 _lib = None
@@ -99,6 +99,8 @@ def load_library(path: Optional[str] = None):
         lib.certkv_trace_enable.restype = ctypes.c_int
         lib.certkv_trace_report.argtypes = [ctypes.c_char_p, SZ]
         lib.certkv_trace_report.restype = ctypes.c_int
+        lib.certkv_decode_attn_noalloc.argtypes = [sp, P, kp, ctypes.c_float, I32, P, P]
+        lib.certkv_decode_attn_noalloc.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -323,4 +325,23 @@ def certkv_trace_report() -> dict:
     for line in buf.value.decode().splitlines():
         name, cnt, ms = line.split()
         out[name] = (int(cnt), float(ms))
+    return out
+
+
+def certkv_decode_attn_noalloc(q, packed: Packed, *, hkv: int, scale: float = 0.0, out=None,
+                               stream=None) -> torch.Tensor:
+    """a9 for callers that cannot provide scratch memory: the library uses its
+    own fixed 16 MiB device array instead (see include/certkv.h for the limit
+    and for calls that overlap on the GPU).  The output tensor is the caller's."""
+    _bf16(q, "q")
+    B, L, Hq, d = q.shape
+    shape = certkv_shape(B, L, Hq, hkv, 2, d, 1)
+    if out is None:
+        out = torch.empty_like(q)
+    st = packed.struct()
+    rc = load_library().certkv_decode_attn_noalloc(ctypes.byref(shape), _ptr(q),
+                                                   ctypes.byref(st), float(scale),
+                                                   int(packed.tail_slot), _ptr(out),
+                                                   _stream(stream))
+    _check(rc, "certkv_decode_attn_noalloc")
     return out

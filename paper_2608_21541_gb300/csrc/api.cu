@@ -332,6 +332,9 @@ const char* certkv_strerror(int code) {
     case CERTKV_EWORKSPACE: return "workspace missing, misaligned or too small";
     case CERTKV_ECAPACITY: return "packed-cache capacity below B*L*B_live slots";
     case CERTKV_ECUDA: return "CUDA runtime error";
+    case CERTKV_ETOOLARGE:
+      return "problem exceeds the fixed 16 MiB scratch of certkv_decode_attn_noalloc "
+             "((B*L*H)*G <= 2016); split the call";
     default: return "unknown error";
   }
 }
