@@ -73,6 +73,8 @@ extern "C" {
 #define CERTKV_STATUS_NONFINITE   1u  /* a score or curve value was NaN/Inf     */
 #define CERTKV_STATUS_ZERO_TAIL   2u  /* an evicted suffix had zero mass: its
                                          tail slot is the uniform mean instead */
+#define CERTKV_STATUS_TIMEOUT     4u  /* a bounded wait inside a tensor-core
+                                         kernel gave up; its outputs are invalid */
 
 /* ---- problem description ------------------------------------------------- */
 typedef struct {

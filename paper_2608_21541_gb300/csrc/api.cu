@@ -59,7 +59,9 @@ int make_prob(const certkv_shape* s, const certkv_params* q, int64_t budget_live
   P.statistic = q->statistic; P.tail_slot = q->tail_slot;
   P.score_warps = (P.R + 15) / 16 < 16 ? (P.R + 15) / 16 : 16;
   P.row_blocks = (P.R + 16 * P.score_warps - 1) / (16 * P.score_warps);
-  P.key_splits = (P.n + kScoreKeysPerCta - 1) / kScoreKeysPerCta;
+  P.score_tc = score_tc_supported(P) ? 1 : 0;
+  P.key_splits = P.score_tc ? (P.n + kKeysPerItemTc - 1) / kKeysPerItemTc
+                            : (P.n + kScoreKeysPerCta - 1) / kScoreKeysPerCta;
   P.sort_tiles = (P.n + kSortTile - 1) / kSortTile;
   P.chunks = (P.n + kChunk - 1) / kChunk;
   if (budget_live >= 0) {

@@ -20,6 +20,7 @@ struct Prob {
   int64_t B_live, B_real;
   int b_min;
   // derived launch geometry
+  int score_tc;     // 1: tcgen05 scorer (R in {128, 256}); 0: mma.sync scorer
   int score_warps;  // warps per score CTA (16 rows each)
   int row_blocks;   // ceil(R / (16 * score_warps))
   int key_splits;   // ceil(n / kScoreKeysPerCta)
@@ -28,7 +29,8 @@ struct Prob {
   int hull_segs;    // ceil((n - b_min) / kHullSeg)
 };
 
-constexpr int kScoreKeysPerCta = 1024;
+constexpr int kScoreKeysPerCta = 1024;   // keys per CTA of the mma.sync scorer
+constexpr int kKeysPerItemTc = 16384;    // keys per CTA of the tcgen05 scorer
 constexpr int kScoreTileKeys = 64;
 
 // Workspace carve-up (byte offsets from the workspace base, 256-B aligned).
@@ -58,6 +60,10 @@ struct Layout {
 Layout make_layout(const Prob& p);
 
 // ---- launchers (all asynchronous on `st`) --------------------------------
+__global__ void lse_merge_kernel(Prob p, const float2* __restrict__ part, float* __restrict__ lse2);
+bool score_tc_supported(const Prob& p);
+bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_part, float* lse2,
+                     float* s_part, uint32_t* status, cudaStream_t st);
 void launch_score(const Prob& p, const Layout& ly, char* ws, const void* K, const void* Q,
                   float* a_out, cudaStream_t st);
 void launch_sort(const Prob& p, const Layout& ly, char* ws, const float* a, cudaStream_t st);

@@ -345,7 +345,12 @@ void launch_score(const Prob& p, const Layout& ly, char* ws, const void* K, cons
     cudaFuncSetAttribute(score_pass_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
     attr_set = true;
   }
+  bool done = false;
+  if (p.score_tc)
+    done = launch_score_tc(p, K, Q, lse_part, lse2, s_part,
+                           reinterpret_cast<uint32_t*>(ws + ly.status), st);
   dim3 grid(p.key_splits, p.row_blocks, p.units);
+  if (!done) {
   {
     TraceScope ts_("score_pass1", st);
     score_pass_kernel<false><<<grid, threads, smem, st>>>(Kb, Qb, p, nullptr, lse_part, nullptr);
@@ -358,6 +363,7 @@ void launch_score(const Prob& p, const Layout& ly, char* ws, const void* K, cons
   {
     TraceScope ts_("score_pass2", st);
     score_pass_kernel<true><<<grid, threads, smem, st>>>(Kb, Qb, p, lse2, nullptr, s_part);
+  }
   }
   {
     TraceScope ts_("score_finalize", st);

@@ -1,0 +1,493 @@
+// score_tc.cu — a1/a2 on the 5th-generation tensor cores (tcgen05 + TMEM).
+//
+// The same two passes as score.cu (§4 observation-window score; the log-sum-
+// exp of every observation row is needed before any column sum), for the
+// observation-row counts R in {128, 256} that fit one MMA instruction:
+//   pass 1  D[rows x keys] = Q K^T.  Each epilogue thread owns one row and
+//           keeps its online (max, sum) over the CTA's keys without shuffles.
+//   pass 2  D[keys x rows] = K Q^T.  Each epilogue thread owns one key and sums
+//           exp(l - LSE_row) over the rows of its TMEM lane without shuffles.
+// Roles per CTA (one work item = one unit x kKeysPerItem keys):
+//   warp 0      TMA producer: Q once, then K tiles of 128 keys (two 128-byte
+//               swizzled boxes of 64 dims) into a kStages-deep ring;
+//   warp 1      TMEM allocation and the single MMA-issuing thread
+//               (tcgen05.mma kind::f16, bf16 x bf16 -> fp32 in TMEM, two
+//               accumulator buffers so MMA and epilogue overlap);
+//   warps 2..9  epilogue: tcgen05.ld, exp2, reductions.
+// Every mbarrier wait is bounded; a timeout sets an abort flag and the status
+// word, every role then drains and the CTA frees its TMEM before returning.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "../../include/certkv.h"
+#include "common.cuh"
+#include "internal.cuh"
+
+namespace certkv {
+namespace tc {
+
+constexpr int kTileKeys = 128;
+constexpr int kStages = 4;
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = (2 + kEpiWarps) * 32;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kSpinLimit = 1u << 22;
+constexpr int kQBytes = 256 * 128 * 2;         // Q region (two 128-B-wide halves)
+constexpr int kStageBytes = kTileKeys * 128 * 2;  // one K tile (two halves)
+constexpr int kBarOff = kQBytes + kStages * kStageBytes;
+constexpr int kMiscBytes = 4096;
+constexpr int kSmemBytes = kBarOff + kMiscBytes + 1024;  // + alignment slack
+constexpr uint32_t kStatusTimeout = CERTKV_STATUS_TIMEOUT;
+
+// ------------------------------------------------------------ primitives --
+__device__ __forceinline__ uint32_t saddr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t a) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred P;\n mbarrier.try_wait.parity.shared::cta.b64 P, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, P;\n}\n"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait: false on timeout or when another role has aborted.
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, volatile int* abort_flag) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if (mbar_try(a, parity)) return true;
+    if ((i & 255u) == 255u && *abort_flag) return false;
+  }
+  *abort_flag = 1;
+  return false;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t mbar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(mbar)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 B, groups of 8 rows 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t smem) {
+  uint64_t d = 0;
+  d |= (uint64_t)((smem >> 4) & 0x3FFFu);
+  d |= (uint64_t)1u << 16;             // leading byte offset (unused with this swizzle)
+  d |= (uint64_t)(1024u >> 4) << 32;   // stride byte offset: 8 rows x 128 B
+  d |= (uint64_t)1u << 46;             // descriptor version
+  d |= (uint64_t)2u << 61;             // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulate, bf16 A and B, both
+// K-major, shape M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
+         ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
+}
+__device__ __forceinline__ void umma_commit(uint32_t mbar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   mbar)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one per thread).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Named barrier over the epilogue warps only; returns the OR of `stop` over
+// them, so that every epilogue warp takes the same decision.
+__device__ __forceinline__ bool epi_sync_or(bool stop) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n"
+      " bar.red.or.pred po, 1, %2, pi;\n selp.u32 %0, 1, 0, po;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)stop), "n"(kEpiWarps * 32)
+      : "memory");
+  return r != 0;
+}
+
+struct Shared {
+  char* base;  // 1024-byte aligned
+  __device__ uint32_t q() const { return saddr(base); }
+  __device__ uint32_t kst(int s) const { return saddr(base + kQBytes + s * kStageBytes); }
+  __device__ uint64_t* bars() const { return reinterpret_cast<uint64_t*>(base + kBarOff); }
+  __device__ uint32_t full(int s) const { return saddr(bars() + s); }
+  __device__ uint32_t empty(int s) const { return saddr(bars() + kStages + s); }
+  __device__ uint32_t accf(int b) const { return saddr(bars() + 2 * kStages + b); }
+  __device__ uint32_t acce(int b) const { return saddr(bars() + 2 * kStages + 2 + b); }
+  __device__ uint32_t qfull() const { return saddr(bars() + 2 * kStages + 4); }
+  __device__ uint32_t done() const { return saddr(bars() + 2 * kStages + 5); }
+  __device__ uint32_t* tmem_slot() const { return reinterpret_cast<uint32_t*>(base + kBarOff + 256); }
+  __device__ volatile int* abort_flag() const {
+    return reinterpret_cast<volatile int*>(base + kBarOff + 260);
+  }
+  __device__ float* lse() const { return reinterpret_cast<float*>(base + kBarOff + 512); }  // 256
+  __device__ float* part() const { return reinterpret_cast<float*>(base + kBarOff + 1536); }  // 2x2x128
+};
+
+__device__ __forceinline__ Shared shared_layout(char* raw) {
+  Shared s;
+  s.base = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~(uintptr_t)1023);
+  return s;
+}
+
+// Set-up common to both passes: barriers, TMEM allocation.
+__device__ __forceinline__ uint32_t setup(const Shared& sh, int warp) {
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(sh.full(s), 1);
+      mbar_init(sh.empty(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(sh.accf(b), 1);
+      mbar_init(sh.acce(b), kEpiWarps);
+    }
+    mbar_init(sh.qfull(), 1);
+    mbar_init(sh.done(), 1);
+    *sh.abort_flag() = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     saddr(sh.tmem_slot())),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  return *sh.tmem_slot();
+}
+
+__device__ __forceinline__ void teardown(const Shared& sh, int warp, uint32_t tmem, uint32_t* status) {
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && *sh.abort_flag()) atomicOr(status, kStatusTimeout);
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kTmemCols)
+                 : "memory");
+  }
+}
+
+// Producer: Q once, then the K tiles of [j_begin, j_begin + ntiles*128).
+__device__ __forceinline__ void produce(const Shared& sh, const CUtensorMap* tmK,
+                                        const CUtensorMap* tmQ, int qrow0, int R, long krow0,
+                                        int ntiles) {
+  volatile int* ab = sh.abort_flag();
+  mbar_expect_tx(sh.qfull(), (uint32_t)R * 256u);
+  tma_load_2d(sh.q(), tmQ, 0, qrow0, sh.qfull());
+  tma_load_2d(sh.q() + kQBytes / 2, tmQ, 64, qrow0, sh.qfull());
+  int issued = 0;
+  for (int t = 0; t < ntiles; ++t) {
+    const int s = t % kStages;
+    if (t >= kStages && !mbar_wait(sh.empty(s), ((t / kStages) - 1) & 1, ab)) break;
+    mbar_expect_tx(sh.full(s), (uint32_t)kStageBytes);
+    const int y = (int)(krow0 + (long)t * kTileKeys);
+    tma_load_2d(sh.kst(s), tmK, 0, y, sh.full(s));
+    tma_load_2d(sh.kst(s) + kStageBytes / 2, tmK, 64, y, sh.full(s));
+    issued = t + 1;
+  }
+  // drain: the copies of the last stages must land before the CTA exits
+  for (int t = (issued > kStages ? issued - kStages : 0); t < issued; ++t) {
+    const int s = t % kStages;
+    volatile int dummy = 0;
+    mbar_wait(sh.full(s), (t / kStages) & 1, &dummy);
+  }
+  volatile int dummy = 0;
+  mbar_wait(sh.qfull(), 0, &dummy);
+}
+
+// grid = units * items_per_unit, block = kThreads.  Pass 1: per-row (max, sum).
+__global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_constant__ CUtensorMap tmK,
+                                                             const __grid_constant__ CUtensorMap tmQ,
+                                                             Prob p, float2* __restrict__ lse_part,
+                                                             uint32_t* status) {
+  extern __shared__ char smem_raw[];
+  const Shared sh = shared_layout(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int u = blockIdx.x / p.key_splits, split = blockIdx.x % p.key_splits;
+  const int n = p.n, R = p.R, halves = R / 128;
+  const int j_begin = split * kKeysPerItemTc;
+  const int j_end = min(n, j_begin + kKeysPerItemTc);
+  const int ntiles = (j_end - j_begin + kTileKeys - 1) / kTileKeys;
+  const uint32_t tmem = setup(sh, warp);
+  volatile int* ab = sh.abort_flag();
+
+  if (warp == 0) {
+    if (lane == 0) produce(sh, &tmK, &tmQ, u * R, R, (long)u * n + j_begin, ntiles);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(128, kTileKeys);
+      bool ok = mbar_wait(sh.qfull(), 0, ab);
+      tc_fence_after();
+      for (int t = 0; ok && t < ntiles; ++t) {
+        const int s = t % kStages, b = t & 1;
+        if (!mbar_wait(sh.full(s), (t / kStages) & 1, ab)) break;
+        if (t >= 2 && !mbar_wait(sh.acce(b), ((t >> 1) - 1) & 1, ab)) break;
+        tc_fence_after();
+        for (int half = 0; half < halves; ++half) {
+          const uint32_t d = tmem + (uint32_t)(b * 256 + half * 128);
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint32_t kh = ks >> 2, koff = (ks & 3) * 32;
+            const uint64_t a = sw128_desc(sh.q() + kh * (kQBytes / 2) + half * 128 * 128 + koff);
+            const uint64_t bdesc = sw128_desc(sh.kst(s) + kh * (kStageBytes / 2) + koff);
+            umma_bf16(d, a, bdesc, idesc, ks > 0);
+          }
+        }
+        umma_commit(sh.empty(s));
+        umma_commit(sh.accf(b));
+      }
+      umma_commit(sh.done());  // every MMA issued above has finished reading smem
+      volatile int dummy = 0;
+      mbar_wait(sh.done(), 0, &dummy);
+    }
+  } else {
+    const int ew = warp - 2, q = warp & 3, half = ew >> 2;
+    const int row = half * 128 + q * 32 + lane;
+    const bool active = half < halves && row < R;
+    const int lim = n - p.w + (row % p.w);
+    const float sl2 = p.scale_log2;
+    float m = -INFINITY, l = 0.f;
+    for (int t = 0; t < ntiles; ++t) {
+      const int b = t & 1;
+      if (!mbar_wait(sh.accf(b), (t >> 1) & 1, ab)) break;
+      tc_fence_after();
+      const int j0 = j_begin + t * kTileKeys;
+      if (half < halves) {
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + half * 128 + c * 32), v);
+          float cm = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int j = j0 + c * 32 + i;
+            v[i] = (j <= lim && j < j_end) ? v[i] * sl2 : -INFINITY;
+            cm = fmaxf(cm, v[i]);
+          }
+          const float nm = fmaxf(m, cm);
+          if (nm > -INFINITY) {
+            float s = 0.f;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) s += exp2f(v[i] - nm);
+            l = l * exp2f(m - nm) + s;
+            m = nm;
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sh.acce(b));
+    }
+    if (active && !*ab) lse_part[((size_t)u * R + row) * p.key_splits + split] = make_float2(m, l);
+  }
+  teardown(sh, warp, tmem, status);
+}
+
+// grid = units * items_per_unit, block = kThreads.  Pass 2: per-key column sums.
+__global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_constant__ CUtensorMap tmK,
+                                                                const __grid_constant__ CUtensorMap tmQ,
+                                                                Prob p, const float* __restrict__ lse2,
+                                                                float* __restrict__ s_part,
+                                                                uint32_t* status) {
+  extern __shared__ char smem_raw[];
+  const Shared sh = shared_layout(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int u = blockIdx.x / p.key_splits, split = blockIdx.x % p.key_splits;
+  const int n = p.n, R = p.R;
+  const int j_begin = split * kKeysPerItemTc;
+  const int j_end = min(n, j_begin + kKeysPerItemTc);
+  const int ntiles = (j_end - j_begin + kTileKeys - 1) / kTileKeys;
+  for (int r = threadIdx.x; r < R; r += blockDim.x) sh.lse()[r] = lse2[(size_t)u * R + r];
+  const uint32_t tmem = setup(sh, warp);
+  volatile int* ab = sh.abort_flag();
+
+  if (warp == 0) {
+    if (lane == 0) produce(sh, &tmK, &tmQ, u * R, R, (long)u * n + j_begin, ntiles);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(kTileKeys, R);
+      bool ok = mbar_wait(sh.qfull(), 0, ab);
+      tc_fence_after();
+      for (int t = 0; ok && t < ntiles; ++t) {
+        const int s = t % kStages, b = t & 1;
+        if (!mbar_wait(sh.full(s), (t / kStages) & 1, ab)) break;
+        if (t >= 2 && !mbar_wait(sh.acce(b), ((t >> 1) - 1) & 1, ab)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(b * 256);
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks) {
+          const uint32_t kh = ks >> 2, koff = (ks & 3) * 32;
+          const uint64_t a = sw128_desc(sh.kst(s) + kh * (kStageBytes / 2) + koff);
+          const uint64_t bdesc = sw128_desc(sh.q() + kh * (kQBytes / 2) + koff);
+          umma_bf16(d, a, bdesc, idesc, ks > 0);
+        }
+        umma_commit(sh.empty(s));
+        umma_commit(sh.accf(b));
+      }
+      umma_commit(sh.done());  // every MMA issued above has finished reading smem
+      volatile int dummy = 0;
+      mbar_wait(sh.done(), 0, &dummy);
+    }
+  } else {
+    const int ew = warp - 2, q = warp & 3, ch = ew >> 2;  // ch: which 128 rows
+    const int key = q * 32 + lane;
+    const bool rows_here = ch * 128 < R;
+    const float sl2 = p.scale_log2;
+    const int nw = n - p.w;
+    float* part = sh.part();
+    for (int t = 0; t < ntiles; ++t) {
+      const int b = t & 1;
+      const bool ok = mbar_wait(sh.accf(b), (t >> 1) & 1, ab);
+      if (epi_sync_or(!ok)) break;  // all epilogue warps stop together
+      tc_fence_after();
+      const int j = j_begin + t * kTileKeys + key;
+      float s = 0.f;
+      if (rows_here) {
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + ch * 128 + c * 32), v);
+          const int r0 = ch * 128 + c * 32;
+          if (j < nw) {  // every observation row sees this key
+#pragma unroll
+            for (int i = 0; i < 32; ++i) s += exp2f(fmaf(v[i], sl2, -sh.lse()[r0 + i]));
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int r = r0 + i;
+              if (j < j_end && j <= nw + (r % p.w)) s += exp2f(fmaf(v[i], sl2, -sh.lse()[r]));
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sh.acce(b));
+      // combine the two row halves of this key
+      float* pb = part + (t & 1) * 256;
+      pb[ch * 128 + key] = s;
+      epi_sync_or(false);
+      if (ch == 0 && j < j_end)
+        s_part[(size_t)u * p.row_blocks * n + j] = pb[key] + pb[128 + key];
+    }
+  }
+  teardown(sh, warp, tmem, status);
+}
+
+}  // namespace tc
+
+// --------------------------------------------------------------- host ----
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// 2-D view [rows][128] of a bf16 tensor, boxes of {64 dims, box_rows rows},
+// 128-byte swizzle.
+bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {128, rows};
+  cuuint64_t strides[1] = {256};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool score_tc_supported(const Prob& p) { return p.R == 128 || p.R == 256; }
+
+bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_part, float* lse2,
+                     float* s_part, uint32_t* status, cudaStream_t st) {
+  CUtensorMap mk, mq;
+  if (!make_map(&mk, K, (uint64_t)p.units * p.n, tc::kTileKeys)) return false;
+  if (!make_map(&mq, Q, (uint64_t)p.units * p.R, (uint32_t)p.R)) return false;
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(tc::lse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         tc::kSmemBytes);
+    cudaFuncSetAttribute(tc::colsum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         tc::kSmemBytes);
+    attr = true;
+  }
+  const unsigned grid = (unsigned)(p.units * p.key_splits);
+  {
+    TraceScope ts_("score_pass1", st);
+    tc::lse_tc_kernel<<<grid, tc::kThreads, tc::kSmemBytes, st>>>(mk, mq, p, lse_part, status);
+  }
+  const size_t rows = (size_t)p.units * p.R;
+  {
+    TraceScope ts_("lse_merge", st);
+    lse_merge_kernel<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(p, lse_part, lse2);
+  }
+  {
+    TraceScope ts_("score_pass2", st);
+    tc::colsum_tc_kernel<<<grid, tc::kThreads, tc::kSmemBytes, st>>>(mk, mq, p, lse2, s_part,
+                                                                     status);
+  }
+  return true;
+}
+
+}  // namespace certkv
