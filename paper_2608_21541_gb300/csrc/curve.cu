@@ -45,6 +45,32 @@ __device__ __forceinline__ DF reduce_scatter32_df(DF (&v)[32], int lane) {
   return v[0];
 }
 
+// As reduce_scatter32_df, from fp32 inputs: the first butterfly level already
+// produces double-float sums (error-free), the later ones add double-floats.
+__device__ __forceinline__ DF reduce_scatter32_f2df(float (&v)[32], int lane) {
+  DF w[16];
+  {
+    const bool upper = (lane & 16) != 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const float keep = upper ? v[i + 16] : v[i];
+      const float send = upper ? v[i] : v[i + 16];
+      w[i] = two_sum(keep, __shfl_xor_sync(kFull, send, 16));
+    }
+  }
+#pragma unroll
+  for (int o = 8; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      DF keep = upper ? w[i + o] : w[i];
+      DF send = upper ? w[i] : w[i + o];
+      w[i] = df_add(keep, shfl_xor_df(send, o));
+    }
+  }
+  return w[0];
+}
+
 // lane t ends with sum over lanes of v[t]  (31 shuffles)
 __device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
 #pragma unroll
@@ -90,7 +116,9 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
     const float at = ok ? key_score(ku[r]) : 0.f;
     const int jt = ok ? pu[r] : 0;
     const int cnt = min(32, r1 - rb);
-    DF yp[32];  // ||v||^2 partials: bf16 squares are exact in fp32, sums in double-float
+    // ||v||^2: per lane the 4 squares of bf16 values (each exact in fp32) are
+    // summed in fp32, the 32 lane partials in double-float.
+    float yp[32];
 #pragma unroll
     for (int s0 = 0; s0 < 32; s0 += 8) {
       // issue the 8 rows' loads first so that they are in flight together
@@ -116,11 +144,10 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
           sv[i] = fmaf(as[t], v[i], sv[i]);
           sk[i] = fmaf(as[t], k4[i], sk[i]);
         }
-        DF y = two_sum(__fmul_rn(v[0], v[0]), __fmul_rn(v[1], v[1]));
-        yp[s0 + t] = df_add(y, two_sum(__fmul_rn(v[2], v[2]), __fmul_rn(v[3], v[3])));
+        yp[s0 + t] = fmaf(v[3], v[3], fmaf(v[2], v[2], fmaf(v[1], v[1], v[0] * v[0])));
       }
     }
-    const DF yt = reduce_scatter32_df(yp, lane);
+    const DF yt = reduce_scatter32_f2df(yp, lane);
     if (ok) yrank[(size_t)u * n + r] = make_float2(yt.hi, yt.lo);
     DF dm = df_make(at);
     DF dq = ok ? df_mul_f(yt, at) : df_make(0.f);

@@ -137,17 +137,11 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Named barrier over the epilogue warps only; returns the OR of `stop` over
-// them, so that every epilogue warp takes the same decision.
-__device__ __forceinline__ bool epi_sync_or(bool stop) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n"
-      " bar.red.or.pred po, 1, %2, pi;\n selp.u32 %0, 1, 0, po;\n}\n"
-      : "=r"(r)
-      : "r"((uint32_t)stop), "n"(kEpiWarps * 32)
-      : "memory");
-  return r != 0;
+// Hardware base-2 exponential (MUFU), flush-to-zero, relative error ~2^-22.
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 struct Shared {
@@ -166,7 +160,6 @@ struct Shared {
     return reinterpret_cast<volatile int*>(base + kBarOff + 260);
   }
   __device__ float* lse() const { return reinterpret_cast<float*>(base + kBarOff + 512); }  // 256
-  __device__ float* part() const { return reinterpret_cast<float*>(base + kBarOff + 1536); }  // 2x2x128
 };
 
 __device__ __forceinline__ Shared shared_layout(char* raw) {
@@ -301,25 +294,44 @@ __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_consta
       if (!mbar_wait(sh.accf(b), (t >> 1) & 1, ab)) break;
       tc_fence_after();
       const int j0 = j_begin + t * kTileKeys;
+      // every row sees every key of an interior tile: no mask needed
+      const bool interior = (j0 + kTileKeys <= j_end) && (j0 + kTileKeys - 1 <= n - p.w);
       if (half < halves) {
 #pragma unroll 1
         for (int c = 0; c < 4; ++c) {
           float v[32];
           tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + half * 128 + c * 32), v);
-          float cm = -INFINITY;
+          if (interior) {
+            float mx = v[0];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int j = j0 + c * 32 + i;
-            v[i] = (j <= lim && j < j_end) ? v[i] * sl2 : -INFINITY;
-            cm = fmaxf(cm, v[i]);
-          }
-          const float nm = fmaxf(m, cm);
-          if (nm > -INFINITY) {
-            float s = 0.f;
+            for (int i = 1; i < 32; ++i) mx = fmaxf(mx, v[i]);
+            const float nm = fmaxf(m, mx * sl2);  // sl2 > 0: the max commutes with scaling
+            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-            for (int i = 0; i < 32; ++i) s += exp2f(v[i] - nm);
-            l = l * exp2f(m - nm) + s;
+            for (int i = 0; i < 32; i += 4) {
+              s0 += ex2(fmaf(v[i], sl2, -nm));
+              s1 += ex2(fmaf(v[i + 1], sl2, -nm));
+              s2 += ex2(fmaf(v[i + 2], sl2, -nm));
+              s3 += ex2(fmaf(v[i + 3], sl2, -nm));
+            }
+            l = fmaf(l, ex2(m - nm), (s0 + s1) + (s2 + s3));
             m = nm;
+          } else {
+            float cm = -INFINITY;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int j = j0 + c * 32 + i;
+              v[i] = (j <= lim && j < j_end) ? v[i] * sl2 : -INFINITY;
+              cm = fmaxf(cm, v[i]);
+            }
+            const float nm = fmaxf(m, cm);
+            if (nm > -INFINITY) {
+              float sum = 0.f;
+#pragma unroll
+              for (int i = 0; i < 32; ++i) sum += ex2(v[i] - nm);
+              l = fmaf(l, ex2(m - nm), sum);
+              m = nm;
+            }
           }
         }
       }
@@ -383,28 +395,37 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
     const bool rows_here = ch * 128 < R;
     const float sl2 = p.scale_log2;
     const int nw = n - p.w;
-    float* part = sh.part();
+    // the two row halves write separate row blocks; the finalize kernel adds them
+    float* out = s_part + ((size_t)u * p.row_blocks + ch) * n;
     for (int t = 0; t < ntiles; ++t) {
       const int b = t & 1;
-      const bool ok = mbar_wait(sh.accf(b), (t >> 1) & 1, ab);
-      if (epi_sync_or(!ok)) break;  // all epilogue warps stop together
+      if (!mbar_wait(sh.accf(b), (t >> 1) & 1, ab)) break;
       tc_fence_after();
-      const int j = j_begin + t * kTileKeys + key;
-      float s = 0.f;
+      const int j0 = j_begin + t * kTileKeys;
+      const int j = j0 + key;
+      const bool interior = (j0 + kTileKeys <= j_end) && (j0 + kTileKeys <= nw);
+      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
       if (rows_here) {
 #pragma unroll 1
         for (int c = 0; c < 4; ++c) {
           float v[32];
           tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + ch * 128 + c * 32), v);
           const int r0 = ch * 128 + c * 32;
-          if (j < nw) {  // every observation row sees this key
+          const float4* L4 = reinterpret_cast<const float4*>(sh.lse() + r0);
+          if (interior) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) s += exp2f(fmaf(v[i], sl2, -sh.lse()[r0 + i]));
+            for (int i = 0; i < 32; i += 4) {
+              const float4 L = L4[i >> 2];
+              s0 += ex2(fmaf(v[i], sl2, -L.x));
+              s1 += ex2(fmaf(v[i + 1], sl2, -L.y));
+              s2 += ex2(fmaf(v[i + 2], sl2, -L.z));
+              s3 += ex2(fmaf(v[i + 3], sl2, -L.w));
+            }
           } else {
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
               const int r = r0 + i;
-              if (j < j_end && j <= nw + (r % p.w)) s += exp2f(fmaf(v[i], sl2, -sh.lse()[r]));
+              if (j < j_end && j <= nw + (r % p.w)) s0 += ex2(fmaf(v[i], sl2, -sh.lse()[r]));
             }
           }
         }
@@ -412,12 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sh.acce(b));
-      // combine the two row halves of this key
-      float* pb = part + (t & 1) * 256;
-      pb[ch * 128 + key] = s;
-      epi_sync_or(false);
-      if (ch == 0 && j < j_end)
-        s_part[(size_t)u * p.row_blocks * n + j] = pb[key] + pb[128 + key];
+      if (j < j_end) out[j] = (s0 + s1) + (s2 + s3);
     }
   }
   teardown(sh, warp, tmem, status);
