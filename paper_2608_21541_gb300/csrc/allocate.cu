@@ -186,7 +186,8 @@ __global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* _
 // (sequence, layer).  Candidates are staged in shared memory when they fit;
 // the repair keeps a 64-value window of each head's upcoming curve values in
 // shared memory, refilled by the whole warp.
-constexpr int kCandCap = 16384;  // staged candidates: 128 KB of values + 64 KB of b (dynamic smem)
+constexpr int kCandCap = 12288;  // staged candidates: 96 KB of values + 48 KB of b (dynamic smem)
+constexpr int kScan = 2048;      // curve values per round of a block extension (16 KB)
 
 __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2* __restrict__ curve,
                                                             const int32_t* __restrict__ cand,
@@ -198,6 +199,7 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
   __shared__ int coff[33];
   __shared__ double lam_sh[2];
   __shared__ float2 win[32][64];
+  __shared__ float2 scanbuf[kScan];
   extern __shared__ __align__(16) char dyn[];
   float2* cy = reinterpret_cast<float2*>(dyn);
   int32_t* cb_ = reinterpret_cast<int32_t*>(dyn + kCandCap * sizeof(float2));
@@ -334,14 +336,79 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
         b = nb;
       }
       ++tot;
-      if (nb + 1 - wbase >= 64 && nb < n - 1) {  // refill the winner's window
-        __syncwarp();
-        const float2* ch = curve + (size_t)(bl * H + who) * n;
-        for (int k = lane; k < 64; k += 32)
-          win[who][k] = (nb + 1 + k < n) ? ch[nb + 1 + k] : make_float2(0.f, 0.f);
-        if (lane == who) base = nb + 1;
-        __syncwarp();
+      const float2* ch = curve + (size_t)(bl * H + who) * n;
+      // The winner keeps every following marginal strictly below its leading
+      // one: those would be picked next one at a time anyway (each is below
+      // every other head's front), so the whole run is taken at once.
+      int bw = nb;
+      DF cw = shfl_df(cur, who);
+      bool more = false;
+      if (tot < B_real && bw < n - 1) {
+        int nbase = wbase;
+        if (bw + 1 - nbase >= 64) nbase = -1;  // next value not in the window
+        DF d1 = kNone;
+        if (nbase >= 0) {
+          const float2 w = win[who][bw + 1 - nbase];
+          d1 = df_add(DF{w.x, w.y}, df_neg(cw));
+        } else {
+          const float2 w = ch[bw + 1];
+          d1 = df_add(DF{w.x, w.y}, df_neg(cw));
+        }
+        more = df_less(d1, mg);
       }
+      bool extended = false;
+      while (more) {  // warp-cooperative scan, kScan values per round
+        extended = true;
+        __syncwarp();
+        for (int k = lane; k < kScan; k += 32)
+          scanbuf[k] = (bw + 1 + k < n) ? ch[bw + 1 + k] : make_float2(0.f, 0.f);
+        __syncwarp();
+        // lane L checks positions e = 64 L .. 64 L + 63: marginal c(bw+e+1) - c(bw+e)
+        int first = 64;
+        for (int i = 0; i < 64; ++i) {
+          const int e = lane * 64 + i;
+          const float2 pv = (e == 0) ? make_float2(cw.hi, cw.lo) : scanbuf[e - 1];
+          const float2 nv = scanbuf[e];
+          const DF d = df_add(DF{nv.x, nv.y}, df_neg(DF{pv.x, pv.y}));
+          const bool stop = (bw + e >= n - 1) || !df_less(d, mg);
+          if (stop) {
+            first = i;
+            break;
+          }
+        }
+        const unsigned stops = __ballot_sync(kFull, first < 64);
+        int run = kScan;
+        if (stops) {
+          const int L = __ffs(stops) - 1;
+          run = L * 64 + __shfl_sync(kFull, first, L);
+        } else {
+          __shfl_sync(kFull, first, 0);
+        }
+        const int64_t room = B_real - tot;
+        if ((int64_t)run > room) run = (int)room;
+        if (run > 0) {
+          const float2 last = scanbuf[run - 1];
+          cw = DF{last.x, last.y};
+        }
+        bw += run;
+        tot += run;
+        more = (run == kScan) && tot < B_real && bw < n - 1;
+      }
+      if (lane == who && extended) {
+        b = bw;
+        cur = cw;
+      }
+      const int wb = extended ? -1 : wbase;
+      if (nb + 1 - wbase >= 64 || extended) {  // refill the winner's window
+        if (bw < n - 1) {
+          __syncwarp();
+          for (int k = lane; k < 64; k += 32)
+            win[who][k] = (bw + 1 + k < n) ? ch[bw + 1 + k] : make_float2(0.f, 0.f);
+          if (lane == who) base = bw + 1;
+          __syncwarp();
+        }
+      }
+      (void)wb;
     }
     // counts and offsets: segment = b_h real slots (+ 1 tail slot)
     const int seg = live ? b + p.tail_slot : 0;
