@@ -13,7 +13,9 @@
 //   warp 1      TMEM allocation and the single MMA-issuing thread
 //               (tcgen05.mma kind::f16, bf16 x bf16 -> fp32 in TMEM, two
 //               accumulator buffers so MMA and epilogue overlap);
-//   warps 2..9  epilogue: tcgen05.ld, exp2, reductions.
+//   warps 2..17 epilogue: two groups of 8 warps, group g reads the
+//               accumulator buffer g (tiles of parity g): tcgen05.ld, exp2,
+//               reductions.
 // Every mbarrier wait is bounded; a timeout sets an abort flag and the status
 // word, every role then drains and the CTA frees its TMEM before returning.
 #include <cuda.h>
@@ -26,18 +28,30 @@
 namespace certkv {
 namespace tc {
 
-constexpr int kTileKeys = 128;
-constexpr int kStages = 4;
-constexpr int kEpiWarps = 8;
+#ifndef CERTKV_TC_STAGES
+#define CERTKV_TC_STAGES 4
+#endif
+constexpr int kEpiWarps = 16;  // two groups of 8, one per TMEM accumulator buffer
 constexpr int kThreads = (2 + kEpiWarps) * 32;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kSpinLimit = 1u << 22;
-constexpr int kQBytes = 256 * 128 * 2;         // Q region (two 128-B-wide halves)
-constexpr int kStageBytes = kTileKeys * 128 * 2;  // one K tile (two halves)
-constexpr int kBarOff = kQBytes + kStages * kStageBytes;
-constexpr int kMiscBytes = 4096;
-constexpr int kSmemBytes = kBarOff + kMiscBytes + 1024;  // + alignment slack
 constexpr uint32_t kStatusTimeout = CERTKV_STATUS_TIMEOUT;
+
+// Shared-memory plan of one pass: Q rows staged once, a ring of K tiles.
+template <int QROWS, int TKEYS, int STAGES>
+struct Cfg {
+  static constexpr int kQRows = QROWS;
+  static constexpr int kTileKeys = TKEYS;
+  static constexpr int kStages = STAGES;
+  static constexpr int kQBytes = QROWS * 128 * 2;        // two 128-B-wide halves
+  static constexpr int kStageBytes = TKEYS * 128 * 2;    // one K tile, two halves
+  static constexpr int kBarOff = kQBytes + STAGES * kStageBytes;
+  static constexpr int kSmemBytes = kBarOff + 8192 + 1024;  // + misc + alignment slack
+};
+// pass 1: one 128-row half of Q per CTA, 256-key tiles (M128 x N256 MMAs)
+using Pass1 = Cfg<128, 256, 2>;
+// pass 2: all (<= 256) rows of Q, 128-key tiles (M128 x N<=256 MMAs)
+using Pass2 = Cfg<256, 128, CERTKV_TC_STAGES>;
 
 // ------------------------------------------------------------ primitives --
 __device__ __forceinline__ uint32_t saddr(const void* p) {
@@ -144,40 +158,74 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// 64 consecutive fp32 columns: two 32-column loads issued before one wait.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
+  uint32_t r[64];
+#define CERTKV_R8(o) "=r"(r[o]), "=r"(r[o + 1]), "=r"(r[o + 2]), "=r"(r[o + 3]), "=r"(r[o + 4]), \
+                     "=r"(r[o + 5]), "=r"(r[o + 6]), "=r"(r[o + 7])
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : CERTKV_R8(0), CERTKV_R8(8), CERTKV_R8(16), CERTKV_R8(24)
+      : "r"(taddr));
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : CERTKV_R8(32), CERTKV_R8(40), CERTKV_R8(48), CERTKV_R8(56)
+      : "r"(taddr + 32u));
+#undef CERTKV_R8
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Named barrier over the epilogue warps only.
+__device__ __forceinline__ void epi_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+}
+
+template <class C>
 struct Shared {
   char* base;  // 1024-byte aligned
   __device__ uint32_t q() const { return saddr(base); }
-  __device__ uint32_t kst(int s) const { return saddr(base + kQBytes + s * kStageBytes); }
-  __device__ uint64_t* bars() const { return reinterpret_cast<uint64_t*>(base + kBarOff); }
+  __device__ uint32_t kst(int s) const { return saddr(base + C::kQBytes + s * C::kStageBytes); }
+  __device__ uint64_t* bars() const { return reinterpret_cast<uint64_t*>(base + C::kBarOff); }
   __device__ uint32_t full(int s) const { return saddr(bars() + s); }
-  __device__ uint32_t empty(int s) const { return saddr(bars() + kStages + s); }
-  __device__ uint32_t accf(int b) const { return saddr(bars() + 2 * kStages + b); }
-  __device__ uint32_t acce(int b) const { return saddr(bars() + 2 * kStages + 2 + b); }
-  __device__ uint32_t qfull() const { return saddr(bars() + 2 * kStages + 4); }
-  __device__ uint32_t done() const { return saddr(bars() + 2 * kStages + 5); }
-  __device__ uint32_t* tmem_slot() const { return reinterpret_cast<uint32_t*>(base + kBarOff + 256); }
-  __device__ volatile int* abort_flag() const {
-    return reinterpret_cast<volatile int*>(base + kBarOff + 260);
+  __device__ uint32_t empty(int s) const { return saddr(bars() + C::kStages + s); }
+  __device__ uint32_t accf(int b) const { return saddr(bars() + 2 * C::kStages + b); }
+  __device__ uint32_t acce(int b) const { return saddr(bars() + 2 * C::kStages + 2 + b); }
+  __device__ uint32_t qfull() const { return saddr(bars() + 2 * C::kStages + 4); }
+  __device__ uint32_t done() const { return saddr(bars() + 2 * C::kStages + 5); }
+  __device__ uint32_t* tmem_slot() const {
+    return reinterpret_cast<uint32_t*>(base + C::kBarOff + 256);
   }
-  __device__ float* lse() const { return reinterpret_cast<float*>(base + kBarOff + 512); }  // 256
+  __device__ volatile int* abort_flag() const {
+    return reinterpret_cast<volatile int*>(base + C::kBarOff + 260);
+  }
+  // misc region: lse[256] (pass 2) or the partial (max, sum) of 4 x 128 rows (pass 1)
+  __device__ float* lse() const { return reinterpret_cast<float*>(base + C::kBarOff + 512); }
+  __device__ float* pm() const { return reinterpret_cast<float*>(base + C::kBarOff + 512); }
+  __device__ float* pl() const { return reinterpret_cast<float*>(base + C::kBarOff + 2560); }
 };
 
-__device__ __forceinline__ Shared shared_layout(char* raw) {
-  Shared s;
+template <class C>
+__device__ __forceinline__ Shared<C> shared_layout(char* raw) {
+  Shared<C> s;
   s.base = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~(uintptr_t)1023);
   return s;
 }
 
 // Set-up common to both passes: barriers, TMEM allocation.
-__device__ __forceinline__ uint32_t setup(const Shared& sh, int warp) {
+template <class C>
+__device__ __forceinline__ uint32_t setup(const Shared<C>& sh, int warp) {
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < C::kStages; ++s) {
       mbar_init(sh.full(s), 1);
       mbar_init(sh.empty(s), 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(sh.accf(b), 1);
-      mbar_init(sh.acce(b), kEpiWarps);
+      mbar_init(sh.acce(b), kEpiWarps / 2);
     }
     mbar_init(sh.qfull(), 1);
     mbar_init(sh.done(), 1);
@@ -197,7 +245,9 @@ __device__ __forceinline__ uint32_t setup(const Shared& sh, int warp) {
   return *sh.tmem_slot();
 }
 
-__device__ __forceinline__ void teardown(const Shared& sh, int warp, uint32_t tmem, uint32_t* status) {
+template <class C>
+__device__ __forceinline__ void teardown(const Shared<C>& sh, int warp, uint32_t tmem,
+                                         uint32_t* status) {
   tc_fence_before();
   __syncthreads();
   if (threadIdx.x == 0 && *sh.abort_flag()) atomicOr(status, kStatusTimeout);
@@ -209,129 +259,142 @@ __device__ __forceinline__ void teardown(const Shared& sh, int warp, uint32_t tm
   }
 }
 
-// Producer: Q once, then the K tiles of [j_begin, j_begin + ntiles*128).
-__device__ __forceinline__ void produce(const Shared& sh, const CUtensorMap* tmK,
-                                        const CUtensorMap* tmQ, int qrow0, int R, long krow0,
+// Producer: qrows rows of Q once, then the K tiles starting at row krow0.
+template <class C>
+__device__ __forceinline__ void produce(const Shared<C>& sh, const CUtensorMap* tmK,
+                                        const CUtensorMap* tmQ, int qrow0, int qrows, long krow0,
                                         int ntiles) {
   volatile int* ab = sh.abort_flag();
-  mbar_expect_tx(sh.qfull(), (uint32_t)R * 256u);
+  mbar_expect_tx(sh.qfull(), (uint32_t)qrows * 256u);
   tma_load_2d(sh.q(), tmQ, 0, qrow0, sh.qfull());
-  tma_load_2d(sh.q() + kQBytes / 2, tmQ, 64, qrow0, sh.qfull());
+  tma_load_2d(sh.q() + C::kQBytes / 2, tmQ, 64, qrow0, sh.qfull());
   int issued = 0;
   for (int t = 0; t < ntiles; ++t) {
-    const int s = t % kStages;
-    if (t >= kStages && !mbar_wait(sh.empty(s), ((t / kStages) - 1) & 1, ab)) break;
-    mbar_expect_tx(sh.full(s), (uint32_t)kStageBytes);
-    const int y = (int)(krow0 + (long)t * kTileKeys);
+    const int s = t % C::kStages;
+    if (t >= C::kStages && !mbar_wait(sh.empty(s), ((t / C::kStages) - 1) & 1, ab)) break;
+    mbar_expect_tx(sh.full(s), (uint32_t)C::kStageBytes);
+    const int y = (int)(krow0 + (long)t * C::kTileKeys);
     tma_load_2d(sh.kst(s), tmK, 0, y, sh.full(s));
-    tma_load_2d(sh.kst(s) + kStageBytes / 2, tmK, 64, y, sh.full(s));
+    tma_load_2d(sh.kst(s) + C::kStageBytes / 2, tmK, 64, y, sh.full(s));
     issued = t + 1;
   }
   // drain: the copies of the last stages must land before the CTA exits
-  for (int t = (issued > kStages ? issued - kStages : 0); t < issued; ++t) {
-    const int s = t % kStages;
+  for (int t = (issued > C::kStages ? issued - C::kStages : 0); t < issued; ++t) {
+    const int s = t % C::kStages;
     volatile int dummy = 0;
-    mbar_wait(sh.full(s), (t / kStages) & 1, &dummy);
+    mbar_wait(sh.full(s), (t / C::kStages) & 1, &dummy);
   }
   volatile int dummy = 0;
   mbar_wait(sh.qfull(), 0, &dummy);
 }
 
-// grid = units * items_per_unit, block = kThreads.  Pass 1: per-row (max, sum).
+// MMA issuer: for each tile, 8 k-steps of one M128 x N MMA into buffer t & 1.
+// `a_of(kh, koff)` / `b_of(stage, kh, koff)` give the operand smem addresses.
+template <class C, class AOf, class BOf>
+__device__ __forceinline__ void issue_mmas(const Shared<C>& sh, uint32_t tmem, uint32_t idesc,
+                                           int ntiles, AOf a_of, BOf b_of) {
+  volatile int* ab = sh.abort_flag();
+  bool ok = mbar_wait(sh.qfull(), 0, ab);
+  tc_fence_after();
+  for (int t = 0; ok && t < ntiles; ++t) {
+    const int s = t % C::kStages, b = t & 1;
+    if (!mbar_wait(sh.full(s), (t / C::kStages) & 1, ab)) break;
+    if (t >= 2 && !mbar_wait(sh.acce(b), ((t >> 1) - 1) & 1, ab)) break;
+    tc_fence_after();
+    const uint32_t d = tmem + (uint32_t)(b * 256);
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+      const uint32_t kh = ks >> 2, koff = (ks & 3) * 32;
+      umma_bf16(d, sw128_desc(a_of(s, kh, koff)), sw128_desc(b_of(s, kh, koff)), idesc, ks > 0);
+    }
+    umma_commit(sh.empty(s));
+    umma_commit(sh.accf(b));
+  }
+  umma_commit(sh.done());  // every MMA issued above has finished reading smem
+  volatile int dummy = 0;
+  mbar_wait(sh.done(), 0, &dummy);
+}
+
+// Pass 1.  grid = units * key_splits * halves; adjacent CTAs are the two
+// 128-row halves of one key range (they stream the same K tiles, the second
+// mostly from L2).  D[rows x 256 keys]; epilogue thread = one row.
 __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_constant__ CUtensorMap tmK,
                                                              const __grid_constant__ CUtensorMap tmQ,
                                                              Prob p, float2* __restrict__ lse_part,
                                                              uint32_t* status) {
+  using C = Pass1;
   extern __shared__ char smem_raw[];
-  const Shared sh = shared_layout(smem_raw);
+  const Shared<C> sh = shared_layout<C>(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int u = blockIdx.x / p.key_splits, split = blockIdx.x % p.key_splits;
-  const int n = p.n, R = p.R, halves = R / 128;
+  const int halves = p.R / 128;
+  const int half = blockIdx.x % halves;
+  const int item = blockIdx.x / halves;
+  const int u = item / p.key_splits, split = item % p.key_splits;
+  const int n = p.n, R = p.R;
   const int j_begin = split * kKeysPerItemTc;
   const int j_end = min(n, j_begin + kKeysPerItemTc);
-  const int ntiles = (j_end - j_begin + kTileKeys - 1) / kTileKeys;
-  const uint32_t tmem = setup(sh, warp);
+  const int ntiles = (j_end - j_begin + C::kTileKeys - 1) / C::kTileKeys;
+  const uint32_t tmem = setup<C>(sh, warp);
   volatile int* ab = sh.abort_flag();
 
   if (warp == 0) {
-    if (lane == 0) produce(sh, &tmK, &tmQ, u * R, R, (long)u * n + j_begin, ntiles);
+    if (lane == 0) produce<C>(sh, &tmK, &tmQ, u * R + half * 128, 128, (long)u * n + j_begin, ntiles);
   } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(128, kTileKeys);
-      bool ok = mbar_wait(sh.qfull(), 0, ab);
-      tc_fence_after();
-      for (int t = 0; ok && t < ntiles; ++t) {
-        const int s = t % kStages, b = t & 1;
-        if (!mbar_wait(sh.full(s), (t / kStages) & 1, ab)) break;
-        if (t >= 2 && !mbar_wait(sh.acce(b), ((t >> 1) - 1) & 1, ab)) break;
-        tc_fence_after();
-        for (int half = 0; half < halves; ++half) {
-          const uint32_t d = tmem + (uint32_t)(b * 256 + half * 128);
-#pragma unroll
-          for (int ks = 0; ks < 8; ++ks) {
-            const uint32_t kh = ks >> 2, koff = (ks & 3) * 32;
-            const uint64_t a = sw128_desc(sh.q() + kh * (kQBytes / 2) + half * 128 * 128 + koff);
-            const uint64_t bdesc = sw128_desc(sh.kst(s) + kh * (kStageBytes / 2) + koff);
-            umma_bf16(d, a, bdesc, idesc, ks > 0);
-          }
-        }
-        umma_commit(sh.empty(s));
-        umma_commit(sh.accf(b));
-      }
-      umma_commit(sh.done());  // every MMA issued above has finished reading smem
-      volatile int dummy = 0;
-      mbar_wait(sh.done(), 0, &dummy);
-    }
+    if (lane == 0)
+      issue_mmas<C>(
+          sh, tmem, idesc_bf16(128, C::kTileKeys), ntiles,
+          [&](int, uint32_t kh, uint32_t koff) { return sh.q() + kh * (C::kQBytes / 2) + koff; },
+          [&](int s, uint32_t kh, uint32_t koff) {
+            return sh.kst(s) + kh * (C::kStageBytes / 2) + koff;
+          });
   } else {
-    const int ew = warp - 2, q = warp & 3, half = ew >> 2;
-    const int row = half * 128 + q * 32 + lane;
-    const bool active = half < halves && row < R;
+    // group grp reads buffer grp (tiles of that parity); within a group, warp
+    // (q, colh) owns rows q*32.. of the half and keys colh*128.. of the tile
+    const int ew = warp - 2, grp = ew >> 3, q = warp & 3, colh = (ew & 7) >> 2;
+    const int rloc = q * 32 + lane;
+    const int row = half * 128 + rloc;
     const int lim = n - p.w + (row % p.w);
     const float sl2 = p.scale_log2;
     float m = -INFINITY, l = 0.f;
-    for (int t = 0; t < ntiles; ++t) {
+    for (int t = grp; t < ntiles; t += 2) {
       const int b = t & 1;
       if (!mbar_wait(sh.accf(b), (t >> 1) & 1, ab)) break;
       tc_fence_after();
-      const int j0 = j_begin + t * kTileKeys;
-      // every row sees every key of an interior tile: no mask needed
-      const bool interior = (j0 + kTileKeys <= j_end) && (j0 + kTileKeys - 1 <= n - p.w);
-      if (half < halves) {
+      const int j0 = j_begin + t * C::kTileKeys + colh * 128;
+      const bool interior = (j0 + 128 <= j_end) && (j0 + 127 <= n - p.w);
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + half * 128 + c * 32), v);
-          if (interior) {
-            float mx = v[0];
+      for (int c = 0; c < 2; ++c) {
+        float v[64];
+        tmem_ld64(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + colh * 128 + c * 64), v);
+        if (interior) {
+          float mx0 = v[0], mx1 = v[1];
 #pragma unroll
-            for (int i = 1; i < 32; ++i) mx = fmaxf(mx, v[i]);
-            const float nm = fmaxf(m, mx * sl2);  // sl2 > 0: the max commutes with scaling
-            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+          for (int i = 2; i < 64; i += 2) {
+            mx0 = fmaxf(mx0, v[i]);
+            mx1 = fmaxf(mx1, v[i + 1]);
+          }
+          const float nm = fmaxf(m, fmaxf(mx0, mx1) * sl2);  // sl2 > 0: max commutes with scaling
+          float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-              s0 += ex2(fmaf(v[i], sl2, -nm));
-              s1 += ex2(fmaf(v[i + 1], sl2, -nm));
-              s2 += ex2(fmaf(v[i + 2], sl2, -nm));
-              s3 += ex2(fmaf(v[i + 3], sl2, -nm));
-            }
-            l = fmaf(l, ex2(m - nm), (s0 + s1) + (s2 + s3));
+          for (int i = 0; i < 64; ++i) acc[i & 7] += ex2(fmaf(v[i], sl2, -nm));
+          const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+          l = fmaf(l, ex2(m - nm), sum);
+          m = nm;
+        } else {
+          float cm = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < 64; ++i) {
+            const int j = j0 + c * 64 + i;
+            v[i] = (j <= lim && j < j_end) ? v[i] * sl2 : -INFINITY;
+            cm = fmaxf(cm, v[i]);
+          }
+          const float nm = fmaxf(m, cm);
+          if (nm > -INFINITY) {
+            float sum = 0.f;
+#pragma unroll
+            for (int i = 0; i < 64; ++i) sum += ex2(v[i] - nm);
+            l = fmaf(l, ex2(m - nm), sum);
             m = nm;
-          } else {
-            float cm = -INFINITY;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int j = j0 + c * 32 + i;
-              v[i] = (j <= lim && j < j_end) ? v[i] * sl2 : -INFINITY;
-              cm = fmaxf(cm, v[i]);
-            }
-            const float nm = fmaxf(m, cm);
-            if (nm > -INFINITY) {
-              float sum = 0.f;
-#pragma unroll
-              for (int i = 0; i < 32; ++i) sum += ex2(v[i] - nm);
-              l = fmaf(l, ex2(m - nm), sum);
-              m = nm;
-            }
           }
         }
       }
@@ -339,93 +402,93 @@ __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_consta
       __syncwarp();
       if (lane == 0) mbar_arrive(sh.acce(b));
     }
-    if (active && !*ab) lse_part[((size_t)u * R + row) * p.key_splits + split] = make_float2(m, l);
+    // merge the four partial (max, sum) of each row: 2 groups x 2 key halves
+    const int slot = grp * 2 + colh;
+    sh.pm()[slot * 128 + rloc] = m;
+    sh.pl()[slot * 128 + rloc] = l;
+    epi_sync();
+    if (slot == 0 && !*ab) {
+      float M = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) M = fmaxf(M, sh.pm()[k * 128 + rloc]);
+      float L = 0.f;
+      if (M > -INFINITY) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) L += sh.pl()[k * 128 + rloc] * ex2(sh.pm()[k * 128 + rloc] - M);
+      }
+      lse_part[((size_t)u * R + row) * p.key_splits + split] = make_float2(M, L);
+    }
   }
-  teardown(sh, warp, tmem, status);
+  teardown<C>(sh, warp, tmem, status);
 }
 
-// grid = units * items_per_unit, block = kThreads.  Pass 2: per-key column sums.
+// Pass 2.  grid = units * key_splits.  D[128 keys x R rows]; epilogue thread
+// = one key, summing exp(l - LSE_row) over 128 rows of its TMEM lane.
 __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_constant__ CUtensorMap tmK,
                                                                 const __grid_constant__ CUtensorMap tmQ,
                                                                 Prob p, const float* __restrict__ lse2,
                                                                 float* __restrict__ s_part,
                                                                 uint32_t* status) {
+  using C = Pass2;
   extern __shared__ char smem_raw[];
-  const Shared sh = shared_layout(smem_raw);
+  const Shared<C> sh = shared_layout<C>(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int u = blockIdx.x / p.key_splits, split = blockIdx.x % p.key_splits;
   const int n = p.n, R = p.R;
   const int j_begin = split * kKeysPerItemTc;
   const int j_end = min(n, j_begin + kKeysPerItemTc);
-  const int ntiles = (j_end - j_begin + kTileKeys - 1) / kTileKeys;
+  const int ntiles = (j_end - j_begin + C::kTileKeys - 1) / C::kTileKeys;
   for (int r = threadIdx.x; r < R; r += blockDim.x) sh.lse()[r] = lse2[(size_t)u * R + r];
-  const uint32_t tmem = setup(sh, warp);
+  const uint32_t tmem = setup<C>(sh, warp);
   volatile int* ab = sh.abort_flag();
 
   if (warp == 0) {
-    if (lane == 0) produce(sh, &tmK, &tmQ, u * R, R, (long)u * n + j_begin, ntiles);
+    if (lane == 0) produce<C>(sh, &tmK, &tmQ, u * R, R, (long)u * n + j_begin, ntiles);
   } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(kTileKeys, R);
-      bool ok = mbar_wait(sh.qfull(), 0, ab);
-      tc_fence_after();
-      for (int t = 0; ok && t < ntiles; ++t) {
-        const int s = t % kStages, b = t & 1;
-        if (!mbar_wait(sh.full(s), (t / kStages) & 1, ab)) break;
-        if (t >= 2 && !mbar_wait(sh.acce(b), ((t >> 1) - 1) & 1, ab)) break;
-        tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(b * 256);
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint32_t kh = ks >> 2, koff = (ks & 3) * 32;
-          const uint64_t a = sw128_desc(sh.kst(s) + kh * (kStageBytes / 2) + koff);
-          const uint64_t bdesc = sw128_desc(sh.q() + kh * (kQBytes / 2) + koff);
-          umma_bf16(d, a, bdesc, idesc, ks > 0);
-        }
-        umma_commit(sh.empty(s));
-        umma_commit(sh.accf(b));
-      }
-      umma_commit(sh.done());  // every MMA issued above has finished reading smem
-      volatile int dummy = 0;
-      mbar_wait(sh.done(), 0, &dummy);
-    }
+    if (lane == 0)
+      issue_mmas<C>(
+          sh, tmem, idesc_bf16(C::kTileKeys, R), ntiles,
+          [&](int s, uint32_t kh, uint32_t koff) {
+            return sh.kst(s) + kh * (C::kStageBytes / 2) + koff;
+          },
+          [&](int, uint32_t kh, uint32_t koff) { return sh.q() + kh * (C::kQBytes / 2) + koff; });
   } else {
-    const int ew = warp - 2, q = warp & 3, ch = ew >> 2;  // ch: which 128 rows
+    const int ew = warp - 2, grp = ew >> 3, q = warp & 3, ch = (ew & 7) >> 2;  // ch: 128-row half
     const int key = q * 32 + lane;
     const bool rows_here = ch * 128 < R;
     const float sl2 = p.scale_log2;
     const int nw = n - p.w;
     // the two row halves write separate row blocks; the finalize kernel adds them
     float* out = s_part + ((size_t)u * p.row_blocks + ch) * n;
-    for (int t = 0; t < ntiles; ++t) {
+    for (int t = grp; t < ntiles; t += 2) {
       const int b = t & 1;
       if (!mbar_wait(sh.accf(b), (t >> 1) & 1, ab)) break;
       tc_fence_after();
-      const int j0 = j_begin + t * kTileKeys;
+      const int j0 = j_begin + t * C::kTileKeys;
       const int j = j0 + key;
-      const bool interior = (j0 + kTileKeys <= j_end) && (j0 + kTileKeys <= nw);
-      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+      const bool interior = (j0 + C::kTileKeys <= j_end) && (j0 + C::kTileKeys <= nw);
+      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
       if (rows_here) {
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + ch * 128 + c * 32), v);
-          const int r0 = ch * 128 + c * 32;
+        for (int c = 0; c < 2; ++c) {
+          float v[64];
+          tmem_ld64(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + ch * 128 + c * 64), v);
+          const int r0 = ch * 128 + c * 64;
           const float4* L4 = reinterpret_cast<const float4*>(sh.lse() + r0);
           if (interior) {
 #pragma unroll
-            for (int i = 0; i < 32; i += 4) {
+            for (int i = 0; i < 64; i += 4) {
               const float4 L = L4[i >> 2];
-              s0 += ex2(fmaf(v[i], sl2, -L.x));
-              s1 += ex2(fmaf(v[i + 1], sl2, -L.y));
-              s2 += ex2(fmaf(v[i + 2], sl2, -L.z));
-              s3 += ex2(fmaf(v[i + 3], sl2, -L.w));
+              acc[(i + 0) & 7] += ex2(fmaf(v[i], sl2, -L.x));
+              acc[(i + 1) & 7] += ex2(fmaf(v[i + 1], sl2, -L.y));
+              acc[(i + 2) & 7] += ex2(fmaf(v[i + 2], sl2, -L.z));
+              acc[(i + 3) & 7] += ex2(fmaf(v[i + 3], sl2, -L.w));
             }
           } else {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
+            for (int i = 0; i < 64; ++i) {
               const int r = r0 + i;
-              if (j < j_end && j <= nw + (r % p.w)) s0 += ex2(fmaf(v[i], sl2, -sh.lse()[r]));
+              if (j < j_end && j <= nw + (r % p.w)) acc[0] += ex2(fmaf(v[i], sl2, -sh.lse()[r]));
             }
           }
         }
@@ -433,10 +496,11 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sh.acce(b));
-      if (j < j_end) out[j] = (s0 + s1) + (s2 + s3);
+      if (j < j_end)
+        out[j] = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
     }
   }
-  teardown(sh, warp, tmem, status);
+  teardown<C>(sh, warp, tmem, status);
 }
 
 }  // namespace tc
@@ -477,21 +541,24 @@ bool score_tc_supported(const Prob& p) { return p.R == 128 || p.R == 256; }
 
 bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_part, float* lse2,
                      float* s_part, uint32_t* status, cudaStream_t st) {
-  CUtensorMap mk, mq;
-  if (!make_map(&mk, K, (uint64_t)p.units * p.n, tc::kTileKeys)) return false;
-  if (!make_map(&mq, Q, (uint64_t)p.units * p.R, (uint32_t)p.R)) return false;
+  CUtensorMap mk1, mq1, mk2, mq2;
+  const uint64_t krows = (uint64_t)p.units * p.n, qrows = (uint64_t)p.units * p.R;
+  if (!make_map(&mk1, K, krows, tc::Pass1::kTileKeys) || !make_map(&mq1, Q, qrows, 128) ||
+      !make_map(&mk2, K, krows, tc::Pass2::kTileKeys) || !make_map(&mq2, Q, qrows, (uint32_t)p.R))
+    return false;
   static bool attr = false;
   if (!attr) {
     cudaFuncSetAttribute(tc::lse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         tc::kSmemBytes);
+                         tc::Pass1::kSmemBytes);
     cudaFuncSetAttribute(tc::colsum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         tc::kSmemBytes);
+                         tc::Pass2::kSmemBytes);
     attr = true;
   }
-  const unsigned grid = (unsigned)(p.units * p.key_splits);
+  const unsigned items = (unsigned)(p.units * p.key_splits);
   {
     TraceScope ts_("score_pass1", st);
-    tc::lse_tc_kernel<<<grid, tc::kThreads, tc::kSmemBytes, st>>>(mk, mq, p, lse_part, status);
+    tc::lse_tc_kernel<<<items * (p.R / 128), tc::kThreads, tc::Pass1::kSmemBytes, st>>>(
+        mk1, mq1, p, lse_part, status);
   }
   const size_t rows = (size_t)p.units * p.R;
   {
@@ -500,8 +567,8 @@ bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_pa
   }
   {
     TraceScope ts_("score_pass2", st);
-    tc::colsum_tc_kernel<<<grid, tc::kThreads, tc::kSmemBytes, st>>>(mk, mq, p, lse2, s_part,
-                                                                     status);
+    tc::colsum_tc_kernel<<<items, tc::kThreads, tc::Pass2::kSmemBytes, st>>>(mk2, mq2, p, lse2,
+                                                                             s_part, status);
   }
   return true;
 }
