@@ -162,7 +162,9 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
 }
 
 // grid = units, block = 128 (one thread per dimension): exclusive suffix sums
-// over chunks, in double-float.
+// over chunks, in double-float, folded from the last chunk down.  The chunk
+// sums are loaded kPrefixBlock chunks at a time so that the loads overlap.
+constexpr int kPrefixBlock = 16;
 __global__ void __launch_bounds__(128) curve_prefix_kernel(Prob p, const float4* __restrict__ agg_mq,
                                                            const float* __restrict__ agg_v,
                                                            const float* __restrict__ agg_k,
@@ -172,24 +174,34 @@ __global__ void __launch_bounds__(128) curve_prefix_kernel(Prob p, const float4*
   const int u = blockIdx.x, i = threadIdx.x;
   const size_t c0 = (size_t)u * p.chunks;
   DF rv = df_make(0.f), rk = df_make(0.f), rm = df_make(0.f), rq = df_make(0.f);
-  float nv = agg_v[(c0 + p.chunks - 1) * kD + i];
-  float nk = need_k ? agg_k[(c0 + p.chunks - 1) * kD + i] : 0.f;
-  float4 nmq = agg_mq[c0 + p.chunks - 1];
-  for (int c = p.chunks - 1; c >= 0; --c) {
-    const float cv = nv, ck = nk;
-    const float4 cmq = nmq;
-    if (c > 0) {  // prefetch the next (lower) chunk
-      nv = agg_v[(c0 + c - 1) * kD + i];
-      if (need_k) nk = agg_k[(c0 + c - 1) * kD + i];
-      nmq = agg_mq[c0 + c - 1];
+  for (int top = p.chunks - 1; top >= 0; top -= kPrefixBlock) {
+    float cv[kPrefixBlock], ck[kPrefixBlock];
+    float4 cmq[kPrefixBlock];
+#pragma unroll
+    for (int e = 0; e < kPrefixBlock; ++e) {
+      const int c = top - e;
+      cv[e] = ck[e] = 0.f;
+      cmq[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (c >= 0) {
+        cv[e] = agg_v[(c0 + c) * kD + i];
+        if (need_k) ck[e] = agg_k[(c0 + c) * kD + i];
+        if (i == 0) cmq[e] = agg_mq[c0 + c];
+      }
     }
-    base_v[(c0 + c) * kD + i] = make_float2(rv.hi, rv.lo);
-    if (need_k) base_k[(c0 + c) * kD + i] = make_float2(rk.hi, rk.lo);
-    if (i == 0) base_mq[c0 + c] = make_float4(rm.hi, rm.lo, rq.hi, rq.lo);
-    rv = df_add_f(rv, cv);
-    if (need_k) rk = df_add_f(rk, ck);
-    rm = df_add(rm, DF{cmq.x, cmq.y});
-    rq = df_add(rq, DF{cmq.z, cmq.w});
+#pragma unroll
+    for (int e = 0; e < kPrefixBlock; ++e) {
+      const int c = top - e;
+      if (c < 0) break;
+      base_v[(c0 + c) * kD + i] = make_float2(rv.hi, rv.lo);
+      if (need_k) base_k[(c0 + c) * kD + i] = make_float2(rk.hi, rk.lo);
+      if (i == 0) base_mq[c0 + c] = make_float4(rm.hi, rm.lo, rq.hi, rq.lo);
+      rv = df_add_f(rv, cv[e]);
+      if (need_k) rk = df_add_f(rk, ck[e]);
+      if (i == 0) {
+        rm = df_add(rm, DF{cmq[e].x, cmq[e].y});
+        rq = df_add(rq, DF{cmq[e].z, cmq[e].w});
+      }
+    }
   }
 }
 
@@ -240,39 +252,71 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
   unsigned long long best = 0ull;
   bool bad = false;
   const int nb = (r1 - r0 + 31) / 32;
+  const uint2* Vrows = reinterpret_cast<const uint2*>(Vu);
+  // The per-rank scalars of batch bi + 1 and the V rows of the next group of
+  // 8 ranks are loaded while the current group is evaluated.
+  float at, at_n = 0.f;
+  int jt, jt_n = 0;
+  float2 yv, yv_n = make_float2(0.f, 0.f);
+  {
+    const int r = r0 + (nb - 1) * 32 + lane;
+    const bool ok = r < r1;
+    at = ok ? key_score(ku[r]) : 0.f;
+    jt = ok ? pu[r] : 0;
+    yv = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
+  }
+  uint2 cur[8];
+  if (!exact) {
+    const int cnt = min(32, r1 - (r0 + (nb - 1) * 32));
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      const int js = __shfl_sync(kFull, jt, 24 + t);
+      cur[t] = (24 + t < cnt) ? __ldg(Vrows + (size_t)js * (kD / 4) + lane) : make_uint2(0u, 0u);
+    }
+  }
   for (int bi = nb - 1; bi >= 0; --bi) {
     const int rb = r0 + bi * 32;
     const int r = rb + lane;
     const bool ok = r < r1;
-    const float at = ok ? key_score(ku[r]) : 0.f;
-    const int jt = ok ? pu[r] : 0;
-    const float2 yv = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
+    if (bi > 0) {  // batch bi - 1 is a full batch
+      const int rn = rb - 32 + lane;
+      at_n = key_score(ku[rn]);
+      jt_n = pu[rn];
+      yv_n = yrank[(size_t)u * n + rn];
+    }
     const int cnt = min(32, r1 - rb);
     DF xt;
     if (!exact) {
       float xp[32];
 #pragma unroll
       for (int s0 = 24; s0 >= 0; s0 -= 8) {
-        uint2 vr[8];
-        float as[8];
+        uint2 nxt[8];
 #pragma unroll
-        for (int t = 7; t >= 0; --t) {  // loads first, highest rank of the group first
-          as[t] = __shfl_sync(kFull, at, s0 + t);
-          const int js = __shfl_sync(kFull, jt, s0 + t);
-          vr[t] = make_uint2(0u, 0u);
-          if (s0 + t < cnt) vr[t] = __ldg(reinterpret_cast<const uint2*>(Vu + (size_t)js * kD) + lane);
+        for (int t = 0; t < 8; ++t) {
+          nxt[t] = make_uint2(0u, 0u);
+          if (s0 > 0) {
+            const int js = __shfl_sync(kFull, jt, s0 - 8 + t);
+            if (s0 - 8 + t < cnt) nxt[t] = __ldg(Vrows + (size_t)js * (kD / 4) + lane);
+          } else {
+            const int js = __shfl_sync(kFull, jt_n, 24 + t);
+            if (bi > 0) nxt[t] = __ldg(Vrows + (size_t)js * (kD / 4) + lane);
+          }
         }
 #pragma unroll
         for (int t = 7; t >= 0; --t) {
-          const float v[4] = {bf16lo(vr[t].x), bf16hi(vr[t].x), bf16lo(vr[t].y), bf16hi(vr[t].y)};
+          const float as = __shfl_sync(kFull, at, s0 + t);
+          const float v[4] = {bf16lo(cur[t].x), bf16hi(cur[t].x), bf16lo(cur[t].y),
+                              bf16hi(cur[t].y)};
           float acc = 0.f;
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            P[i] = fmaf(as[t], v[i], P[i]);
+            P[i] = fmaf(as, v[i], P[i]);
             acc = fmaf(wb2x[i] + P[i], P[i], acc);
           }
           xp[s0 + t] = (s0 + t < cnt) ? acc : 0.f;
         }
+#pragma unroll
+        for (int t = 0; t < 8; ++t) cur[t] = nxt[t];
       }
       xt = df_make(reduce_scatter32(xp, lane));
     } else {
@@ -326,6 +370,9 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
     }
     carry_m = df_add(carry_m, shfl_df(sm, 0));
     carry_q = df_add(carry_q, shfl_df(sq, 0));
+    at = at_n;
+    jt = jt_n;
+    yv = yv_n;
   }
 #pragma unroll
   for (int o = 16; o >= 1; o >>= 1) {
