@@ -42,6 +42,7 @@
  *         q      bf16  [B][L][Hq][d]      one decode query per head
  *     Query head qh reads KV head qh / G.  Observation row t of a query head
  *     sits at absolute position n - w + t and sees keys j <= n - w + t.
+ *     Every tensor pointer must be 16-byte aligned (CERTKV_EINVAL otherwise).
  *   - A "unit" is one (sequence, layer, KV head): u = (b * L + l) * H + h.
  *   - Device-side problems (non-finite scores, an evicted suffix with zero
  *     mass) are recorded in a status word inside the workspace; read it with

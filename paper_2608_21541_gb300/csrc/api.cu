@@ -219,6 +219,7 @@ int certkv_score(const certkv_shape* shape, const void* K, const void* Q_obs,
   int rc = make_prob(shape, params, -1, &p);
   if (rc) return rc;
   if (!K || !Q_obs || !a_out) return CERTKV_EINVAL;
+  if (!aligned(K, 16) || !aligned(Q_obs, 16)) return CERTKV_EINVAL;
   Layout ly;
   if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -235,6 +236,7 @@ int certkv_curves(const certkv_shape* shape, const void* V, const float* a,
   int rc = make_prob(shape, params, -1, &p);
   if (rc) return rc;
   if (!V || !a || (!perm_out && !c_out)) return CERTKV_EINVAL;
+  if (!aligned(V, 16)) return CERTKV_EINVAL;
   Layout ly;
   if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -261,6 +263,7 @@ int certkv_compress_scored(const certkv_shape* shape, const void* K, const void*
   int rc = make_prob(shape, params, budget_live, &p);
   if (rc) return rc;
   if (!K || !V || !a) return CERTKV_EINVAL;
+  if (!aligned(K, 16) || !aligned(V, 16)) return CERTKV_EINVAL;
   if ((rc = check_packed(p, out))) return rc;
   Layout ly;
   if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
@@ -284,6 +287,7 @@ int certkv_compress(const certkv_shape* shape, const void* K, const void* V, con
   int rc = make_prob(shape, params, budget_live, &p);
   if (rc) return rc;
   if (!K || !V || !Q_obs) return CERTKV_EINVAL;
+  if (!aligned(K, 16) || !aligned(V, 16) || !aligned(Q_obs, 16)) return CERTKV_EINVAL;
   if ((rc = check_packed(p, out))) return rc;
   Layout ly;
   if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;

@@ -22,31 +22,9 @@ namespace certkv {
 
 namespace {
 
-__device__ __forceinline__ void load_row4(const __nv_bfloat16* row, int lane, float (&x)[4]) {
-  uint2 raw = __ldg(reinterpret_cast<const uint2*>(row) + lane);
-  x[0] = bf16lo(raw.x);
-  x[1] = bf16hi(raw.x);
-  x[2] = bf16lo(raw.y);
-  x[3] = bf16hi(raw.y);
-}
-
-// lane t ends with the double-float sum over lanes of v[t]  (62 shuffles)
-__device__ __forceinline__ DF reduce_scatter32_df(DF (&v)[32], int lane) {
-#pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) {
-    const bool upper = (lane & o) != 0;
-#pragma unroll
-    for (int i = 0; i < o; ++i) {
-      DF keep = upper ? v[i + o] : v[i];
-      DF send = upper ? v[i] : v[i + o];
-      v[i] = df_add(keep, shfl_xor_df(send, o));
-    }
-  }
-  return v[0];
-}
-
-// As reduce_scatter32_df, from fp32 inputs: the first butterfly level already
-// produces double-float sums (error-free), the later ones add double-floats.
+// lane t ends with the double-float sum over lanes of v[t], from fp32 inputs:
+// the first butterfly level already produces double-float sums (error-free),
+// the later ones add double-floats.
 __device__ __forceinline__ DF reduce_scatter32_f2df(float (&v)[32], int lane) {
   DF w[16];
   {
@@ -69,21 +47,6 @@ __device__ __forceinline__ DF reduce_scatter32_f2df(float (&v)[32], int lane) {
     }
   }
   return w[0];
-}
-
-// lane t ends with sum over lanes of v[t]  (31 shuffles)
-__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
-#pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) {
-    const bool upper = (lane & o) != 0;
-#pragma unroll
-    for (int i = 0; i < o; ++i) {
-      float keep = upper ? v[i + o] : v[i];
-      float send = upper ? v[i] : v[i + o];
-      v[i] = keep + __shfl_xor_sync(kFull, send, o);
-    }
-  }
-  return v[0];
 }
 
 }  // namespace
@@ -205,7 +168,56 @@ __global__ void __launch_bounds__(128) curve_prefix_kernel(Prob p, const float4*
   }
 }
 
-// grid = (ceil(chunks / 4), units), block = 128 (one warp per chunk)
+// Eight per-lane partials of rows 0..7 -> every lane l holds the lane sum of
+// row (l & 7).
+__device__ __forceinline__ float reduce8(float (&v)[8], int lane) {
+#pragma unroll
+  for (int o = 4; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const float keep = upper ? v[i + o] : v[i];
+      const float send = upper ? v[i] : v[i + o];
+      v[i] = keep + __shfl_xor_sync(kFull, send, o);
+    }
+  }
+  float x = v[0];
+  x += __shfl_xor_sync(kFull, x, 8);
+  x += __shfl_xor_sync(kFull, x, 16);
+  return x;
+}
+__device__ __forceinline__ DF reduce8_df(DF (&v)[8], int lane) {
+#pragma unroll
+  for (int o = 4; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const DF keep = upper ? v[i + o] : v[i];
+      const DF send = upper ? v[i] : v[i + o];
+      v[i] = df_add(keep, shfl_xor_df(send, o));
+    }
+  }
+  DF x = v[0];
+  x = df_add(x, shfl_xor_df(x, 8));
+  x = df_add(x, shfl_xor_df(x, 16));
+  return x;
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+constexpr int kEvalGroup = 8;                  // V rows per staged group
+constexpr int kEvalAhead = 3;                  // groups in flight ahead of the one in use
+constexpr int kEvalRing = kEvalAhead + 1;
+constexpr int kEvalGroupBytes = kEvalGroup * kD * 2;
+
+// grid = (ceil(chunks / 4), units), block = 128 (one warp per chunk).  The V
+// rows of a chunk are staged in groups of 8 ranks (descending) through a
+// per-warp ring in shared memory, kEvalAhead groups ahead of the evaluation.
 __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t* __restrict__ keys,
                                                          const int32_t* __restrict__ perm,
                                                          const __nv_bfloat16* __restrict__ V,
@@ -215,6 +227,10 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
                                                          float2* __restrict__ curve,
                                                          unsigned long long* __restrict__ cmax,
                                                          uint32_t* status) {
+  __shared__ __align__(16) unsigned char s_ring[4][kEvalRing][kEvalGroupBytes];
+  __shared__ float s_a[4][kChunk];
+  __shared__ int s_j[4][kChunk];
+  __shared__ float2 s_y[4][kChunk];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int chunk = blockIdx.x * 4 + warp;
   const int u = blockIdx.y;
@@ -223,8 +239,42 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
   const int r0 = chunk * kChunk, r1 = min(n, r0 + kChunk);
   const uint32_t* ku = keys + (size_t)u * n;
   const int32_t* pu = perm + (size_t)u * n;
-  const __nv_bfloat16* Vu = V + (size_t)u * n * kD;
+  const unsigned char* Vu = reinterpret_cast<const unsigned char*>(V + (size_t)u * n * kD);
   const size_t ci = (size_t)u * p.chunks + chunk;
+  float* sa = s_a[warp];
+  int* sj = s_j[warp];
+  float2* sy = s_y[warp];
+  const uint32_t ring = (uint32_t)__cvta_generic_to_shared(s_ring[warp][0]);
+
+  // per-rank scalars of the whole chunk (zero past the end)
+#pragma unroll
+  for (int e = 0; e < kChunk / 32; ++e) {
+    const int r = r0 + e * 32 + lane;
+    const bool ok = r < r1;
+    sa[e * 32 + lane] = ok ? key_score(ku[r]) : 0.f;
+    sj[e * 32 + lane] = ok ? pu[r] : 0;
+    sy[e * 32 + lane] = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
+  }
+  __syncwarp();
+  const int nb = (r1 - r0 + 31) / 32;
+  const int ngroups = nb * 4;  // group g: ranks r0 + 32*(nb-1-g/4) + 24 - 8*(g%4) + 0..7
+  // lane l copies 16-byte piece (l & 15) of rows (l >> 4) + 2k, k = 0..3
+  auto stage = [&](int g) {
+    if (g < ngroups) {
+      const int rl = 32 * (nb - 1 - g / 4) + 24 - 8 * (g % 4);  // first rank of the group, chunk-local
+      const uint32_t dst = ring + (uint32_t)((g % kEvalRing) * kEvalGroupBytes);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int t = (lane >> 4) + 2 * k;
+        if (r0 + rl + t < r1)
+          cp_async16(dst + t * (kD * 2) + (lane & 15) * 16,
+                     Vu + (size_t)sj[rl + t] * (kD * 2) + (lane & 15) * 16);
+      }
+    }
+    cp_async_commit();
+  };
+#pragma unroll
+  for (int g = 0; g < kEvalAhead; ++g) stage(g);
 
   const float4 bmq = base_mq[ci];
   const DF M0{bmq.x, bmq.y}, Q0{bmq.z, bmq.w};
@@ -251,94 +301,68 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
   DF carry_m = df_make(0.f), carry_q = df_make(0.f);
   unsigned long long best = 0ull;
   bool bad = false;
-  const int nb = (r1 - r0 + 31) / 32;
-  const uint2* Vrows = reinterpret_cast<const uint2*>(Vu);
-  // The per-rank scalars of batch bi + 1 and the V rows of the next group of
-  // 8 ranks are loaded while the current group is evaluated.
-  float at, at_n = 0.f;
-  int jt, jt_n = 0;
-  float2 yv, yv_n = make_float2(0.f, 0.f);
-  {
-    const int r = r0 + (nb - 1) * 32 + lane;
-    const bool ok = r < r1;
-    at = ok ? key_score(ku[r]) : 0.f;
-    jt = ok ? pu[r] : 0;
-    yv = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
-  }
-  uint2 cur[8];
-  if (!exact) {
-    const int cnt = min(32, r1 - (r0 + (nb - 1) * 32));
-#pragma unroll
-    for (int t = 0; t < 8; ++t) {
-      const int js = __shfl_sync(kFull, jt, 24 + t);
-      cur[t] = (24 + t < cnt) ? __ldg(Vrows + (size_t)js * (kD / 4) + lane) : make_uint2(0u, 0u);
-    }
-  }
-  for (int bi = nb - 1; bi >= 0; --bi) {
-    const int rb = r0 + bi * 32;
-    const int r = rb + lane;
-    const bool ok = r < r1;
-    if (bi > 0) {  // batch bi - 1 is a full batch
-      const int rn = rb - 32 + lane;
-      at_n = key_score(ku[rn]);
-      jt_n = pu[rn];
-      yv_n = yrank[(size_t)u * n + rn];
-    }
-    const int cnt = min(32, r1 - rb);
-    DF xt;
+  DF xt = df_make(0.f);  // lane r: ||W_base + P(b)||^2 - ||W_base||^2 for rank r of the batch
+  for (int g = 0; g < ngroups; ++g) {
+    stage(g + kEvalAhead);
+    asm volatile("cp.async.wait_group %0;" ::"n"(kEvalAhead) : "memory");
+    __syncwarp();
+    const int bi = nb - 1 - g / 4;
+    const int s0 = 24 - 8 * (g % 4);
+    const int rl = 32 * bi + s0;
+    const int cnt = r1 - (r0 + rl);  // rows of the group that exist (may exceed 8)
+    const unsigned char* rows = s_ring[warp][g % kEvalRing];
     if (!exact) {
-      float xp[32];
+      float xg[8];
 #pragma unroll
-      for (int s0 = 24; s0 >= 0; s0 -= 8) {
-        uint2 nxt[8];
-#pragma unroll
-        for (int t = 0; t < 8; ++t) {
-          nxt[t] = make_uint2(0u, 0u);
-          if (s0 > 0) {
-            const int js = __shfl_sync(kFull, jt, s0 - 8 + t);
-            if (s0 - 8 + t < cnt) nxt[t] = __ldg(Vrows + (size_t)js * (kD / 4) + lane);
-          } else {
-            const int js = __shfl_sync(kFull, jt_n, 24 + t);
-            if (bi > 0) nxt[t] = __ldg(Vrows + (size_t)js * (kD / 4) + lane);
-          }
+      for (int t = 7; t >= 0; --t) {
+        const float as = sa[rl + t];
+        float v[4] = {0.f, 0.f, 0.f, 0.f};
+        if (t < cnt) {
+          const uint2 raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
+          v[0] = bf16lo(raw.x);
+          v[1] = bf16hi(raw.x);
+          v[2] = bf16lo(raw.y);
+          v[3] = bf16hi(raw.y);
         }
+        float acc = 0.f;
 #pragma unroll
-        for (int t = 7; t >= 0; --t) {
-          const float as = __shfl_sync(kFull, at, s0 + t);
-          const float v[4] = {bf16lo(cur[t].x), bf16hi(cur[t].x), bf16lo(cur[t].y),
-                              bf16hi(cur[t].y)};
-          float acc = 0.f;
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            P[i] = fmaf(as, v[i], P[i]);
-            acc = fmaf(wb2x[i] + P[i], P[i], acc);
-          }
-          xp[s0 + t] = (s0 + t < cnt) ? acc : 0.f;
+        for (int i = 0; i < 4; ++i) {
+          P[i] = fmaf(as, v[i], P[i]);
+          acc = fmaf(wb2x[i] + P[i], P[i], acc);
         }
-#pragma unroll
-        for (int t = 0; t < 8; ++t) cur[t] = nxt[t];
+        xg[t] = (t < cnt) ? acc : 0.f;
       }
-      xt = df_make(reduce_scatter32(xp, lane));
+      const float x = reduce8(xg, lane);
+      if ((lane >> 3) == (s0 >> 3)) xt = df_make(x);
     } else {
-      DF xp[32];
-      for (int s = 31; s >= 0; --s) {
-        const float as = __shfl_sync(kFull, at, s);
-        const int js = __shfl_sync(kFull, jt, s);
-        xp[s] = df_make(0.f);
-        if (s < cnt) {
-          float v[4];
-          load_row4(Vu + (size_t)js * kD, lane, v);
+      DF xg[8];
+#pragma unroll
+      for (int t = 7; t >= 0; --t) {
+        const float as = sa[rl + t];
+        xg[t] = df_make(0.f);
+        if (t < cnt) {
+          const uint2 raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
+          const float v[4] = {bf16lo(raw.x), bf16hi(raw.x), bf16lo(raw.y), bf16hi(raw.y)};
           DF acc = df_make(0.f);
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
             Pd[i] = df_add(Pd[i], two_prod(as, v[i]));
             acc = df_add(acc, df_mul(Pd[i], Pd[i]));
           }
-          xp[s] = acc;
+          xg[t] = acc;
         }
       }
-      xt = reduce_scatter32_df(xp, lane);
+      const DF x = reduce8_df(xg, lane);
+      if ((lane >> 3) == (s0 >> 3)) xt = x;
     }
+    __syncwarp();  // the ring slot of group g is free once every lane has read it
+    if (s0 != 0) continue;
+
+    // ---- end of batch bi: the curve at its 32 ranks ----
+    const int r = r0 + 32 * bi + lane;
+    const bool ok = r < r1;
+    const float at = sa[32 * bi + lane];
+    const float2 yv = sy[32 * bi + lane];
     // in-batch inclusive suffix sums over lanes >= t
     DF sm = df_make(at);
     DF sq = ok ? df_mul_f(DF{yv.x, yv.y}, at) : df_make(0.f);
@@ -370,10 +394,8 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
     }
     carry_m = df_add(carry_m, shfl_df(sm, 0));
     carry_q = df_add(carry_q, shfl_df(sq, 0));
-    at = at_n;
-    jt = jt_n;
-    yv = yv_n;
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
 #pragma unroll
   for (int o = 16; o >= 1; o >>= 1) {
     unsigned long long other = __shfl_xor_sync(kFull, best, o);

@@ -67,13 +67,15 @@ def test_workspace_size_grows_with_the_problem(lib):
     assert ck.certkv_decode_workspace_bytes(shape()) > 0
 
 
-def _call_compress(lib, shp, budget, params=None, ws_bytes=None, ws_ptr=256, cap=None):
+def _call_compress(lib, shp, budget, params=None, ws_bytes=None, ws_ptr=256, cap=None,
+                   k_ptr=1 << 20):
     params = params or ck.certkv_default_params()
     fake = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
     need = lib.certkv_workspace_bytes(ctypes.byref(shp), ctypes.byref(params))
     packed = ck.certkv_packed(fake, fake, fake, fake, fake,
                               cap if cap is not None else 1 << 40, None, None)
-    return lib.certkv_compress(ctypes.byref(shp), fake, fake, fake, budget, ctypes.byref(params),
+    return lib.certkv_compress(ctypes.byref(shp), ctypes.c_void_p(k_ptr), fake, fake, budget,
+                               ctypes.byref(params),
                                ctypes.byref(packed),
                                ctypes.c_void_p(ws_ptr) if ws_ptr else None,
                                need if ws_bytes is None else ws_bytes, None)
@@ -89,6 +91,7 @@ def test_host_validation_errors(lib):
     assert _call_compress(lib, s, 2 * H, ws_ptr=0) == ck.EWORKSPACE
     assert _call_compress(lib, s, 2 * H, ws_ptr=257) == ck.EWORKSPACE  # misaligned
     assert _call_compress(lib, s, 2 * H, ws_bytes=1024) == ck.EWORKSPACE
+    assert _call_compress(lib, s, 2 * H, k_ptr=(1 << 20) + 8) == ck.EINVAL  # K not 16-B aligned
     assert _call_compress(lib, s, 40 * H, cap=10) == ck.ECAPACITY
     bad = ck.certkv_default_params(pool_kernel=4)
     assert _call_compress(lib, s, 2 * H, params=bad) == ck.EINVAL
