@@ -22,36 +22,94 @@ namespace certkv {
 
 namespace {
 
-// lane t ends with the double-float sum over lanes of v[t], from fp32 inputs:
-// the first butterfly level already produces double-float sums (error-free),
-// the later ones add double-floats.
-__device__ __forceinline__ DF reduce_scatter32_f2df(float (&v)[32], int lane) {
-  DF w[16];
-  {
-    const bool upper = (lane & 16) != 0;
+// Eight per-lane partials of rows 0..7 -> every lane l holds the lane sum of
+// row (l & 7).
+__device__ __forceinline__ float reduce8(float (&v)[8], int lane) {
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const float keep = upper ? v[i + 16] : v[i];
-      const float send = upper ? v[i] : v[i + 16];
-      w[i] = two_sum(keep, __shfl_xor_sync(kFull, send, 16));
-    }
-  }
-#pragma unroll
-  for (int o = 8; o >= 1; o >>= 1) {
+  for (int o = 4; o >= 1; o >>= 1) {
     const bool upper = (lane & o) != 0;
 #pragma unroll
     for (int i = 0; i < o; ++i) {
-      DF keep = upper ? w[i + o] : w[i];
-      DF send = upper ? w[i] : w[i + o];
+      const float keep = upper ? v[i + o] : v[i];
+      const float send = upper ? v[i] : v[i + o];
+      v[i] = keep + __shfl_xor_sync(kFull, send, o);
+    }
+  }
+  float x = v[0];
+  x += __shfl_xor_sync(kFull, x, 8);
+  x += __shfl_xor_sync(kFull, x, 16);
+  return x;
+}
+__device__ __forceinline__ DF reduce8_df(DF (&v)[8], int lane) {
+#pragma unroll
+  for (int o = 4; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const DF keep = upper ? v[i + o] : v[i];
+      const DF send = upper ? v[i] : v[i + o];
+      v[i] = df_add(keep, shfl_xor_df(send, o));
+    }
+  }
+  DF x = v[0];
+  x = df_add(x, shfl_xor_df(x, 8));
+  x = df_add(x, shfl_xor_df(x, 16));
+  return x;
+}
+
+// As reduce8, from fp32 inputs, in double-float (the first level is an
+// error-free two_sum).
+__device__ __forceinline__ DF reduce8_f2df(float (&v)[8], int lane) {
+  DF w[4];
+  {
+    const bool upper = (lane & 4) != 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float keep = upper ? v[i + 4] : v[i];
+      const float send = upper ? v[i] : v[i + 4];
+      w[i] = two_sum(keep, __shfl_xor_sync(kFull, send, 4));
+    }
+  }
+#pragma unroll
+  for (int o = 2; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const DF keep = upper ? w[i + o] : w[i];
+      const DF send = upper ? w[i] : w[i + o];
       w[i] = df_add(keep, shfl_xor_df(send, o));
     }
   }
-  return w[0];
+  DF x = w[0];
+  x = df_add(x, shfl_xor_df(x, 8));
+  x = df_add(x, shfl_xor_df(x, 16));
+  return x;
 }
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+constexpr int kEvalGroup = 8;                  // V rows per staged group
+constexpr int kEvalAhead = 3;                  // groups in flight ahead of the one in use
+constexpr int kEvalRing = kEvalAhead + 1;
+constexpr int kEvalGroupBytes = kEvalGroup * kD * 2;
 
 }  // namespace
 
-// grid = (ceil(chunks / 4), units), block = 128 (one warp per chunk)
+constexpr int kAggAhead = 2;                   // groups in flight ahead of the one in use
+constexpr int kAggRing = kAggAhead + 1;
+constexpr int kAggRingBytes = 4 * kAggRing * 2 * kEvalGroupBytes;  // [warp][slot][V, K]
+constexpr int kAggSmemBytes = kAggRingBytes + 4 * kChunk * 8;      // + a and token per rank
+
+// grid = (ceil(chunks / 4), units), block = 128 (one warp per chunk), dynamic
+// shared memory kAggSmemBytes.  The V (and K) rows of a chunk are staged in
+// groups of 8 ranks (ascending) through a per-warp ring, kAggAhead groups
+// ahead of their use.  Chunk sums of a and a||v||^2 are carried per lane in
+// double-float and summed over the warp once at the end.
 __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* __restrict__ keys,
                                                         const int32_t* __restrict__ perm,
                                                         const __nv_bfloat16* __restrict__ K,
@@ -60,6 +118,7 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
                                                         float* __restrict__ agg_v,
                                                         float* __restrict__ agg_k,
                                                         float2* __restrict__ yrank) {
+  extern __shared__ __align__(16) unsigned char agg_smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int chunk = blockIdx.x * 4 + warp;
   const int u = blockIdx.y;
@@ -68,55 +127,98 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
   const int r0 = chunk * kChunk, r1 = min(n, r0 + kChunk);
   const uint32_t* ku = keys + (size_t)u * n;
   const int32_t* pu = perm + (size_t)u * n;
-  const __nv_bfloat16* Vu = V + (size_t)u * n * kD;
-  const __nv_bfloat16* Ku = K + (size_t)u * n * kD;
+  const unsigned char* Vu = reinterpret_cast<const unsigned char*>(V + (size_t)u * n * kD);
+  const unsigned char* Ku = reinterpret_cast<const unsigned char*>(K + (size_t)u * n * kD);
+  unsigned char* ring_w = agg_smem + warp * (kAggRing * 2 * kEvalGroupBytes);
+  const uint32_t ring = (uint32_t)__cvta_generic_to_shared(ring_w);
+  float* sa = reinterpret_cast<float*>(agg_smem + kAggRingBytes) + warp * kChunk;
+  int* sj = reinterpret_cast<int*>(agg_smem + kAggRingBytes + 4 * kChunk * 4) + warp * kChunk;
 
-  float sv[4] = {0.f, 0.f, 0.f, 0.f}, sk[4] = {0.f, 0.f, 0.f, 0.f};
-  DF m = df_make(0.f), q = df_make(0.f);
-  for (int rb = r0; rb < r1; rb += 32) {
-    const int r = rb + lane;
+#pragma unroll
+  for (int e = 0; e < kChunk / 32; ++e) {
+    const int r = r0 + e * 32 + lane;
     const bool ok = r < r1;
-    const float at = ok ? key_score(ku[r]) : 0.f;
-    const int jt = ok ? pu[r] : 0;
-    const int cnt = min(32, r1 - rb);
-    // ||v||^2: per lane the 4 squares of bf16 values (each exact in fp32) are
-    // summed in fp32, the 32 lane partials in double-float.
-    float yp[32];
+    sa[e * 32 + lane] = ok ? key_score(ku[r]) : 0.f;
+    sj[e * 32 + lane] = ok ? pu[r] : 0;
+  }
+  __syncwarp();
+  const int ngroups = (r1 - r0 + kEvalGroup - 1) / kEvalGroup;  // group g: chunk ranks 8g .. 8g+7
+  // lane l copies 16-byte piece (l & 15) of rows (l >> 4) + 2k, k = 0..3
+  auto stage = [&](int g) {
+    if (g < ngroups) {
+      const uint32_t dst = ring + (uint32_t)((g % kAggRing) * 2 * kEvalGroupBytes);
 #pragma unroll
-    for (int s0 = 0; s0 < 32; s0 += 8) {
-      // issue the 8 rows' loads first so that they are in flight together
-      uint2 vr[8], kr[8];
-      float as[8];
-#pragma unroll
-      for (int t = 0; t < 8; ++t) {
-        as[t] = __shfl_sync(kFull, at, s0 + t);
-        const int js = __shfl_sync(kFull, jt, s0 + t);
-        vr[t] = make_uint2(0u, 0u);
-        kr[t] = make_uint2(0u, 0u);
-        if (s0 + t < cnt) {
-          vr[t] = __ldg(reinterpret_cast<const uint2*>(Vu + (size_t)js * kD) + lane);
-          if (need_k) kr[t] = __ldg(reinterpret_cast<const uint2*>(Ku + (size_t)js * kD) + lane);
+      for (int k = 0; k < 4; ++k) {
+        const int t = (lane >> 4) + 2 * k;
+        const int rl = kEvalGroup * g + t;
+        if (r0 + rl < r1) {
+          const size_t src = (size_t)sj[rl] * (kD * 2) + (lane & 15) * 16;
+          const uint32_t off = t * (kD * 2) + (lane & 15) * 16;
+          cp_async16(dst + off, Vu + src);
+          if (need_k) cp_async16(dst + kEvalGroupBytes + off, Ku + src);
         }
-      }
-#pragma unroll
-      for (int t = 0; t < 8; ++t) {
-        const float v[4] = {bf16lo(vr[t].x), bf16hi(vr[t].x), bf16lo(vr[t].y), bf16hi(vr[t].y)};
-        const float k4[4] = {bf16lo(kr[t].x), bf16hi(kr[t].x), bf16lo(kr[t].y), bf16hi(kr[t].y)};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          sv[i] = fmaf(as[t], v[i], sv[i]);
-          sk[i] = fmaf(as[t], k4[i], sk[i]);
-        }
-        yp[s0 + t] = fmaf(v[3], v[3], fmaf(v[2], v[2], fmaf(v[1], v[1], v[0] * v[0])));
       }
     }
-    const DF yt = reduce_scatter32_f2df(yp, lane);
-    if (ok) yrank[(size_t)u * n + r] = make_float2(yt.hi, yt.lo);
-    DF dm = df_make(at);
-    DF dq = ok ? df_mul_f(yt, at) : df_make(0.f);
-    m = df_add(m, warp_sum_df(dm));
-    q = df_add(q, warp_sum_df(dq));
+    cp_async_commit();
+  };
+#pragma unroll
+  for (int g = 0; g < kAggAhead; ++g) stage(g);
+
+  float sv[4] = {0.f, 0.f, 0.f, 0.f}, sk[4] = {0.f, 0.f, 0.f, 0.f};
+  DF ml = df_make(0.f), ql = df_make(0.f);
+  DF ylane = df_make(0.f);  // lane r: ||v||^2 of rank r of the current batch
+  for (int g = 0; g < ngroups; ++g) {
+    stage(g + kAggAhead);
+    asm volatile("cp.async.wait_group %0;" ::"n"(kAggAhead) : "memory");
+    __syncwarp();
+    const unsigned char* rows = ring_w + (g % kAggRing) * 2 * kEvalGroupBytes;
+    const int rl0 = kEvalGroup * g;
+    const int cnt = r1 - (r0 + rl0);
+    // ||v||^2: per lane the 4 squares of bf16 values (each exact in fp32) are
+    // summed in fp32, the 32 lane partials in double-float.
+    float yp[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      const float as = sa[rl0 + t];
+      float v[4] = {0.f, 0.f, 0.f, 0.f}, k4[4] = {0.f, 0.f, 0.f, 0.f};
+      if (t < cnt) {
+        const uint2 rv = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
+        v[0] = bf16lo(rv.x);
+        v[1] = bf16hi(rv.x);
+        v[2] = bf16lo(rv.y);
+        v[3] = bf16hi(rv.y);
+        if (need_k) {
+          const uint2 rk =
+              *reinterpret_cast<const uint2*>(rows + kEvalGroupBytes + t * (kD * 2) + lane * 8);
+          k4[0] = bf16lo(rk.x);
+          k4[1] = bf16hi(rk.x);
+          k4[2] = bf16lo(rk.y);
+          k4[3] = bf16hi(rk.y);
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        sv[i] = fmaf(as, v[i], sv[i]);
+        sk[i] = fmaf(as, k4[i], sk[i]);
+      }
+      yp[t] = fmaf(v[3], v[3], fmaf(v[2], v[2], fmaf(v[1], v[1], v[0] * v[0])));
+    }
+    const DF y = reduce8_f2df(yp, lane);
+    if ((lane >> 3) == (g & 3)) ylane = y;
+    __syncwarp();  // the ring slot of group g is free once every lane has read it
+    if ((g & 3) == 3 || g == ngroups - 1) {  // end of batch g / 4
+      const int rl = 32 * (g >> 2) + lane;
+      const bool ok = r0 + rl < r1;
+      const float at = sa[rl];
+      if (ok) {
+        yrank[(size_t)u * n + r0 + rl] = make_float2(ylane.hi, ylane.lo);
+        ml = df_add_f(ml, at);
+        ql = df_add(ql, df_mul_f(ylane, at));
+      }
+    }
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  const DF m = warp_sum_df(ml), q = warp_sum_df(ql);
   const size_t ci = (size_t)u * p.chunks + chunk;
   reinterpret_cast<float4*>(agg_v + ci * kD)[lane] = make_float4(sv[0], sv[1], sv[2], sv[3]);
   if (need_k)
@@ -167,53 +269,6 @@ __global__ void __launch_bounds__(128) curve_prefix_kernel(Prob p, const float4*
     }
   }
 }
-
-// Eight per-lane partials of rows 0..7 -> every lane l holds the lane sum of
-// row (l & 7).
-__device__ __forceinline__ float reduce8(float (&v)[8], int lane) {
-#pragma unroll
-  for (int o = 4; o >= 1; o >>= 1) {
-    const bool upper = (lane & o) != 0;
-#pragma unroll
-    for (int i = 0; i < o; ++i) {
-      const float keep = upper ? v[i + o] : v[i];
-      const float send = upper ? v[i] : v[i + o];
-      v[i] = keep + __shfl_xor_sync(kFull, send, o);
-    }
-  }
-  float x = v[0];
-  x += __shfl_xor_sync(kFull, x, 8);
-  x += __shfl_xor_sync(kFull, x, 16);
-  return x;
-}
-__device__ __forceinline__ DF reduce8_df(DF (&v)[8], int lane) {
-#pragma unroll
-  for (int o = 4; o >= 1; o >>= 1) {
-    const bool upper = (lane & o) != 0;
-#pragma unroll
-    for (int i = 0; i < o; ++i) {
-      const DF keep = upper ? v[i + o] : v[i];
-      const DF send = upper ? v[i] : v[i + o];
-      v[i] = df_add(keep, shfl_xor_df(send, o));
-    }
-  }
-  DF x = v[0];
-  x = df_add(x, shfl_xor_df(x, 8));
-  x = df_add(x, shfl_xor_df(x, 16));
-  return x;
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-
-constexpr int kEvalGroup = 8;                  // V rows per staged group
-constexpr int kEvalAhead = 3;                  // groups in flight ahead of the one in use
-constexpr int kEvalRing = kEvalAhead + 1;
-constexpr int kEvalGroupBytes = kEvalGroup * kD * 2;
 
 // grid = (ceil(chunks / 4), units), block = 128 (one warp per chunk).  The V
 // rows of a chunk are staged in groups of 8 ranks (descending) through a
@@ -444,9 +499,15 @@ void launch_curves(const Prob& p, const Layout& ly, char* ws, const void* K, con
     TraceScope ts_("cmax_clear", st);
     cmax_clear_kernel<<<(p.units + 255) / 256, 256, 0, st>>>(cmax, p.units);
   }
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(curve_agg_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         kAggSmemBytes);
+    attr = true;
+  }
   {
     TraceScope ts_("curve_agg", st);
-    curve_agg_kernel<<<grid, 128, 0, st>>>(p, keys, perm, Kb, Vb, need_k, agg_mq, agg_v, agg_k,
+    curve_agg_kernel<<<grid, 128, kAggSmemBytes, st>>>(p, keys, perm, Kb, Vb, need_k, agg_mq, agg_v, agg_k,
                                            yrank);
   }
   {
