@@ -12,7 +12,7 @@ constexpr int kD = 128;          // head dimension supported by the kernels
 constexpr int kChunk = 128;      // ranks per dispersion chunk (one warp)
 constexpr int kHullSeg = 256;    // curve points per hull-filter thread
 constexpr int kGroupSegs = 16;   // hull-filter segments per group
-constexpr int kSortTile = 4096;  // keys per radix-sort tile
+constexpr int kSortTile = 2048;  // keys per radix-sort tile
 constexpr int kSortThreads = 256;
 constexpr int kDecodeSplits = 16;
 constexpr uint32_t kFull = 0xffffffffu;

@@ -13,7 +13,20 @@ namespace certkv {
 
 namespace {
 constexpr int kWarps = kSortThreads / 32;
-constexpr int kPerLane = kSortTile / kSortThreads;  // 16 keys per lane, striped per warp
+constexpr int kPerLane = kSortTile / kSortThreads;  // 8 keys per lane, striped per warp
+
+// Lanes of the warp whose 8-bit digit equals this lane's, among the lanes with
+// `ok` set (0 for a lane without it): one ballot per digit bit.
+__device__ __forceinline__ uint32_t same_digit_lanes(uint32_t dgt, bool ok) {
+  uint32_t peers = __ballot_sync(kFull, ok);
+#pragma unroll
+  for (int b = 0; b < 8; ++b) {
+    const uint32_t bit = (dgt >> b) & 1u;
+    const uint32_t bal = __ballot_sync(kFull, bit != 0u);
+    peers &= bit ? bal : ~bal;
+  }
+  return ok ? peers : 0u;
+}
 }  // namespace
 
 // grid = (tiles, units): per-tile digit histogram, stored [u][digit][tile].
@@ -26,10 +39,15 @@ __global__ void __launch_bounds__(kSortThreads) radix_hist_kernel(const uint32_t
   __syncthreads();
   const uint32_t* ku = keys + (size_t)u * n;
   const int base = tile * kSortTile;
-  for (int i = threadIdx.x; i < kSortTile; i += kSortThreads) {
-    int j = base + i;
-    if (j < n) atomicAdd(&cnt[(ku[j] >> shift) & 255u], 1u);
+  uint32_t k[kPerLane];
+#pragma unroll
+  for (int e = 0; e < kPerLane; ++e) {  // all loads in flight before the counting
+    const int j = base + e * kSortThreads + threadIdx.x;
+    k[e] = j < n ? ku[j] : 0u;
   }
+#pragma unroll
+  for (int e = 0; e < kPerLane; ++e)
+    if (base + e * kSortThreads + (int)threadIdx.x < n) atomicAdd(&cnt[(k[e] >> shift) & 255u], 1u);
   __syncthreads();
   hist[((size_t)u * 256 + threadIdx.x) * tiles + tile] = cnt[threadIdx.x];
 }
@@ -72,12 +90,19 @@ __global__ void __launch_bounds__(1024) radix_scan_kernel(uint32_t* __restrict__
   }
 }
 
-// grid = (tiles, units): stable scatter of one tile.
+// grid = (tiles, units): stable scatter of one tile.  The tile is first
+// ordered by digit in shared memory (stable ranks from per-warp counts), then
+// written out so that consecutive threads store consecutive positions of a
+// digit's run.
 __global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
     const uint32_t* __restrict__ kin, const int32_t* __restrict__ vin, uint32_t* __restrict__ kout,
     int32_t* __restrict__ vout, int n, int tiles, int shift, const uint32_t* __restrict__ hist) {
   __shared__ uint32_t wcnt[kWarps][256];
   __shared__ uint32_t gbase[256];
+  __shared__ uint32_t tstart[256];
+  __shared__ uint32_t wsum[kWarps];
+  __shared__ uint32_t skey[kSortTile];
+  __shared__ int32_t sval[kSortTile];
   const int tile = blockIdx.x, u = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < kWarps * 256; i += kSortThreads) (&wcnt[0][0])[i] = 0;
@@ -97,18 +122,19 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
     val[i] = ok ? vu[j] : 0;
   }
   const uint32_t lt = (1u << lane) - 1u;
-  // 1. per-warp digit counts
+  // 1. per-warp digit counts; peers[i] = lanes holding the same digit
+  uint32_t peers[kPerLane];
 #pragma unroll
   for (int i = 0; i < kPerLane; ++i) {
-    int j = wbase + i * 32 + lane;
-    bool ok = j < n;
-    uint32_t dgt = ok ? ((key[i] >> shift) & 255u) : 256u + lane;  // unique dummy digit
-    uint32_t peers = __match_any_sync(kFull, dgt);
-    if (ok && (peers & lt) == 0u) wcnt[warp][dgt] += __popc(peers);
+    const int j = wbase + i * 32 + lane;
+    const bool ok = j < n;
+    const uint32_t dgt = (key[i] >> shift) & 255u;
+    peers[i] = same_digit_lanes(dgt, ok);
+    if (ok && (peers[i] & lt) == 0u) wcnt[warp][dgt] += __popc(peers[i]);
     __syncwarp();
   }
   __syncthreads();
-  // 2. exclusive scan across warps per digit
+  // 2. per digit: exclusive scan across warps, then over digits (tile start)
   {
     const int d = threadIdx.x;
     uint32_t run = 0;
@@ -118,27 +144,52 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
       wcnt[wi][d] = run;
       run += t;
     }
+    uint32_t x = run;  // inclusive scan over digits: warp level, then warp totals
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      uint32_t y = __shfl_up_sync(kFull, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) wsum[warp] = x;
+    __syncthreads();
+    uint32_t before = 0;
+#pragma unroll
+    for (int wi = 0; wi < kWarps; ++wi)
+      if (wi < warp) before += wsum[wi];
+    const uint32_t start = before + x - run;
+    tstart[d] = start;
+#pragma unroll
+    for (int wi = 0; wi < kWarps; ++wi) wcnt[wi][d] += start;
   }
   __syncthreads();
-  // 3. ranks and scatter, in element order
-  uint32_t* ko = kout + (size_t)u * n;
-  int32_t* vo = vout + (size_t)u * n;
+  // 3. stable tile-local ranks -> shared memory, in digit order
 #pragma unroll
   for (int i = 0; i < kPerLane; ++i) {
-    int j = wbase + i * 32 + lane;
-    bool ok = j < n;
-    uint32_t dgt = ok ? ((key[i] >> shift) & 255u) : 256u + lane;
-    uint32_t peers = __match_any_sync(kFull, dgt);
+    const int j = wbase + i * 32 + lane;
+    const bool ok = j < n;
+    const uint32_t dgt = (key[i] >> shift) & 255u;
     uint32_t before = 0;
     if (ok) before = wcnt[warp][dgt];
     __syncwarp();
     if (ok) {
-      uint32_t pos = gbase[dgt] + before + __popc(peers & lt);
-      ko[pos] = key[i];
-      vo[pos] = val[i];
-      if ((peers & lt) == 0u) wcnt[warp][dgt] = before + __popc(peers);
+      const uint32_t pos = before + __popc(peers[i] & lt);
+      skey[pos] = key[i];
+      sval[pos] = val[i];
+      if ((peers[i] & lt) == 0u) wcnt[warp][dgt] = before + __popc(peers[i]);
     }
     __syncwarp();
+  }
+  __syncthreads();
+  // 4. coalesced write-out of the digit runs
+  uint32_t* ko = kout + (size_t)u * n;
+  int32_t* vo = vout + (size_t)u * n;
+  const int count = min(kSortTile, n - tile * kSortTile);
+  for (int i = threadIdx.x; i < count; i += kSortThreads) {
+    const uint32_t k = skey[i];
+    const uint32_t d = (k >> shift) & 255u;
+    const uint32_t pos = gbase[d] + (uint32_t)i - tstart[d];
+    ko[pos] = k;
+    vo[pos] = sval[i];
   }
 }
 
