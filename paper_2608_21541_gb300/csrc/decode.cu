@@ -95,17 +95,24 @@ __global__ void __launch_bounds__(128) decode_split_kernel(Prob p, const __nv_bf
     }
     // values: lane = 4 dims
     const int cnt = min(32, slots - t * 32);
-    for (int j = 0; j < cnt; ++j) {
-      const uint2 raw =
-          __ldg(reinterpret_cast<const uint2*>(pv + (size_t)(off + t * 32 + j) * kD) + lane);
-      const float v0 = bf16lo(raw.x), v1 = bf16hi(raw.x), v2 = bf16lo(raw.y), v3 = bf16hi(raw.y);
+    const uint2* vrow = reinterpret_cast<const uint2*>(pv + (size_t)(off + t * 32) * kD) + lane;
+    for (int j0 = 0; j0 < cnt; j0 += 8) {  // 8 rows' loads in flight, then their FMAs
+      uint2 raw[8];
 #pragma unroll
-      for (int g = 0; g < G; ++g) {
-        const float pj = __shfl_sync(kFull, pr[g], j);
-        acc[g][0] = fmaf(pj, v0, acc[g][0]);
-        acc[g][1] = fmaf(pj, v1, acc[g][1]);
-        acc[g][2] = fmaf(pj, v2, acc[g][2]);
-        acc[g][3] = fmaf(pj, v3, acc[g][3]);
+      for (int e = 0; e < 8; ++e)
+        raw[e] = (j0 + e < cnt) ? __ldg(vrow + (size_t)(j0 + e) * (kD / 4)) : make_uint2(0u, 0u);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float v0 = bf16lo(raw[e].x), v1 = bf16hi(raw[e].x), v2 = bf16lo(raw[e].y),
+                    v3 = bf16hi(raw[e].y);
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          const float pj = __shfl_sync(kFull, pr[g], j0 + e);  // 0 past the last slot
+          acc[g][0] = fmaf(pj, v0, acc[g][0]);
+          acc[g][1] = fmaf(pj, v1, acc[g][1]);
+          acc[g][2] = fmaf(pj, v2, acc[g][2]);
+          acc[g][3] = fmaf(pj, v3, acc[g][3]);
+        }
       }
     }
   }

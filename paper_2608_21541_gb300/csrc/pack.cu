@@ -157,13 +157,31 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloa
   const uint4* Vu = reinterpret_cast<const uint4*>(V + (size_t)u * p.n * kD);
   uint4* PK = reinterpret_cast<uint4*>(pk);
   uint4* PV = reinterpret_cast<uint4*>(pv);
-  // 16 uint4 per row; 256 threads = 16 rows per step
+  // 16 uint4 per row; 256 threads = 16 rows per step, 4 steps' loads in flight
   const int sub = threadIdx.x & 15;
-  for (int row = blockIdx.y * 16 + (threadIdx.x >> 4); row < b; row += gridDim.y * 16) {
-    const int j = positions[off + row];
-    if (j < 0 || j >= p.n) continue;  // unreachable when the selection is consistent
-    PK[(size_t)(off + row) * 16 + sub] = __ldg(Ku + (size_t)j * 16 + sub);
-    PV[(size_t)(off + row) * 16 + sub] = __ldg(Vu + (size_t)j * 16 + sub);
+  const int stride = gridDim.y * 16;
+  for (int row0 = blockIdx.y * 16 + (threadIdx.x >> 4); row0 < b; row0 += 4 * stride) {
+    int j[4];
+    uint4 kx[4], vx[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int row = row0 + e * stride;
+      j[e] = row < b ? positions[off + row] : -1;
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const bool ok = j[e] >= 0 && j[e] < p.n;  // false only past b (the selection is consistent)
+      kx[e] = ok ? __ldg(Ku + (size_t)j[e] * 16 + sub) : make_uint4(0u, 0u, 0u, 0u);
+      vx[e] = ok ? __ldg(Vu + (size_t)j[e] * 16 + sub) : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int row = row0 + e * stride;
+      if (j[e] >= 0 && j[e] < p.n) {
+        PK[(size_t)(off + row) * 16 + sub] = kx[e];
+        PV[(size_t)(off + row) * 16 + sub] = vx[e];
+      }
+    }
   }
 }
 
