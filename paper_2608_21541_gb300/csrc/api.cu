@@ -98,6 +98,7 @@ Layout make_layout(const Prob& p) {
   ly.lse = take(U * p.R * sizeof(float));
   ly.s_part = take(U * p.row_blocks * n * sizeof(float));
   ly.s_tmp = take(U * n * sizeof(float));
+  ly.fin_part = take(U * ((n + kFinSpan - 1) / kFinSpan) * sizeof(float4));
   ly.a = take(U * n * sizeof(float));
   ly.keys0 = take(U * n * 4);
   ly.keys1 = take(U * n * 4);

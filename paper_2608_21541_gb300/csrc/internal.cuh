@@ -32,6 +32,7 @@ struct Prob {
 constexpr int kScoreKeysPerCta = 1024;   // keys per CTA of the mma.sync scorer
 constexpr int kKeysPerItemTc = 16384;    // keys per CTA of the tcgen05 scorer
 constexpr int kScoreTileKeys = 64;
+constexpr int kFinSpan = 8192;           // keys per CTA of the score finalize kernels
 
 // Workspace carve-up (byte offsets from the workspace base, 256-B aligned).
 struct Layout {
@@ -40,6 +41,7 @@ struct Layout {
   size_t lse;        // float  [U][R]   log2-domain LSE of each observation row
   size_t s_part;     // float  [U][row_blocks][n]
   size_t s_tmp;      // float  [U][n]   pooled scores
+  size_t fin_part;   // float4 [U][ceil(n / kFinSpan)]  per-slice (max, sum.hi, sum.lo, 0)
   size_t a;          // float  [U][n]   scores (when the caller gives none)
   size_t keys0, keys1, vals0, vals1;  // uint32/int32 [U][n]
   size_t hist;       // uint32 [U][256][sort_tiles]

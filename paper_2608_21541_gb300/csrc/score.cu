@@ -252,76 +252,105 @@ __global__ void lse_merge_kernel(Prob p, const float2* __restrict__ part, float*
   lse2[i] = M + log2f(L);
 }
 
-// Mean over rows, average pool (zero padding, / width, non-window keys only),
-// window protection, normalisation; writes a and the sort keys.  grid = units.
-__global__ void __launch_bounds__(1024) score_finalize_kernel(Prob p, const float* __restrict__ s_part,
-                                                              float* __restrict__ s_pool,
-                                                              float* __restrict__ a_out,
-                                                              uint32_t* __restrict__ keys,
-                                                              int32_t* __restrict__ vals,
-                                                              uint32_t* status) {
-  __shared__ float red_max[32];
-  __shared__ DF red_sum[32];
-  __shared__ float bcast[2];
-  const int u = blockIdx.x;
+// Finalize (a2), in two position-parallel kernels over slices of
+// kFinSpan keys.  pool: s_j = (1/R) sum of the row blocks, average-pooled
+// over non-window keys (zero padding, divided by the width; the slice loads a
+// halo of pool/2 keys on each side), written to s_pool; per slice the max of
+// the pooled scores and the double-float sum of the clipped ones.
+// scale: the unit's max and total from its slices (window keys count as the
+// max when protected), then a_j = (s_j)+ / total, the sort keys and indices.
+__global__ void __launch_bounds__(256) score_pool_kernel(Prob p, const float* __restrict__ s_part,
+                                                         float* __restrict__ s_pool,
+                                                         float4* __restrict__ fin_part,
+                                                         uint32_t* status) {
+  extern __shared__ float s_win[];  // s over [j0 - half, j1 + half)
+  __shared__ float red_max[8];
+  __shared__ DF red_sum[8];
+  const int slice = blockIdx.x, u = blockIdx.y;
   const int n = p.n, nw = n - p.w, half = p.pool / 2;
+  const int j0 = slice * kFinSpan, j1 = min(n, j0 + kFinSpan);
   const float invR = 1.0f / (float)p.R;
   const float invPool = 1.0f / (float)p.pool;
-  float* sp = s_pool + (size_t)u * n;
-  float* au = a_out + (size_t)u * n;
-
-  // 1. s_j = (1/R) sum over row blocks  (written into a_out as scratch)
-  for (int j = threadIdx.x; j < n; j += blockDim.x) {
+  const int lo = j0 - half, cnt = (j1 + half) - lo;
+  for (int t = threadIdx.x; t < cnt; t += blockDim.x) {
+    const int i = lo + t;
     float s = 0.f;
-    for (int rb = 0; rb < p.row_blocks; ++rb) s += s_part[((size_t)u * p.row_blocks + rb) * n + j];
-    au[j] = s * invR;
+    if (i >= 0 && i < n)
+      for (int rb = 0; rb < p.row_blocks; ++rb) s += s_part[((size_t)u * p.row_blocks + rb) * n + i];
+    s_win[t] = s * invR;
   }
   __syncthreads();
-  // 2. pooled scores for non-window keys, running max
+  float* sp = s_pool + (size_t)u * n;
   float mx = -INFINITY;
-  for (int j = threadIdx.x; j < nw; j += blockDim.x) {
-    float acc = 0.f;
-    for (int i = j - half; i <= j + half; ++i)
-      if (i >= 0 && i < nw) acc += au[i];
-    float v = acc * invPool;
-    if (p.pool == 1) v = au[j];
-    sp[j] = v;
-    mx = fmaxf(mx, v);
-  }
-  mx = warp_max(mx);
-  if ((threadIdx.x & 31) == 0) red_max[threadIdx.x >> 5] = mx;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    float v = threadIdx.x < (blockDim.x >> 5) ? red_max[threadIdx.x] : -INFINITY;
-    v = warp_max(v);
-    if (threadIdx.x == 0) bcast[0] = v;
-  }
-  __syncthreads();
-  const float smax = bcast[0];
-  // 3. window keys, clip, total (double-float)
   DF tot = df_make(0.f);
-  for (int j = threadIdx.x; j < n; j += blockDim.x) {
-    float v = (j < nw) ? sp[j] : (p.protect ? smax : au[j]);
-    if (!(fabsf(v) <= 3.0e38f)) raise_status(status, 1u);  // NaN or Inf
-    v = v > 0.f ? v : 0.f;
-    if (j >= nw) sp[j] = v;
-    tot = df_add_f(tot, v);
+  bool bad = false;
+  for (int j = j0 + threadIdx.x; j < j1; j += blockDim.x) {
+    float v;
+    if (j < nw) {
+      if (p.pool == 1) {
+        v = s_win[j - lo];
+      } else {
+        float acc = 0.f;
+        for (int i = j - half; i <= j + half; ++i)
+          if (i >= 0 && i < nw) acc += s_win[i - lo];
+        v = acc * invPool;
+      }
+      mx = fmaxf(mx, v);
+    } else {
+      if (p.protect) continue;  // the unit's max, known only after every slice
+      v = s_win[j - lo];
+    }
+    sp[j] = v;
+    if (!(fabsf(v) <= 3.0e38f)) bad = true;  // NaN or Inf
+    tot = df_add_f(tot, v > 0.f ? v : 0.f);
   }
+  if (bad) raise_status(status, 1u);
+  mx = warp_max(mx);
   tot = warp_sum_df(tot);
-  if ((threadIdx.x & 31) == 0) red_sum[threadIdx.x >> 5] = tot;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    DF v = threadIdx.x < (blockDim.x >> 5) ? red_sum[threadIdx.x] : df_make(0.f);
-    v = warp_sum_df(v);
-    if (threadIdx.x == 0) bcast[1] = v.hi;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    red_max[warp] = mx;
+    red_sum[warp] = tot;
   }
   __syncthreads();
-  const float total = bcast[1];
-  // 4. a_j = s_j / total
-  for (int j = threadIdx.x; j < n; j += blockDim.x) {
-    float v = sp[j];
+  if (threadIdx.x == 0) {
+    float m = -INFINITY;
+    DF t = df_make(0.f);
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+      m = fmaxf(m, red_max[w]);
+      t = df_add(t, red_sum[w]);
+    }
+    fin_part[(size_t)u * gridDim.x + slice] = make_float4(m, t.hi, t.lo, 0.f);
+  }
+}
+
+__global__ void __launch_bounds__(256) score_scale_kernel(Prob p, const float* __restrict__ s_pool,
+                                                          const float4* __restrict__ fin_part,
+                                                          float* __restrict__ a_out,
+                                                          uint32_t* __restrict__ keys,
+                                                          int32_t* __restrict__ vals,
+                                                          uint32_t* status) {
+  const int slice = blockIdx.x, u = blockIdx.y;
+  const int n = p.n, nw = n - p.w;
+  float smax = -INFINITY;
+  DF tot = df_make(0.f);
+  for (int k = 0; k < (int)gridDim.x; ++k) {  // every thread, same order
+    const float4 f = fin_part[(size_t)u * gridDim.x + k];
+    smax = fmaxf(smax, f.x);
+    tot = df_add(tot, DF{f.y, f.z});
+  }
+  if (p.protect) {
+    if (!(fabsf(smax) <= 3.0e38f) && slice == 0 && threadIdx.x == 0) raise_status(status, 1u);
+    tot = df_add(tot, two_prod(smax > 0.f ? smax : 0.f, (float)p.w));
+  }
+  const float total = tot.hi;
+  const float* sp = s_pool + (size_t)u * n;
+  float* au = a_out + (size_t)u * n;
+  const int j0 = slice * kFinSpan, j1 = min(n, j0 + kFinSpan);
+  for (int j = j0 + threadIdx.x; j < j1; j += blockDim.x) {
+    float v = (j >= nw && p.protect) ? smax : sp[j];
     v = v > 0.f ? v : 0.f;
-    float a = __fdiv_rn(v, total);
+    const float a = __fdiv_rn(v, total);
     au[j] = a;
     if (keys) {
       keys[(size_t)u * n + j] = score_key(a);
@@ -365,12 +394,20 @@ void launch_score(const Prob& p, const Layout& ly, char* ws, const void* K, cons
     score_pass_kernel<true><<<grid, threads, smem, st>>>(Kb, Qb, p, lse2, nullptr, s_part);
   }
   }
+  const dim3 fgrid((p.n + kFinSpan - 1) / kFinSpan, p.units);
+  float* s_pool = reinterpret_cast<float*>(ws + ly.s_tmp);
+  float4* fin_part = reinterpret_cast<float4*>(ws + ly.fin_part);
+  uint32_t* status = reinterpret_cast<uint32_t*>(ws + ly.status);
   {
-    TraceScope ts_("score_finalize", st);
-    score_finalize_kernel<<<p.units, 1024, 0, st>>>(
-        p, s_part, reinterpret_cast<float*>(ws + ly.s_tmp), a_out,
-        reinterpret_cast<uint32_t*>(ws + ly.keys0), reinterpret_cast<int32_t*>(ws + ly.vals0),
-        reinterpret_cast<uint32_t*>(ws + ly.status));
+    TraceScope ts_("score_pool", st);
+    const size_t fsmem = (size_t)(kFinSpan + p.pool) * sizeof(float);
+    score_pool_kernel<<<fgrid, 256, fsmem, st>>>(p, s_part, s_pool, fin_part, status);
+  }
+  {
+    TraceScope ts_("score_scale", st);
+    score_scale_kernel<<<fgrid, 256, 0, st>>>(
+        p, s_pool, fin_part, a_out, reinterpret_cast<uint32_t*>(ws + ly.keys0),
+        reinterpret_cast<int32_t*>(ws + ly.vals0), status);
   }
 }
 
