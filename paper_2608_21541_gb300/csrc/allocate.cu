@@ -182,14 +182,14 @@ __global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* _
   nc[p.hull_segs + g] = top;
 }
 
-// grid = B*L, block = 256: bisection, repair, counts and offsets of one
+// grid = B*L, block = 1024: bisection, repair, counts and offsets of one
 // (sequence, layer).  Candidates are staged in shared memory when they fit;
 // the repair keeps a 64-value window of each head's upcoming curve values in
 // shared memory, refilled by the whole warp.
 constexpr int kCandCap = 12288;  // staged candidates: 96 KB of values + 48 KB of b (dynamic smem)
 constexpr int kScan = 2048;      // curve values per round of a block extension (16 KB)
 
-__global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2* __restrict__ curve,
+__global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float2* __restrict__ curve,
                                                             const int32_t* __restrict__ cand,
                                                             const int32_t* __restrict__ ncand,
                                                             const unsigned long long* __restrict__ cmax,
@@ -197,7 +197,10 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
                                                             int64_t* __restrict__ offsets) {
   __shared__ int bsel[32];
   __shared__ int coff[33];
+  __shared__ DF wbest_f[32];  // per-warp argmin, combined per head
+  __shared__ int wbest_b[32];
   __shared__ double lam_sh[2];
+  __shared__ DF lam_df;  // the step's multiplier as double-float, for every warp
   __shared__ float2 win[32][64];
   __shared__ float2 scanbuf[kScan];
   extern __shared__ __align__(16) char dyn[];
@@ -227,28 +230,31 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
   }
   __syncthreads();
   const bool staged = coff[H] <= kCandCap;
-  if (staged) {  // gather the group survivors of every head, in order
-    for (int h = warp; h < H; h += nwarps) {
+  if (staged) {  // gather the group survivors of every head, in order; warp per (head, group)
+    for (int hg = warp; hg < H * groups; hg += nwarps) {
+      const int h = hg / groups, g = hg - h * groups;
       const int u = bl * H + h;
       const int32_t* nc = ncand + (size_t)u * stride + p.hull_segs;
       const int32_t* cl = cand + (size_t)u * n;
       int acc = coff[h];
-      for (int g = 0; g < groups; ++g) {
-        const int cnt = nc[g];
-        for (int k = lane; k < cnt; k += 32) {
-          const int b = cl[(size_t)g * kGroupSegs * kHullSeg + k];
-          cb_[acc + k] = b;
-          cy[acc + k] = curve[(size_t)u * n + b];
-        }
-        acc += cnt;
+      for (int g2 = 0; g2 < g; ++g2) acc += nc[g2];
+      const int cnt = nc[g];
+      for (int k = lane; k < cnt; k += 32) {
+        const int b = cl[(size_t)g * kGroupSegs * kHullSeg + k];
+        cb_[acc + k] = b;
+        cy[acc + k] = curve[(size_t)u * n + b];
       }
     }
   }
   __syncthreads();
 
-  auto argmin_heads = [&](double lam) {
-    const DF ld = df_from_double(lam);
-    for (int h = warp; h < H; h += nwarps) {
+  // Head h is scanned by warps h * wph .. h * wph + wph - 1 (wph = warps per
+  // head); the lexicographic (value, b) minimum does not depend on the split.
+  const int wph = nwarps / H;  // >= 1 since H <= 32
+  auto argmin_heads = [&]() {
+    const DF ld = lam_df;
+    const int h = warp / wph, sub = warp - h * wph;
+    if (h < H) {
       const int u = bl * H + h;
       DF bf{INFINITY, 0.f};
       int bb = INT_MAX;
@@ -260,33 +266,59 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
         }
       };
       if (staged) {
-        for (int k = coff[h] + lane; k < coff[h + 1]; k += 32) consider(cb_[k], cy[k]);
+        for (int k = coff[h] + sub * 32 + lane; k < coff[h + 1]; k += wph * 32) consider(cb_[k], cy[k]);
       } else {
         const int32_t* nc = ncand + (size_t)u * stride + p.hull_segs;
         const int32_t* cl = cand + (size_t)u * n;
         for (int g = 0; g < groups; ++g)
-          for (int k = lane; k < nc[g]; k += 32) {
+          for (int k = sub * 32 + lane; k < nc[g]; k += wph * 32) {
             const int b = cl[(size_t)g * kGroupSegs * kHullSeg + k];
             consider(b, curve[(size_t)u * n + b]);
           }
       }
       warp_argmin_df(bf, bb);
-      if (lane == 0) bsel[h] = (bb == INT_MAX) ? p.b_min : bb;
+      if (lane == 0) {
+        wbest_f[warp] = bf;
+        wbest_b[warp] = bb;
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x < H) {
+      const int hh = threadIdx.x;
+      DF bf = wbest_f[hh * wph];
+      int bb = wbest_b[hh * wph];
+      for (int w = 1; w < wph; ++w) {
+        const DF f = wbest_f[hh * wph + w];
+        const int b = wbest_b[hh * wph + w];
+        if (df_less(f, bf) || (f.hi == bf.hi && f.lo == bf.lo && b < bb)) {
+          bf = f;
+          bb = b;
+        }
+      }
+      bsel[hh] = (bb == INT_MAX) ? p.b_min : bb;
     }
   };
 
+  // float64 bisection of the multiplier, by one thread; the argmin runs in
+  // double-float on every warp
+  if (threadIdx.x == 0) lam_df = df_from_double(__dmul_rn(__dadd_rn(lam_sh[0], lam_sh[1]), 0.5));
+  __syncthreads();
   for (int t = 0; t < p.T; ++t) {
-    const double lam = __dmul_rn(__dadd_rn(lam_sh[0], lam_sh[1]), 0.5);
-    argmin_heads(lam);
+    argmin_heads();
     __syncthreads();
     if (threadIdx.x == 0) {
+      const double lam = __dmul_rn(__dadd_rn(lam_sh[0], lam_sh[1]), 0.5);
       int64_t tot = 0;
       for (int h = 0; h < H; ++h) tot += bsel[h];
       if (tot > B_real) lam_sh[0] = lam; else lam_sh[1] = lam;
+      lam_df = (t + 1 < p.T) ? df_from_double(__dmul_rn(__dadd_rn(lam_sh[0], lam_sh[1]), 0.5))
+                             : df_from_double(lam_sh[1]);
     }
     __syncthreads();
   }
-  argmin_heads(lam_sh[1]);
+  if (p.T == 0 && threadIdx.x == 0) lam_df = df_from_double(lam_sh[1]);
+  __syncthreads();
+  argmin_heads();
   __syncthreads();
 
   if (warp == 0) {
@@ -356,6 +388,40 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
         }
         more = df_less(d1, mg);
       }
+      // the run inside the winner's window first (no global loads): lane e
+      // checks marginal c(bw+1+e) - c(bw+e) for window positions, 32 at a time
+      if (more && bw + 1 - wbase < 64) {
+        const int i0 = bw + 1 - wbase;  // window index of c(bw + 1); c(bw) sits at i0 - 1
+        int run = 64 - i0;              // whole rest of the window, unless a check fails
+        for (int e0 = 0; e0 < 64 - i0; e0 += 32) {
+          const int e = e0 + lane, i = i0 + e;
+          bool stop = false;
+          if (i < 64) {
+            const float2 pv = win[who][i - 1], nv = win[who][i];
+            const DF d = df_add(DF{nv.x, nv.y}, df_neg(DF{pv.x, pv.y}));
+            stop = (bw + e >= n - 1) || !df_less(d, mg);
+          }
+          const unsigned stops = __ballot_sync(kFull, stop);
+          if (stops) {
+            run = e0 + __ffs(stops) - 1;
+            break;
+          }
+        }
+        const int64_t room = B_real - tot;
+        if ((int64_t)run > room) run = (int)room;
+        const bool whole = (run == 64 - i0);
+        if (run > 0) {
+          const float2 last = win[who][i0 + run - 1];
+          cw = DF{last.x, last.y};
+        }
+        bw += run;
+        tot += run;
+        more = whole && tot < B_real && bw < n - 1;
+        if (more) {  // does the run go on past the window?
+          const float2 w = ch[bw + 1];
+          more = df_less(df_add(DF{w.x, w.y}, df_neg(cw)), mg);
+        }
+      }
       bool extended = false;
       while (more) {  // warp-cooperative scan, kScan values per round
         extended = true;
@@ -394,12 +460,12 @@ __global__ void __launch_bounds__(256) bisect_repair_kernel(Prob p, const float2
         tot += run;
         more = (run == kScan) && tot < B_real && bw < n - 1;
       }
-      if (lane == who && extended) {
+      if (lane == who && bw > nb) {
         b = bw;
         cur = cw;
       }
       const int wb = extended ? -1 : wbase;
-      if (nb + 1 - wbase >= 64 || extended) {  // refill the winner's window
+      if (bw + 1 - wbase >= 64 || extended) {  // refill the winner's window
         if (bw < n - 1) {
           __syncwarp();
           for (int k = lane; k < 64; k += 32)
@@ -450,7 +516,7 @@ void launch_allocate(const Prob& p, const Layout& ly, char* ws, int32_t* counts,
                            (int)smem);
       attr = true;
     }
-    bisect_repair_kernel<<<p.bl, 256, smem, st>>>(
+    bisect_repair_kernel<<<p.bl, 1024, smem, st>>>(
         p, curve, cand, ncand, reinterpret_cast<const unsigned long long*>(ws + ly.cmax), counts,
         offsets);
   }
