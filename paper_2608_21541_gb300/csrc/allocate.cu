@@ -144,11 +144,13 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   if (seg >= p.hull_segs) return;
   const int n = p.n;
   const float2* cu = curve + (size_t)u * n;
-  int32_t* st = cand + (size_t)u * n + (size_t)seg * kHullSeg;
+  int32_t* out = cand + (size_t)u * n + (size_t)seg * kHullSeg;
   const int b0 = p.b_min + seg * kHullSeg;
   const int b1 = min(n, b0 + kHullSeg);
   const Shear sh = make_shear(cu, b0, b1 - 1);
+  int32_t st[kHullSeg];  // thread-private (L1-resident) chain stack
   const int top = tolerant_chain(sh, b1 - b0, [&](int i) { return b0 + i; }, st);
+  for (int i = 0; i < top; ++i) out[i] = st[i];
   ncand[(size_t)u * ncand_stride(p) + seg] = top;
 }
 
