@@ -173,6 +173,28 @@ int certkv_compress(const certkv_shape* shape, const void* K, const void* V,
                     const certkv_params* params, certkv_packed* out,
                     void* workspace, size_t workspace_bytes, void* stream);
 
+/* a1-a8 from HOST inputs, with the host->device copies overlapped with the
+ * compression (a runtime convenience; the paper's method is certkv_compress).
+ * hK, hV, hQ_obs: host memory in the layouts above; page-locked (pinned)
+ * memory makes the copies asynchronous, pageable memory works but its copies
+ * block the calling thread.  The (sequence, layer) pairs are processed
+ * `chunk` at a time (0: about 1 GiB of K and V per chunk): chunk c + 1 is
+ * copied into the other half of a double-buffered staging area inside the
+ * workspace, on a stream of the library's own, while chunk c compresses on
+ * `stream`.  Each pair is compressed independently, so `out` (device memory,
+ * as for certkv_compress) receives exactly what certkv_compress writes for the
+ * whole problem.  The host buffers must stay valid and unchanged until the
+ * work enqueued on `stream` has finished.  Workspace:
+ * certkv_host_workspace_bytes(shape, params, chunk) bytes, 256-byte aligned;
+ * certkv_read_status reads it as for the other entry points.  Returns the
+ * codes of certkv_compress; CERTKV_EINVAL also for chunk < 0. */
+size_t certkv_host_workspace_bytes(const certkv_shape* shape, const certkv_params* params,
+                                   int32_t chunk);
+int certkv_compress_host(const certkv_shape* shape, const void* hK, const void* hV,
+                         const void* hQ_obs, int64_t budget_live, const certkv_params* params,
+                         int32_t chunk, certkv_packed* out, void* workspace,
+                         size_t workspace_bytes, void* stream);
+
 /* a9: decode attention over the packed cache: for every query head qh of
  * unit u = (b, l, qh / G), out[b][l][qh] = sum_s softmax_s(scale <q, k_s>) v_s
  * over the real_counts[u] (+ 1 tail) slots of segment u.  q, out: bf16

@@ -48,7 +48,8 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_decode_workspace_bytes", "certkv_score", "certkv_curves",
             "certkv_compress_scored", "certkv_compress", "certkv_decode_attn",
             "certkv_read_status", "certkv_strerror", "certkv_trace_enable",
-            "certkv_trace_report", "certkv_decode_attn_noalloc")
+            "certkv_trace_report", "certkv_decode_attn_noalloc", "certkv_host_workspace_bytes",
+            "certkv_compress_host")
 
 _lock = threading.Lock()
 _lib = None
@@ -101,6 +102,10 @@ def load_library(path: Optional[str] = None):
         lib.certkv_trace_report.restype = ctypes.c_int
         lib.certkv_decode_attn_noalloc.argtypes = [sp, P, kp, ctypes.c_float, I32, P, P]
         lib.certkv_decode_attn_noalloc.restype = ctypes.c_int
+        lib.certkv_host_workspace_bytes.argtypes = [sp, pp, I32]
+        lib.certkv_host_workspace_bytes.restype = SZ
+        lib.certkv_compress_host.argtypes = [sp, P, P, P, I64, pp, I32, kp, P, SZ, P]
+        lib.certkv_compress_host.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -149,6 +154,13 @@ def certkv_workspace_bytes(shape: certkv_shape, params: Optional[certkv_params] 
     return int(load_library().certkv_workspace_bytes(ctypes.byref(shape), ctypes.byref(params)))
 
 
+def certkv_host_workspace_bytes(shape: certkv_shape, params: Optional[certkv_params] = None,
+                                chunk: int = 0) -> int:
+    params = params or certkv_default_params()
+    return int(load_library().certkv_host_workspace_bytes(ctypes.byref(shape),
+                                                          ctypes.byref(params), int(chunk)))
+
+
 def certkv_decode_workspace_bytes(shape: certkv_shape) -> int:
     return int(load_library().certkv_decode_workspace_bytes(ctypes.byref(shape)))
 
@@ -164,6 +176,12 @@ def _ptr(t: Optional[torch.Tensor]):
         return None
     if not t.is_cuda or not t.is_contiguous():
         raise ValueError("tensors passed to the CertKV library must be contiguous CUDA tensors")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _host_ptr(t: torch.Tensor):
+    if t.is_cuda or not t.is_contiguous():
+        raise ValueError("host inputs must be contiguous CPU tensors (pinned for asynchronous copies)")
     return ctypes.c_void_p(t.data_ptr())
 
 
@@ -284,6 +302,29 @@ def certkv_compress(K, V, Q_obs, budget_live: int, params=None, *, out: Optional
                                         int(budget_live), ctypes.byref(params), ctypes.byref(st),
                                         _ptr(ws), ws.numel(), _stream(stream))
     _check(rc, "certkv_compress")
+    return out
+
+
+def certkv_compress_host(hK, hV, hQ_obs, budget_live: int, params=None, *, chunk: int = 0,
+                         out: Optional[Packed] = None, ws=None, device=None, with_tail: bool = False,
+                         stream=None) -> Packed:
+    """a1-a8 from host tensors, copies overlapped with the compression."""
+    _bf16(hK, "K"); _bf16(hV, "V"); _bf16(hQ_obs, "Q_obs")
+    params = params or certkv_default_params()
+    shape = shape_of(hK, hQ_obs)
+    device = torch.device(device) if device is not None else torch.device("cuda",
+                                                                          torch.cuda.current_device())
+    if out is None:
+        out = Packed.empty(shape.batch, shape.layers, shape.hkv, shape.d, budget_live, device,
+                           with_tail, params.tail_slot)
+    if ws is None:
+        ws = workspace(certkv_host_workspace_bytes(shape, params, chunk), device)
+    st = out.struct()
+    rc = load_library().certkv_compress_host(ctypes.byref(shape), _host_ptr(hK), _host_ptr(hV),
+                                             _host_ptr(hQ_obs),
+                                             int(budget_live), ctypes.byref(params), int(chunk),
+                                             ctypes.byref(st), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "certkv_compress_host")
     return out
 
 

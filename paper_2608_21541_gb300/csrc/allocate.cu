@@ -488,9 +488,9 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
     }
     if (live) {
       counts[(size_t)bl * H + h] = b;
-      offsets[(size_t)bl * H + h] = (int64_t)bl * p.B_live + (incl - seg);
+      offsets[(size_t)bl * H + h] = p.slot_base + (int64_t)bl * p.B_live + (incl - seg);
     }
-    if (bl == p.bl - 1 && lane == 0) offsets[(size_t)p.bl * H] = (int64_t)p.bl * p.B_live;
+    if (bl == p.bl - 1 && lane == 0) offsets[(size_t)p.bl * H] = p.slot_base + (int64_t)p.bl * p.B_live;
   }
 }
 

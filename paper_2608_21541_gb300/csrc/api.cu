@@ -280,6 +280,133 @@ int certkv_compress_scored(const certkv_shape* shape, const void* K, const void*
   return run_scored(p, ly, ws, K, V, a, out, st);
 }
 
+namespace {
+// (sequence, layer) pairs per chunk of certkv_compress_host: 0 picks about
+// 1 GiB of K and V per chunk (at least 1 pair, at most all of them).
+int host_chunk(const Prob& p, int32_t chunk) {
+  if (chunk > 0) return chunk < p.bl ? chunk : p.bl;
+  const size_t per_bl = (size_t)2 * p.H * p.n * kD * 2;
+  size_t c = ((size_t)1 << 30) / per_bl;
+  if (c < 1) c = 1;
+  if (c > (size_t)p.bl) c = (size_t)p.bl;
+  return (int)c;
+}
+// Shape of a chunk of `cnt` consecutive (sequence, layer) pairs: one
+// sequence with cnt layers (the pairs are independent).
+certkv_shape chunk_shape(const certkv_shape* s, int cnt) {
+  certkv_shape c = *s;
+  c.batch = 1;
+  c.layers = cnt;
+  return c;
+}
+struct HostPlan {
+  Prob full, sub;
+  int chunk;
+  size_t ws_sub, stage_k, stage_q, stage, total;
+};
+int host_plan(const certkv_shape* shape, const certkv_params* params, int64_t budget, int32_t chunk,
+              HostPlan* hp) {
+  int rc = make_prob(shape, params, budget, &hp->full);
+  if (rc) return rc;
+  hp->chunk = host_chunk(hp->full, chunk);
+  const certkv_shape cs = chunk_shape(shape, hp->chunk);
+  if ((rc = make_prob(&cs, params, budget, &hp->sub))) return rc;
+  hp->ws_sub = align256(make_layout(hp->sub).total);
+  hp->stage_k = align256((size_t)hp->chunk * hp->full.H * hp->full.n * kD * 2);
+  hp->stage_q = align256((size_t)hp->chunk * hp->full.Hq * hp->full.w * kD * 2);
+  hp->stage = 2 * hp->stage_k + hp->stage_q;
+  hp->total = hp->ws_sub + 2 * hp->stage;
+  return CERTKV_OK;
+}
+}  // namespace
+
+size_t certkv_host_workspace_bytes(const certkv_shape* shape, const certkv_params* params,
+                                   int32_t chunk) {
+  HostPlan hp;
+  if (chunk < 0 || host_plan(shape, params, -1, chunk, &hp)) return 0;
+  return hp.total;
+}
+
+int certkv_compress_host(const certkv_shape* shape, const void* hK, const void* hV,
+                         const void* hQ_obs, int64_t budget_live, const certkv_params* params,
+                         int32_t chunk, certkv_packed* out, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  if (budget_live < 0) return CERTKV_EBUDGET;
+  if (chunk < 0) return CERTKV_EINVAL;
+  HostPlan hp;
+  int rc = host_plan(shape, params, budget_live, chunk, &hp);
+  if (rc) return rc;
+  if (!hK || !hV || !hQ_obs) return CERTKV_EINVAL;
+  if ((rc = check_packed(hp.full, out))) return rc;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < hp.total) return CERTKV_EWORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = reinterpret_cast<char*>(workspace);
+  char* stage[2] = {ws + hp.ws_sub, ws + hp.ws_sub + hp.stage};
+  // a private copy stream and its events, released when their work is done
+  cudaStream_t cs = nullptr;
+  cudaEvent_t start = nullptr, staged[2] = {nullptr, nullptr}, freed[2] = {nullptr, nullptr};
+  auto release = [&]() {
+    for (int i = 0; i < 2; ++i) {
+      if (staged[i]) cudaEventDestroy(staged[i]);
+      if (freed[i]) cudaEventDestroy(freed[i]);
+    }
+    if (start) cudaEventDestroy(start);
+    if (cs) cudaStreamDestroy(cs);
+  };
+  if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&start, cudaEventDisableTiming) != cudaSuccess) {
+    release();
+    return CERTKV_ECUDA;
+  }
+  for (int i = 0; i < 2; ++i)
+    if (cudaEventCreateWithFlags(&staged[i], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&freed[i], cudaEventDisableTiming) != cudaSuccess) {
+      release();
+      return CERTKV_ECUDA;
+    }
+  const Prob& F = hp.full;
+  const size_t kv_bl = (size_t)F.H * F.n * kD * 2, q_bl = (size_t)F.Hq * F.w * kD * 2;
+  const Layout ly_sub = make_layout(hp.sub);
+  rc = cuda_ok(cudaMemsetAsync(ws + ly_sub.status, 0, 256, st));
+  if (!rc) rc = cuda_ok(cudaEventRecord(start, st));
+  if (!rc) rc = cuda_ok(cudaStreamWaitEvent(cs, start, 0));
+  for (int bl0 = 0, c = 0; !rc && bl0 < F.bl; bl0 += hp.chunk, ++c) {
+    const int cnt = (F.bl - bl0) < hp.chunk ? (F.bl - bl0) : hp.chunk;
+    const int s = c & 1;
+    char* sK = stage[s];
+    char* sV = stage[s] + hp.stage_k;
+    char* sQ = stage[s] + 2 * hp.stage_k;
+    // copy stream: wait until chunk c - 2 has left this half, then stage chunk c
+    if (c >= 2) rc = cuda_ok(cudaStreamWaitEvent(cs, freed[s], 0));
+    if (!rc) rc = cuda_ok(cudaMemcpyAsync(sK, (const char*)hK + bl0 * kv_bl, cnt * kv_bl,
+                                          cudaMemcpyHostToDevice, cs));
+    if (!rc) rc = cuda_ok(cudaMemcpyAsync(sV, (const char*)hV + bl0 * kv_bl, cnt * kv_bl,
+                                          cudaMemcpyHostToDevice, cs));
+    if (!rc) rc = cuda_ok(cudaMemcpyAsync(sQ, (const char*)hQ_obs + bl0 * q_bl, cnt * q_bl,
+                                          cudaMemcpyHostToDevice, cs));
+    if (!rc) rc = cuda_ok(cudaEventRecord(staged[s], cs));
+    if (!rc) rc = cuda_ok(cudaStreamWaitEvent(st, staged[s], 0));
+    if (rc) break;
+    // compute stream: the chunk as its own problem, writing global slots
+    Prob p;
+    certkv_shape csub = chunk_shape(shape, cnt);
+    if ((rc = make_prob(&csub, params, budget_live, &p))) break;
+    p.slot_base = (int64_t)bl0 * F.B_live;
+    const Layout ly = make_layout(p);
+    certkv_packed o = *out;
+    o.offsets = out->offsets + (size_t)bl0 * F.H;
+    o.real_counts = out->real_counts + (size_t)bl0 * F.H;
+    if (out->tail_f32) o.tail_f32 = out->tail_f32 + (size_t)bl0 * F.H * 2 * kD;
+    if (out->tail_mass) o.tail_mass = out->tail_mass + (size_t)bl0 * F.H;
+    float* a = reinterpret_cast<float*>(ws + ly.a);
+    launch_score(p, ly, ws, sK, sQ, a, st);
+    rc = run_scored(p, ly, ws, sK, sV, a, &o, st);
+    if (!rc) rc = cuda_ok(cudaEventRecord(freed[s], st));
+  }
+  release();
+  return rc;
+}
+
 int certkv_compress(const certkv_shape* shape, const void* K, const void* V, const void* Q_obs,
                     int64_t budget_live, const certkv_params* params, certkv_packed* out,
                     void* workspace, size_t workspace_bytes, void* stream) {

@@ -19,6 +19,7 @@ struct Prob {
   int alpha_num, alpha_den, T, statistic, tail_slot;
   int64_t B_live, B_real;
   int b_min;
+  int64_t slot_base;  // packed slot of this problem's first (sequence, layer): offsets are global
   // derived launch geometry
   int score_tc;     // 1: tcgen05 scorer (R in {128, 256}); 0: mma.sync scorer
   int score_warps;  // warps per score CTA (16 rows each)

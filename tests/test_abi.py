@@ -113,3 +113,27 @@ def test_binding_refuses_a_missing_library(tmp_path):
             ck.load_library(str(tmp_path / "missing.so"))
     finally:
         ck._lib = saved
+
+
+def test_host_entry_point_validation(lib):
+    s = shape()
+    params = ck.certkv_default_params()
+    need_dev = lib.certkv_workspace_bytes(ctypes.byref(s), ctypes.byref(params))
+    need = lib.certkv_host_workspace_bytes(ctypes.byref(s), ctypes.byref(params), 0)
+    assert need > need_dev  # device workspace of a chunk plus two staging halves
+    assert lib.certkv_host_workspace_bytes(ctypes.byref(s), ctypes.byref(params), -1) == 0
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
+    packed = ck.certkv_packed(fake, fake, fake, fake, fake, 1 << 40, None, None)
+
+    def call(chunk=0, ws=256, ws_bytes=None, budget=2 * s.hkv, k=fake):
+        return lib.certkv_compress_host(ctypes.byref(s), k, fake, fake, budget,
+                                        ctypes.byref(params), chunk, ctypes.byref(packed),
+                                        ctypes.c_void_p(ws) if ws else None,
+                                        need if ws_bytes is None else ws_bytes, None)
+
+    assert call(chunk=-1) == ck.EINVAL
+    assert call(k=None) == ck.EINVAL
+    assert call(budget=-3) == ck.EBUDGET
+    assert call(ws=0) == ck.EWORKSPACE
+    assert call(ws=257) == ck.EWORKSPACE
+    assert call(ws_bytes=need - 1) == ck.EWORKSPACE

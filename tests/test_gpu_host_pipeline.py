@@ -1,0 +1,55 @@
+"""certkv_compress_host (host inputs, copies overlapped with the compression)
+gives exactly what certkv_compress gives on the same data, for every chunk
+size, with pinned and with pageable host memory."""
+import pytest
+import torch
+
+from paper_2608_21541_gb300 import certkv as ck
+from paper_2608_21541_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+WL = W.Workload("S", B=2, L=3, Hq=8, H=2, n=3000, d=128, w=20, keep=(1, 10), kind="planted")
+
+
+def _reference(K, V, Q, B_live, params):
+    return ck.certkv_compress(K, V, Q, B_live, params, with_tail=True)
+
+
+def _same(a: ck.Packed, b: ck.Packed):
+    assert torch.equal(a.real_counts, b.real_counts)
+    assert torch.equal(a.offsets, b.offsets)
+    n = int(a.offsets[-1])
+    assert torch.equal(a.positions[:n], b.positions[:n])
+    assert torch.equal(a.k[:n].view(torch.int16), b.k[:n].view(torch.int16))
+    assert torch.equal(a.v[:n].view(torch.int16), b.v[:n].view(torch.int16))
+    assert torch.equal(a.tail_f32, b.tail_f32)
+    assert torch.equal(a.tail_mass, b.tail_mass)
+
+
+@pytest.mark.parametrize("chunk", [1, 4, 0])
+@pytest.mark.parametrize("pinned", [True, False])
+def test_host_pipeline_equals_device_call(chunk, pinned):
+    K, V, Q = W.draw(WL, device="cuda")
+    params = ck.certkv_default_params()
+    ref = _reference(K, V, Q, WL.B_live, params)
+    hK, hV, hQ = K.cpu(), V.cpu(), Q.cpu()
+    if pinned:
+        hK, hV, hQ = hK.pin_memory(), hV.pin_memory(), hQ.pin_memory()
+    got = ck.certkv_compress_host(hK, hV, hQ, WL.B_live, params, chunk=chunk, with_tail=True)
+    torch.cuda.synchronize()
+    _same(got, ref)
+
+
+def test_host_pipeline_status_and_reuse():
+    # two calls in a row on one workspace; the status word stays clean
+    K, V, Q = W.draw(WL, device="cuda")
+    params = ck.certkv_default_params()
+    shape = ck.shape_of(K, Q)
+    ws = ck.workspace(ck.certkv_host_workspace_bytes(shape, params, 2), K.device)
+    hK, hV, hQ = K.cpu().pin_memory(), V.cpu().pin_memory(), Q.cpu().pin_memory()
+    a = ck.certkv_compress_host(hK, hV, hQ, WL.B_live, params, chunk=2, ws=ws, with_tail=True)
+    b = ck.certkv_compress_host(hK, hV, hQ, WL.B_live, params, chunk=2, ws=ws, with_tail=True)
+    torch.cuda.synchronize()
+    _same(a, b)
+    assert ck.certkv_read_status(ws) == 0
