@@ -59,7 +59,7 @@ int make_prob(const certkv_shape* s, const certkv_params* q, int64_t budget_live
   P.statistic = q->statistic; P.tail_slot = q->tail_slot;
   P.score_warps = (P.R + 15) / 16 < 16 ? (P.R + 15) / 16 : 16;
   P.row_blocks = (P.R + 16 * P.score_warps - 1) / (16 * P.score_warps);
-  if (score_tc_supported(P)) P.row_blocks = 2;  // one per 128-row half of the tcgen05 pass 2
+  if (score_tc_supported(P)) P.row_blocks = P.R / 64;  // one per 64-row quarter of the tcgen05 pass 2
   P.score_tc = score_tc_supported(P) ? 1 : 0;
   P.key_splits = P.score_tc ? (P.n + kKeysPerItemTc - 1) / kKeysPerItemTc
                             : (P.n + kScoreKeysPerCta - 1) / kScoreKeysPerCta;

@@ -31,7 +31,7 @@ namespace tc {
 #ifndef CERTKV_TC_STAGES
 #define CERTKV_TC_STAGES 4
 #endif
-constexpr int kEpiWarps = 16;  // two groups of 8, one per TMEM accumulator buffer
+constexpr int kEpiWarps = 16;  // warp (q, cq): TMEM lane quadrant q, 64-column quarter cq
 constexpr int kThreads = (2 + kEpiWarps) * 32;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kSpinLimit = 1u << 22;
@@ -225,7 +225,7 @@ __device__ __forceinline__ uint32_t setup(const Shared<C>& sh, int warp) {
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(sh.accf(b), 1);
-      mbar_init(sh.acce(b), kEpiWarps / 2);
+      mbar_init(sh.acce(b), kEpiWarps);
     }
     mbar_init(sh.qfull(), 1);
     mbar_init(sh.done(), 1);
@@ -317,7 +317,8 @@ __device__ __forceinline__ void issue_mmas(const Shared<C>& sh, uint32_t tmem, u
 
 // Pass 1.  grid = units * key_splits * halves; adjacent CTAs are the two
 // 128-row halves of one key range (they stream the same K tiles, the second
-// mostly from L2).  D[rows x 256 keys]; epilogue thread = one row.
+// mostly from L2).  D[rows x 256 keys]; epilogue thread = one row and a
+// 64-key quarter of every tile.
 __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_constant__ CUtensorMap tmK,
                                                              const __grid_constant__ CUtensorMap tmQ,
                                                              Prob p, float2* __restrict__ lse_part,
@@ -348,66 +349,63 @@ __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_consta
             return sh.kst(s) + kh * (C::kStageBytes / 2) + koff;
           });
   } else {
-    // group grp reads buffer grp (tiles of that parity); within a group, warp
-    // (q, colh) owns rows q*32.. of the half and keys colh*128.. of the tile
-    const int ew = warp - 2, grp = ew >> 3, q = warp & 3, colh = (ew & 7) >> 2;
+    // every warp takes every tile: warp (q, cq) owns rows q*32.. of the half
+    // (its TMEM lane quadrant) and keys cq*64 .. cq*64+63 of each 256-key tile.
+    // It releases the accumulator as soon as its columns are in registers.
+    const int ew = warp - 2, q = warp & 3, cq = ew >> 2;
     const int rloc = q * 32 + lane;
     const int row = half * 128 + rloc;
     const int lim = n - p.w + (row % p.w);
     const float sl2 = p.scale_log2;
     float m = -INFINITY, l = 0.f;
-    for (int t = grp; t < ntiles; t += 2) {
+    for (int t = 0; t < ntiles; ++t) {
       const int b = t & 1;
       if (!mbar_wait(sh.accf(b), (t >> 1) & 1, ab)) break;
       tc_fence_after();
-      const int j0 = j_begin + t * C::kTileKeys + colh * 128;
-      const bool interior = (j0 + 128 <= j_end) && (j0 + 127 <= n - p.w);
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
-        float v[64];
-        tmem_ld64(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + colh * 128 + c * 64), v);
-        if (interior) {
-          float mx0 = v[0], mx1 = v[1];
-#pragma unroll
-          for (int i = 2; i < 64; i += 2) {
-            mx0 = fmaxf(mx0, v[i]);
-            mx1 = fmaxf(mx1, v[i + 1]);
-          }
-          const float nm = fmaxf(m, fmaxf(mx0, mx1) * sl2);  // sl2 > 0: max commutes with scaling
-          float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-          for (int i = 0; i < 64; ++i) acc[i & 7] += ex2(fmaf(v[i], sl2, -nm));
-          const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
-          l = fmaf(l, ex2(m - nm), sum);
-          m = nm;
-        } else {
-          float cm = -INFINITY;
-#pragma unroll
-          for (int i = 0; i < 64; ++i) {
-            const int j = j0 + c * 64 + i;
-            v[i] = (j <= lim && j < j_end) ? v[i] * sl2 : -INFINITY;
-            cm = fmaxf(cm, v[i]);
-          }
-          const float nm = fmaxf(m, cm);
-          if (nm > -INFINITY) {
-            float sum = 0.f;
-#pragma unroll
-            for (int i = 0; i < 64; ++i) sum += ex2(v[i] - nm);
-            l = fmaf(l, ex2(m - nm), sum);
-            m = nm;
-          }
-        }
-      }
+      float v[64];
+      tmem_ld64(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + cq * 64), v);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(sh.acce(b));
+      const int jc = j_begin + t * C::kTileKeys + cq * 64;
+      const bool interior = (jc + 64 <= j_end) && (jc + 63 <= n - p.w);
+      if (interior) {
+        float mx0 = v[0], mx1 = v[1];
+#pragma unroll
+        for (int i = 2; i < 64; i += 2) {
+          mx0 = fmaxf(mx0, v[i]);
+          mx1 = fmaxf(mx1, v[i + 1]);
+        }
+        const float nm = fmaxf(m, fmaxf(mx0, mx1) * sl2);  // sl2 > 0: max commutes with scaling
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < 64; ++i) acc[i & 7] += ex2(fmaf(v[i], sl2, -nm));
+        const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+        l = fmaf(l, ex2(m - nm), sum);
+        m = nm;
+      } else {
+        float cm = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 64; ++i) {
+          const int j = jc + i;
+          v[i] = (j <= lim && j < j_end) ? v[i] * sl2 : -INFINITY;
+          cm = fmaxf(cm, v[i]);
+        }
+        const float nm = fmaxf(m, cm);
+        if (nm > -INFINITY) {
+          float sum = 0.f;
+#pragma unroll
+          for (int i = 0; i < 64; ++i) sum += ex2(v[i] - nm);
+          l = fmaf(l, ex2(m - nm), sum);
+          m = nm;
+        }
+      }
     }
-    // merge the four partial (max, sum) of each row: 2 groups x 2 key halves
-    const int slot = grp * 2 + colh;
-    sh.pm()[slot * 128 + rloc] = m;
-    sh.pl()[slot * 128 + rloc] = l;
+    // merge the four partial (max, sum) of each row, one per key quarter
+    sh.pm()[cq * 128 + rloc] = m;
+    sh.pl()[cq * 128 + rloc] = l;
     epi_sync();
-    if (slot == 0 && !*ab) {
+    if (cq == 0 && !*ab) {
       float M = -INFINITY;
 #pragma unroll
       for (int k = 0; k < 4; ++k) M = fmaxf(M, sh.pm()[k * 128 + rloc]);
@@ -423,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_consta
 }
 
 // Pass 2.  grid = units * key_splits.  D[128 keys x R rows]; epilogue thread
-// = one key, summing exp(l - LSE_row) over 128 rows of its TMEM lane.
+// = one key, summing exp(l - LSE_row) over a 64-row quarter of its TMEM lane.
 __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_constant__ CUtensorMap tmK,
                                                                 const __grid_constant__ CUtensorMap tmQ,
                                                                 Prob p, const float* __restrict__ lse2,
@@ -453,49 +451,48 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
           },
           [&](int, uint32_t kh, uint32_t koff) { return sh.q() + kh * (C::kQBytes / 2) + koff; });
   } else {
-    const int ew = warp - 2, grp = ew >> 3, q = warp & 3, ch = (ew & 7) >> 2;  // ch: 128-row half
+    // every warp takes every tile: warp (q, cq) owns keys q*32.. of the tile
+    // (its TMEM lane quadrant) and rows cq*64 .. cq*64+63, summed into row
+    // block cq.  It releases the accumulator as soon as its columns are read.
+    const int ew = warp - 2, q = warp & 3, cq = ew >> 2;
     const int key = q * 32 + lane;
-    const bool rows_here = ch * 128 < R;
+    const bool rows_here = cq * 64 < R;
     const float sl2 = p.scale_log2;
     const int nw = n - p.w;
-    // the two row halves write separate row blocks; the finalize kernel adds them
-    float* out = s_part + ((size_t)u * p.row_blocks + ch) * n;
-    for (int t = grp; t < ntiles; t += 2) {
+    float* out = s_part + ((size_t)u * p.row_blocks + cq) * n;
+    const int r0 = cq * 64;
+    const float4* L4 = reinterpret_cast<const float4*>(sh.lse() + r0);
+    for (int t = 0; t < ntiles; ++t) {
       const int b = t & 1;
       if (!mbar_wait(sh.accf(b), (t >> 1) & 1, ab)) break;
       tc_fence_after();
+      float v[64];
+      if (rows_here)
+        tmem_ld64(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + cq * 64), v);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sh.acce(b));
+      if (!rows_here) continue;
       const int j0 = j_begin + t * C::kTileKeys;
       const int j = j0 + key;
       const bool interior = (j0 + C::kTileKeys <= j_end) && (j0 + C::kTileKeys <= nw);
       float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      if (rows_here) {
-#pragma unroll 1
-        for (int c = 0; c < 2; ++c) {
-          float v[64];
-          tmem_ld64(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * 256 + ch * 128 + c * 64), v);
-          const int r0 = ch * 128 + c * 64;
-          const float4* L4 = reinterpret_cast<const float4*>(sh.lse() + r0);
-          if (interior) {
+      if (interior) {
 #pragma unroll
-            for (int i = 0; i < 64; i += 4) {
-              const float4 L = L4[i >> 2];
-              acc[(i + 0) & 7] += ex2(fmaf(v[i], sl2, -L.x));
-              acc[(i + 1) & 7] += ex2(fmaf(v[i + 1], sl2, -L.y));
-              acc[(i + 2) & 7] += ex2(fmaf(v[i + 2], sl2, -L.z));
-              acc[(i + 3) & 7] += ex2(fmaf(v[i + 3], sl2, -L.w));
-            }
-          } else {
+        for (int i = 0; i < 64; i += 4) {
+          const float4 L = L4[i >> 2];
+          acc[(i + 0) & 7] += ex2(fmaf(v[i], sl2, -L.x));
+          acc[(i + 1) & 7] += ex2(fmaf(v[i + 1], sl2, -L.y));
+          acc[(i + 2) & 7] += ex2(fmaf(v[i + 2], sl2, -L.z));
+          acc[(i + 3) & 7] += ex2(fmaf(v[i + 3], sl2, -L.w));
+        }
+      } else {
 #pragma unroll
-            for (int i = 0; i < 64; ++i) {
-              const int r = r0 + i;
-              if (j < j_end && j <= nw + (r % p.w)) acc[0] += ex2(fmaf(v[i], sl2, -sh.lse()[r]));
-            }
-          }
+        for (int i = 0; i < 64; ++i) {
+          const int r = r0 + i;
+          if (j < j_end && j <= nw + (r % p.w)) acc[0] += ex2(fmaf(v[i], sl2, -sh.lse()[r]));
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(sh.acce(b));
       if (j < j_end)
         out[j] = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
     }
