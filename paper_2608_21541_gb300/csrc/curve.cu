@@ -367,26 +367,25 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
     const int cnt = r1 - (r0 + rl);  // rows of the group that exist (may exceed 8)
     const unsigned char* rows = s_ring[warp][g % kEvalRing];
     if (!exact) {
+      // dimension pairs (0,1) and (2,3) of this lane in two-wide arithmetic
+      float2 P01 = make_float2(P[0], P[1]), P23 = make_float2(P[2], P[3]);
+      const float2 W01 = make_float2(wb2x[0], wb2x[1]), W23 = make_float2(wb2x[2], wb2x[3]);
       float xg[8];
 #pragma unroll
       for (int t = 7; t >= 0; --t) {
         const float as = sa[rl + t];
-        float v[4] = {0.f, 0.f, 0.f, 0.f};
-        if (t < cnt) {
-          const uint2 raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
-          v[0] = bf16lo(raw.x);
-          v[1] = bf16hi(raw.x);
-          v[2] = bf16lo(raw.y);
-          v[3] = bf16hi(raw.y);
-        }
-        float acc = 0.f;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          P[i] = fmaf(as, v[i], P[i]);
-          acc = fmaf(wb2x[i] + P[i], P[i], acc);
-        }
-        xg[t] = (t < cnt) ? acc : 0.f;
+        uint2 raw = make_uint2(0u, 0u);
+        if (t < cnt) raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
+        const float2 a2 = make_float2(as, as);
+        P01 = ffma2(a2, make_float2(bf16lo(raw.x), bf16hi(raw.x)), P01);
+        P23 = ffma2(a2, make_float2(bf16lo(raw.y), bf16hi(raw.y)), P23);
+        const float2 acc = ffma2(fadd2(W23, P23), P23, fmul2(fadd2(W01, P01), P01));
+        xg[t] = (t < cnt) ? acc.x + acc.y : 0.f;
       }
+      P[0] = P01.x;
+      P[1] = P01.y;
+      P[2] = P23.x;
+      P[3] = P23.y;
       const float x = reduce8(xg, lane);
       if ((lane >> 3) == (s0 >> 3)) xt = df_make(x);
     } else {
