@@ -84,6 +84,16 @@ __device__ __forceinline__ DF df_add(DF x, DF y) {
   return fast_two_sum(v.hi, e);
 }
 
+// x + y for x and y of the same sign (both >= 0 here): the high parts are
+// added exactly (two_sum), the low parts folded into the error, one
+// renormalisation.  Without cancellation this simplified double-float sum is
+// accurate to a few units of 2^-48 (Dekker 1971); it is not used where the
+// operands can have opposite signs.
+__device__ __forceinline__ DF df_add_same_sign(DF x, DF y) {
+  const DF s = two_sum(x.hi, y.hi);
+  return fast_two_sum(s.hi, __fadd_rn(s.lo, __fadd_rn(x.lo, y.lo)));
+}
+
 __device__ __forceinline__ DF df_add_f(DF x, float y) {
   DF s = two_sum(x.hi, y);
   float e = __fadd_rn(s.lo, x.lo);
@@ -121,6 +131,20 @@ __device__ __forceinline__ DF df_sqrt(DF x) {
   float r = __fadd_rn(__fsub_rn(__fsub_rn(x.hi, s2.hi), s2.lo), x.lo);
   float corr = __fdiv_rn(r, __fmul_rn(2.0f, s));
   return fast_two_sum(s, corr);
+}
+
+// sqrt of a non-negative df value from the hardware reciprocal square root:
+// s = x * rsqrt(x) is within a few 2^-23 of sqrt(x); one Newton step for the
+// square root, s + (x - s^2) / (2 s), with x - s^2 formed exactly (two_prod)
+// and 1 / (2 s) taken as rsqrt(x) / 2, squares that error to ~2^-44.
+__device__ __forceinline__ DF df_sqrt_newton(DF x) {
+  if (!(x.hi > 0.0f)) return DF{0.0f, 0.0f};
+  if (x.hi < 7.8886091e-31f) return df_sqrt(x);  // below 2^-100: keep clear of subnormals
+  const float r = rsqrtf(x.hi);
+  const float s = __fmul_rn(x.hi, r);
+  const DF s2 = two_prod(s, s);
+  const float e = __fadd_rn(__fsub_rn(__fsub_rn(x.hi, s2.hi), s2.lo), x.lo);
+  return fast_two_sum(s, __fmul_rn(e, __fmul_rn(0.5f, r)));
 }
 
 __device__ __forceinline__ double df_to_double(DF x) { return (double)x.hi + (double)x.lo; }

@@ -353,7 +353,7 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
   const bool exact = (chunk == p.chunks - 1);
   float P[4] = {0.f, 0.f, 0.f, 0.f};
   DF Pd[4] = {df_make(0.f), df_make(0.f), df_make(0.f), df_make(0.f)};
-  DF carry_m = df_make(0.f), carry_q = df_make(0.f);
+  DF base_m = M0, base_q = Q0;  // sums over the ranks after the current batch
   unsigned long long best = 0ull;
   bool bad = false;
   DF xt = df_make(0.f);  // lane r: ||W_base + P(b)||^2 - ||W_base||^2 for rank r of the batch
@@ -417,7 +417,8 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
     const bool ok = r < r1;
     const float at = sa[32 * bi + lane];
     const float2 yv = sy[32 * bi + lane];
-    // in-batch inclusive suffix sums over lanes >= t
+    // in-batch inclusive suffix sums over lanes >= t (a and a||v||^2 are
+    // non-negative: same-sign double-float additions)
     DF sm = df_make(at);
     DF sq = ok ? df_mul_f(DF{yv.x, yv.y}, at) : df_make(0.f);
 #pragma unroll
@@ -425,20 +426,20 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
       DF om{__shfl_down_sync(kFull, sm.hi, o), __shfl_down_sync(kFull, sm.lo, o)};
       DF oq{__shfl_down_sync(kFull, sq.hi, o), __shfl_down_sync(kFull, sq.lo, o)};
       if (lane + o < 32) {
-        sm = df_add(sm, om);
-        sq = df_add(sq, oq);
+        sm = df_add_same_sign(sm, om);
+        sq = df_add_same_sign(sq, oq);
       }
     }
-    const DF Mt = df_add(M0, df_add(carry_m, sm));
-    const DF Qt = df_add(Q0, df_add(carry_q, sq));
+    const DF Mt = df_add_same_sign(base_m, sm);
+    const DF Qt = df_add_same_sign(base_q, sq);
     DF c;
     if (p.statistic == 2) {
       c = Mt;
     } else if (p.statistic == 1) {
-      c = df_sqrt(df_mul(Mt, Qt));
+      c = df_sqrt_newton(df_mul(Mt, Qt));
     } else {
       const DF W2 = df_add(wb2, xt);
-      c = df_sqrt(df_add(df_mul(Mt, Qt), df_neg(W2)));
+      c = df_sqrt_newton(df_add(df_mul(Mt, Qt), df_neg(W2)));
     }
     if (ok) {
       curve[(size_t)u * n + r] = make_float2(c.hi, c.lo);
@@ -446,8 +447,8 @@ __global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t*
       unsigned long long k = df_order_key(c);
       best = k > best ? k : best;
     }
-    carry_m = df_add(carry_m, shfl_df(sm, 0));
-    carry_q = df_add(carry_q, shfl_df(sq, 0));
+    base_m = df_add_same_sign(base_m, shfl_df(sm, 0));
+    base_q = df_add_same_sign(base_q, shfl_df(sq, 0));
   }
   asm volatile("cp.async.wait_all;" ::: "memory");
 #pragma unroll
