@@ -57,9 +57,12 @@ __global__ void __launch_bounds__(128) decode_split_kernel(Prob p, const __nv_bf
     for (int g = 0; g < G; ++g) x[g] = 0.f;
     if (ok) {
       const uint4* kr = reinterpret_cast<const uint4*>(pk + (size_t)(off + s) * kD);
-#pragma unroll 4
+      uint4 krow[16];  // the whole 256-byte row in flight before the dot products
+#pragma unroll
+      for (int c = 0; c < 16; ++c) krow[c] = __ldg(kr + c);
+#pragma unroll
       for (int c = 0; c < 16; ++c) {
-        const uint4 raw = __ldg(kr + c);
+        const uint4 raw = krow[c];
         const float kf[8] = {bf16lo(raw.x), bf16hi(raw.x), bf16lo(raw.y), bf16hi(raw.y),
                              bf16lo(raw.z), bf16hi(raw.z), bf16lo(raw.w), bf16hi(raw.w)};
 #pragma unroll
