@@ -105,7 +105,18 @@ typedef struct {
   int32_t statistic;      /* CERTKV_STAT_* (default CERTKV_STAT_CENTERED)             */
   int32_t tail_slot;      /* 1 (default): one synthetic tail slot per head is charged
                              to the budget; 0: no slot, the slot goes to a real token */
+  int32_t allocator;      /* CERTKV_ALLOC_* (default CERTKV_ALLOC_LAGRANGIAN)          */
 } certkv_params;
+
+/* Cross-head allocator (paper: one-factor ablations, "Allocator" block).  The
+ * paper names the two ablations without defining them; the readings used:
+ * UNIFORM gives every head floor(B_real / H) real tokens and one more to each
+ * of the lowest (B_real mod H) heads; GREEDY starts every head at b_min and
+ * adds one token at a time to the head with the smallest c_h(b_h+1) - c_h(b_h)
+ * (lowest head on ties), the repair rule of Algorithm 1 run from b_min. */
+#define CERTKV_ALLOC_LAGRANGIAN 0  /* T-step bisection on lambda + repair (Algorithm 1) */
+#define CERTKV_ALLOC_UNIFORM    1
+#define CERTKV_ALLOC_GREEDY     2
 
 /* Ragged packed cache.  Segment u (one per unit) holds real_counts[u] real
  * slots in ascending original position followed, when params.tail_slot = 1,

@@ -52,6 +52,8 @@ def _bind(lib):
     lib.oracle_b_min.restype = I64
     lib.oracle_allocate.argtypes = [P, I, I, I64, I64, I64, I, P, P]
     lib.oracle_allocate.restype = I
+    lib.oracle_allocate_mode.argtypes = [P, I, I, I64, I64, I64, I, I, P, P]
+    lib.oracle_allocate_mode.restype = I
     lib.oracle_select.argtypes = [P, I, P]
     lib.oracle_select.restype = None
     lib.oracle_tail.argtypes = [P, P, P, P, I, I, I, P, P, P]
@@ -153,8 +155,10 @@ def b_min(B_real: int, H: int, alpha_num: int = 1, alpha_den: int = 5, *, lib=No
     return int((lib or _load()).oracle_b_min(int(B_real), int(H), int(alpha_num), int(alpha_den)))
 
 
-def allocate(curves, B_real: int, alpha_num: int = 1, alpha_den: int = 5, T: int = 40, *, lib=None):
-    """a5: per-head real-token budgets.  curves [H][n] float64.
+def allocate(curves, B_real: int, alpha_num: int = 1, alpha_den: int = 5, T: int = 40, *,
+             mode: int = 0, lib=None):
+    """a5: per-head real-token budgets.  curves [H][n] float64.  mode 0: Lagrangian
+    bisection + repair (the method); 1: true uniform; 2: greedy marginal from b_min.
 
     Returns (b [H] int32, repairs) or raises ValueError on an infeasible budget."""
     curves = np.ascontiguousarray(curves, dtype=np.float64)
@@ -162,8 +166,9 @@ def allocate(curves, B_real: int, alpha_num: int = 1, alpha_den: int = 5, T: int
     ptrs = (ctypes.c_void_p * H)(*[curves.ctypes.data + h * n * 8 for h in range(H)])
     b = np.empty(H, dtype=np.int32)
     rep = np.zeros(1, dtype=np.int64)
-    rc = (lib or _load()).oracle_allocate(ctypes.cast(ptrs, ctypes.c_void_p), H, n, int(B_real),
-                                 int(alpha_num), int(alpha_den), int(T), _ptr(b), _ptr(rep))
+    rc = (lib or _load()).oracle_allocate_mode(ctypes.cast(ptrs, ctypes.c_void_p), H, n,
+                                               int(B_real), int(alpha_num), int(alpha_den),
+                                               int(T), int(mode), _ptr(b), _ptr(rep))
     if rc != 0:
         raise ValueError("infeasible budget")
     return b, int(rep[0])
@@ -196,7 +201,8 @@ def tail(a, K, V, perm, b: int, *, lib=None):
 def compress(K, V, Q, *, B: int, L: int, Hq: int, H: int, n: int, d: int, w: int,
              B_live: int, scale: float = 0.0, pool: int = 5, protect: int = 1,
              alpha_num: int = 1, alpha_den: int = 5, T: int = 40, statistic: int = 0,
-             tail_slot: int = 1, a_in=None, threads: int | None = None, lib=None) -> dict:
+             tail_slot: int = 1, allocator: int = 0, a_in=None, threads: int | None = None,
+             lib=None) -> dict:
     """The whole compression pass in the packed layout of the CUDA library.
 
     K, V: uint16 [B][L][H][n][d]; Q: uint16 [B][L][Hq][w][d] (may be None when
@@ -213,7 +219,7 @@ def compress(K, V, Q, *, B: int, L: int, Hq: int, H: int, n: int, d: int, w: int
     if scale == 0.0:
         scale = 1.0 / np.sqrt(d)
     cfg = np.array([B, L, Hq, H, n, d, w, pool, protect, alpha_num, alpha_den, T,
-                    statistic, tail_slot], dtype=np.int32)
+                    statistic, tail_slot, allocator], dtype=np.int32)
     slots = B * L * B_live
     out = dict(
         a=np.empty((units, n), np.float64), perm=np.empty((units, n), np.int32),

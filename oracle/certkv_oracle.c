@@ -27,7 +27,9 @@
  *        one from the head with the smallest c(b-1) - c(b);
  *   R-A10 the tail slot stores the centroids k* = sum a k / m, v* = sum a v / m;
  *   R-A11 if m == 0 in floating point the slot is the uniform tail mean;
- *   R-A12 the tail slot enters decode as a plain key/value pair (no logit bias).
+ *   R-A12 the tail slot enters decode as a plain key/value pair (no logit bias);
+ *   R-A15 / R-A16 the "true uniform" and "greedy marginal" allocator ablations
+ *        (see oracle_allocate_mode).
  *
  * Build: cc -O2 -ffp-contract=off -fPIC -shared (no fused multiply-add, so that
  * x86 and Arm builds round identically).
@@ -209,12 +211,37 @@ static int argmin_penalised(const double* c, int lo, int hi, double lambda) {
  * when one tail slot per head is charged).  Writes b[H]; *repairs = number of
  * one-token repairs.  Returns 0, or 2 if the budget is infeasible.
  */
+int oracle_allocate_mode(const double* const* curves, int H, int n, int64_t B_real,
+                         int64_t alpha_num, int64_t alpha_den, int T, int mode, int32_t* b,
+                         int64_t* repairs);
+
 int oracle_allocate(const double* const* curves, int H, int n, int64_t B_real,
                     int64_t alpha_num, int64_t alpha_den, int T, int32_t* b,
                     int64_t* repairs) {
+  return oracle_allocate_mode(curves, H, n, B_real, alpha_num, alpha_den, T, 0, b, repairs);
+}
+
+/*
+ * The one-factor allocator ablations (ablation table, "Allocator" block),
+ * with `mode`:
+ *   0  Lagrangian bisection + repair (the method, above);
+ *   1  true uniform: READING R-A15, b_h = floor(B_real / H), the remainder
+ *      going one token each to the lowest-index heads;
+ *   2  greedy marginal: READING R-A16, every head starts at b_min and the
+ *      repair rule above (smallest c_h(b_h+1) - c_h(b_h), lowest head on
+ *      ties) adds one token at a time until B_real.
+ */
+int oracle_allocate_mode(const double* const* curves, int H, int n, int64_t B_real,
+                         int64_t alpha_num, int64_t alpha_den, int T, int mode, int32_t* b,
+                         int64_t* repairs) {
   const int64_t bmin = oracle_b_min(B_real, H, alpha_num, alpha_den);
   if (B_real < (int64_t)H * bmin || B_real > (int64_t)H * (n - 1)) return 2;
   const int lo_b = (int)bmin, hi_b = n - 1;
+  if (mode == 1) {
+    for (int h = 0; h < H; ++h) b[h] = (int32_t)(B_real / H + (h < B_real % H ? 1 : 0));
+    if (repairs) *repairs = 0;
+    return 0;
+  }
 
   double cmax = 0.0;
   for (int h = 0; h < H; ++h)
@@ -222,16 +249,22 @@ int oracle_allocate(const double* const* curves, int H, int n, int64_t B_real,
       if (curves[h][bb] > cmax) cmax = curves[h][bb];
   double lam_lo = 0.0, lam_hi = 2.0 * cmax + 1.0;
 
-  for (int t = 0; t < T; ++t) {
-    const double lam = (lam_lo + lam_hi) / 2.0;
-    int64_t total = 0;
-    for (int h = 0; h < H; ++h) total += argmin_penalised(curves[h], lo_b, hi_b, lam);
-    if (total > B_real) lam_lo = lam; else lam_hi = lam;
-  }
   int64_t total = 0;
-  for (int h = 0; h < H; ++h) {
-    b[h] = argmin_penalised(curves[h], lo_b, hi_b, lam_hi);
-    total += b[h];
+  if (mode == 2) {
+    for (int h = 0; h < H; ++h) b[h] = lo_b;
+    total = (int64_t)H * lo_b;
+  } else {
+    for (int t = 0; t < T; ++t) {
+      const double lam = (lam_lo + lam_hi) / 2.0;
+      total = 0;
+      for (int h = 0; h < H; ++h) total += argmin_penalised(curves[h], lo_b, hi_b, lam);
+      if (total > B_real) lam_lo = lam; else lam_hi = lam;
+    }
+    total = 0;
+    for (int h = 0; h < H; ++h) {
+      b[h] = argmin_penalised(curves[h], lo_b, hi_b, lam_hi);
+      total += b[h];
+    }
   }
   int64_t steps = 0;
   while (total < B_real) { /* best-marginal repair: add one token */
@@ -312,7 +345,7 @@ double oracle_tail(const double* a, const uint16_t* K, const uint16_t* V,
 typedef struct {
   int B, L, Hq, H, n, d, w;
   double scale;
-  int pool, protect, alpha_num, alpha_den, T, statistic, tail_slot;
+  int pool, protect, alpha_num, alpha_den, T, statistic, tail_slot, allocator;
   int64_t B_live;
 } oracle_cfg;
 
@@ -366,8 +399,9 @@ static void* worker(void* arg) {
       const double* curves[64];
       for (int h = 0; h < g->H; ++h) curves[h] = jb->c + ((size_t)bl * g->H + h) * n;
       const int64_t B_real = g->B_live - (g->tail_slot ? g->H : 0);
-      int rc = oracle_allocate(curves, g->H, g->n, B_real, g->alpha_num, g->alpha_den,
-                               g->T, jb->counts + (size_t)bl * g->H, jb->repairs + bl);
+      int rc = oracle_allocate_mode(curves, g->H, g->n, B_real, g->alpha_num, g->alpha_den,
+                                    g->T, g->allocator, jb->counts + (size_t)bl * g->H,
+                                    jb->repairs + bl);
       for (int h = 0; h < g->H; ++h) jb->status[bl * g->H + h] = rc;
     }
   } else { /* tail per unit */
@@ -398,7 +432,8 @@ static void run_phase(job_t* jb, int phase, int threads) {
 /*
  * The whole compression pass over B*L*H units plus the packed cache, in the
  * library's packed layout.  cfg_i holds {B, L, Hq, H, n, d, w, pool, protect,
- * alpha_num, alpha_den, T, statistic, tail_slot}; scale and B_live separately.
+ * alpha_num, alpha_den, T, statistic, tail_slot, allocator}; scale and B_live
+ * separately.
  * a_in (fp32 [units][n]) may be NULL; when given, scoring is skipped and the
  * pass starts from these scores (conditioned mode).  Outputs (all required):
  *   a [units][n], perm [units][n], c [units][n], counts [units],
@@ -417,7 +452,7 @@ int oracle_compress(const int32_t* cfg_i, double scale, int64_t B_live,
   g.B = cfg_i[0]; g.L = cfg_i[1]; g.Hq = cfg_i[2]; g.H = cfg_i[3]; g.n = cfg_i[4];
   g.d = cfg_i[5]; g.w = cfg_i[6]; g.pool = cfg_i[7]; g.protect = cfg_i[8];
   g.alpha_num = cfg_i[9]; g.alpha_den = cfg_i[10]; g.T = cfg_i[11];
-  g.statistic = cfg_i[12]; g.tail_slot = cfg_i[13];
+  g.statistic = cfg_i[12]; g.tail_slot = cfg_i[13]; g.allocator = cfg_i[14];
   g.scale = scale; g.B_live = B_live;
   if (g.H > 64) return 1;
   const int units = g.B * g.L * g.H;

@@ -34,7 +34,8 @@ class certkv_params(ctypes.Structure):
     _fields_ = [("scale", ctypes.c_float), ("pool_kernel", ctypes.c_int32),
                 ("protect_window", ctypes.c_int32), ("alpha_num", ctypes.c_int32),
                 ("alpha_den", ctypes.c_int32), ("bisect_steps", ctypes.c_int32),
-                ("statistic", ctypes.c_int32), ("tail_slot", ctypes.c_int32)]
+                ("statistic", ctypes.c_int32), ("tail_slot", ctypes.c_int32),
+                ("allocator", ctypes.c_int32)]
 
 
 class certkv_packed(ctypes.Structure):

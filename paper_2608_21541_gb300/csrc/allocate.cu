@@ -21,6 +21,7 @@
 #include <float.h>
 #include <limits.h>
 
+#include "../../include/certkv.h"
 #include "common.cuh"
 #include "internal.cuh"
 
@@ -224,14 +225,16 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
       mx = v > mx ? v : mx;
       coff[h] = acc;
       const int32_t* nc = ncand + (size_t)(bl * H + h) * stride + p.hull_segs;
-      for (int g = 0; g < groups; ++g) acc += nc[g];
+      if (p.allocator == CERTKV_ALLOC_LAGRANGIAN)  // the hull filter ran only for it
+        for (int g = 0; g < groups; ++g) acc += nc[g];
     }
     coff[H] = acc;
     lam_sh[0] = 0.0;
     lam_sh[1] = __dadd_rn(__dmul_rn(2.0, mx), 1.0);
   }
   __syncthreads();
-  const bool staged = coff[H] <= kCandCap;
+  const bool lagrangian = p.allocator == CERTKV_ALLOC_LAGRANGIAN;
+  const bool staged = lagrangian && coff[H] <= kCandCap;
   if (staged) {  // gather the group survivors of every head, in order; warp per (head, group)
     for (int hg = warp; hg < H * groups; hg += nwarps) {
       const int h = hg / groups, g = hg - h * groups;
@@ -305,7 +308,7 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
   // double-float on every warp
   if (threadIdx.x == 0) lam_df = df_from_double(__dmul_rn(__dadd_rn(lam_sh[0], lam_sh[1]), 0.5));
   __syncthreads();
-  for (int t = 0; t < p.T; ++t) {
+  for (int t = 0; lagrangian && t < p.T; ++t) {
     argmin_heads();
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -320,7 +323,14 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
   }
   if (p.T == 0 && threadIdx.x == 0) lam_df = df_from_double(lam_sh[1]);
   __syncthreads();
-  argmin_heads();
+  if (lagrangian) {
+    argmin_heads();
+  } else if (threadIdx.x < H) {  // the allocator ablations' starting points
+    const int h = threadIdx.x;
+    bsel[h] = (p.allocator == CERTKV_ALLOC_UNIFORM)
+                  ? (int)(B_real / H + (h < B_real % H ? 1 : 0))  // already sums to B_real
+                  : p.b_min;  // greedy: the repair below adds the rest
+  }
   __syncthreads();
 
   if (warp == 0) {
@@ -500,6 +510,7 @@ void launch_allocate(const Prob& p, const Layout& ly, char* ws, int32_t* counts,
   int32_t* cand = reinterpret_cast<int32_t*>(ws + ly.cand);
   int32_t* ncand = reinterpret_cast<int32_t*>(ws + ly.ncand);
   const int groups = (p.hull_segs + kGroupSegs - 1) / kGroupSegs;
+  if (p.allocator == CERTKV_ALLOC_LAGRANGIAN) {  // candidates for the bisection only
   {
     TraceScope ts_("hull_seg", st);
     hull_seg_kernel<<<dim3((p.hull_segs + 127) / 128, p.units), 128, 0, st>>>(p, curve, cand,
@@ -508,6 +519,7 @@ void launch_allocate(const Prob& p, const Layout& ly, char* ws, int32_t* counts,
   {
     TraceScope ts_("hull_group", st);
     hull_group_kernel<<<dim3((groups + 127) / 128, p.units), 128, 0, st>>>(p, curve, cand, ncand);
+  }
   }
   {
     TraceScope ts_("bisect_repair", st);

@@ -37,6 +37,7 @@ int check_params(const certkv_params* q) {
   if (q->bisect_steps < 0 || q->bisect_steps > 200) return CERTKV_EINVAL;
   if (q->statistic < 0 || q->statistic > 2) return CERTKV_EINVAL;
   if (q->tail_slot != 0 && q->tail_slot != 1) return CERTKV_EINVAL;
+  if (q->allocator < CERTKV_ALLOC_LAGRANGIAN || q->allocator > CERTKV_ALLOC_GREEDY) return CERTKV_EINVAL;
   return CERTKV_OK;
 }
 
@@ -56,7 +57,7 @@ int make_prob(const certkv_shape* s, const certkv_params* q, int64_t budget_live
   P.scale_log2 = P.scale * 1.4426950408889634f;
   P.pool = q->pool_kernel; P.protect = q->protect_window;
   P.alpha_num = q->alpha_num; P.alpha_den = q->alpha_den; P.T = q->bisect_steps;
-  P.statistic = q->statistic; P.tail_slot = q->tail_slot;
+  P.statistic = q->statistic; P.tail_slot = q->tail_slot; P.allocator = q->allocator;
   P.score_warps = (P.R + 15) / 16 < 16 ? (P.R + 15) / 16 : 16;
   P.row_blocks = (P.R + 16 * P.score_warps - 1) / (16 * P.score_warps);
   if (score_tc_supported(P)) P.row_blocks = P.R / 64;  // one per 64-row quarter of the tcgen05 pass 2
@@ -191,6 +192,7 @@ void certkv_default_params(certkv_params* p) {
   p->bisect_steps = 40;
   p->statistic = CERTKV_STAT_CENTERED;
   p->tail_slot = 1;
+  p->allocator = CERTKV_ALLOC_LAGRANGIAN;
 }
 
 int64_t certkv_live_budget(int32_t n, int32_t hkv, int64_t keep_num, int64_t keep_den) {

@@ -17,6 +17,7 @@ struct Prob {
   float scale_log2;                // scale * log2(e)
   int pool, protect;
   int alpha_num, alpha_den, T, statistic, tail_slot;
+  int allocator;  // CERTKV_ALLOC_*
   int64_t B_live, B_real;
   int b_min;
   int64_t slot_base;  // packed slot of this problem's first (sequence, layer): offsets are global

@@ -264,6 +264,47 @@ def pin_allocation_equalities_and_optimality(lib=None):
                 assert obj >= best - 1e-12
 
 
+def pin_allocator_true_uniform(lib=None):
+    """Allocator ablation "true uniform" (reading R-A15): the budget split as
+    evenly as integers allow, the remainder to the lowest heads, whatever the
+    curves."""
+    rng = np.random.default_rng(21)
+    for H, n, B_real in ((3, 9, 7), (4, 20, 40), (5, 6, 25), (2, 33, 2)):
+        curves = rng.uniform(0, 5, size=(H, n))
+        b, rep = oracle.allocate(curves, B_real, 1, 5, 40, mode=1, lib=lib)
+        assert b.sum() == B_real and rep == 0
+        assert b.max() - b.min() <= 1
+        assert all(b[h] >= b[h + 1] for h in range(H - 1)), b  # extra tokens go to low heads
+
+
+def pin_allocator_greedy_marginal(lib=None):
+    """Allocator ablation "greedy marginal" (reading R-A16): from b_min, one
+    token at a time to the smallest marginal.  For separable convex curves
+    greedy marginal allocation is optimal (textbook resource allocation), so
+    it must match the exhaustive optimum; on the hand-worked non-convex pair
+    it takes c_0's two steepest marginals first, then the tie -0.5 / -0.5 goes
+    to head 0: b = [4, 1] after 3 single-token steps."""
+    rng = np.random.default_rng(5)
+    H, n = 3, 8
+    for _ in range(6):
+        steps = -np.sort(rng.uniform(0.05, 1.0, size=(H, n - 1)), axis=1)[:, ::-1]
+        curves = np.concatenate([np.full((H, 1), 10.0), 10.0 + np.cumsum(steps, 1)], 1)
+        for B_real in (H, 8, 13, H * (n - 1)):
+            bmin = oracle.b_min(B_real, H, 1, 5, lib=lib)
+            b, _ = oracle.allocate(curves, B_real, 1, 5, 40, mode=2, lib=lib)
+            assert b.sum() == B_real and (b >= bmin).all()
+            _, arg = _brute_force(curves, B_real, bmin)
+            assert list(b) == list(arg), (b, arg)
+    c = np.array([[10, 6, 4, 3, 2.5, 2.2], [9, 8, 7.5, 3, 2, 1.9]], float)
+    b, rep = oracle.allocate(c, 5, 1, 5, 40, mode=2, lib=lib)
+    assert b.tolist() == [4, 1] and rep == 3, (b, rep)
+    # the safeguard binds: b_min = floor(30 / (5 * 2)) = 3, and head 1 is flat,
+    # so greedy keeps it at exactly b_min and gives head 0 the other 27
+    c = np.stack([100.0 - np.arange(40.0), np.full(40, 5.0)])
+    b, rep = oracle.allocate(c, 30, 1, 5, 40, mode=2, lib=lib)
+    assert b.tolist() == [27, 3], b
+
+
 def pin_allocation_infeasible(lib=None):
     """B_real above H (n - 1) cannot be met with b_h <= n - 1."""
     curves = np.ones((2, 5))

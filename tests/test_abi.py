@@ -99,6 +99,8 @@ def test_host_validation_errors(lib):
     assert _call_compress(lib, s, 2 * H, params=bad) == ck.EINVAL
     bad = ck.certkv_default_params(statistic=3)
     assert _call_compress(lib, s, 2 * H, params=bad) == ck.EINVAL
+    bad = ck.certkv_default_params(allocator=3)
+    assert _call_compress(lib, s, 2 * H, params=bad) == ck.EINVAL
     # without a tail slot the smallest budget is H
     ns = ck.certkv_default_params(tail_slot=0)
     assert _call_compress(lib, s, H - 1, params=ns) == ck.EBUDGET

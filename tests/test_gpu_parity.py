@@ -52,7 +52,8 @@ def run_case(name, wl=None, params=None, B_live=None, seed=0):
     kw = dict(B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, n=wl.n, d=wl.d, w=wl.w, B_live=B_live,
               scale=params.scale, pool=params.pool_kernel, protect=params.protect_window,
               alpha_num=params.alpha_num, alpha_den=params.alpha_den, T=params.bisect_steps,
-              statistic=params.statistic, tail_slot=params.tail_slot)
+              statistic=params.statistic, tail_slot=params.tail_slot,
+              allocator=params.allocator)
     ref_e2e = oracle.compress(host["K"], host["V"], host["Q"], **kw)
     ref_cond = oracle.compress(host["K"], host["V"], None, a_in=host["a"], **kw)
     res = dict(wl=wl, params=params, B_live=B_live, K=K, V=V, Q=Q, a=a, packed=packed,
@@ -128,6 +129,8 @@ VARIANTS = {
     "alpha04": dict(alpha_num=2, alpha_den=5),
     "no_pool_no_protect": dict(pool_kernel=1, protect_window=0),
     "pool7_scale": dict(pool_kernel=7, scale=0.05),
+    "allocator_uniform": dict(allocator=1),
+    "allocator_greedy": dict(allocator=2),
 }
 
 

@@ -34,6 +34,9 @@ MUTANTS = {
                                 "    const int j = perm[r];\n    m += a[j];"),
     "repair_largest_marginal": ("if (best_h < 0 || delta < best) { best = delta; best_h = h; }",
                                 "if (best_h < 0 || delta > best) { best = delta; best_h = h; }"),
+    "uniform_remainder_to_high_heads": ("(h < B_real % H ? 1 : 0)", "(h >= H - B_real % H ? 1 : 0)"),
+    "greedy_ignores_safeguard": ("for (int h = 0; h < H; ++h) b[h] = lo_b;",
+                                 "for (int h = 0; h < H; ++h) b[h] = 1;"),
     "bisection_inverted": ("if (total > B_real) lam_lo = lam; else lam_hi = lam;",
                            "if (total > B_real) lam_hi = lam; else lam_lo = lam;"),
     "kept_not_sorted": ("qsort(kept, (size_t)b, sizeof(int32_t), cmp_int32);", ""),
