@@ -106,7 +106,13 @@ typedef struct {
   int32_t tail_slot;      /* 1 (default): one synthetic tail slot per head is charged
                              to the budget; 0: no slot, the slot goes to a real token */
   int32_t allocator;      /* CERTKV_ALLOC_* (default CERTKV_ALLOC_LAGRANGIAN)          */
+  int32_t tail_clusters;  /* m >= 0 (default 0): cluster summaries of each head's evicted
+                             tail, for certkv_decode_certified; each costs one slot of
+                             the budget (B_real = B_live - H (tail_slot + m)); at most
+                             CERTKV_MAX_CLUSTERS                                       */
 } certkv_params;
+
+#define CERTKV_MAX_CLUSTERS 64
 
 /* Cross-head allocator (paper: one-factor ablations, "Allocator" block).  The
  * paper names the two ablations without defining them; the readings used:
@@ -120,8 +126,12 @@ typedef struct {
 
 /* Ragged packed cache.  Segment u (one per unit) holds real_counts[u] real
  * slots in ascending original position followed, when params.tail_slot = 1,
- * by the tail slot; offsets[u] is its first slot.  Each (sequence, layer)
- * owns exactly B_live consecutive slots: offsets[(b*L+l)*H] = (b*L+l)*B_live. */
+ * by the tail slot, then, when params.tail_clusters = m > 0, by m cluster
+ * summary slots (positions -2 - g; k, v = the bf16-rounded unweighted means of
+ * cluster g of the evicted ranks, which is ranks b + floor(g T / m) ..
+ * b + floor((g + 1) T / m) - 1 with T = n - b); offsets[u] is its first slot.
+ * Each (sequence, layer) owns exactly B_live consecutive slots:
+ * offsets[(b*L+l)*H] = (b*L+l)*B_live. */
 typedef struct {
   void*    k;               /* bf16 [capacity_slots][d]                          */
   void*    v;               /* bf16 [capacity_slots][d]                          */
@@ -132,6 +142,10 @@ typedef struct {
   float*   tail_f32;        /* optional (NULL = skip) [B*L*H][2][d]: k*, v* in fp32
                                before rounding to bf16                            */
   double*  tail_mass;       /* optional (NULL = skip) [B*L*H]: m_h(b_h)          */
+  float*   cluster_meta;    /* with params.tail_clusters = m > 0 (else NULL):
+                               [B*L*H][m][4] = (count n_g, key radius R_g, value
+                               radius rho_g, 0) of each cluster summary slot     */
+  float*   kept_vmax;       /* with m > 0: [B*L*H] largest ||v|| of the real slots */
 } certkv_packed;
 
 /* Fill `p` with the defaults listed above.  Host call. */
@@ -215,6 +229,25 @@ int certkv_decode_attn(const certkv_shape* shape, const void* q,
                        const certkv_packed* packed, float scale, int32_t tail_slot,
                        void* out, void* workspace, size_t workspace_bytes,
                        void* stream);
+
+/* Clustered-tail decode with its runtime output-error bound (appendix:
+ * deterministic output-error bound for clustered tail summaries, theorem and
+ * runtime remark).  For each query head: O-hat = (sum over the real slots of
+ * e^l v + sum_g n_g e^{lbar_g} vbar_g) / Z-hat with lbar_g = scale <q, kbar_g>
+ * (the plain tail slot, if present, is not used), and
+ * bound = (3 / Z-hat) (D_N + V'max D_Z), D_Z = sum_g (e^{r_g} - 1) e^{r_g} Zhat_g,
+ * D_N = sum_g e^{r_g} Zhat_g ((e^{r_g} - 1) ||vbar_g|| + rho_g),
+ * V'max = max(kept_vmax, max_g ||vbar_g|| + rho_g), with logit radius
+ * r_g = scale ||q|| R_g (Cauchy-Schwarz).  certified = 1 when D_Z <= Z-hat / 3,
+ * the condition under which ||O-hat - O|| <= bound for exact attention O over
+ * every original token.  packed comes from a compression with
+ * params.tail_clusters = clusters and params.tail_slot = tail_slot.
+ * out: bf16 [B][L][Hq][d]; bound: fp32 [B][L][Hq]; certified: int32 [B][L][Hq].
+ * Workspace: certkv_decode_workspace_bytes(shape). */
+int certkv_decode_certified(const certkv_shape* shape, const void* q, const certkv_packed* packed,
+                            float scale, int32_t tail_slot, int32_t clusters, void* out,
+                            float* bound, int32_t* certified, void* workspace,
+                            size_t workspace_bytes, void* stream);
 
 /* Decode attention that allocates nothing.  The paper has no counterpart: this
  * entry point exists for callers that cannot hand the library a scratch

@@ -58,7 +58,11 @@ def _bind(lib):
     lib.oracle_select.restype = None
     lib.oracle_tail.argtypes = [P, P, P, P, I, I, I, P, P, P]
     lib.oracle_tail.restype = D
-    lib.oracle_compress.argtypes = [P, D, I64, P, P, P, P, I] + [P] * 11
+    lib.oracle_compress.argtypes = [P, D, I64, P, P, P, P, I] + [P] * 13
+    lib.oracle_tail_clusters.argtypes = [P, P, P, I, I, I, I, P, P, P, P, P, P]
+    lib.oracle_tail_clusters.restype = None
+    lib.oracle_decode_certified.argtypes = [P, P, P, I, I, D, P, P, P, P, P, I, P, P, P]
+    lib.oracle_decode_certified.restype = D
     lib.oracle_compress.restype = I
     lib.oracle_decode.argtypes = [P, D, P, P, P, P, P, I, P]
     lib.oracle_decode.restype = None
@@ -201,8 +205,8 @@ def tail(a, K, V, perm, b: int, *, lib=None):
 def compress(K, V, Q, *, B: int, L: int, Hq: int, H: int, n: int, d: int, w: int,
              B_live: int, scale: float = 0.0, pool: int = 5, protect: int = 1,
              alpha_num: int = 1, alpha_den: int = 5, T: int = 40, statistic: int = 0,
-             tail_slot: int = 1, allocator: int = 0, a_in=None, threads: int | None = None,
-             lib=None) -> dict:
+             tail_slot: int = 1, allocator: int = 0, clusters: int = 0, a_in=None,
+             threads: int | None = None, lib=None) -> dict:
     """The whole compression pass in the packed layout of the CUDA library.
 
     K, V: uint16 [B][L][H][n][d]; Q: uint16 [B][L][Hq][w][d] (may be None when
@@ -219,7 +223,7 @@ def compress(K, V, Q, *, B: int, L: int, Hq: int, H: int, n: int, d: int, w: int
     if scale == 0.0:
         scale = 1.0 / np.sqrt(d)
     cfg = np.array([B, L, Hq, H, n, d, w, pool, protect, alpha_num, alpha_den, T,
-                    statistic, tail_slot, allocator], dtype=np.int32)
+                    statistic, tail_slot, allocator, clusters], dtype=np.int32)
     slots = B * L * B_live
     out = dict(
         a=np.empty((units, n), np.float64), perm=np.empty((units, n), np.int32),
@@ -227,7 +231,9 @@ def compress(K, V, Q, *, B: int, L: int, Hq: int, H: int, n: int, d: int, w: int
         offsets=np.empty(units + 1, np.int64), positions=np.empty(slots, np.int32),
         pk=np.empty((slots, d), np.uint16), pv=np.empty((slots, d), np.uint16),
         tail=np.zeros((units, 2, d), np.float64), tail_mass=np.zeros(units, np.float64),
-        repairs=np.zeros(B * L, np.int64))
+        repairs=np.zeros(B * L, np.int64),
+        cl_meta=np.zeros((units, max(clusters, 1), 3), np.float64),
+        kept_vmax=np.zeros(units, np.float64))
     if threads is None:
         threads = os.cpu_count() or 1
     rc = (lib or _load()).oracle_compress(
@@ -235,12 +241,44 @@ def compress(K, V, Q, *, B: int, L: int, Hq: int, H: int, n: int, d: int, w: int
         _ptr(a_in) if a_in is not None else None, int(threads),
         _ptr(out["a"]), _ptr(out["perm"]), _ptr(out["c"]), _ptr(out["counts"]),
         _ptr(out["offsets"]), _ptr(out["positions"]), _ptr(out["pk"]), _ptr(out["pv"]),
-        _ptr(out["tail"]), _ptr(out["tail_mass"]), _ptr(out["repairs"]))
+        _ptr(out["tail"]), _ptr(out["tail_mass"]), _ptr(out["repairs"]),
+        _ptr(out["cl_meta"]), _ptr(out["kept_vmax"]))
     if rc == 2:
         raise ValueError("infeasible budget")
     out["zero_tail"] = bool(rc & 0x100)
     out["threads"] = threads
     return out
+
+
+def tail_clusters(K, V, perm, b: int, m: int, *, lib=None):
+    """Cluster summaries of the evicted ranks b..n-1 of one unit.  K, V uint16
+    [n][d]; perm int32 [n].  Returns (kbar bits [m][d], vbar bits [m][d],
+    count [m], key radius [m], value radius [m], kept value-norm max)."""
+    K = _u16(K); V = _u16(V)
+    n, d = K.shape
+    perm = np.ascontiguousarray(perm, dtype=np.int32)
+    kb = np.zeros((m, d), np.uint16); vb = np.zeros((m, d), np.uint16)
+    cnt = np.zeros(m, np.int32); rk = np.zeros(m); rv = np.zeros(m); vm = np.zeros(1)
+    (lib or _load()).oracle_tail_clusters(_ptr(K), _ptr(V), _ptr(perm), n, d, int(b), int(m),
+                                          _ptr(kb), _ptr(vb), _ptr(cnt), _ptr(rk), _ptr(rv),
+                                          _ptr(vm))
+    return kb, vb, cnt, rk, rv, float(vm[0])
+
+
+def decode_certified(q, pk, pv, kbar, vbar, count, rk, rv, *, scale: float, lib=None):
+    """Certified decode of one query head: q uint16 [d]; kept rows pk, pv uint16
+    [b][d]; clusters as from tail_clusters.  Returns (O-hat [d], bound,
+    certified, structural form)."""
+    q = _u16(q); pk = _u16(pk); pv = _u16(pv); kbar = _u16(kbar); vbar = _u16(vbar)
+    b, d = pk.shape if pk.size else (0, q.shape[0])
+    m = kbar.shape[0]
+    count = np.ascontiguousarray(count, dtype=np.int32)
+    rk = np.ascontiguousarray(rk, dtype=np.float64); rv = np.ascontiguousarray(rv, dtype=np.float64)
+    out = np.zeros(d); cert = np.zeros(1, np.int32); struct = np.zeros(1)
+    bound = (lib or _load()).oracle_decode_certified(
+        _ptr(q), _ptr(pk), _ptr(pv), int(b), int(d), float(scale), _ptr(kbar), _ptr(vbar),
+        _ptr(count), _ptr(rk), _ptr(rv), int(m), _ptr(out), _ptr(cert), _ptr(struct))
+    return out, float(bound), bool(cert[0]), float(struct[0])
 
 
 def decode(q, pk, pv, offsets, counts, *, B: int, L: int, Hq: int, H: int, d: int,

@@ -340,12 +340,16 @@ double oracle_tail(const double* a, const uint16_t* K, const uint16_t* V,
   return m;
 }
 
+void oracle_tail_clusters(const uint16_t* K, const uint16_t* V, const int32_t* perm, int n, int d,
+                          int b, int m, uint16_t* kbar_bits, uint16_t* vbar_bits,
+                          int32_t* count, double* rk, double* rv, double* kept_vmax);
+
 /* -------------------------------------------------------- whole pass ----- */
 
 typedef struct {
   int B, L, Hq, H, n, d, w;
   double scale;
-  int pool, protect, alpha_num, alpha_den, T, statistic, tail_slot, allocator;
+  int pool, protect, alpha_num, alpha_den, T, statistic, tail_slot, allocator, clusters;
   int64_t B_live;
 } oracle_cfg;
 
@@ -398,7 +402,8 @@ static void* worker(void* arg) {
     for (int bl; (bl = take(jb, g->B * g->L)) >= 0;) {
       const double* curves[64];
       for (int h = 0; h < g->H; ++h) curves[h] = jb->c + ((size_t)bl * g->H + h) * n;
-      const int64_t B_real = g->B_live - (g->tail_slot ? g->H : 0);
+      /* every head is charged its tail slot and its cluster summaries */
+      const int64_t B_real = g->B_live - (int64_t)g->H * ((g->tail_slot ? 1 : 0) + g->clusters);
       int rc = oracle_allocate_mode(curves, g->H, g->n, B_real, g->alpha_num, g->alpha_den,
                                     g->T, g->allocator, jb->counts + (size_t)bl * g->H,
                                     jb->repairs + bl);
@@ -432,8 +437,11 @@ static void run_phase(job_t* jb, int phase, int threads) {
 /*
  * The whole compression pass over B*L*H units plus the packed cache, in the
  * library's packed layout.  cfg_i holds {B, L, Hq, H, n, d, w, pool, protect,
- * alpha_num, alpha_den, T, statistic, tail_slot, allocator}; scale and B_live
- * separately.
+ * alpha_num, alpha_den, T, statistic, tail_slot, allocator, clusters}; scale and
+ * B_live separately.  With clusters = m > 0 each segment ends with m summary
+ * slots (stored representatives, positions -2 - g), cl_meta [units][m][3]
+ * receives (count, key radius, value radius) and kept_vmax [units] the largest
+ * kept value norm (both may be NULL when m = 0).
  * a_in (fp32 [units][n]) may be NULL; when given, scoring is skipped and the
  * pass starts from these scores (conditioned mode).  Outputs (all required):
  *   a [units][n], perm [units][n], c [units][n], counts [units],
@@ -447,12 +455,14 @@ int oracle_compress(const int32_t* cfg_i, double scale, int64_t B_live,
                     const float* a_in, int threads,
                     double* a, int32_t* perm, double* c, int32_t* counts,
                     int64_t* offsets, int32_t* positions, uint16_t* pk, uint16_t* pv,
-                    double* tail, double* tail_mass, int64_t* repairs) {
+                    double* tail, double* tail_mass, int64_t* repairs,
+                    double* cl_meta, double* kept_vmax) {
   oracle_cfg g;
   g.B = cfg_i[0]; g.L = cfg_i[1]; g.Hq = cfg_i[2]; g.H = cfg_i[3]; g.n = cfg_i[4];
   g.d = cfg_i[5]; g.w = cfg_i[6]; g.pool = cfg_i[7]; g.protect = cfg_i[8];
   g.alpha_num = cfg_i[9]; g.alpha_den = cfg_i[10]; g.T = cfg_i[11];
   g.statistic = cfg_i[12]; g.tail_slot = cfg_i[13]; g.allocator = cfg_i[14];
+  g.clusters = cfg_i[15];
   g.scale = scale; g.B_live = B_live;
   if (g.H > 64) return 1;
   const int units = g.B * g.L * g.H;
@@ -499,6 +509,23 @@ int oracle_compress(const int32_t* cfg_i, double scale, int64_t B_live,
       positions[off] = -1;
       off += 1;
     }
+    if (g.clusters > 0) {  /* the m summary slots (clustered-tail certificate) */
+      const int m = g.clusters;
+      int32_t* cnt = (int32_t*)malloc((size_t)m * sizeof(int32_t));
+      double* rk = (double*)malloc((size_t)m * 2 * sizeof(double));
+      oracle_tail_clusters(K + (size_t)u * n * d, V + (size_t)u * n * d, perm + (size_t)u * n,
+                           g.n, g.d, bu, m, pk + (size_t)off * d, pv + (size_t)off * d, cnt, rk,
+                           rk + m, kept_vmax + u);
+      for (int c = 0; c < m; ++c) {
+        positions[off + c] = -2 - c;
+        cl_meta[((size_t)u * m + c) * 3 + 0] = (double)cnt[c];
+        cl_meta[((size_t)u * m + c) * 3 + 1] = rk[c];
+        cl_meta[((size_t)u * m + c) * 3 + 2] = rk[m + c];
+      }
+      off += m;
+      free(cnt);
+      free(rk);
+    }
   }
   offsets[units] = (int64_t)g.B * g.L * g.B_live;
   free(kept);
@@ -542,4 +569,147 @@ void oracle_decode(const int32_t* cfg_i, double scale, const uint16_t* q,
       free(lg);
     }
   }
+}
+
+/* ------------------------------------------- clustered tail summaries ---- */
+
+/*
+ * Summaries of the evicted ranks b..n-1 of one unit for the clustered-tail
+ * output-error bound (appendix: deterministic output-error bound for
+ * clustered tail summaries, Eq. (cluster-summaries), (cluster-radii)).
+ * READING R-C1: m groups of consecutive ranks, group g = ranks
+ * b + floor(g T / m) .. b + floor((g + 1) T / m) - 1 with T = n - b (an empty
+ * group has count 0).  READING R-C2: the representatives are the unweighted
+ * means of the group's keys and values, rounded to bf16 as they are stored
+ * (kbar_bits, vbar_bits [m][d]); the radii are the largest Euclidean distances
+ * of the group's rows to those stored representatives.  kept_vmax = max over
+ * the kept ranks 0..b-1 of ||v_j||_2.
+ */
+void oracle_tail_clusters(const uint16_t* K, const uint16_t* V, const int32_t* perm, int n, int d,
+                          int b, int m, uint16_t* kbar_bits, uint16_t* vbar_bits,
+                          int32_t* count, double* rk, double* rv, double* kept_vmax) {
+  const int T = n - b;
+  double* mk = (double*)malloc((size_t)d * sizeof(double));
+  double* mv = (double*)malloc((size_t)d * sizeof(double));
+  for (int g = 0; g < m; ++g) {
+    const int r0 = b + (int)(((int64_t)g * T) / m), r1 = b + (int)(((int64_t)(g + 1) * T) / m);
+    count[g] = r1 - r0;
+    for (int i = 0; i < d; ++i) { mk[i] = 0.0; mv[i] = 0.0; }
+    for (int r = r0; r < r1; ++r) {
+      const int j = perm[r];
+      for (int i = 0; i < d; ++i) {
+        mk[i] += bf16_to_f64(K[(size_t)j * d + i]);
+        mv[i] += bf16_to_f64(V[(size_t)j * d + i]);
+      }
+    }
+    for (int i = 0; i < d; ++i) {
+      const double ck = count[g] > 0 ? mk[i] / count[g] : 0.0;
+      const double cv = count[g] > 0 ? mv[i] / count[g] : 0.0;
+      kbar_bits[(size_t)g * d + i] = oracle_f64_to_bf16(ck);
+      vbar_bits[(size_t)g * d + i] = oracle_f64_to_bf16(cv);
+    }
+    double rkg = 0.0, rvg = 0.0;
+    for (int r = r0; r < r1; ++r) {
+      const int j = perm[r];
+      double sk = 0.0, sv = 0.0;
+      for (int i = 0; i < d; ++i) {
+        const double dk = bf16_to_f64(K[(size_t)j * d + i]) - bf16_to_f64(kbar_bits[(size_t)g * d + i]);
+        const double dv = bf16_to_f64(V[(size_t)j * d + i]) - bf16_to_f64(vbar_bits[(size_t)g * d + i]);
+        sk += dk * dk;
+        sv += dv * dv;
+      }
+      if (sqrt(sk) > rkg) rkg = sqrt(sk);
+      if (sqrt(sv) > rvg) rvg = sqrt(sv);
+    }
+    rk[g] = rkg;
+    rv[g] = rvg;
+  }
+  double vm = 0.0;
+  for (int r = 0; r < b; ++r) {
+    const int j = perm[r];
+    double s = 0.0;
+    for (int i = 0; i < d; ++i) s += bf16_to_f64(V[(size_t)j * d + i]) * bf16_to_f64(V[(size_t)j * d + i]);
+    if (sqrt(s) > vm) vm = sqrt(s);
+  }
+  *kept_vmax = vm;
+  free(mk);
+  free(mv);
+}
+
+/*
+ * Certified decode of one query head (Theorem: runtime-computable output-error
+ * bound for clustered tail summaries, Eq. (certificate-estimator),
+ * (certificate-quantities), (certificate-bound), (certificate-structure)).
+ * Kept set S = the b packed real rows pk, pv [b][d]; clusters g = 0..m-1 with
+ * stored representatives kbar, vbar (bf16 bits [m][d]), counts, key radii rk
+ * and value radii rv.  READING R-C3: the representative logit is
+ * scale <q, kbar_g> and the logit radius r_g = scale ||q||_2 rk_g
+ * (Cauchy-Schwarz, the paper's runtime remark).  Empty clusters are skipped.
+ * Writes O-hat [d]; returns the bound (3 / Zhat)(D_N + V'max D_Z); *certified
+ * = (D_Z <= Zhat / 3); *structural = the bound's structural form.  Every
+ * exponential is taken relative to one shift, to which the bound is invariant.
+ */
+double oracle_decode_certified(const uint16_t* q, const uint16_t* pk, const uint16_t* pv, int b,
+                               int d, double scale, const uint16_t* kbar, const uint16_t* vbar,
+                               const int32_t* count, const double* rk, const double* rv, int m,
+                               double* out, int* certified, double* structural) {
+  double qn = 0.0;
+  for (int i = 0; i < d; ++i) qn += bf16_to_f64(q[i]) * bf16_to_f64(q[i]);
+  qn = sqrt(qn);
+  double* lg = (double*)malloc((size_t)(b + m) * sizeof(double));
+  double M = -INFINITY;
+  for (int s = 0; s < b; ++s) {
+    double dot = 0.0;
+    for (int i = 0; i < d; ++i) dot += bf16_to_f64(q[i]) * bf16_to_f64(pk[(size_t)s * d + i]);
+    lg[s] = scale * dot;
+    if (lg[s] > M) M = lg[s];
+  }
+  for (int g = 0; g < m; ++g) {  /* log of n_g e^{lbar_g} */
+    double dot = 0.0;
+    for (int i = 0; i < d; ++i) dot += bf16_to_f64(q[i]) * bf16_to_f64(kbar[(size_t)g * d + i]);
+    lg[b + g] = count[g] > 0 ? scale * dot + log((double)count[g]) : -INFINITY;
+    if (lg[b + g] > M) M = lg[b + g];
+  }
+  double Z = 0.0, ZS = 0.0, DZ = 0.0, DN = 0.0, vmax = 0.0, smax = 0.0;
+  for (int i = 0; i < d; ++i) out[i] = 0.0;
+  for (int s = 0; s < b; ++s) {
+    const double w = exp(lg[s] - M);
+    Z += w;
+    ZS += w;
+    double vv = 0.0;
+    for (int i = 0; i < d; ++i) {
+      const double x = bf16_to_f64(pv[(size_t)s * d + i]);
+      out[i] += w * x;
+      vv += x * x;
+    }
+    if (sqrt(vv) > vmax) vmax = sqrt(vv);
+  }
+  for (int g = 0; g < m; ++g) {
+    if (count[g] <= 0) continue;
+    const double zg = exp(lg[b + g] - M);
+    const double r = scale * qn * rk[g];
+    const double er = exp(r);
+    double vn = 0.0;
+    for (int i = 0; i < d; ++i) {
+      const double x = bf16_to_f64(vbar[(size_t)g * d + i]);
+      out[i] += zg * x;
+      vn += x * x;
+    }
+    vn = sqrt(vn);
+    Z += zg;
+    DZ += (er - 1.0) * er * zg;
+    DN += er * zg * ((er - 1.0) * vn + rv[g]);
+    if (vn + rv[g] > vmax) vmax = vn + rv[g];
+  }
+  for (int i = 0; i < d; ++i) out[i] /= Z;
+  for (int g = 0; g < m; ++g) {
+    if (count[g] <= 0) continue;
+    const double er = exp(scale * qn * rk[g]);
+    const double t = er * (2.0 * vmax * (er - 1.0) + rv[g]);
+    if (t > smax) smax = t;
+  }
+  *certified = DZ <= Z / 3.0;
+  *structural = 3.0 * (1.0 - ZS / Z) * smax;
+  free(lg);
+  return 3.0 / Z * (DN + vmax * DZ);
 }

@@ -35,14 +35,15 @@ class certkv_params(ctypes.Structure):
                 ("protect_window", ctypes.c_int32), ("alpha_num", ctypes.c_int32),
                 ("alpha_den", ctypes.c_int32), ("bisect_steps", ctypes.c_int32),
                 ("statistic", ctypes.c_int32), ("tail_slot", ctypes.c_int32),
-                ("allocator", ctypes.c_int32)]
+                ("allocator", ctypes.c_int32), ("tail_clusters", ctypes.c_int32)]
 
 
 class certkv_packed(ctypes.Structure):
     _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("offsets", ctypes.c_void_p),
                 ("real_counts", ctypes.c_void_p), ("positions", ctypes.c_void_p),
                 ("capacity_slots", ctypes.c_int64), ("tail_f32", ctypes.c_void_p),
-                ("tail_mass", ctypes.c_void_p)]
+                ("tail_mass", ctypes.c_void_p), ("cluster_meta", ctypes.c_void_p),
+                ("kept_vmax", ctypes.c_void_p)]
 
 
 EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_bytes",
@@ -50,7 +51,7 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_compress_scored", "certkv_compress", "certkv_decode_attn",
             "certkv_read_status", "certkv_strerror", "certkv_trace_enable",
             "certkv_trace_report", "certkv_decode_attn_noalloc", "certkv_host_workspace_bytes",
-            "certkv_compress_host")
+            "certkv_compress_host", "certkv_decode_certified")
 
 _lock = threading.Lock()
 _lib = None
@@ -107,6 +108,9 @@ def load_library(path: Optional[str] = None):
         lib.certkv_host_workspace_bytes.restype = SZ
         lib.certkv_compress_host.argtypes = [sp, P, P, P, I64, pp, I32, kp, P, SZ, P]
         lib.certkv_compress_host.restype = ctypes.c_int
+        lib.certkv_decode_certified.argtypes = [sp, P, kp, ctypes.c_float, I32, I32, P, P, P, P,
+                                                SZ, P]
+        lib.certkv_decode_certified.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -208,18 +212,27 @@ class Packed:
     tail_f32: Optional[torch.Tensor] = None
     tail_mass: Optional[torch.Tensor] = None
     tail_slot: int = 1
+    clusters: int = 0
+    cluster_meta: Optional[torch.Tensor] = None  # fp32 [units][m][4]
+    kept_vmax: Optional[torch.Tensor] = None     # fp32 [units]
 
     def struct(self) -> certkv_packed:
         return certkv_packed(_ptr(self.k), _ptr(self.v), _ptr(self.offsets),
                              _ptr(self.real_counts), _ptr(self.positions), self.k.shape[0],
-                             _ptr(self.tail_f32), _ptr(self.tail_mass))
+                             _ptr(self.tail_f32), _ptr(self.tail_mass), _ptr(self.cluster_meta),
+                             _ptr(self.kept_vmax))
 
     @staticmethod
     def empty(B: int, L: int, H: int, d: int, B_live: int, device, with_tail: bool = False,
-              tail_slot: int = 1) -> "Packed":
+              tail_slot: int = 1, clusters: int = 0) -> "Packed":
         slots = B * L * B_live
         units = B * L * H
         return Packed(
+            clusters=clusters,
+            cluster_meta=(torch.empty((units, clusters, 4), dtype=torch.float32, device=device)
+                          if clusters else None),
+            kept_vmax=(torch.empty(units, dtype=torch.float32, device=device)
+                       if clusters else None),
             k=torch.empty((slots, d), dtype=torch.bfloat16, device=device),
             v=torch.empty((slots, d), dtype=torch.bfloat16, device=device),
             offsets=torch.empty(units + 1, dtype=torch.int64, device=device),
@@ -275,7 +288,7 @@ def certkv_compress_scored(K, V, a, budget_live: int, params=None, *, hq: Option
     shape = shape_of(K, None, hq=hq, w=w)
     if out is None:
         out = Packed.empty(shape.batch, shape.layers, shape.hkv, shape.d, budget_live, K.device,
-                           with_tail, params.tail_slot)
+                           with_tail, params.tail_slot, params.tail_clusters)
     if ws is None:
         ws = workspace(certkv_workspace_bytes(shape, params), K.device)
     st = out.struct()
@@ -295,7 +308,7 @@ def certkv_compress(K, V, Q_obs, budget_live: int, params=None, *, out: Optional
     shape = shape_of(K, Q_obs)
     if out is None:
         out = Packed.empty(shape.batch, shape.layers, shape.hkv, shape.d, budget_live, K.device,
-                           with_tail, params.tail_slot)
+                           with_tail, params.tail_slot, params.tail_clusters)
     if ws is None:
         ws = workspace(certkv_workspace_bytes(shape, params), K.device)
     st = out.struct()
@@ -317,7 +330,7 @@ def certkv_compress_host(hK, hV, hQ_obs, budget_live: int, params=None, *, chunk
                                                                           torch.cuda.current_device())
     if out is None:
         out = Packed.empty(shape.batch, shape.layers, shape.hkv, shape.d, budget_live, device,
-                           with_tail, params.tail_slot)
+                           with_tail, params.tail_slot, params.tail_clusters)
     if ws is None:
         ws = workspace(certkv_host_workspace_bytes(shape, params, chunk), device)
     st = out.struct()
@@ -345,6 +358,33 @@ def certkv_decode_attn(q, packed: Packed, *, hkv: int, scale: float = 0.0, out=N
                                            _ptr(ws), ws.numel(), _stream(stream))
     _check(rc, "certkv_decode_attn")
     return out
+
+
+def certkv_decode_certified(q, packed: Packed, *, hkv: int, scale: float = 0.0, out=None,
+                            bound=None, certified=None, ws=None, stream=None):
+    """Clustered-tail decode with its runtime error bound: (out bf16 [B][L][Hq][d],
+    bound fp32 [B][L][Hq], certified int32 [B][L][Hq])."""
+    _bf16(q, "q")
+    if packed.clusters < 1:
+        raise ValueError("packed cache has no cluster summaries (params.tail_clusters = 0)")
+    B, L, Hq, d = q.shape
+    shape = certkv_shape(B, L, Hq, hkv, 2, d, 1)
+    if out is None:
+        out = torch.empty_like(q)
+    if bound is None:
+        bound = torch.empty((B, L, Hq), dtype=torch.float32, device=q.device)
+    if certified is None:
+        certified = torch.empty((B, L, Hq), dtype=torch.int32, device=q.device)
+    if ws is None:
+        ws = workspace(certkv_decode_workspace_bytes(shape), q.device)
+    st = packed.struct()
+    rc = load_library().certkv_decode_certified(ctypes.byref(shape), _ptr(q), ctypes.byref(st),
+                                                float(scale), int(packed.tail_slot),
+                                                int(packed.clusters), _ptr(out), _ptr(bound),
+                                                _ptr(certified), _ptr(ws), ws.numel(),
+                                                _stream(stream))
+    _check(rc, "certkv_decode_certified")
+    return out, bound, certified
 
 
 def certkv_read_status(ws: torch.Tensor, stream=None) -> int:

@@ -488,8 +488,8 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
       }
       (void)wb;
     }
-    // counts and offsets: segment = b_h real slots (+ 1 tail slot)
-    const int seg = live ? b + p.tail_slot : 0;
+    // counts and offsets: segment = b_h real slots (+ 1 tail slot) (+ m cluster summaries)
+    const int seg = live ? b + p.tail_slot + p.clusters : 0;
     int incl = seg;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {

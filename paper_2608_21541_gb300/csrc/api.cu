@@ -38,6 +38,7 @@ int check_params(const certkv_params* q) {
   if (q->statistic < 0 || q->statistic > 2) return CERTKV_EINVAL;
   if (q->tail_slot != 0 && q->tail_slot != 1) return CERTKV_EINVAL;
   if (q->allocator < CERTKV_ALLOC_LAGRANGIAN || q->allocator > CERTKV_ALLOC_GREEDY) return CERTKV_EINVAL;
+  if (q->tail_clusters < 0 || q->tail_clusters > CERTKV_MAX_CLUSTERS) return CERTKV_EINVAL;
   return CERTKV_OK;
 }
 
@@ -58,6 +59,7 @@ int make_prob(const certkv_shape* s, const certkv_params* q, int64_t budget_live
   P.pool = q->pool_kernel; P.protect = q->protect_window;
   P.alpha_num = q->alpha_num; P.alpha_den = q->alpha_den; P.T = q->bisect_steps;
   P.statistic = q->statistic; P.tail_slot = q->tail_slot; P.allocator = q->allocator;
+  P.clusters = q->tail_clusters;
   P.score_warps = (P.R + 15) / 16 < 16 ? (P.R + 15) / 16 : 16;
   P.row_blocks = (P.R + 16 * P.score_warps - 1) / (16 * P.score_warps);
   if (score_tc_supported(P)) P.row_blocks = P.R / 64;  // one per 64-row quarter of the tcgen05 pass 2
@@ -68,10 +70,10 @@ int make_prob(const certkv_shape* s, const certkv_params* q, int64_t budget_live
   P.chunks = (P.n + kChunk - 1) / kChunk;
   if (budget_live >= 0) {
     const int64_t H = P.H;
-    const int64_t lo = P.tail_slot ? 2 * H : H;
-    if (budget_live < lo || budget_live > H * (int64_t)P.n) return CERTKV_EBUDGET;
+    const int64_t charged = H * ((P.tail_slot ? 1 : 0) + P.clusters);  // summary slots
+    if (budget_live < charged + H || budget_live > H * (int64_t)P.n) return CERTKV_EBUDGET;
     P.B_live = budget_live;
-    P.B_real = budget_live - (P.tail_slot ? H : 0);
+    P.B_real = budget_live - charged;
     int64_t bmin = ((int64_t)P.alpha_num * P.B_real) / ((int64_t)P.alpha_den * H);
     if (bmin < 1) bmin = 1;
     if (P.B_real < H * bmin || P.B_real > H * (int64_t)(P.n - 1)) return CERTKV_EBUDGET;
@@ -162,6 +164,7 @@ int check_packed(const Prob& p, const certkv_packed* out) {
     return CERTKV_EINVAL;
   if (!aligned(out->k, 16) || !aligned(out->v, 16)) return CERTKV_EINVAL;
   if (out->capacity_slots < (int64_t)p.bl * p.B_live) return CERTKV_ECAPACITY;
+  if (p.clusters > 0 && (!out->cluster_meta || !out->kept_vmax)) return CERTKV_EINVAL;
   return CERTKV_OK;
 }
 
@@ -171,7 +174,7 @@ int run_scored(const Prob& p, const Layout& ly, char* ws, const void* K, const v
   launch_curves(p, ly, ws, K, V, p.tail_slot != 0, st);
   launch_allocate(p, ly, ws, out->real_counts, out->offsets, st);
   launch_pack(p, ly, ws, K, V, a, out->k, out->v, out->offsets, out->real_counts, out->positions,
-              out->tail_f32, out->tail_mass, st);
+              out->tail_f32, out->tail_mass, out->cluster_meta, out->kept_vmax, st);
   return cuda_ok(cudaGetLastError());
 }
 
@@ -193,6 +196,7 @@ void certkv_default_params(certkv_params* p) {
   p->statistic = CERTKV_STAT_CENTERED;
   p->tail_slot = 1;
   p->allocator = CERTKV_ALLOC_LAGRANGIAN;
+  p->tail_clusters = 0;
 }
 
 int64_t certkv_live_budget(int32_t n, int32_t hkv, int64_t keep_num, int64_t keep_den) {
@@ -400,6 +404,8 @@ int certkv_compress_host(const certkv_shape* shape, const void* hK, const void* 
     o.real_counts = out->real_counts + (size_t)bl0 * F.H;
     if (out->tail_f32) o.tail_f32 = out->tail_f32 + (size_t)bl0 * F.H * 2 * kD;
     if (out->tail_mass) o.tail_mass = out->tail_mass + (size_t)bl0 * F.H;
+    if (out->cluster_meta) o.cluster_meta = out->cluster_meta + (size_t)bl0 * F.H * F.clusters * 4;
+    if (out->kept_vmax) o.kept_vmax = out->kept_vmax + (size_t)bl0 * F.H;
     float* a = reinterpret_cast<float*>(ws + ly.a);
     launch_score(p, ly, ws, sK, sQ, a, st);
     rc = run_scored(p, ly, ws, sK, sV, a, &o, st);
@@ -449,6 +455,33 @@ int certkv_decode_attn(const certkv_shape* shape, const void* q, const certkv_pa
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   launch_decode(p, q, packed->k, packed->v, packed->offsets, packed->real_counts, tail_slot, sc,
                 out, reinterpret_cast<char*>(workspace), st);
+  return cuda_ok(cudaGetLastError());
+}
+
+int certkv_decode_certified(const certkv_shape* shape, const void* q, const certkv_packed* packed,
+                            float scale, int32_t tail_slot, int32_t clusters, void* out,
+                            float* bound, int32_t* certified, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  int rc = check_shape(shape);
+  if (rc) return rc;
+  if (!q || !packed || !packed->k || !packed->v || !packed->offsets || !packed->real_counts ||
+      !packed->cluster_meta || !packed->kept_vmax || !out || !bound || !certified)
+    return CERTKV_EINVAL;
+  if (!aligned(packed->k, 16) || !aligned(packed->v, 16) || !aligned(q, 16)) return CERTKV_EINVAL;
+  if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
+  if (clusters < 1 || clusters > CERTKV_MAX_CLUSTERS) return CERTKV_EINVAL;
+  if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
+  certkv_params prm;
+  certkv_default_params(&prm);
+  Prob p;
+  if ((rc = make_prob(shape, &prm, -1, &p))) return rc;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < decode_workspace(p))
+    return CERTKV_EWORKSPACE;
+  const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  launch_decode_certified(p, q, packed->k, packed->v, packed->offsets, packed->real_counts,
+                          tail_slot, clusters, packed->cluster_meta, packed->kept_vmax, sc, out,
+                          bound, certified, reinterpret_cast<char*>(workspace), st);
   return cuda_ok(cudaGetLastError());
 }
 

@@ -8,6 +8,7 @@
 // share of 32-slot tiles and keep online (max, sum, acc) for the G query
 // heads that share the unit, so every packed K/V byte is read once per step;
 // a merge kernel combines the splits in the log-sum-exp domain.
+#include "../../include/certkv.h"
 #include "common.cuh"
 #include "internal.cuh"
 
@@ -179,6 +180,95 @@ __global__ void __launch_bounds__(128) decode_merge_kernel(Prob p, int G,
   out[((size_t)bl * p.Hq + (size_t)h * G + g) * kD + i] = __float2bfloat16_rn(A / L);
 }
 
+// Sum over the 128 threads of the block (one per dimension).
+__device__ __forceinline__ float block_sum128(float x, float* red) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) x += __shfl_xor_sync(kFull, x, o);
+  __syncthreads();  // red may still be read from the previous reduction
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = x;
+  __syncthreads();
+  return (red[0] + red[1]) + (red[2] + red[3]);
+}
+
+// grid = units * G, block = 128 (thread = dimension): the real-slot splits of
+// one query head merged as in decode_merge_kernel, then the m cluster
+// summaries added with weight n_g e^{lbar_g} (all weights relative to one
+// log2-domain shift, to which the bound is invariant), then the certificate.
+__global__ void __launch_bounds__(128) decode_certified_merge_kernel(
+    Prob p, int G, int m, int tail_slot, float scale, const __nv_bfloat16* __restrict__ q,
+    const __nv_bfloat16* __restrict__ pk, const __nv_bfloat16* __restrict__ pv,
+    const int64_t* __restrict__ offsets, const int32_t* __restrict__ counts,
+    const float4* __restrict__ cluster_meta, const float* __restrict__ kept_vmax,
+    const float2* __restrict__ part_ml, const float* __restrict__ part_acc,
+    __nv_bfloat16* __restrict__ out, float* __restrict__ bound, int32_t* __restrict__ certified) {
+  __shared__ float red[4];
+  __shared__ float s_lam[CERTKV_MAX_CLUSTERS], s_r[CERTKV_MAX_CLUSTERS];
+  __shared__ float s_vn[CERTKV_MAX_CLUSTERS], s_rho[CERTKV_MAX_CLUSTERS];
+  const int ug = blockIdx.x;
+  const int u = ug / G, g = ug - u * G;
+  const int i = threadIdx.x;
+  const float kLog2e = 1.4426950408889634f;
+  // real slots: merge of the splits (log2 domain)
+  float MS = -INFINITY;
+  for (int s = 0; s < kDecodeSplits; ++s)
+    MS = fmaxf(MS, part_ml[((size_t)u * kDecodeSplits + s) * G + g].x);
+  float LS = 0.f, AS = 0.f;
+  for (int s = 0; s < kDecodeSplits; ++s) {
+    const size_t pi = ((size_t)u * kDecodeSplits + s) * G + g;
+    const float2 ml = part_ml[pi];
+    if (ml.x > -INFINITY) {
+      const float f = exp2f(ml.x - MS);
+      LS += ml.y * f;
+      AS += part_acc[pi * kD + i] * f;
+    }
+  }
+  const int bl = u / p.H, h = u - bl * p.H;
+  const size_t qi = (size_t)bl * p.Hq + (size_t)h * G + g;
+  const float qv = __bfloat162float(q[qi * kD + i]);
+  const float qn = sqrtf(block_sum128(qv * qv, red));
+  const int64_t s0 = offsets[u] + counts[u] + tail_slot;  // first summary slot
+  // clusters: lbar (log2 domain, with log2 n_g), logit radius, ||vbar||, rho
+  float M = MS;
+  for (int c = 0; c < m; ++c) {
+    const float4 meta = cluster_meta[(size_t)u * m + c];
+    const float kb = __bfloat162float(pk[(s0 + c) * kD + i]);
+    const float vb = __bfloat162float(pv[(s0 + c) * kD + i]);
+    const float dot = block_sum128(qv * kb, red);
+    const float vn = sqrtf(block_sum128(vb * vb, red));
+    const float lam = meta.x > 0.f ? fmaf(dot, scale * kLog2e, log2f(meta.x)) : -INFINITY;
+    if (i == 0) {
+      s_lam[c] = lam;
+      s_r[c] = scale * qn * meta.y;
+      s_vn[c] = vn;
+      s_rho[c] = meta.z;
+    }
+    M = fmaxf(M, lam);
+  }
+  __syncthreads();
+  const float fS = MS > -INFINITY ? exp2f(MS - M) : 0.f;
+  float num = AS * fS, Z = LS * fS;
+  for (int c = 0; c < m; ++c) {
+    if (!(s_lam[c] > -INFINITY)) continue;
+    const float zg = exp2f(s_lam[c] - M);
+    num = fmaf(zg, __bfloat162float(pv[(s0 + c) * kD + i]), num);
+    Z += zg;
+  }
+  out[qi * kD + i] = __float2bfloat16_rn(num / Z);
+  if (i == 0) {
+    float DZ = 0.f, DN = 0.f, vmax = kept_vmax[u];
+    for (int c = 0; c < m; ++c) {
+      if (!(s_lam[c] > -INFINITY)) continue;
+      const float zg = exp2f(s_lam[c] - M);
+      const float er = expf(s_r[c]);
+      DZ += (er - 1.f) * er * zg;
+      DN += er * zg * ((er - 1.f) * s_vn[c] + s_rho[c]);
+      vmax = fmaxf(vmax, s_vn[c] + s_rho[c]);
+    }
+    bound[qi] = 3.f / Z * (DN + vmax * DZ);
+    certified[qi] = DZ <= Z / 3.f ? 1 : 0;
+  }
+}
+
 size_t decode_workspace(const Prob& p) {
   const size_t parts = (size_t)p.units * kDecodeSplits * p.G;
   return parts * sizeof(float2) + parts * kD * sizeof(float) + 512;
@@ -219,6 +309,37 @@ void launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
     TraceScope ts_("decode_merge", st);
     decode_merge_kernel<<<p.units * p.G, 128, 0, st>>>(p, p.G, ml, acc,
                                                        reinterpret_cast<__nv_bfloat16*>(out));
+  }
+}
+
+void launch_decode_certified(const Prob& p, const void* q, const void* pk, const void* pv,
+                             const int64_t* offsets, const int32_t* counts, int tail_slot,
+                             int clusters, const float* cluster_meta, const float* kept_vmax,
+                             float scale, void* out, float* bound, int32_t* certified, char* ws,
+                             cudaStream_t st) {
+  const size_t parts = (size_t)p.units * kDecodeSplits * p.G;
+  float2* ml = reinterpret_cast<float2*>(ws);
+  size_t acc_off = (parts * sizeof(float2) + 255) / 256 * 256;
+  float* acc = reinterpret_cast<float*>(ws + acc_off);
+  const float sl2 = scale * 1.4426950408889634f;
+  const __nv_bfloat16* qb = reinterpret_cast<const __nv_bfloat16*>(q);
+  const __nv_bfloat16* kb = reinterpret_cast<const __nv_bfloat16*>(pk);
+  const __nv_bfloat16* vb = reinterpret_cast<const __nv_bfloat16*>(pv);
+  // the real slots only: the splits see no tail slot
+  switch (p.G) {
+    case 1: launch_split<1>(p, qb, kb, vb, offsets, counts, 0, sl2, ml, acc, st); break;
+    case 2: launch_split<2>(p, qb, kb, vb, offsets, counts, 0, sl2, ml, acc, st); break;
+    case 4: launch_split<4>(p, qb, kb, vb, offsets, counts, 0, sl2, ml, acc, st); break;
+    case 8: launch_split<8>(p, qb, kb, vb, offsets, counts, 0, sl2, ml, acc, st); break;
+    case 16: launch_split<16>(p, qb, kb, vb, offsets, counts, 0, sl2, ml, acc, st); break;
+    default: return;
+  }
+  {
+    TraceScope ts_("decode_certified_merge", st);
+    decode_certified_merge_kernel<<<p.units * p.G, 128, 0, st>>>(
+        p, p.G, clusters, tail_slot, scale, qb, kb, vb, offsets, counts,
+        reinterpret_cast<const float4*>(cluster_meta), kept_vmax, ml, acc,
+        reinterpret_cast<__nv_bfloat16*>(out), bound, certified);
   }
 }
 

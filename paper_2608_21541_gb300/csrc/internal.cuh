@@ -18,6 +18,7 @@ struct Prob {
   int pool, protect;
   int alpha_num, alpha_den, T, statistic, tail_slot;
   int allocator;  // CERTKV_ALLOC_*
+  int clusters;   // m cluster summaries per head over the evicted tail (0 = none)
   int64_t B_live, B_real;
   int b_min;
   int64_t slot_base;  // packed slot of this problem's first (sequence, layer): offsets are global
@@ -78,13 +79,18 @@ void launch_allocate(const Prob& p, const Layout& ly, char* ws, int32_t* counts,
 void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const void* V,
                  const float* a, void* pk, void* pv, const int64_t* offsets,
                  const int32_t* counts, int32_t* positions, float* tail_f32,
-                 double* tail_mass, cudaStream_t st);
+                 double* tail_mass, float* cluster_meta, float* kept_vmax, cudaStream_t st);
 void launch_export_curves(const Prob& p, const Layout& ly, char* ws, int32_t* perm_out,
                           double* c_out, cudaStream_t st);
 void launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
                    const int64_t* offsets, const int32_t* counts, int tail_slot, float scale,
                    void* out, char* ws, cudaStream_t st);
 size_t decode_workspace(const Prob& p);
+void launch_decode_certified(const Prob& p, const void* q, const void* pk, const void* pv,
+                             const int64_t* offsets, const int32_t* counts, int tail_slot,
+                             int clusters, const float* cluster_meta, const float* kept_vmax,
+                             float scale, void* out, float* bound, int32_t* certified, char* ws,
+                             cudaStream_t st);
 
 // ---- optional kernel timing (off by default) ------------------------------
 // When enabled with certkv_trace_enable(), every kernel launch is bracketed

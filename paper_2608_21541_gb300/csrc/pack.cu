@@ -185,10 +185,134 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloa
   }
 }
 
+// Clustered-tail summaries (appendix: deterministic output-error bound for
+// clustered tail summaries; readings R-C1, R-C2): group g of unit u = ranks
+// b + floor(g T / m) .. b + floor((g + 1) T / m) - 1 of the evicted tail
+// (T = n - b); stored representatives = the bf16-rounded unweighted means,
+// radii = the largest distances of the group's rows to them, rounded up by
+// 1e-5 relative (the fp32 sum of 128 squares and the square root are within
+// a few 1e-6 of exact).  grid = (units, m + 1), block = 512 (warp per row,
+// 4 rows in flight); blockIdx.y = m computes the kept rows' largest ||v||.
+constexpr int kClusterWarps = 16;
+constexpr float kRadiusRoundUp = 1.0f + 1e-5f;
+__global__ void __launch_bounds__(kClusterWarps * 32) cluster_kernel(
+    Prob p, const int32_t* __restrict__ perm, const __nv_bfloat16* __restrict__ K,
+    const __nv_bfloat16* __restrict__ V, const int32_t* __restrict__ counts,
+    const int64_t* __restrict__ offsets, __nv_bfloat16* __restrict__ pk,
+    __nv_bfloat16* __restrict__ pv, int32_t* __restrict__ positions,
+    float4* __restrict__ cluster_meta, float* __restrict__ kept_vmax) {
+  __shared__ DF s_sum[kClusterWarps][2][kD];
+  __shared__ float s_mean[2][kD];
+  __shared__ float s_max[kClusterWarps][2];
+  const int u = blockIdx.x, g = blockIdx.y, m = p.clusters;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = p.n, b = counts[u];
+  const int32_t* pu = perm + (size_t)u * n;
+  const uint2* Ku = reinterpret_cast<const uint2*>(K + (size_t)u * n * kD);
+  const uint2* Vu = reinterpret_cast<const uint2*>(V + (size_t)u * n * kD);
+  auto row4 = [&](const uint2* base, int j, float (&x)[4]) {
+    const uint2 raw = __ldg(base + (size_t)j * (kD / 4) + lane);
+    x[0] = bf16lo(raw.x);
+    x[1] = bf16hi(raw.x);
+    x[2] = bf16lo(raw.y);
+    x[3] = bf16hi(raw.y);
+  };
+  auto block_max = [&](float a, float c, float& ra, float& rc) {
+    if (lane == 0) {
+      s_max[warp][0] = a;
+      s_max[warp][1] = c;
+    }
+    __syncthreads();
+    ra = rc = 0.f;
+    for (int w = 0; w < kClusterWarps; ++w) {
+      ra = fmaxf(ra, s_max[w][0]);
+      rc = fmaxf(rc, s_max[w][1]);
+    }
+  };
+  if (g == m) {  // largest value norm over the kept ranks 0 .. b-1
+    float mx = 0.f;
+    for (int r = warp; r < b; r += kClusterWarps) {
+      float v[4];
+      row4(Vu, pu[r], v);
+      float sq = fmaf(v[3], v[3], fmaf(v[2], v[2], fmaf(v[1], v[1], v[0] * v[0])));
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) sq += __shfl_xor_sync(kFull, sq, o);
+      mx = fmaxf(mx, sqrtf(sq));
+    }
+    float ra, rc;
+    block_max(mx, 0.f, ra, rc);
+    if (threadIdx.x == 0) kept_vmax[u] = ra * kRadiusRoundUp;
+    return;
+  }
+  const int T = n - b;
+  const int r0 = b + (int)(((int64_t)g * T) / m), r1 = b + (int)(((int64_t)(g + 1) * T) / m);
+  const int cnt = r1 - r0;
+  // 1. unweighted means: double-float sums per lane (4 dimensions), then per dimension
+  DF sk[4], sv[4];
+#pragma unroll
+  for (int c = 0; c < 4; ++c) sk[c] = sv[c] = df_make(0.f);
+  for (int r = r0 + warp; r < r1; r += kClusterWarps) {
+    const int j = pu[r];
+    float k4[4], v4[4];
+    row4(Ku, j, k4);
+    row4(Vu, j, v4);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      sk[c] = df_add_f(sk[c], k4[c]);
+      sv[c] = df_add_f(sv[c], v4[c]);
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    s_sum[warp][0][lane * 4 + c] = sk[c];
+    s_sum[warp][1][lane * 4 + c] = sv[c];
+  }
+  __syncthreads();
+  const int64_t slot = offsets[u] + b + p.tail_slot + g;
+  if (threadIdx.x < 2 * kD) {
+    const int t = threadIdx.x / kD, i = threadIdx.x % kD;
+    DF sum = df_make(0.f);
+    for (int w = 0; w < kClusterWarps; ++w) sum = df_add(sum, s_sum[w][t][i]);
+    const DF mean = cnt > 0 ? df_div(sum, df_make((float)cnt)) : df_make(0.f);
+    const uint16_t bits = df_to_bf16(mean.hi, mean.lo);
+    reinterpret_cast<uint16_t*>(t == 0 ? pk : pv)[slot * kD + i] = bits;
+    s_mean[t][i] = __uint_as_float((uint32_t)bits << 16);
+  }
+  if (threadIdx.x == 0) positions[slot] = -2 - g;
+  __syncthreads();
+  // 2. radii to the stored representatives: warp per row
+  float mk = 0.f, mv = 0.f;
+  for (int r = r0 + warp; r < r1; r += kClusterWarps) {
+    const int j = pu[r];
+    float k4[4], v4[4];
+    row4(Ku, j, k4);
+    row4(Vu, j, v4);
+    float qk = 0.f, qv = 0.f;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const float dk = k4[c] - s_mean[0][lane * 4 + c], dv = v4[c] - s_mean[1][lane * 4 + c];
+      qk = fmaf(dk, dk, qk);
+      qv = fmaf(dv, dv, qv);
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+      qk += __shfl_xor_sync(kFull, qk, o);
+      qv += __shfl_xor_sync(kFull, qv, o);
+    }
+    mk = fmaxf(mk, sqrtf(qk));
+    mv = fmaxf(mv, sqrtf(qv));
+  }
+  float rk, rv;
+  block_max(mk, mv, rk, rv);
+  if (threadIdx.x == 0)
+    cluster_meta[(size_t)u * m + g] = make_float4((float)cnt, rk * kRadiusRoundUp,
+                                                  rv * kRadiusRoundUp, 0.f);
+}
+
 void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const void* V,
                  const float* a, void* pk, void* pv, const int64_t* offsets,
                  const int32_t* counts, int32_t* positions, float* tail_f32,
-                 double* tail_mass, cudaStream_t st) {
+                 double* tail_mass, float* cluster_meta, float* kept_vmax, cudaStream_t st) {
   const uint32_t* keys = reinterpret_cast<const uint32_t*>(ws + ly.keys0);
   const int32_t* perm = reinterpret_cast<const int32_t*>(ws + ly.vals0);
   const __nv_bfloat16* Kb = reinterpret_cast<const __nv_bfloat16*>(K);
@@ -206,6 +330,12 @@ void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const
     TraceScope ts("copy_rows", st);
     copy_rows_kernel<<<dim3(p.units, ysplit), 256, 0, st>>>(p, Kb, Vb, counts, offsets,
                                                            positions, PK, PV);
+  }
+  if (p.clusters > 0) {
+    TraceScope ts("clusters", st);
+    cluster_kernel<<<dim3(p.units, p.clusters + 1), kClusterWarps * 32, 0, st>>>(
+        p, perm, Kb, Vb, counts, offsets, PK, PV, positions,
+        reinterpret_cast<float4*>(cluster_meta), kept_vmax);
   }
   if (p.tail_slot) {
     TraceScope ts("tail", st);

@@ -305,6 +305,158 @@ def pin_allocator_greedy_marginal(lib=None):
     assert b.tolist() == [27, 3], b
 
 
+def _full_attention(q, K, V, scale):
+    lg = scale * (K @ q)
+    w = np.exp(lg - lg.max())
+    return (w[:, None] * V).sum(0) / w.sum()
+
+
+def _certificate_case(rng, n, d, b, m, spread, scale, lib):
+    """A unit with a kept set of b rows and m clusters over the rest; returns
+    (O-hat, bound, certified, structural, exact O)."""
+    K = to_bf16_bits(rng.normal(size=(n, d)) * spread)
+    V = to_bf16_bits(rng.normal(size=(n, d)))
+    q = to_bf16_bits(rng.normal(size=d))
+    perm = rng.permutation(n).astype(np.int32)
+    kb, vb, cnt, rk, rv, _ = oracle.tail_clusters(K, V, perm, b, m, lib=lib)
+    kept = perm[:b]
+    est, bound, cert, struct = oracle.decode_certified(q, K[kept], V[kept], kb, vb, cnt, rk, rv,
+                                                       scale=scale, lib=lib)
+    exact = _full_attention(bf(q), bf(K), bf(V), scale)
+    return est, bound, cert, struct, exact
+
+
+def pin_certificate_singleton_clusters_exact(lib=None):
+    """Clustered-tail certificate (appendix theorem): with one token per
+    cluster every radius is 0 (the stored bf16 representative is the token
+    itself), so D_Z = D_N = 0, the bound is 0 and O-hat is exact attention."""
+    rng = np.random.default_rng(31)
+    n, d, b = 24, 16, 9
+    est, bound, cert, struct, exact = _certificate_case(rng, n, d, b, n - b, 1.0, 0.25, lib)
+    assert cert and bound == 0.0 and struct == 0.0
+    assert np.abs(est - exact).max() < 1e-12
+
+
+def pin_certificate_bound_holds(lib=None):
+    """The runtime bound dominates the true output error whenever its
+    checkable condition D_Z <= Z-hat / 3 holds (appendix theorem, Eq.
+    (certificate-bound)), and it is at most its structural form (Eq.
+    (certificate-structure)); tighter key clusters give smaller bounds."""
+    rng = np.random.default_rng(32)
+    held = 0
+    for trial in range(40):
+        n, d = int(rng.integers(20, 60)), int(rng.choice([8, 16, 32]))
+        b = int(rng.integers(1, n - 2))
+        m = int(rng.integers(1, n - b + 1))
+        spread = float(rng.choice([0.02, 0.1, 0.5]))
+        est, bound, cert, struct, exact = _certificate_case(rng, n, d, b, m, spread, 0.3, lib)
+        if cert:
+            held += 1
+            assert np.linalg.norm(est - exact) <= bound * (1 + 1e-9) + 1e-12, (trial, bound)
+            assert bound <= struct * (1 + 1e-9) + 1e-12, (trial, bound, struct)
+    assert held >= 20
+    rng = np.random.default_rng(33)
+    loose = _certificate_case(rng, 40, 16, 10, 3, 0.5, 0.3, lib)[1]
+    rng = np.random.default_rng(33)
+    tight = _certificate_case(rng, 40, 16, 10, 3, 0.05, 0.3, lib)[1]
+    assert tight < loose
+
+
+def pin_certificate_value_radius(lib=None):
+    """Identical keys inside each cluster make every logit radius 0, so the
+    only error left is the value representative (rounded to bf16): it must be
+    covered by the value-radius term rho_g of D_N alone."""
+    rng = np.random.default_rng(36)
+    n, d, b, m = 48, 16, 8, 4
+    T = n - b
+    perm = rng.permutation(n).astype(np.int32)
+    Kf = rng.normal(size=(n, d))
+    for g in range(m):  # one key per cluster
+        rows = perm[b + g * T // m: b + (g + 1) * T // m]
+        Kf[rows] = rng.normal(size=d)
+    K, V = to_bf16_bits(Kf), to_bf16_bits(rng.normal(size=(n, d)) * 3.0)
+    q = to_bf16_bits(rng.normal(size=d))
+    kb, vb, cnt, rk, rv, _ = oracle.tail_clusters(K, V, perm, b, m, lib=lib)
+    assert np.allclose(rk, 0.0)
+    est, bound, cert, _ = oracle.decode_certified(q, K[perm[:b]], V[perm[:b]], kb, vb, cnt, rk, rv,
+                                                  scale=0.25, lib=lib)
+    err = np.linalg.norm(est - _full_attention(bf(q), bf(K), bf(V), 0.25))
+    assert cert and 0.0 < err <= bound, (err, bound)
+
+
+def pin_certificate_logit_radius(lib=None):
+    """Hand-built case where the logit radius matters: q = (32, 0, 0, 0),
+    scale 1/2; one kept token (key e1 / 2, value e1, logit 8) and one tail cluster
+    of three keys (2, -1, -1) e1 / 32 (centroid exactly 0, key radius 1/16,
+    logits 1, -1/2, -1/2) sharing the value e2 (value radius 0).  The logit
+    radius is scale ||q|| 1/16 = 1; the estimator puts weight 3 on e2 where
+    exact attention puts e + 2 e^{-1/2} = 3.93 beside e^8 on e1, an output error
+    of 4.41e-4, inside the bound 3/Z-hat (D_N + V'max D_Z) = 0.0282 but not
+    inside what a radius without the query norm (1/32) would give (1.98e-4)."""
+    d = 4
+    K = to_bf16_bits(np.array([[0.5, 0, 0, 0], [2 / 32, 0, 0, 0], [-1 / 32, 0, 0, 0],
+                               [-1 / 32, 0, 0, 0]], float))
+    V = to_bf16_bits(np.array([[1, 0, 0, 0], [0, 1, 0, 0], [0, 1, 0, 0], [0, 1, 0, 0]], float))
+    q = to_bf16_bits(np.array([32.0, 0, 0, 0]))
+    perm = np.arange(4, dtype=np.int32)
+    kb, vb, cnt, rk, rv, _ = oracle.tail_clusters(K, V, perm, 1, 1, lib=lib)
+    assert cnt.tolist() == [3] and rk[0] == 1 / 16 and rv[0] == 0.0
+    est, bound, cert, _ = oracle.decode_certified(q, K[:1], V[:1], kb, vb, cnt, rk, rv,
+                                                  scale=0.5, lib=lib)
+    err = np.linalg.norm(est - _full_attention(bf(q), bf(K), bf(V), 0.5))
+    assert cert and abs(err - 4.408e-4) < 1e-6 and err <= bound, (err, bound)
+    assert abs(bound - 0.02818) < 1e-4, bound
+
+
+def pin_cluster_summaries(lib=None):
+    """Cluster summaries: consecutive rank groups of the evicted tail (reading
+    R-C1) with the bf16-rounded unweighted means and the largest distances to
+    them as radii (reading R-C2), checked by direct computation."""
+    rng = np.random.default_rng(34)
+    n, d, b, m = 30, 8, 7, 4
+    K = to_bf16_bits(rng.normal(size=(n, d)))
+    V = to_bf16_bits(rng.normal(size=(n, d)))
+    perm = rng.permutation(n).astype(np.int32)
+    kb, vb, cnt, rk, rv, vmax = oracle.tail_clusters(K, V, perm, b, m, lib=lib)
+    T = n - b
+    assert cnt.tolist() == [(g + 1) * T // m - g * T // m for g in range(m)]
+    for g in range(m):
+        rows = perm[b + g * T // m: b + (g + 1) * T // m]
+        assert (kb[g] == to_bf16_bits(bf(K[rows]).mean(0))).all()
+        assert (vb[g] == to_bf16_bits(bf(V[rows]).mean(0))).all()
+        assert abs(rk[g] - np.linalg.norm(bf(K[rows]) - bf(kb[g]), axis=1).max()) < 1e-12
+        assert abs(rv[g] - np.linalg.norm(bf(V[rows]) - bf(vb[g]), axis=1).max()) < 1e-12
+    assert abs(vmax - np.linalg.norm(bf(V[perm[:b]]), axis=1).max()) < 1e-12
+
+
+def pin_packed_layout_with_clusters(lib=None):
+    """With m cluster summaries per head every head is charged m more slots
+    (exact-budget accounting): sum_h b_h = B_live - H (tail_slot + m), each
+    segment is its b_h real slots, the tail slot, then the m summary slots
+    (positions -2 - g), and every (sequence, layer) still fills exactly B_live
+    slots."""
+    rng = np.random.default_rng(35)
+    B, L, Hq, H, n, d, w, m = 1, 2, 4, 2, 64, 8, 4, 3
+    K = to_bf16_bits(rng.normal(size=(B, L, H, n, d)))
+    V = to_bf16_bits(rng.normal(size=(B, L, H, n, d)))
+    Q = to_bf16_bits(rng.normal(size=(B, L, Hq, w, d)))
+    B_live = 30
+    r = oracle.compress(K, V, Q, B=B, L=L, Hq=Hq, H=H, n=n, d=d, w=w, B_live=B_live,
+                        clusters=m, threads=1, lib=lib)
+    for bl in range(B * L):
+        cnt = r["counts"][bl * H:(bl + 1) * H]
+        assert cnt.sum() == B_live - H * (1 + m), cnt
+        for h in range(H):
+            u = bl * H + h
+            off, end = r["offsets"][u], r["offsets"][u + 1]
+            assert end - off == cnt[h] + 1 + m
+            pos = r["positions"][off:end]
+            assert (pos[:cnt[h]] >= 0).all() and pos[cnt[h]] == -1
+            assert pos[cnt[h] + 1:].tolist() == [-2 - g for g in range(m)]
+            assert int(r["cl_meta"][u, :, 0].sum()) == n - cnt[h]
+    assert r["offsets"][-1] == B * L * B_live
+
+
 def pin_allocation_infeasible(lib=None):
     """B_real above H (n - 1) cannot be met with b_h <= n - 1."""
     curves = np.ones((2, 5))

@@ -37,6 +37,12 @@ MUTANTS = {
     "uniform_remainder_to_high_heads": ("(h < B_real % H ? 1 : 0)", "(h >= H - B_real % H ? 1 : 0)"),
     "greedy_ignores_safeguard": ("for (int h = 0; h < H; ++h) b[h] = lo_b;",
                                  "for (int h = 0; h < H; ++h) b[h] = 1;"),
+    "certificate_radius_without_query_norm": ("const double r = scale * qn * rk[g];",
+                                              "const double r = scale * rk[g];"),
+    "certificate_drops_value_radius": ("DN += er * zg * ((er - 1.0) * vn + rv[g]);",
+                                       "DN += er * zg * ((er - 1.0) * vn);"),
+    "cluster_groups_overlap_kept": ("const int r0 = b + (int)(((int64_t)g * T) / m),",
+                                    "const int r0 = (g == 0 ? b - 1 : b) + (int)(((int64_t)g * T) / m),"),
     "bisection_inverted": ("if (total > B_real) lam_lo = lam; else lam_hi = lam;",
                            "if (total > B_real) lam_hi = lam; else lam_lo = lam;"),
     "kept_not_sorted": ("qsort(kept, (size_t)b, sizeof(int32_t), cmp_int32);", ""),
