@@ -249,6 +249,27 @@ int certkv_decode_certified(const certkv_shape* shape, const void* q, const cert
                             float* bound, int32_t* certified, void* workspace,
                             size_t workspace_bytes, void* stream);
 
+/* Fixed-row diagnostics (an evaluation tool: it reads the full original K and
+ * V, like the paper's fixed-row experiments; Theorem: fixed-row tail
+ * factorization).  For every query head qh of unit u with its decode query q
+ * and the realized softmax row A_j = softmax_j(scale <q, k_j>) over all n
+ * original tokens, and S = the real tokens kept in `packed`, writes stats
+ * fp32 [B][L][Hq][8]:
+ *   0  p_S = sum_{j in S} A_j (kept mass)
+ *   1  ||O||_2 of exact attention O = sum_j A_j v_j
+ *   2  ||O~_S - O||_2, O~_S = sum_{j in S} A_j v_j / p_S (subset-only output)
+ *   3  ||u*||_2, u* = sum_{j not in S} A_j v_j (the fixed-row correction)
+ *   4  2 V_max (1 - p_S), V_max = max_j ||v_j||_2 (the theorem's mass bound)
+ *   5  ||O-hat - O||_2 for O-hat = certkv_decode_attn(q, packed, tail_slot)
+ *   6  V_max
+ *   7  ||p_S O~_S + (1 - p_S) V-bar_T - O||_2, the factorization residual
+ * q bf16 [B][L][Hq][d]; K, V as for certkv_compress; workspace:
+ * certkv_fixed_row_workspace_bytes(shape). */
+size_t certkv_fixed_row_workspace_bytes(const certkv_shape* shape);
+int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void* K, const void* V,
+                           const certkv_packed* packed, float scale, int32_t tail_slot,
+                           float* stats, void* workspace, size_t workspace_bytes, void* stream);
+
 /* Decode attention that allocates nothing.  The paper has no counterpart: this
  * entry point exists for callers that cannot hand the library a scratch
  * buffer, for example a plugin that an inference server gives only its input

@@ -63,6 +63,8 @@ def _bind(lib):
     lib.oracle_tail_clusters.restype = None
     lib.oracle_decode_certified.argtypes = [P, P, P, I, I, D, P, P, P, P, P, I, P, P, P]
     lib.oracle_decode_certified.restype = D
+    lib.oracle_fixed_row.argtypes = [P, P, P, P, I, I, D, P, P]
+    lib.oracle_fixed_row.restype = None
     lib.oracle_compress.restype = I
     lib.oracle_decode.argtypes = [P, D, P, P, P, P, P, I, P]
     lib.oracle_decode.restype = None
@@ -279,6 +281,20 @@ def decode_certified(q, pk, pv, kbar, vbar, count, rk, rv, *, scale: float, lib=
         _ptr(q), _ptr(pk), _ptr(pv), int(b), int(d), float(scale), _ptr(kbar), _ptr(vbar),
         _ptr(count), _ptr(rk), _ptr(rv), int(m), _ptr(out), _ptr(cert), _ptr(struct))
     return out, float(bound), bool(cert[0]), float(struct[0])
+
+
+def fixed_row(q, K, V, kept, *, scale: float, ohat=None, lib=None) -> np.ndarray:
+    """Fixed-row quantities of one query row over all n tokens of a unit:
+    q uint16 [d], K, V uint16 [n][d], kept bool [n], ohat float64 [d] or None.
+    Returns stats [8] (see oracle_fixed_row)."""
+    q = _u16(q); K = _u16(K); V = _u16(V)
+    n, d = K.shape
+    kept = np.ascontiguousarray(kept, dtype=np.uint8)
+    st = np.zeros(8)
+    oh = None if ohat is None else np.ascontiguousarray(ohat, dtype=np.float64)
+    (lib or _load()).oracle_fixed_row(_ptr(q), _ptr(K), _ptr(V), _ptr(kept), n, d, float(scale),
+                                      _ptr(oh) if oh is not None else None, _ptr(st))
+    return st
 
 
 def decode(q, pk, pv, offsets, counts, *, B: int, L: int, Hq: int, H: int, d: int,

@@ -713,3 +713,74 @@ double oracle_decode_certified(const uint16_t* q, const uint16_t* pk, const uint
   free(lg);
   return 3.0 / Z * (DN + vmax * DZ);
 }
+
+/* ------------------------------------------------- fixed-row diagnostics ---- */
+
+/*
+ * Fixed-row quantities of one realized query row over all n original tokens
+ * of a unit (Theorem: fixed-row tail factorization).  A_j = softmax_j(scale
+ * <q, k_j>); S = the tokens with kept[j] != 0.  Writes stats[8]:
+ *   0 p_S = sum_{j in S} A_j
+ *   1 ||O||_2, O = sum_j A_j v_j (exact attention)
+ *   2 ||O~_S - O||_2, O~_S = sum_{j in S} A_j v_j / p_S (subset-only output)
+ *   3 ||u*||_2, u* = sum_{j not in S} A_j v_j (the unique fixed-row correction)
+ *   4 2 V_max (1 - p_S), V_max = max_j ||v_j||_2 (the theorem's mass bound)
+ *   5 ||ohat - O||_2 for the given output ohat [d] (NULL: 0)
+ *   6 V_max
+ *   7 ||O~_S + (1 - p_S) (V-bar_T - O~_S) - O||_2, the factorization residual
+ *     (0 up to rounding; V-bar_T = u* / (1 - p_S))
+ */
+void oracle_fixed_row(const uint16_t* q, const uint16_t* K, const uint16_t* V,
+                      const uint8_t* kept, int n, int d, double scale, const double* ohat,
+                      double* stats) {
+  double* lg = (double*)malloc((size_t)n * sizeof(double));
+  double* O = (double*)calloc((size_t)d, sizeof(double));
+  double* OS = (double*)calloc((size_t)d, sizeof(double));
+  double mx = -INFINITY, vmax = 0.0;
+  for (int j = 0; j < n; ++j) {
+    double dot = 0.0, vv = 0.0;
+    for (int i = 0; i < d; ++i) {
+      dot += bf16_to_f64(q[i]) * bf16_to_f64(K[(size_t)j * d + i]);
+      vv += bf16_to_f64(V[(size_t)j * d + i]) * bf16_to_f64(V[(size_t)j * d + i]);
+    }
+    lg[j] = scale * dot;
+    if (lg[j] > mx) mx = lg[j];
+    if (sqrt(vv) > vmax) vmax = sqrt(vv);
+  }
+  double Z = 0.0, ZS = 0.0;
+  for (int j = 0; j < n; ++j) {
+    const double w = exp(lg[j] - mx);
+    Z += w;
+    if (kept[j]) ZS += w;
+    for (int i = 0; i < d; ++i) {
+      const double x = w * bf16_to_f64(V[(size_t)j * d + i]);
+      O[i] += x;
+      if (kept[j]) OS[i] += x;
+    }
+  }
+  const double pS = ZS / Z;
+  double nO = 0.0, eS = 0.0, nu = 0.0, eh = 0.0, res = 0.0;
+  for (int i = 0; i < d; ++i) {
+    const double o = O[i] / Z;
+    const double os = ZS > 0.0 ? OS[i] / ZS : 0.0;
+    const double u = (O[i] - OS[i]) / Z;
+    const double vbt = pS < 1.0 ? u / (1.0 - pS) : 0.0;
+    nO += o * o;
+    eS += (os - o) * (os - o);
+    nu += u * u;
+    if (ohat) eh += (ohat[i] - o) * (ohat[i] - o);
+    const double f = os + (1.0 - pS) * (vbt - os) - o;
+    res += f * f;
+  }
+  stats[0] = pS;
+  stats[1] = sqrt(nO);
+  stats[2] = sqrt(eS);
+  stats[3] = sqrt(nu);
+  stats[4] = 2.0 * vmax * (1.0 - pS);
+  stats[5] = sqrt(eh);
+  stats[6] = vmax;
+  stats[7] = sqrt(res);
+  free(lg);
+  free(O);
+  free(OS);
+}

@@ -51,7 +51,8 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_compress_scored", "certkv_compress", "certkv_decode_attn",
             "certkv_read_status", "certkv_strerror", "certkv_trace_enable",
             "certkv_trace_report", "certkv_decode_attn_noalloc", "certkv_host_workspace_bytes",
-            "certkv_compress_host", "certkv_decode_certified")
+            "certkv_compress_host", "certkv_decode_certified", "certkv_fixed_row_workspace_bytes",
+            "certkv_fixed_row_stats")
 
 _lock = threading.Lock()
 _lib = None
@@ -111,6 +112,10 @@ def load_library(path: Optional[str] = None):
         lib.certkv_decode_certified.argtypes = [sp, P, kp, ctypes.c_float, I32, I32, P, P, P, P,
                                                 SZ, P]
         lib.certkv_decode_certified.restype = ctypes.c_int
+        lib.certkv_fixed_row_workspace_bytes.argtypes = [sp]
+        lib.certkv_fixed_row_workspace_bytes.restype = SZ
+        lib.certkv_fixed_row_stats.argtypes = [sp, P, P, P, kp, ctypes.c_float, I32, P, P, SZ, P]
+        lib.certkv_fixed_row_stats.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -385,6 +390,31 @@ def certkv_decode_certified(q, packed: Packed, *, hkv: int, scale: float = 0.0, 
                                                 _stream(stream))
     _check(rc, "certkv_decode_certified")
     return out, bound, certified
+
+
+FIXED_ROW_FIELDS = ("kept_mass", "norm_O", "err_subset", "norm_correction", "mass_bound",
+                    "err_decode", "v_max", "factorization_residual")
+
+
+def certkv_fixed_row_stats(q, K, V, packed: Packed, *, scale: float = 0.0, stats=None, ws=None,
+                           stream=None) -> torch.Tensor:
+    """Fixed-row diagnostics per query head: fp32 [B][L][Hq][8] in the order of
+    FIXED_ROW_FIELDS (evaluation tool; reads the full K and V)."""
+    _bf16(q, "q"); _bf16(K, "K"); _bf16(V, "V")
+    B, L, Hq, d = q.shape
+    shape = certkv_shape(B, L, Hq, K.shape[2], K.shape[3], d, 1)
+    if stats is None:
+        stats = torch.empty((B, L, Hq, 8), dtype=torch.float32, device=q.device)
+    if ws is None:
+        ws = workspace(int(load_library().certkv_fixed_row_workspace_bytes(ctypes.byref(shape))),
+                       q.device)
+    st = packed.struct()
+    rc = load_library().certkv_fixed_row_stats(ctypes.byref(shape), _ptr(q), _ptr(K), _ptr(V),
+                                               ctypes.byref(st), float(scale),
+                                               int(packed.tail_slot), _ptr(stats), _ptr(ws),
+                                               ws.numel(), _stream(stream))
+    _check(rc, "certkv_fixed_row_stats")
+    return stats
 
 
 def certkv_read_status(ws: torch.Tensor, stream=None) -> int:

@@ -457,6 +457,46 @@ def pin_packed_layout_with_clusters(lib=None):
     assert r["offsets"][-1] == B * L * B_live
 
 
+def pin_fixed_row_three_tokens(lib=None):
+    """Fixed-row quantities in closed form: q = e1, scale 1, keys 0, 0, e1
+    (logits 0, 0, 1, so A = (1, 1, e) / (2 + e)), values e1, e2, (1, 1), the
+    first token kept: p_S = 1/(2+e), O = (1+e)(1, 1)/(2+e), O~_S = e1,
+    u* = (e, 1+e)/(2+e), V_max = sqrt 2."""
+    e = math.e
+    o = (1 + e) / (2 + e)
+    want = [1 / (2 + e), math.sqrt(2) * o, math.hypot(1 - o, o), math.hypot(e / (2 + e), o),
+            2 * math.sqrt(2) * (1 - 1 / (2 + e))]
+    st = oracle.fixed_row(to_bf16_bits([1.0, 0.0]), to_bf16_bits([[0, 0], [0, 0], [1, 0]]),
+                          to_bf16_bits([[1, 0], [0, 1], [1, 1]]), np.array([1, 0, 0]), scale=1.0,
+                          lib=lib)
+    for i, w in enumerate(want):
+        assert abs(st[i] - w) < 1e-12, (i, st[i], w)
+
+
+def pin_fixed_row_factorization(lib=None):
+    """Theorem (fixed-row tail factorization) on random rows: O = p_S O~_S +
+    (1 - p_S) V-bar_T exactly (residual at rounding level), the subset-only
+    error obeys ||O~_S - O|| <= 2 V_max (1 - p_S), keeping every token gives
+    p_S = 1 and no error, and ohat = O gives no error."""
+    rng = np.random.default_rng(41)
+    for _ in range(20):
+        n, d = int(rng.integers(5, 80)), int(rng.choice([4, 16]))
+        K = to_bf16_bits(rng.normal(size=(n, d)))
+        V = to_bf16_bits(rng.normal(size=(n, d)))
+        q = to_bf16_bits(rng.normal(size=d))
+        kept = rng.random(n) < 0.3
+        kept[0] = True
+        st = oracle.fixed_row(q, K, V, kept, scale=0.5, lib=lib)
+        assert st[7] < 1e-12 and st[2] <= st[4] * (1 + 1e-12)
+        lg = 0.5 * (bf(K) @ bf(q))
+        w = np.exp(lg - lg.max())
+        exact = (w[:, None] * bf(V)).sum(0) / w.sum()
+        st2 = oracle.fixed_row(q, K, V, kept, scale=0.5, ohat=exact, lib=lib)
+        assert st2[5] < 1e-12
+        st3 = oracle.fixed_row(q, K, V, np.ones(n, bool), scale=0.5, lib=lib)
+        assert abs(st3[0] - 1.0) < 1e-15 and st3[2] < 1e-12 and st3[3] < 1e-12
+
+
 def pin_allocation_infeasible(lib=None):
     """B_real above H (n - 1) cannot be met with b_h <= n - 1."""
     curves = np.ones((2, 5))

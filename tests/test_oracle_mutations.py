@@ -43,6 +43,8 @@ MUTANTS = {
                                        "DN += er * zg * ((er - 1.0) * vn);"),
     "cluster_groups_overlap_kept": ("const int r0 = b + (int)(((int64_t)g * T) / m),",
                                     "const int r0 = (g == 0 ? b - 1 : b) + (int)(((int64_t)g * T) / m),"),
+    "fixed_row_subset_not_renormalised": ("const double os = ZS > 0.0 ? OS[i] / ZS : 0.0;",
+                                          "const double os = OS[i] / Z;"),
     "bisection_inverted": ("if (total > B_real) lam_lo = lam; else lam_hi = lam;",
                            "if (total > B_real) lam_hi = lam; else lam_lo = lam;"),
     "kept_not_sorted": ("qsort(kept, (size_t)b, sizeof(int32_t), cmp_int32);", ""),
