@@ -123,6 +123,10 @@ Layout make_layout(const Prob& p) {
   const size_t segs = (size_t)((p.n - 1 + kHullSeg - 1) / kHullSeg);
   const size_t groups = (segs + kGroupSegs - 1) / kGroupSegs;
   ly.ncand = take(U * (segs + groups) * sizeof(int32_t));
+  const size_t mc = (size_t)p.clusters;
+  ly.cl_sum = take(U * mc * 8 * 2 * kD * sizeof(float) * 2);
+  ly.cl_mean = take(U * mc * 2 * kD * sizeof(float));
+  ly.cl_max = take(U * mc * 8 * sizeof(float) * 2);
   ly.total = off;
   return ly;
 }

@@ -59,6 +59,9 @@ struct Layout {
   size_t cmax;       // uint64 [U]     order key of max_b c(b)
   size_t cand;       // int32  [U][n]  allocator candidates
   size_t ncand;      // int32  [U][hull_segs + groups] survivors per segment, per group
+  size_t cl_sum;     // float2 [U][m][8 parts][2][d]  cluster part sums (m = clusters)
+  size_t cl_mean;    // float  [U][m][2][d]           stored cluster means
+  size_t cl_max;     // float2 [U][m][8 parts]        cluster part radii
   size_t total;
 };
 

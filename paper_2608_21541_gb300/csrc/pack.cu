@@ -13,6 +13,10 @@
 
 namespace certkv {
 
+// stored radii and norms are rounded up by this factor so that they stay upper
+// bounds (fp32 sums of 128 squares and square roots are within a few 1e-6)
+constexpr float kRadiusRoundUp = 1.0f + 1e-5f;
+
 // grid = units, block = 128 (one thread per dimension)
 __global__ void __launch_bounds__(128) tail_kernel(
     Prob p, const uint32_t* __restrict__ keys, const int32_t* __restrict__ perm,
@@ -149,7 +153,8 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloa
                                                         const int64_t* __restrict__ offsets,
                                                         const int32_t* __restrict__ positions,
                                                         __nv_bfloat16* __restrict__ pk,
-                                                        __nv_bfloat16* __restrict__ pv) {
+                                                        __nv_bfloat16* __restrict__ pv,
+                                                        float* __restrict__ kept_vmax) {
   const int u = blockIdx.x;
   const int b = counts[u];
   const int64_t off = offsets[u];
@@ -160,7 +165,11 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloa
   // 16 uint4 per row; 256 threads = 16 rows per step, 4 steps' loads in flight
   const int sub = threadIdx.x & 15;
   const int stride = gridDim.y * 16;
-  for (int row0 = blockIdx.y * 16 + (threadIdx.x >> 4); row0 < b; row0 += 4 * stride) {
+  float vmax = 0.f;
+  // the loop bound is the warp's first row, so both half-warps run the same
+  // iterations (the row-norm shuffles need the whole warp)
+  for (int wrow0 = blockIdx.y * 16 + (threadIdx.x >> 5) * 2; wrow0 < b; wrow0 += 4 * stride) {
+    const int row0 = wrow0 + ((threadIdx.x >> 4) & 1);
     int j[4];
     uint4 kx[4], vx[4];
 #pragma unroll
@@ -182,6 +191,29 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloa
         PV[(size_t)(off + row) * 16 + sub] = vx[e];
       }
     }
+    if (kept_vmax) {  // largest ||v|| of the kept rows (for the clustered-tail bound)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const uint32_t w[4] = {vx[e].x, vx[e].y, vx[e].z, vx[e].w};
+        float sq = 0.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const float a = bf16lo(w[c]), b2 = bf16hi(w[c]);
+          sq = fmaf(a, a, fmaf(b2, b2, sq));
+        }
+#pragma unroll
+        for (int o = 8; o >= 1; o >>= 1) sq += __shfl_xor_sync(kFull, sq, o);  // the row's 16 threads
+        vmax = fmaxf(vmax, sqrtf(sq));
+      }
+    }
+  }
+  if (kept_vmax) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) vmax = fmaxf(vmax, __shfl_xor_sync(kFull, vmax, o));
+    // non-negative floats order like their bit patterns
+    if ((threadIdx.x & 31) == 0)
+      atomicMax(reinterpret_cast<unsigned int*>(kept_vmax) + u,
+                __float_as_uint(vmax * kRadiusRoundUp));
   }
 }
 
@@ -191,122 +223,205 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloa
 // (T = n - b); stored representatives = the bf16-rounded unweighted means,
 // radii = the largest distances of the group's rows to them, rounded up by
 // 1e-5 relative (the fp32 sum of 128 squares and the square root are within
-// a few 1e-6 of exact).  grid = (units, m + 1), block = 512 (warp per row,
-// 4 rows in flight); blockIdx.y = m computes the kept rows' largest ||v||.
-constexpr int kClusterWarps = 16;
-constexpr float kRadiusRoundUp = 1.0f + 1e-5f;
-__global__ void __launch_bounds__(kClusterWarps * 32) cluster_kernel(
-    Prob p, const int32_t* __restrict__ perm, const __nv_bfloat16* __restrict__ K,
-    const __nv_bfloat16* __restrict__ V, const int32_t* __restrict__ counts,
-    const int64_t* __restrict__ offsets, __nv_bfloat16* __restrict__ pk,
-    __nv_bfloat16* __restrict__ pv, int32_t* __restrict__ positions,
-    float4* __restrict__ cluster_meta, float* __restrict__ kept_vmax) {
-  __shared__ DF s_sum[kClusterWarps][2][kD];
-  __shared__ float s_mean[2][kD];
-  __shared__ float s_max[kClusterWarps][2];
-  const int u = blockIdx.x, g = blockIdx.y, m = p.clusters;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n = p.n, b = counts[u];
-  const int32_t* pu = perm + (size_t)u * n;
-  const uint2* Ku = reinterpret_cast<const uint2*>(K + (size_t)u * n * kD);
-  const uint2* Vu = reinterpret_cast<const uint2*>(V + (size_t)u * n * kD);
-  auto row4 = [&](const uint2* base, int j, float (&x)[4]) {
-    const uint2 raw = __ldg(base + (size_t)j * (kD / 4) + lane);
-    x[0] = bf16lo(raw.x);
-    x[1] = bf16hi(raw.x);
-    x[2] = bf16lo(raw.y);
-    x[3] = bf16hi(raw.y);
-  };
-  auto block_max = [&](float a, float c, float& ra, float& rc) {
-    if (lane == 0) {
-      s_max[warp][0] = a;
-      s_max[warp][1] = c;
-    }
-    __syncthreads();
-    ra = rc = 0.f;
-    for (int w = 0; w < kClusterWarps; ++w) {
-      ra = fmaxf(ra, s_max[w][0]);
-      rc = fmaxf(rc, s_max[w][1]);
-    }
-  };
-  if (g == m) {  // largest value norm over the kept ranks 0 .. b-1
-    float mx = 0.f;
-    for (int r = warp; r < b; r += kClusterWarps) {
-      float v[4];
-      row4(Vu, pu[r], v);
-      float sq = fmaf(v[3], v[3], fmaf(v[2], v[2], fmaf(v[1], v[1], v[0] * v[0])));
-#pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) sq += __shfl_xor_sync(kFull, sq, o);
-      mx = fmaxf(mx, sqrtf(sq));
-    }
-    float ra, rc;
-    block_max(mx, 0.f, ra, rc);
-    if (threadIdx.x == 0) kept_vmax[u] = ra * kRadiusRoundUp;
-    return;
-  }
+// a few 1e-6 of exact).  Each group is cut into kClusterParts contiguous
+// parts, one CTA each (warp per row, four rows in flight):
+//   cluster_sum     part sums of the keys and values (fp32 over 32 rows,
+//                   folded into double-float);
+//   cluster_mean    the parts added in a fixed order, the mean rounded and
+//                   stored in the summary slot;
+//   cluster_radius  part maxima of the distances to the stored means;
+//   cluster_meta    the maxima over the parts, rounded up.
+constexpr int kClusterParts = 8;
+constexpr int kClusterWarps = 8;
+
+namespace {
+__device__ __forceinline__ void cluster_rows(const Prob& p, const int32_t* counts, int u, int g,
+                                             int part, int& lo, int& hi) {
+  const int n = p.n, b = counts[u], m = p.clusters;
   const int T = n - b;
   const int r0 = b + (int)(((int64_t)g * T) / m), r1 = b + (int)(((int64_t)(g + 1) * T) / m);
   const int cnt = r1 - r0;
-  // 1. unweighted means: double-float sums per lane (4 dimensions), then per dimension
+  lo = r0 + (int)(((int64_t)part * cnt) / kClusterParts);
+  hi = r0 + (int)(((int64_t)(part + 1) * cnt) / kClusterParts);
+}
+__device__ __forceinline__ void load_row4(const uint2* base, int j, int lane, float (&x)[4]) {
+  const uint2 raw = __ldg(base + (size_t)j * (kD / 4) + lane);
+  x[0] = bf16lo(raw.x);
+  x[1] = bf16hi(raw.x);
+  x[2] = bf16lo(raw.y);
+  x[3] = bf16hi(raw.y);
+}
+}  // namespace
+
+// grid = (units, m, kClusterParts), block = 32 * kClusterWarps.
+// part_sum [u][g][part][2][kD] double-float (hi, lo).
+__global__ void __launch_bounds__(kClusterWarps * 32) cluster_sum_kernel(
+    Prob p, const int32_t* __restrict__ perm, const __nv_bfloat16* __restrict__ K,
+    const __nv_bfloat16* __restrict__ V, const int32_t* __restrict__ counts,
+    float2* __restrict__ part_sum) {
+  __shared__ DF s_sum[kClusterWarps][2][kD];
+  const int u = blockIdx.x, g = blockIdx.y, part = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = p.n;
+  const int32_t* pu = perm + (size_t)u * n;
+  const uint2* Ku = reinterpret_cast<const uint2*>(K + (size_t)u * n * kD);
+  const uint2* Vu = reinterpret_cast<const uint2*>(V + (size_t)u * n * kD);
+  int lo, hi;
+  cluster_rows(p, counts, u, g, part, lo, hi);
   DF sk[4], sv[4];
 #pragma unroll
   for (int c = 0; c < 4; ++c) sk[c] = sv[c] = df_make(0.f);
-  for (int r = r0 + warp; r < r1; r += kClusterWarps) {
-    const int j = pu[r];
-    float k4[4], v4[4];
-    row4(Ku, j, k4);
-    row4(Vu, j, v4);
+  int in_block = 0;
+  float fk[4] = {0.f, 0.f, 0.f, 0.f}, fv[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int rb = lo + warp; rb < hi; rb += 4 * kClusterWarps) {
+    float k4[4][4], v4[4][4];
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      sk[c] = df_add_f(sk[c], k4[c]);
-      sv[c] = df_add_f(sv[c], v4[c]);
+    for (int e = 0; e < 4; ++e) {
+      const int r = rb + e * kClusterWarps;
+      if (r < hi) {
+        const int j = pu[r];
+        load_row4(Ku, j, lane, k4[e]);
+        load_row4(Vu, j, lane, v4[e]);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      if (rb + e * kClusterWarps >= hi) break;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        fk[c] += k4[e][c];
+        fv[c] += v4[e][c];
+      }
+    }
+    in_block += 4;
+    if (in_block >= 32) {  // fp32 over 32 rows, then double-float
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        sk[c] = df_add_f(sk[c], fk[c]);
+        sv[c] = df_add_f(sv[c], fv[c]);
+        fk[c] = fv[c] = 0.f;
+      }
+      in_block = 0;
     }
   }
 #pragma unroll
   for (int c = 0; c < 4; ++c) {
-    s_sum[warp][0][lane * 4 + c] = sk[c];
-    s_sum[warp][1][lane * 4 + c] = sv[c];
+    s_sum[warp][0][lane * 4 + c] = df_add_f(sk[c], fk[c]);
+    s_sum[warp][1][lane * 4 + c] = df_add_f(sv[c], fv[c]);
   }
   __syncthreads();
+  const int t = threadIdx.x / kD, i = threadIdx.x % kD;  // 256 threads = 2 tensors x kD
+  DF sum = df_make(0.f);
+  for (int w = 0; w < kClusterWarps; ++w) sum = df_add(sum, s_sum[w][t][i]);
+  part_sum[((((size_t)u * p.clusters + g) * kClusterParts + part) * 2 + t) * kD + i] =
+      make_float2(sum.hi, sum.lo);
+}
+
+// grid = (units, m), block = 256.  means [u][g][2][kD] fp32 = the stored
+// bf16 values.
+__global__ void __launch_bounds__(256) cluster_mean_kernel(
+    Prob p, const int32_t* __restrict__ counts, const int64_t* __restrict__ offsets,
+    const float2* __restrict__ part_sum, float* __restrict__ means, __nv_bfloat16* __restrict__ pk,
+    __nv_bfloat16* __restrict__ pv, int32_t* __restrict__ positions) {
+  const int u = blockIdx.x, g = blockIdx.y, m = p.clusters;
+  const int n = p.n, b = counts[u];
+  const int T = n - b;
+  const int cnt = (int)(((int64_t)(g + 1) * T) / m) - (int)(((int64_t)g * T) / m);
+  const int t = threadIdx.x / kD, i = threadIdx.x % kD;
+  DF sum = df_make(0.f);
+  for (int part = 0; part < kClusterParts; ++part) {
+    const float2 x = part_sum[((((size_t)u * m + g) * kClusterParts + part) * 2 + t) * kD + i];
+    sum = df_add(sum, DF{x.x, x.y});
+  }
+  const DF mean = cnt > 0 ? df_div(sum, df_make((float)cnt)) : df_make(0.f);
+  const uint16_t bits = df_to_bf16(mean.hi, mean.lo);
   const int64_t slot = offsets[u] + b + p.tail_slot + g;
-  if (threadIdx.x < 2 * kD) {
-    const int t = threadIdx.x / kD, i = threadIdx.x % kD;
-    DF sum = df_make(0.f);
-    for (int w = 0; w < kClusterWarps; ++w) sum = df_add(sum, s_sum[w][t][i]);
-    const DF mean = cnt > 0 ? df_div(sum, df_make((float)cnt)) : df_make(0.f);
-    const uint16_t bits = df_to_bf16(mean.hi, mean.lo);
-    reinterpret_cast<uint16_t*>(t == 0 ? pk : pv)[slot * kD + i] = bits;
-    s_mean[t][i] = __uint_as_float((uint32_t)bits << 16);
-  }
+  reinterpret_cast<uint16_t*>(t == 0 ? pk : pv)[slot * kD + i] = bits;
+  means[(((size_t)u * m + g) * 2 + t) * kD + i] = __uint_as_float((uint32_t)bits << 16);
   if (threadIdx.x == 0) positions[slot] = -2 - g;
+}
+
+// grid = (units, m, kClusterParts), block = 32 * kClusterWarps.
+// part_max [u][g][part] = (largest key distance, largest value distance).
+__global__ void __launch_bounds__(kClusterWarps * 32) cluster_radius_kernel(
+    Prob p, const int32_t* __restrict__ perm, const __nv_bfloat16* __restrict__ K,
+    const __nv_bfloat16* __restrict__ V, const int32_t* __restrict__ counts,
+    const float* __restrict__ means, float2* __restrict__ part_max) {
+  __shared__ float s_mean[2][kD];
+  __shared__ float s_max[kClusterWarps][2];
+  const int u = blockIdx.x, g = blockIdx.y, part = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = p.n;
+  const int32_t* pu = perm + (size_t)u * n;
+  const uint2* Ku = reinterpret_cast<const uint2*>(K + (size_t)u * n * kD);
+  const uint2* Vu = reinterpret_cast<const uint2*>(V + (size_t)u * n * kD);
+  (&s_mean[0][0])[threadIdx.x] = means[((size_t)u * p.clusters + g) * 2 * kD + threadIdx.x];
   __syncthreads();
-  // 2. radii to the stored representatives: warp per row
+  int lo, hi;
+  cluster_rows(p, counts, u, g, part, lo, hi);
   float mk = 0.f, mv = 0.f;
-  for (int r = r0 + warp; r < r1; r += kClusterWarps) {
-    const int j = pu[r];
-    float k4[4], v4[4];
-    row4(Ku, j, k4);
-    row4(Vu, j, v4);
-    float qk = 0.f, qv = 0.f;
+  for (int rb = lo + warp; rb < hi; rb += 4 * kClusterWarps) {
+    float k4[4][4], v4[4][4];
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const float dk = k4[c] - s_mean[0][lane * 4 + c], dv = v4[c] - s_mean[1][lane * 4 + c];
-      qk = fmaf(dk, dk, qk);
-      qv = fmaf(dv, dv, qv);
+    for (int e = 0; e < 4; ++e) {
+      const int r = rb + e * kClusterWarps;
+      if (r < hi) {
+        const int j = pu[r];
+        load_row4(Ku, j, lane, k4[e]);
+        load_row4(Vu, j, lane, v4[e]);
+      }
     }
 #pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-      qk += __shfl_xor_sync(kFull, qk, o);
-      qv += __shfl_xor_sync(kFull, qv, o);
+    for (int e = 0; e < 4; ++e) {
+      if (rb + e * kClusterWarps >= hi) break;
+      float qk = 0.f, qv = 0.f;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float dk = k4[e][c] - s_mean[0][lane * 4 + c];
+        const float dv = v4[e][c] - s_mean[1][lane * 4 + c];
+        qk = fmaf(dk, dk, qk);
+        qv = fmaf(dv, dv, qv);
+      }
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) {
+        qk += __shfl_xor_sync(kFull, qk, o);
+        qv += __shfl_xor_sync(kFull, qv, o);
+      }
+      mk = fmaxf(mk, sqrtf(qk));
+      mv = fmaxf(mv, sqrtf(qv));
     }
-    mk = fmaxf(mk, sqrtf(qk));
-    mv = fmaxf(mv, sqrtf(qv));
   }
-  float rk, rv;
-  block_max(mk, mv, rk, rv);
-  if (threadIdx.x == 0)
-    cluster_meta[(size_t)u * m + g] = make_float4((float)cnt, rk * kRadiusRoundUp,
-                                                  rv * kRadiusRoundUp, 0.f);
+  if (lane == 0) {
+    s_max[warp][0] = mk;
+    s_max[warp][1] = mv;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float a = 0.f, c = 0.f;
+    for (int w = 0; w < kClusterWarps; ++w) {
+      a = fmaxf(a, s_max[w][0]);
+      c = fmaxf(c, s_max[w][1]);
+    }
+    part_max[((size_t)u * p.clusters + g) * kClusterParts + part] = make_float2(a, c);
+  }
+}
+
+// grid = units, block = 64 (thread = group g < m)
+__global__ void cluster_meta_kernel(Prob p, const int32_t* __restrict__ counts,
+                                    const float2* __restrict__ part_max,
+                                    float4* __restrict__ cluster_meta) {
+  const int u = blockIdx.x, g = threadIdx.x, m = p.clusters;
+  if (g >= m) return;
+  const int T = p.n - counts[u];
+  const int cnt = (int)(((int64_t)(g + 1) * T) / m) - (int)(((int64_t)g * T) / m);
+  float a = 0.f, c = 0.f;
+  for (int part = 0; part < kClusterParts; ++part) {
+    const float2 x = part_max[((size_t)u * m + g) * kClusterParts + part];
+    a = fmaxf(a, x.x);
+    c = fmaxf(c, x.y);
+  }
+  cluster_meta[(size_t)u * m + g] =
+      make_float4((float)cnt, a * kRadiusRoundUp, c * kRadiusRoundUp, 0.f);
 }
 
 void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const void* V,
@@ -328,14 +443,34 @@ void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const
   if (ysplit > 64) ysplit = 64;
   {
     TraceScope ts("copy_rows", st);
-    copy_rows_kernel<<<dim3(p.units, ysplit), 256, 0, st>>>(p, Kb, Vb, counts, offsets,
-                                                           positions, PK, PV);
+    if (p.clusters > 0) cudaMemsetAsync(kept_vmax, 0, (size_t)p.units * sizeof(float), st);
+    copy_rows_kernel<<<dim3(p.units, ysplit), 256, 0, st>>>(
+        p, Kb, Vb, counts, offsets, positions, PK, PV, p.clusters > 0 ? kept_vmax : nullptr);
   }
   if (p.clusters > 0) {
-    TraceScope ts("clusters", st);
-    cluster_kernel<<<dim3(p.units, p.clusters + 1), kClusterWarps * 32, 0, st>>>(
-        p, perm, Kb, Vb, counts, offsets, PK, PV, positions,
-        reinterpret_cast<float4*>(cluster_meta), kept_vmax);
+    float2* part_sum = reinterpret_cast<float2*>(ws + ly.cl_sum);
+    float* means = reinterpret_cast<float*>(ws + ly.cl_mean);
+    float2* part_max = reinterpret_cast<float2*>(ws + ly.cl_max);
+    const dim3 gp(p.units, p.clusters, kClusterParts);
+    {
+      TraceScope ts("cluster_sum", st);
+      cluster_sum_kernel<<<gp, kClusterWarps * 32, 0, st>>>(p, perm, Kb, Vb, counts, part_sum);
+    }
+    {
+      TraceScope ts("cluster_mean", st);
+      cluster_mean_kernel<<<dim3(p.units, p.clusters), 256, 0, st>>>(p, counts, offsets, part_sum,
+                                                                     means, PK, PV, positions);
+    }
+    {
+      TraceScope ts("cluster_radius", st);
+      cluster_radius_kernel<<<gp, kClusterWarps * 32, 0, st>>>(p, perm, Kb, Vb, counts, means,
+                                                               part_max);
+    }
+    {
+      TraceScope ts("cluster_meta", st);
+      cluster_meta_kernel<<<p.units, 64, 0, st>>>(p, counts, part_max,
+                                                  reinterpret_cast<float4*>(cluster_meta));
+    }
   }
   if (p.tail_slot) {
     TraceScope ts("tail", st);
