@@ -65,6 +65,8 @@ def _bind(lib):
     lib.oracle_decode_certified.restype = D
     lib.oracle_fixed_row.argtypes = [P, P, P, P, I, I, D, P, P]
     lib.oracle_fixed_row.restype = None
+    lib.oracle_future_query_lift.argtypes = [P, P, P, P, P, P, P, I, I, D, P]
+    lib.oracle_future_query_lift.restype = None
     lib.oracle_compress.restype = I
     lib.oracle_decode.argtypes = [P, D, P, P, P, P, P, I, P]
     lib.oracle_decode.restype = None
@@ -294,6 +296,25 @@ def fixed_row(q, K, V, kept, *, scale: float, ohat=None, lib=None) -> np.ndarray
     oh = None if ohat is None else np.ascontiguousarray(ohat, dtype=np.float64)
     (lib or _load()).oracle_fixed_row(_ptr(q), _ptr(K), _ptr(V), _ptr(kept), n, d, float(scale),
                                       _ptr(oh) if oh is not None else None, _ptr(st))
+    return st
+
+
+def future_query_lift(q, K, V, kept, s, *, scale: float, kstar=None, vstar=None,
+                      lib=None) -> np.ndarray:
+    """Future-query lift quantities of one query row (see
+    oracle_future_query_lift): q uint16 [d], K, V uint16 [n][d], kept bool
+    [n], s float32 [n] (the compression scores; only the tail entries are
+    read), kstar, vstar uint16 [d] or None (no synthetic slot).  Returns [8]."""
+    q = _u16(q); K = _u16(K); V = _u16(V)
+    n, d = K.shape
+    kept = np.ascontiguousarray(kept, dtype=np.uint8)
+    s = np.ascontiguousarray(s, dtype=np.float32)
+    ks = None if kstar is None else _u16(kstar)
+    vs = None if vstar is None else _u16(vstar)
+    st = np.zeros(8)
+    (lib or _load()).oracle_future_query_lift(
+        _ptr(q), _ptr(K), _ptr(V), _ptr(kept), _ptr(s), _ptr(ks) if ks is not None else None,
+        _ptr(vs) if vs is not None else None, n, d, float(scale), _ptr(st))
     return st
 
 

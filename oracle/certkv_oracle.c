@@ -784,3 +784,102 @@ void oracle_fixed_row(const uint16_t* q, const uint16_t* K, const uint16_t* V,
   free(O);
   free(OS);
 }
+
+/*
+ * Future-query lift and summary mismatch (Theorem: future-query lift), for
+ * one realized query row over all n original tokens of a unit.  S = the
+ * tokens with kept[j] != 0, T = the others (nonempty); the compressed cache
+ * holds S and, when kstar != NULL, one synthetic slot (kstar, vstar) whose
+ * value stands for the mixture sum_T r_j v_j with r_j = s_j / sum_T s (the
+ * uniform 1/|T| when that sum is 0).  z_j = scale <q, k_j>, A = softmax(z)
+ * over all n tokens, Ahat = softmax over S and the slot.  Writes stats[8]:
+ *   0 p = A(T), the exact attention mass of the tail
+ *   1 q = Ahat_star, the slot's weight in compressed attention (0 without a slot)
+ *   2 ||a - r||_1 over T with a = A_T / p (a = 0 when p = 0)
+ *   3 Lambda_T - z_star, Lambda_T = log sum_T e^{z_j}, z_star = scale <q, kstar>
+ *     (NaN without a slot)
+ *   4 V_max (2 |p - q| + min(p, q) ||a - r||_1), the theorem's bound on
+ *     ||O - Ohat|| when the slot value is the exact mixture
+ *   5 tanh(|Lambda_T - z_star| / 4), the theorem's bound on |p - q| (NaN without a slot)
+ *   6 ||A - Abar||_1, Abar = Ahat on S and q r_j on T (the lifted distribution)
+ *   7 ||vstar - sum_T r_j v_j||_2, the stored slot value against the exact
+ *     mixture (NaN without a slot or when sum_T s = 0)
+ */
+void oracle_future_query_lift(const uint16_t* q, const uint16_t* K, const uint16_t* V,
+                              const uint8_t* kept, const float* s, const uint16_t* kstar,
+                              const uint16_t* vstar, int n, int d, double scale,
+                              double* stats) {
+  double* z = (double*)malloc((size_t)n * sizeof(double));
+  double zmax = -INFINITY, zmaxS = -INFINITY, zmaxT = -INFINITY, vmax = 0.0, sT = 0.0;
+  int nT = 0;
+  for (int j = 0; j < n; ++j) {
+    double dot = 0.0, vv = 0.0;
+    for (int i = 0; i < d; ++i) {
+      dot += bf16_to_f64(q[i]) * bf16_to_f64(K[(size_t)j * d + i]);
+      vv += bf16_to_f64(V[(size_t)j * d + i]) * bf16_to_f64(V[(size_t)j * d + i]);
+    }
+    z[j] = scale * dot;
+    if (z[j] > zmax) zmax = z[j];
+    if (kept[j]) { if (z[j] > zmaxS) zmaxS = z[j]; }
+    else { if (z[j] > zmaxT) zmaxT = z[j]; sT += (double)s[j]; ++nT; }
+    if (sqrt(vv) > vmax) vmax = sqrt(vv);
+  }
+  /* exact attention and the tail mass p */
+  double Z = 0.0, ZT = 0.0;
+  for (int j = 0; j < n; ++j) {
+    const double w = exp(z[j] - zmax);
+    Z += w;
+    if (!kept[j]) ZT += w;
+  }
+  const double p = ZT / Z;
+  /* compressed attention over S and the slot */
+  const int slot = kstar != NULL;
+  double zstar = 0.0;
+  if (slot) {
+    for (int i = 0; i < d; ++i) zstar += bf16_to_f64(q[i]) * bf16_to_f64(kstar[i]);
+    zstar *= scale;
+  }
+  const double c = (slot && zstar > zmaxS) ? zstar : zmaxS;
+  double Zhat = slot ? exp(zstar - c) : 0.0;
+  for (int j = 0; j < n; ++j)
+    if (kept[j]) Zhat += exp(z[j] - c);
+  const double qstar = slot ? exp(zstar - c) / Zhat : 0.0;
+  /* tail log-partition */
+  double sumT = 0.0;
+  for (int j = 0; j < n; ++j)
+    if (!kept[j]) sumT += exp(z[j] - zmaxT);
+  const double LamT = zmaxT + log(sumT);
+  /* the tail distributions a and r, and the lifted distribution Abar */
+  double l1_ar = 0.0, l1_lift = 0.0;
+  double* mix = (double*)calloc((size_t)d, sizeof(double));
+  for (int j = 0; j < n; ++j) {
+    const double A = exp(z[j] - zmax) / Z;
+    if (kept[j]) {
+      const double Ahat = exp(z[j] - c) / Zhat;
+      l1_lift += fabs(A - Ahat);
+    } else {
+      const double r = sT > 0.0 ? (double)s[j] / sT : 1.0 / nT;
+      const double a = p > 0.0 ? A / p : 0.0;
+      l1_ar += fabs(a - r);
+      l1_lift += fabs(A - qstar * r);
+      for (int i = 0; i < d; ++i) mix[i] += r * bf16_to_f64(V[(size_t)j * d + i]);
+    }
+  }
+  double dv = 0.0;
+  if (slot)
+    for (int i = 0; i < d; ++i) {
+      const double e = bf16_to_f64(vstar[i]) - mix[i];
+      dv += e * e;
+    }
+  const double dpq = fabs(p - qstar);
+  stats[0] = p;
+  stats[1] = qstar;
+  stats[2] = l1_ar;
+  stats[3] = slot ? LamT - zstar : NAN;
+  stats[4] = vmax * (2.0 * dpq + (p < qstar ? p : qstar) * l1_ar);
+  stats[5] = slot ? tanh(fabs(LamT - zstar) / 4.0) : NAN;
+  stats[6] = l1_lift;
+  stats[7] = (slot && sT > 0.0) ? sqrt(dv) : NAN;
+  free(mix);
+  free(z);
+}

@@ -497,6 +497,96 @@ def pin_fixed_row_factorization(lib=None):
         assert abs(st3[0] - 1.0) < 1e-15 and st3[2] < 1e-12 and st3[3] < 1e-12
 
 
+def pin_future_query_lift_worked(lib=None):
+    """Theorem (future-query lift) on a hand-built row: q = e1, scale 1, keys
+    0, 0, e1 (logits 0, 0, 1), values e1, e2, (1, 1), the first token kept;
+    tail weights r = (1/4, 3/4) and the slot (k*, v*) = (e1/2, (3/4, 1)), so
+    z* = 1/2 and v* is exactly the r-mixture.  Closed forms: p = (1+e)/(2+e),
+    q = sqrt(e)/(1+sqrt(e)), a = (1, e)/(1+e), Lambda_T = log(1+e)."""
+    e, se = math.e, math.sqrt(math.e)
+    p, qs = (1 + e) / (2 + e), se / (1 + se)
+    l1 = abs(1 / (1 + e) - 0.25) + abs(e / (1 + e) - 0.75)
+    lam = math.log(1 + e) - 0.5
+    lift = (abs(1 / (2 + e) - 1 / (1 + se)) + abs(1 / (2 + e) - qs / 4)
+            + abs(e / (2 + e) - 3 * qs / 4))
+    want = [p, qs, l1, lam, math.sqrt(2) * (2 * abs(p - qs) + min(p, qs) * l1),
+            math.tanh(abs(lam) / 4), lift, 0.0]
+    st = oracle.future_query_lift(
+        to_bf16_bits([1.0, 0.0]), to_bf16_bits([[0, 0], [0, 0], [1, 0]]),
+        to_bf16_bits([[1, 0], [0, 1], [1, 1]]), np.array([1, 0, 0]),
+        np.array([0.5, 0.25, 0.75], np.float32), scale=1.0,
+        kstar=to_bf16_bits([0.5, 0.0]), vstar=to_bf16_bits([0.75, 1.0]), lib=lib)
+    for i, w in enumerate(want):
+        assert abs(st[i] - w) < 1e-12, (i, st[i], w)
+    # without a slot the compressed row is the kept set alone: q = 0 and
+    # ||A - Abar||_1 = 2p, the bound 2 V_max p
+    st0 = oracle.future_query_lift(
+        to_bf16_bits([1.0, 0.0]), to_bf16_bits([[0, 0], [0, 0], [1, 0]]),
+        to_bf16_bits([[1, 0], [0, 1], [1, 1]]), np.array([1, 0, 0]),
+        np.array([0.5, 0.25, 0.75], np.float32), scale=1.0, lib=lib)
+    assert st0[1] == 0.0 and abs(st0[6] - 2 * p) < 1e-12
+    assert abs(st0[4] - 2 * math.sqrt(2) * p) < 1e-12
+    assert math.isnan(st0[3]) and math.isnan(st0[5]) and math.isnan(st0[7])
+
+
+def pin_future_query_lift_single_tail_token(lib=None):
+    """With one evicted token t and the slot equal to (k_t, v_t) the compressed
+    row is the exact row: p = q, a = r = the point mass, Lambda_T = z*, and
+    every mismatch and bound vanishes."""
+    rng = np.random.default_rng(43)
+    for _ in range(10):
+        n, d = int(rng.integers(3, 40)), int(rng.choice([4, 16]))
+        K = to_bf16_bits(rng.normal(size=(n, d)))
+        V = to_bf16_bits(rng.normal(size=(n, d)))
+        q = to_bf16_bits(rng.normal(size=d))
+        t = int(rng.integers(n))
+        kept = np.ones(n, bool)
+        kept[t] = False
+        s = rng.random(n).astype(np.float32)
+        st = oracle.future_query_lift(q, K, V, kept, s, scale=0.3, kstar=K[t], vstar=V[t],
+                                      lib=lib)
+        assert abs(st[0] - st[1]) < 1e-15 and 0.0 < st[0] < 1.0
+        for i in (2, 3, 4, 5, 6, 7):
+            assert abs(st[i]) < 1e-12, (i, st[i])
+
+
+def pin_future_query_lift_bounds(lib=None):
+    """The theorem's inequalities on random rows with a bf16 tail slot built
+    from score weights: ||O - Ohat|| <= V_max ||A - Abar||_1 + q ||v* - mixture||
+    (Ohat computed here, by plain softmax over S and the slot), ||A - Abar||_1 <=
+    2|p - q| + min(p, q) ||a - r||_1, |p - q| <= tanh(|Lambda_T - z*|/4) <=
+    |Lambda_T - z*|/4, and p + p_S = 1 with p_S from the fixed-row quantities."""
+    rng = np.random.default_rng(47)
+    for _ in range(30):
+        n, d = int(rng.integers(6, 90)), int(rng.choice([4, 16]))
+        K = to_bf16_bits(rng.normal(size=(n, d)) * rng.choice([0.5, 2.0]))
+        V = to_bf16_bits(rng.normal(size=(n, d)))
+        q = to_bf16_bits(rng.normal(size=d))
+        kept = rng.random(n) < 0.4
+        kept[0], kept[-1] = True, False
+        s = (rng.random(n) ** 3).astype(np.float32)
+        Kf, Vf, qf = bf(K), bf(V), bf(q)
+        r = np.where(kept, 0.0, s.astype(np.float64))
+        r /= r.sum()
+        ks, vs = to_bf16_bits(r @ Kf), to_bf16_bits(r @ Vf)
+        st = oracle.future_query_lift(q, K, V, kept, s, scale=0.25, kstar=ks, vstar=vs, lib=lib)
+        z = 0.25 * (Kf @ qf)
+        A = softmax(z)
+        O = A @ Vf
+        zh = np.concatenate([z[kept], [0.25 * (bf(ks) @ qf)]])
+        Ah = softmax(zh)
+        Oh = Ah[:-1] @ Vf[kept] + Ah[-1] * bf(vs)
+        vmax = np.linalg.norm(Vf, axis=1).max()
+        err = np.linalg.norm(O - Oh)
+        assert abs(st[1] - Ah[-1]) < 1e-12 and abs(st[0] - A[~kept].sum()) < 1e-12
+        assert err <= vmax * st[6] + st[1] * st[7] + 1e-12
+        assert st[6] <= 2 * abs(st[0] - st[1]) + min(st[0], st[1]) * st[2] + 1e-12
+        assert abs(st[0] - st[1]) <= st[5] + 1e-12 and st[5] <= abs(st[3]) / 4 + 1e-12
+        assert st[4] >= vmax * st[6] - 1e-12
+        fr = oracle.fixed_row(q, K, V, kept, scale=0.25, lib=lib)
+        assert abs(fr[0] + st[0] - 1.0) < 1e-12
+
+
 def pin_allocation_infeasible(lib=None):
     """B_real above H (n - 1) cannot be met with b_h <= n - 1."""
     curves = np.ones((2, 5))

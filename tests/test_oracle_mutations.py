@@ -45,6 +45,12 @@ MUTANTS = {
                                     "const int r0 = (g == 0 ? b - 1 : b) + (int)(((int64_t)g * T) / m),"),
     "fixed_row_subset_not_renormalised": ("const double os = ZS > 0.0 ? OS[i] / ZS : 0.0;",
                                           "const double os = OS[i] / Z;"),
+    "lift_slot_weight_over_all_tokens": ("    if (kept[j]) Zhat += exp(z[j] - c);",
+                                         "    Zhat += exp(z[j] - c);"),
+    "lift_tail_partition_over_all": ("if (!kept[j]) sumT += exp(z[j] - zmaxT);",
+                                     "sumT += exp(z[j] - zmaxT);"),
+    "lift_tail_weights_not_renormalised": ("const double a = p > 0.0 ? A / p : 0.0;",
+                                           "const double a = A;"),
     "bisection_inverted": ("if (total > B_real) lam_lo = lam; else lam_hi = lam;",
                            "if (total > B_real) lam_hi = lam; else lam_lo = lam;"),
     "kept_not_sorted": ("qsort(kept, (size_t)b, sizeof(int32_t), cmp_int32);", ""),
