@@ -250,25 +250,44 @@ int certkv_decode_certified(const certkv_shape* shape, const void* q, const cert
                             size_t workspace_bytes, void* stream);
 
 /* Fixed-row diagnostics (an evaluation tool: it reads the full original K and
- * V, like the paper's fixed-row experiments; Theorem: fixed-row tail
- * factorization).  For every query head qh of unit u with its decode query q
- * and the realized softmax row A_j = softmax_j(scale <q, k_j>) over all n
- * original tokens, and S = the real tokens kept in `packed`, writes stats
- * fp32 [B][L][Hq][8]:
+ * V, like the paper's fixed-row experiments).  For every query head qh of unit
+ * u with its decode query q, the realized logits z_j = scale <q, k_j> and
+ * softmax row A_j over all n original tokens, S = the real tokens kept in
+ * `packed` and T = the evicted ones, writes stats fp32
+ * [B][L][Hq][CERTKV_FIXED_ROW_STATS]:
+ *   Theorem (fixed-row tail factorization):
  *   0  p_S = sum_{j in S} A_j (kept mass)
  *   1  ||O||_2 of exact attention O = sum_j A_j v_j
  *   2  ||O~_S - O||_2, O~_S = sum_{j in S} A_j v_j / p_S (subset-only output)
- *   3  ||u*||_2, u* = sum_{j not in S} A_j v_j (the fixed-row correction)
+ *   3  ||u*||_2, u* = sum_{j in T} A_j v_j (the fixed-row correction)
  *   4  2 V_max (1 - p_S), V_max = max_j ||v_j||_2 (the theorem's mass bound)
  *   5  ||O-hat - O||_2 for O-hat = certkv_decode_attn(q, packed, tail_slot)
  *   6  V_max
  *   7  ||p_S O~_S + (1 - p_S) V-bar_T - O||_2, the factorization residual
- * q bf16 [B][L][Hq][d]; K, V as for certkv_compress; workspace:
- * certkv_fixed_row_workspace_bytes(shape). */
+ *   Theorem (future-query lift and summary mismatch), with Ahat the softmax
+ *   over S and the synthetic slot (logit z* = scale <q, k*>), and the slot's
+ *   tail weights r_j = s_j / sum_T s (uniform 1/|T| when that sum is 0):
+ *   8  p = A(T), the tail mass (computed from the evicted tokens, not 1 - p_S)
+ *   9  q = Ahat_star, the slot's compressed weight (0 when tail_slot = 0)
+ *   10 ||a - r||_1 over T, a = A_T / p (a = 0 when p = 0)
+ *   11 Lambda_T - z*, Lambda_T = log sum_{j in T} e^{z_j} (NaN without a slot)
+ *   12 V_max (2 |p - q| + min(p, q) ||a - r||_1), the theorem's bound on
+ *      ||O - O-hat|| for a slot value equal to the r-mixture
+ *   13 tanh(|Lambda_T - z*| / 4), the theorem's bound on |p - q| (NaN without a slot)
+ *   14 ||A - Abar||_1 for the lifted row Abar (Ahat on S, q r_j on T)
+ *   15 ||v*_stored - sum_T r_j v_j||_2, the packed slot value against the
+ *      exact mixture (bf16 rounding; NaN without a slot or when sum_T s = 0)
+ * Fields 10, 12, 14 and 15 need `scores` (fp32 [B*L*H][n], the a_j the
+ * compression used, e.g. from certkv_score with the same inputs and params);
+ * with scores = NULL they are NaN.  q bf16 [B][L][Hq][d]; K, V as for
+ * certkv_compress; workspace: certkv_fixed_row_workspace_bytes(shape) (it
+ * holds every logit, 4 (B*L*Hq) n bytes). */
+#define CERTKV_FIXED_ROW_STATS 16
 size_t certkv_fixed_row_workspace_bytes(const certkv_shape* shape);
 int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void* K, const void* V,
-                           const certkv_packed* packed, float scale, int32_t tail_slot,
-                           float* stats, void* workspace, size_t workspace_bytes, void* stream);
+                           const float* scores, const certkv_packed* packed, float scale,
+                           int32_t tail_slot, float* stats, void* workspace,
+                           size_t workspace_bytes, void* stream);
 
 /* Decode attention that allocates nothing.  The paper has no counterpart: this
  * entry point exists for callers that cannot hand the library a scratch

@@ -114,7 +114,8 @@ def load_library(path: Optional[str] = None):
         lib.certkv_decode_certified.restype = ctypes.c_int
         lib.certkv_fixed_row_workspace_bytes.argtypes = [sp]
         lib.certkv_fixed_row_workspace_bytes.restype = SZ
-        lib.certkv_fixed_row_stats.argtypes = [sp, P, P, P, kp, ctypes.c_float, I32, P, P, SZ, P]
+        lib.certkv_fixed_row_stats.argtypes = [sp, P, P, P, P, kp, ctypes.c_float, I32, P, P, SZ,
+                                                    P]
         lib.certkv_fixed_row_stats.restype = ctypes.c_int
         _lib = lib
         return lib
@@ -393,24 +394,33 @@ def certkv_decode_certified(q, packed: Packed, *, hkv: int, scale: float = 0.0, 
 
 
 FIXED_ROW_FIELDS = ("kept_mass", "norm_O", "err_subset", "norm_correction", "mass_bound",
-                    "err_decode", "v_max", "factorization_residual")
+                    "err_decode", "v_max", "factorization_residual", "tail_mass", "slot_weight",
+                    "l1_tail_weights", "logpartition_gap", "lift_bound", "tanh_bound",
+                    "l1_lifted_row", "slot_mixture_error")
 
 
-def certkv_fixed_row_stats(q, K, V, packed: Packed, *, scale: float = 0.0, stats=None, ws=None,
-                           stream=None) -> torch.Tensor:
-    """Fixed-row diagnostics per query head: fp32 [B][L][Hq][8] in the order of
-    FIXED_ROW_FIELDS (evaluation tool; reads the full K and V)."""
+def certkv_fixed_row_stats(q, K, V, packed: Packed, *, scores=None, scale: float = 0.0,
+                           stats=None, ws=None, stream=None) -> torch.Tensor:
+    """Fixed-row diagnostics per query head: fp32 [B][L][Hq][16] in the order
+    of FIXED_ROW_FIELDS (evaluation tool; reads the full K and V).  `scores`:
+    fp32 [B*L*H][n] compression scores (certkv_score), or None (the fields
+    that need the slot's tail weights are then NaN)."""
     _bf16(q, "q"); _bf16(K, "K"); _bf16(V, "V")
     B, L, Hq, d = q.shape
     shape = certkv_shape(B, L, Hq, K.shape[2], K.shape[3], d, 1)
+    if scores is not None:
+        if scores.dtype != torch.float32 or not scores.is_contiguous() or \
+                scores.numel() != B * L * K.shape[2] * K.shape[3]:
+            raise ValueError("scores must be contiguous fp32 [B*L*H][n]")
     if stats is None:
-        stats = torch.empty((B, L, Hq, 8), dtype=torch.float32, device=q.device)
+        stats = torch.empty((B, L, Hq, len(FIXED_ROW_FIELDS)), dtype=torch.float32,
+                            device=q.device)
     if ws is None:
         ws = workspace(int(load_library().certkv_fixed_row_workspace_bytes(ctypes.byref(shape))),
                        q.device)
     st = packed.struct()
     rc = load_library().certkv_fixed_row_stats(ctypes.byref(shape), _ptr(q), _ptr(K), _ptr(V),
-                                               ctypes.byref(st), float(scale),
+                                               _ptr(scores), ctypes.byref(st), float(scale),
                                                int(packed.tail_slot), _ptr(stats), _ptr(ws),
                                                ws.numel(), _stream(stream))
     _check(rc, "certkv_fixed_row_stats")

@@ -498,8 +498,9 @@ size_t certkv_fixed_row_workspace_bytes(const certkv_shape* shape) {
 }
 
 int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void* K, const void* V,
-                           const certkv_packed* packed, float scale, int32_t tail_slot,
-                           float* stats, void* workspace, size_t workspace_bytes, void* stream) {
+                           const float* scores, const certkv_packed* packed, float scale,
+                           int32_t tail_slot, float* stats, void* workspace,
+                           size_t workspace_bytes, void* stream) {
   certkv_params prm;
   certkv_default_params(&prm);
   Prob p;
@@ -509,14 +510,14 @@ int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void*
       !packed->real_counts || !packed->positions || !stats)
     return CERTKV_EINVAL;
   if (!aligned(q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(packed->k, 16) ||
-      !aligned(packed->v, 16))
+      !aligned(packed->v, 16) || !aligned(scores, 4))
     return CERTKV_EINVAL;
   if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
   if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < fixed_row_workspace(p))
     return CERTKV_EWORKSPACE;
   const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
-  launch_fixed_row(p, q, K, V, packed->offsets, packed->real_counts, packed->positions, packed->k,
+  launch_fixed_row(p, q, K, V, scores, packed->offsets, packed->real_counts, packed->positions, packed->k,
                    packed->v, tail_slot, sc, stats, reinterpret_cast<char*>(workspace),
                    reinterpret_cast<cudaStream_t>(stream));
   return cuda_ok(cudaGetLastError());

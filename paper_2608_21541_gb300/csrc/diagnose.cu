@@ -3,11 +3,17 @@
 //
 // For each query head and its realized softmax row A over all n original
 // tokens of the unit (Theorem: fixed-row tail factorization), with S = the
-// kept real tokens of a packed cache: the kept mass p_S, exact attention O,
-// the subset-only output O~_S = sum_S A v / p_S, the fixed-row correction
-// u* = sum_{not S} A v, the mass bound 2 V_max (1 - p_S), and the error of
-// the compressed decode.  One split-K pass keeps two online softmax states
-// (all tokens, kept tokens) under one shared running maximum.
+// kept real tokens of a packed cache and T the evicted ones: the kept mass
+// p_S, exact attention O, the subset-only output O~_S = sum_S A v / p_S, the
+// fixed-row correction u* = sum_T A v, the mass bound 2 V_max (1 - p_S), and
+// the error of the compressed decode; and the quantities of the future-query
+// lift (Theorem: future-query lift and summary mismatch): the tail mass p, the
+// synthetic slot's compressed weight q, ||a - r||_1 between the exact tail
+// distribution and the slot's tail weights, Lambda_T - z*, both of the
+// theorem's bounds and the exact lifted L1 mismatch.  One split-K pass keeps
+// two online softmax states (kept tokens, evicted tokens) under one shared
+// running maximum and stores every logit; the merge reads the logits back for
+// the per-token L1 sums.
 #include "../../include/certkv.h"
 #include "common.cuh"
 #include "internal.cuh"
@@ -29,19 +35,26 @@ __global__ void kept_mask_kernel(Prob p, const int64_t* __restrict__ offsets,
 }
 
 struct DiagPart {  // one (unit, split, query head)
-  float m, l_all, l_kept, vmax;
+  float m, l_kept, l_tail, vmax;
 };
 
+constexpr int kSvStride = kD + 1;  // per (unit, split): sum_T s_j v_j [kD], sum_T s_j
+
 // grid = (units, kDiagSplits), block = 128 (4 warps); 32-token tiles, lane =
-// token for the logits, lane = 4 dimensions for the value sums.
+// token for the logits, lane = 4 dimensions for the value sums.  With scores
+// `sc` (may be null) it also sums s_j v_j and s_j over the evicted tokens.
+// z2[u][g][j] receives every log2-domain logit.
 template <int G>
 __global__ void __launch_bounds__(128) fixed_row_split_kernel(
     Prob p, const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ K,
-    const __nv_bfloat16* __restrict__ V, const uint32_t* __restrict__ mask, float scale_log2,
-    DiagPart* __restrict__ part, float* __restrict__ part_acc) {
+    const __nv_bfloat16* __restrict__ V, const uint32_t* __restrict__ mask,
+    const float* __restrict__ sc, float scale_log2, DiagPart* __restrict__ part,
+    float* __restrict__ part_acc, float* __restrict__ z2, float* __restrict__ part_sv) {
   __shared__ __align__(16) float qs[G][kD];
   __shared__ DiagPart wp[4][G];
   __shared__ float wacc[4][2][kD];  // one query head at a time
+  __shared__ float wsv[4][kD];
+  __shared__ float wss[4];
   const int u = blockIdx.x, split = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bl = u / p.H, h = u - bl * p.H;
@@ -52,15 +65,15 @@ __global__ void __launch_bounds__(128) fixed_row_split_kernel(
   __syncthreads();
   const uint4* Ku = reinterpret_cast<const uint4*>(K + (size_t)u * n * kD);
   const uint2* Vu = reinterpret_cast<const uint2*>(V + (size_t)u * n * kD);
-  float m[G], la[G], lk[G], aa[G][4], ak[G][4];
+  float m[G], lk[G], lt[G], ak[G][4], at[G][4];
 #pragma unroll
   for (int g = 0; g < G; ++g) {
     m[g] = -INFINITY;
-    la[g] = lk[g] = 0.f;
+    lk[g] = lt[g] = 0.f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) aa[g][i] = ak[g][i] = 0.f;
+    for (int i = 0; i < 4; ++i) ak[g][i] = at[g][i] = 0.f;
   }
-  float vmax = 0.f;
+  float vmax = 0.f, ssum = 0.f, sv[4] = {0.f, 0.f, 0.f, 0.f};
   const int ntiles = (n + 31) / 32;
   for (int t = split * 4 + warp; t < ntiles; t += kDiagSplits * 4) {
     const int j = t * 32 + lane;
@@ -86,23 +99,30 @@ __global__ void __launch_bounds__(128) fixed_row_split_kernel(
           for (int e = 0; e < 8; ++e) x[g] = fmaf(qs[g][c * 8 + e], kf[e], x[g]);
       }
     }
-    float pa[G], pk[G];
+    if (ok) {
+#pragma unroll
+      for (int g = 0; g < G; ++g) z2[((size_t)u * G + g) * n + j] = x[g];
+    }
+    const float sj = (sc != nullptr && ok && !kept) ? sc[(size_t)u * n + j] : 0.f;
+    ssum += sj;
+    float pk[G], pt[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       const float nm = fmaxf(m[g], warp_max(x[g]));
       const float corr = exp2f(m[g] - nm);
       m[g] = nm;
-      la[g] *= corr;
       lk[g] *= corr;
+      lt[g] *= corr;
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        aa[g][i] *= corr;
         ak[g][i] *= corr;
+        at[g][i] *= corr;
       }
-      pa[g] = ok ? exp2f(x[g] - nm) : 0.f;
-      pk[g] = kept ? pa[g] : 0.f;
-      la[g] += pa[g];
+      const float pe = ok ? exp2f(x[g] - nm) : 0.f;
+      pk[g] = kept ? pe : 0.f;
+      pt[g] = kept ? 0.f : pe;
       lk[g] += pk[g];
+      lt[g] += pt[g];
     }
     const int cnt = min(32, n - t * 32);
     for (int r = 0; r < cnt; ++r) {
@@ -114,45 +134,50 @@ __global__ void __launch_bounds__(128) fixed_row_split_kernel(
       vmax = fmaxf(vmax, sqrtf(sq));
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        const float wa = __shfl_sync(kFull, pa[g], r), wk = __shfl_sync(kFull, pk[g], r);
+        const float wk = __shfl_sync(kFull, pk[g], r), wt = __shfl_sync(kFull, pt[g], r);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          aa[g][i] = fmaf(wa, v[i], aa[g][i]);
           ak[g][i] = fmaf(wk, v[i], ak[g][i]);
+          at[g][i] = fmaf(wt, v[i], at[g][i]);
         }
+      }
+      if (sc != nullptr) {
+        const float ws = __shfl_sync(kFull, sj, r);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) sv[i] = fmaf(ws, v[i], sv[i]);
       }
     }
   }
   // combine the 4 warps, one query head at a time
+  const int i = threadIdx.x;  // 128 threads = kD dimensions
 #pragma unroll
   for (int g = 0; g < G; ++g) {
-    float ta = la[g], tk = lk[g];
+    float tk = lk[g], tt = lt[g];
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) {
-      ta += __shfl_xor_sync(kFull, ta, o);
       tk += __shfl_xor_sync(kFull, tk, o);
+      tt += __shfl_xor_sync(kFull, tt, o);
     }
-    if (lane == 0) wp[warp][g] = DiagPart{m[g], ta, tk, vmax};
+    if (lane == 0) wp[warp][g] = DiagPart{m[g], tk, tt, vmax};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      wacc[warp][0][lane * 4 + i] = aa[g][i];
-      wacc[warp][1][lane * 4 + i] = ak[g][i];
+    for (int e = 0; e < 4; ++e) {
+      wacc[warp][0][lane * 4 + e] = ak[g][e];
+      wacc[warp][1][lane * 4 + e] = at[g][e];
     }
     __syncthreads();
-    const int i = threadIdx.x;  // 128 threads = kD dimensions
     float M = -INFINITY, vm = 0.f;
 #pragma unroll
     for (int wi = 0; wi < 4; ++wi) {
       M = fmaxf(M, wp[wi][g].m);
       vm = fmaxf(vm, wp[wi][g].vmax);
     }
-    float LA = 0.f, LK = 0.f, A = 0.f, B = 0.f;
+    float LK = 0.f, LT = 0.f, A = 0.f, B = 0.f;
 #pragma unroll
     for (int wi = 0; wi < 4; ++wi) {
       if (wp[wi][g].m > -INFINITY) {
         const float f = exp2f(wp[wi][g].m - M);
-        LA += wp[wi][g].l_all * f;
         LK += wp[wi][g].l_kept * f;
+        LT += wp[wi][g].l_tail * f;
         A += wacc[wi][0][i] * f;
         B += wacc[wi][1][i] * f;
       }
@@ -160,8 +185,19 @@ __global__ void __launch_bounds__(128) fixed_row_split_kernel(
     const size_t pi = ((size_t)u * kDiagSplits + split) * G + g;
     part_acc[(pi * 2 + 0) * kD + i] = A;
     part_acc[(pi * 2 + 1) * kD + i] = B;
-    if (i == 0) part[pi] = DiagPart{M, LA, LK, vm};
+    if (i == 0) part[pi] = DiagPart{M, LK, LT, vm};
     __syncthreads();
+  }
+  if (sc != nullptr) {  // block-uniform
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) ssum += __shfl_xor_sync(kFull, ssum, o);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) wsv[warp][lane * 4 + e] = sv[e];
+    if (lane == 0) wss[warp] = ssum;
+    __syncthreads();
+    float* ps = part_sv + ((size_t)u * kDiagSplits + split) * kSvStride;
+    ps[i] = (wsv[0][i] + wsv[1][i]) + (wsv[2][i] + wsv[3][i]);
+    if (i == 0) ps[kD] = (wss[0] + wss[1]) + (wss[2] + wss[3]);
   }
 }
 
@@ -175,36 +211,44 @@ __device__ __forceinline__ float block_sum_128(float x, float* red) {
 }
 
 // grid = units * G, block = 128 (thread = dimension): merge the splits of one
-// query head and write its 8 statistics.
+// query head, write its fixed-row statistics, then (with scores) sweep the
+// stored logits of the evicted tokens for the two L1 sums of the lift.
 __global__ void __launch_bounds__(128) fixed_row_merge_kernel(
     Prob p, int G, const DiagPart* __restrict__ part, const float* __restrict__ part_acc,
-    const __nv_bfloat16* __restrict__ ohat, float* __restrict__ stats) {
+    const __nv_bfloat16* __restrict__ ohat, const __nv_bfloat16* __restrict__ q,
+    const __nv_bfloat16* __restrict__ pk, const __nv_bfloat16* __restrict__ pv,
+    const int64_t* __restrict__ offsets, const int32_t* __restrict__ counts, int tail_slot,
+    float scale_log2, const float* __restrict__ sc, const float* __restrict__ z2,
+    const float* __restrict__ part_sv, const uint32_t* __restrict__ mask,
+    float* __restrict__ stats) {
   __shared__ float red[4];
   const int ug = blockIdx.x;
   const int u = ug / G, g = ug - u * G;
   const int i = threadIdx.x;
+  const int n = p.n, words = (n + 31) / 32;
   float M = -INFINITY, vm = 0.f;
   for (int s = 0; s < kDiagSplits; ++s) {
-    const DiagPart q = part[((size_t)u * kDiagSplits + s) * G + g];
-    M = fmaxf(M, q.m);
-    vm = fmaxf(vm, q.vmax);
+    const DiagPart d = part[((size_t)u * kDiagSplits + s) * G + g];
+    M = fmaxf(M, d.m);
+    vm = fmaxf(vm, d.vmax);
   }
-  float LA = 0.f, LK = 0.f, A = 0.f, B = 0.f;
+  float LK = 0.f, LT = 0.f, AK = 0.f, AT = 0.f;
   for (int s = 0; s < kDiagSplits; ++s) {
     const size_t pi = ((size_t)u * kDiagSplits + s) * G + g;
-    const DiagPart q = part[pi];
-    if (q.m > -INFINITY) {
-      const float f = exp2f(q.m - M);
-      LA += q.l_all * f;
-      LK += q.l_kept * f;
-      A += part_acc[(pi * 2 + 0) * kD + i] * f;
-      B += part_acc[(pi * 2 + 1) * kD + i] * f;
+    const DiagPart d = part[pi];
+    if (d.m > -INFINITY) {
+      const float f = exp2f(d.m - M);
+      LK += d.l_kept * f;
+      LT += d.l_tail * f;
+      AK += part_acc[(pi * 2 + 0) * kD + i] * f;
+      AT += part_acc[(pi * 2 + 1) * kD + i] * f;
     }
   }
-  const float o = A / LA;                       // exact attention
-  const float os = LK > 0.f ? B / LK : 0.f;     // subset-only output
-  const float uu = (A - B) / LA;                // fixed-row correction
-  const float pS = LK / LA;
+  const float LA = LK + LT;
+  const float o = (AK + AT) / LA;               // exact attention
+  const float os = LK > 0.f ? AK / LK : 0.f;    // subset-only output
+  const float uu = AT / LA;                     // fixed-row correction
+  const float pS = LK / LA, pT = LT / LA;
   const int bl = u / p.H, h = u - bl * p.H;
   const size_t qi = (size_t)bl * p.Hq + (size_t)h * G + g;
   const float oh = __bfloat162float(ohat[qi * kD + i]);
@@ -215,8 +259,51 @@ __global__ void __launch_bounds__(128) fixed_row_merge_kernel(
   const float nu = block_sum_128(uu * uu, red);
   const float eh = block_sum_128((oh - o) * (oh - o), red);
   const float res = block_sum_128(f * f, red);
+
+  // the synthetic slot: its logit z* (log2 domain), compressed weight q and
+  // Lambda_T - z* (natural log units)
+  const bool slot = tail_slot != 0;
+  float qstar = 0.f, dlam = NAN, dmix = NAN;
+  const size_t srow = slot ? (size_t)(offsets[u] + counts[u]) : 0;
+  if (slot) {
+    const float xs =
+        block_sum_128(__bfloat162float(q[qi * kD + i]) * __bfloat162float(pk[srow * kD + i]), red) *
+        scale_log2;
+    qstar = 1.f / (1.f + exp2f(M + log2f(LK) - xs));
+    dlam = 0.6931471805599453f * (M + log2f(LT) - xs);
+  }
+  float d1 = NAN, d2 = NAN;
+  if (sc != nullptr) {
+    float ST = 0.f, SV = 0.f;
+    for (int s = 0; s < kDiagSplits; ++s) {
+      const float* ps = part_sv + ((size_t)u * kDiagSplits + s) * kSvStride;
+      SV += ps[i];
+      ST += ps[kD];
+    }
+    if (slot && ST > 0.f) {  // the stored value against the exact r-mixture
+      const float e = __bfloat162float(pv[srow * kD + i]) - SV / ST;
+      dmix = sqrtf(block_sum_128(e * e, red));
+    }
+    const int nT = n - counts[u];
+    const float invLT = LT > 0.f ? 1.f / LT : 0.f, invLA = 1.f / LA;
+    const float invST = ST > 0.f ? 1.f / ST : 0.f, uni = 1.f / (float)nT;
+    const float* zz = z2 + ((size_t)u * G + g) * n;
+    const float* su = sc + (size_t)u * n;
+    const uint32_t* mu = mask + (size_t)u * words;
+    float a1 = 0.f, a2 = 0.f;
+    for (int j = i; j < n; j += 128) {
+      if ((mu[j >> 5] >> (j & 31)) & 1u) continue;
+      const float e = exp2f(zz[j] - M);
+      const float r = ST > 0.f ? su[j] * invST : uni;
+      a1 += fabsf(e * invLT - r);          // |a_j - r_j|
+      a2 += fabsf(e * invLA - qstar * r);  // |A_j - q r_j|
+    }
+    d1 = block_sum_128(a1, red);
+    // on S the lifted row is Ahat = A * Z / Zhat, so sum_S |A - Ahat| = |p_S - (1 - q)|
+    d2 = fabsf(pS - (1.f - qstar)) + block_sum_128(a2, red);
+  }
   if (i == 0) {
-    float* st = stats + qi * 8;
+    float* st = stats + qi * CERTKV_FIXED_ROW_STATS;
     st[0] = pS;
     st[1] = sqrtf(nO);
     st[2] = sqrtf(eS);
@@ -225,31 +312,54 @@ __global__ void __launch_bounds__(128) fixed_row_merge_kernel(
     st[5] = sqrtf(eh);
     st[6] = vm;
     st[7] = sqrtf(res);
+    st[8] = pT;
+    st[9] = qstar;
+    st[10] = d1;
+    st[11] = dlam;
+    st[12] = sc != nullptr ? vm * (2.f * fabsf(pT - qstar) + fminf(pT, qstar) * d1) : NAN;
+    st[13] = slot ? tanhf(0.25f * fabsf(dlam)) : NAN;
+    st[14] = d2;
+    st[15] = dmix;
   }
 }
 
-size_t fixed_row_workspace(const Prob& p) {
+namespace {
+struct FixedRowLayout {
+  size_t mask, part, acc, z2, sv, ohat, dec, total;
+};
+FixedRowLayout fixed_row_layout(const Prob& p) {
   const size_t words = (size_t)(p.n + 31) / 32;
   const size_t parts = (size_t)p.units * kDiagSplits * p.G;
   auto a = [](size_t x) { return (x + 255) / 256 * 256; };
-  return a(p.units * words * 4) + a(parts * sizeof(DiagPart)) + a(parts * 2 * kD * 4) +
-         a((size_t)p.units * p.G * kD * 2) + a(decode_workspace(p));
+  FixedRowLayout ly;
+  ly.mask = 0;
+  ly.part = ly.mask + a(p.units * words * 4);
+  ly.acc = ly.part + a(parts * sizeof(DiagPart));
+  ly.z2 = ly.acc + a(parts * 2 * kD * 4);
+  ly.sv = ly.z2 + a((size_t)p.units * p.G * p.n * 4);
+  ly.ohat = ly.sv + a((size_t)p.units * kDiagSplits * kSvStride * 4);
+  ly.dec = ly.ohat + a((size_t)p.units * p.G * kD * 2);
+  ly.total = ly.dec + a(decode_workspace(p));
+  return ly;
 }
+}  // namespace
+
+size_t fixed_row_workspace(const Prob& p) { return fixed_row_layout(p).total; }
 
 void launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V,
-                      const int64_t* offsets, const int32_t* counts, const int32_t* positions,
-                      const void* pk, const void* pv, int tail_slot, float scale, float* stats,
-                      char* ws, cudaStream_t st) {
+                      const float* scores, const int64_t* offsets, const int32_t* counts,
+                      const int32_t* positions, const void* pk, const void* pv, int tail_slot,
+                      float scale, float* stats, char* ws, cudaStream_t st) {
+  const FixedRowLayout ly = fixed_row_layout(p);
   const size_t words = (size_t)(p.n + 31) / 32;
-  const size_t parts = (size_t)p.units * kDiagSplits * p.G;
-  auto a = [](size_t x) { return (x + 255) / 256 * 256; };
-  uint32_t* mask = reinterpret_cast<uint32_t*>(ws);
-  DiagPart* part = reinterpret_cast<DiagPart*>(ws + a(p.units * words * 4));
-  float* acc = reinterpret_cast<float*>(ws + a(p.units * words * 4) + a(parts * sizeof(DiagPart)));
-  char* ohat = ws + a(p.units * words * 4) + a(parts * sizeof(DiagPart)) + a(parts * 2 * kD * 4);
-  char* dws = ohat + a((size_t)p.units * p.G * kD * 2);
+  uint32_t* mask = reinterpret_cast<uint32_t*>(ws + ly.mask);
+  DiagPart* part = reinterpret_cast<DiagPart*>(ws + ly.part);
+  float* acc = reinterpret_cast<float*>(ws + ly.acc);
+  float* z2 = reinterpret_cast<float*>(ws + ly.z2);
+  float* psv = reinterpret_cast<float*>(ws + ly.sv);
+  char* ohat = ws + ly.ohat;
   // the compressed decode's output, for its error against O
-  launch_decode(p, q, pk, pv, offsets, counts, tail_slot, scale, ohat, dws, st);
+  launch_decode(p, q, pk, pv, offsets, counts, tail_slot, scale, ohat, ws + ly.dec, st);
   cudaMemsetAsync(mask, 0, p.units * words * 4, st);
   {
     TraceScope ts_("kept_mask", st);
@@ -262,19 +372,25 @@ void launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V
   const dim3 grid(p.units, kDiagSplits);
   {
     TraceScope ts_("fixed_row_split", st);
+#define CERTKV_FR_SPLIT(GG)                                                                  \
+  fixed_row_split_kernel<GG><<<grid, 128, 0, st>>>(p, qb, kb, vb, mask, scores, sl2, part, acc, \
+                                                  z2, psv)
     switch (p.G) {
-      case 1: fixed_row_split_kernel<1><<<grid, 128, 0, st>>>(p, qb, kb, vb, mask, sl2, part, acc); break;
-      case 2: fixed_row_split_kernel<2><<<grid, 128, 0, st>>>(p, qb, kb, vb, mask, sl2, part, acc); break;
-      case 4: fixed_row_split_kernel<4><<<grid, 128, 0, st>>>(p, qb, kb, vb, mask, sl2, part, acc); break;
-      case 8: fixed_row_split_kernel<8><<<grid, 128, 0, st>>>(p, qb, kb, vb, mask, sl2, part, acc); break;
-      case 16: fixed_row_split_kernel<16><<<grid, 128, 0, st>>>(p, qb, kb, vb, mask, sl2, part, acc); break;
+      case 1: CERTKV_FR_SPLIT(1); break;
+      case 2: CERTKV_FR_SPLIT(2); break;
+      case 4: CERTKV_FR_SPLIT(4); break;
+      case 8: CERTKV_FR_SPLIT(8); break;
+      case 16: CERTKV_FR_SPLIT(16); break;
       default: return;
     }
+#undef CERTKV_FR_SPLIT
   }
   {
     TraceScope ts_("fixed_row_merge", st);
     fixed_row_merge_kernel<<<p.units * p.G, 128, 0, st>>>(
-        p, p.G, part, acc, reinterpret_cast<const __nv_bfloat16*>(ohat), stats);
+        p, p.G, part, acc, reinterpret_cast<const __nv_bfloat16*>(ohat), qb,
+        reinterpret_cast<const __nv_bfloat16*>(pk), reinterpret_cast<const __nv_bfloat16*>(pv),
+        offsets, counts, tail_slot, sl2, scores, z2, psv, mask, stats);
   }
 }
 

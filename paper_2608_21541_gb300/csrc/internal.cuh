@@ -91,7 +91,8 @@ void launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
 size_t decode_workspace(const Prob& p);
 size_t fixed_row_workspace(const Prob& p);
 void launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V,
-                      const int64_t* offsets, const int32_t* counts, const int32_t* positions,
+                      const float* scores, const int64_t* offsets, const int32_t* counts,
+                      const int32_t* positions,
                       const void* pk, const void* pv, int tail_slot, float scale, float* stats,
                       char* ws, cudaStream_t st);
 void launch_decode_certified(const Prob& p, const void* q, const void* pk, const void* pv,
