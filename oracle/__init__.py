@@ -67,6 +67,8 @@ def _bind(lib):
     lib.oracle_fixed_row.restype = None
     lib.oracle_future_query_lift.argtypes = [P, P, P, P, P, P, P, I, I, D, P]
     lib.oracle_future_query_lift.restype = None
+    lib.oracle_coverage_profile.argtypes = [P, P, I, I, D, P, I, P, I, P, I, P, P, P, P, P, P]
+    lib.oracle_coverage_profile.restype = None
     lib.oracle_compress.restype = I
     lib.oracle_decode.argtypes = [P, D, P, P, P, P, P, I, P]
     lib.oracle_decode.restype = None
@@ -316,6 +318,31 @@ def future_query_lift(q, K, V, kept, s, *, scale: float, kstar=None, vstar=None,
         _ptr(q), _ptr(K), _ptr(V), _ptr(kept), _ptr(s), _ptr(ks) if ks is not None else None,
         _ptr(vs) if vs is not None else None, n, d, float(scale), _ptr(st))
     return st
+
+
+def coverage_profile(q, K, *, scale: float, eta=(0.1,), rel_eps=(0.1,), abs_eps=(),
+                     lib=None) -> dict:
+    """Coverage profile of one query row over the n keys K (see
+    oracle_coverage_profile): q uint16 [d], K uint16 [n][d].  Returns order
+    int32 [n], gap float64 [n] (G(j) for ranks j = 1..n), K_eta, rel, abs
+    int32 per threshold, and top = (z_(1), log sum e^z)."""
+    q = _u16(q); K = _u16(K)
+    n, d = K.shape
+    eta = np.ascontiguousarray(eta, dtype=np.float64)
+    rel_eps = np.ascontiguousarray(rel_eps, dtype=np.float64)
+    abs_eps = np.ascontiguousarray(abs_eps, dtype=np.float64)
+    order = np.zeros(n, np.int32)
+    gap = np.zeros(n)
+    K_eta = np.zeros(max(len(eta), 1), np.int32)
+    rel = np.zeros(max(len(rel_eps), 1), np.int32)
+    ab = np.zeros(max(len(abs_eps), 1), np.int32)
+    top = np.zeros(2)
+    (lib or _load()).oracle_coverage_profile(
+        _ptr(q), _ptr(K), n, d, float(scale), _ptr(eta), len(eta), _ptr(rel_eps), len(rel_eps),
+        _ptr(abs_eps), len(abs_eps), _ptr(order), _ptr(gap), _ptr(K_eta), _ptr(rel), _ptr(ab),
+        _ptr(top))
+    return dict(order=order, gap=gap, K_eta=K_eta[:len(eta)], rel=rel[:len(rel_eps)],
+                abs=ab[:len(abs_eps)], top=top)
 
 
 def decode(q, pk, pv, offsets, counts, *, B: int, L: int, Hq: int, H: int, d: int,

@@ -714,6 +714,67 @@ double oracle_decode_certified(const uint16_t* q, const uint16_t* pk, const uint
   return 3.0 / Z * (DN + vmax * DZ);
 }
 
+/* ------------------------------------------------ coverage profile ------ */
+
+/*
+ * Coverage profile of one realized query row over n keys (§3: the ranked gap
+ * profile and the coverage budget; the count definitions; appendix: the
+ * gap-profile instrument, which recomputes row logits).  z_j = scale <q, k_j>,
+ * A = softmax(z).  pi orders the logits nonincreasingly, ties by lower index.
+ * Writes
+ *   order[r]  = pi(r + 1), the token at rank r (0-based ranks; NULL: skipped)
+ *   gap[r]    = G(r + 1) = z_(1) - z_(r+1) (NULL: skipped)
+ *   K_eta[e]  = min{k : sum_{j <= k} A_(j) >= 1 - eta[e]}
+ *   rel[e]    = #{j : A_j > rel_eps[e] A_(1)} (relative-weight count)
+ *   abs_[e]   = #{j : A_j > abs_eps[e]} (calibrated count k(eps))
+ *   top[0] = z_(1), top[1] = log sum_j e^{z_j}
+ */
+void oracle_coverage_profile(const uint16_t* q, const uint16_t* K, int n, int d, double scale,
+                             const double* eta, int n_eta, const double* rel_eps, int n_rel,
+                             const double* abs_eps, int n_abs, int32_t* order, double* gap,
+                             int32_t* K_eta, int32_t* rel, int32_t* abs_, double* top) {
+  scored_t* t = (scored_t*)malloc((size_t)n * sizeof(scored_t));
+  for (int j = 0; j < n; ++j) {
+    double dot = 0.0;
+    for (int i = 0; i < d; ++i) dot += bf16_to_f64(q[i]) * bf16_to_f64(K[(size_t)j * d + i]);
+    t[j].a = scale * dot;
+    t[j].j = j;
+  }
+  qsort(t, (size_t)n, sizeof(scored_t), cmp_desc_then_index);
+  const double z1 = t[0].a;
+  double Z = 0.0;
+  for (int r = 0; r < n; ++r) Z += exp(t[r].a - z1);
+  for (int r = 0; r < n; ++r) {
+    if (order) order[r] = t[r].j;
+    if (gap) gap[r] = z1 - t[r].a;
+  }
+  for (int e = 0; e < n_eta; ++e) {
+    double c = 0.0;
+    int k = n;
+    for (int r = 0; r < n; ++r) {
+      c += exp(t[r].a - z1) / Z;
+      if (c >= 1.0 - eta[e]) { k = r + 1; break; }
+    }
+    K_eta[e] = k;
+  }
+  const double A1 = 1.0 / Z;
+  for (int e = 0; e < n_rel; ++e) {
+    int cnt = 0;
+    for (int r = 0; r < n; ++r)
+      if (exp(t[r].a - z1) / Z > rel_eps[e] * A1) ++cnt;
+    rel[e] = cnt;
+  }
+  for (int e = 0; e < n_abs; ++e) {
+    int cnt = 0;
+    for (int r = 0; r < n; ++r)
+      if (exp(t[r].a - z1) / Z > abs_eps[e]) ++cnt;
+    abs_[e] = cnt;
+  }
+  top[0] = z1;
+  top[1] = z1 + log(Z);
+  free(t);
+}
+
 /* ------------------------------------------------- fixed-row diagnostics ---- */
 
 /*

@@ -759,6 +759,80 @@ def pin_gaussian_kept_fraction(lib=None):
     assert abs(k_eta / n - limit) < 0.01, (k_eta / n, limit)
 
 
+def pin_coverage_worked(lib=None):
+    """Coverage profile of a hand-built row (§3: ranked gap profile G(j) =
+    z_(1) - z_(j), coverage budget K_eta, relative and calibrated counts): q =
+    e1, scale 1, logits (0, 1, 2, 1/2, 1).  Order 2, 1, 4, 3, 0 (the tied
+    logits 1 by lower index), gaps (0, 1, 1, 3/2, 2), Z = e^2 + 2e + sqrt(e) + 1
+    (15.474): cumulative ranked mass 0.478, 0.653, 0.829, 0.935, 1, so K_0.5 =
+    2, K_0.2 = 3, K_0.05 = 5; A_j > eps A_(1) iff z_j > 2 + log eps (eps 0.3:
+    3 tokens, 0.5: 1, 0.1: 5); weights (0.065, 0.176, 0.478, 0.107, 0.176), so
+    3 tokens above 0.15 and 4 above 0.1."""
+    K = np.zeros((5, 2))
+    K[:, 0] = [0.0, 1.0, 2.0, 0.5, 1.0]
+    r = oracle.coverage_profile(to_bf16_bits([1.0, 0.0]), to_bf16_bits(K), scale=1.0,
+                                eta=[0.5, 0.2, 0.05], rel_eps=[0.3, 0.5, 0.1],
+                                abs_eps=[0.15, 0.1], lib=lib)
+    assert r["order"].tolist() == [2, 1, 4, 3, 0]
+    assert np.allclose(r["gap"], [0.0, 1.0, 1.0, 1.5, 2.0], rtol=0, atol=1e-15)
+    assert r["K_eta"].tolist() == [2, 3, 5]
+    assert r["rel"].tolist() == [3, 1, 5]
+    assert r["abs"].tolist() == [3, 4]
+    Z = math.e ** 2 + 2 * math.e + math.sqrt(math.e) + 1
+    assert abs(r["top"][0] - 2.0) < 1e-15 and abs(r["top"][1] - math.log(Z)) < 1e-12
+
+
+def pin_coverage_flat_row(lib=None):
+    """A flat row (all logits equal, A_j = 1/n exactly): index order, zero
+    gaps, K_eta = ceil((1 - eta) n) with the threshold met exactly at eta =
+    1/2 (the definition's >=), every token above eps A_(1) for eps < 1 and none
+    at eps = 1, and A_j = 1/8 is not above 1/8."""
+    n = 8
+    r = oracle.coverage_profile(to_bf16_bits([1.0, 0.0]), to_bf16_bits(np.zeros((n, 2))),
+                                scale=1.0, eta=[0.5, 0.1, 0.3], rel_eps=[0.5, 1.0],
+                                abs_eps=[0.125, 0.1], lib=lib)
+    assert r["order"].tolist() == list(range(n)) and (r["gap"] == 0).all()
+    assert r["K_eta"].tolist() == [4, 8, 6]
+    assert r["rel"].tolist() == [8, 0] and r["abs"].tolist() == [0, 8]
+    assert abs(r["top"][1] - math.log(n)) < 1e-15
+
+
+def pin_coverage_gaussian_and_envelopes(lib=None):
+    """iid N(0, 1) logits: K_eta / n close to Phi(Phi^-1(1 - eta) - 1) (§3);
+    the order-statistic mass bound 1 - p(k) <= (n - k)/(k + 1) caps K_eta; and
+    on power-law rows the global gap envelopes of Theorem (coverage regimes from
+    global gap envelopes) bound K_eta from above (gamma > 1) and below (gamma' <
+    1), with b and b' read off the returned gap profile."""
+    g = golden("gaussian_kept_fraction")
+    rng = np.random.default_rng(19)
+    n = 100_000
+    K = np.zeros((n, 2))
+    K[:, 0] = rng.standard_normal(n)
+    r = oracle.coverage_profile(to_bf16_bits([1.0, 0.0]), to_bf16_bits(K), scale=g["sigma"],
+                                eta=[g["eta"]], lib=lib)
+    limit = norm.cdf(norm.ppf(1 - g["eta"]) - g["sigma"])
+    assert abs(r["K_eta"][0] / n - limit) < 0.01, (r["K_eta"][0] / n, limit)
+    for n, gamma in ((4000, 2.0), (4000, 1.5), (20000, 0.5), (20000, 0.2)):
+        j = np.arange(1, n + 1)
+        G = gamma * np.log(j) + rng.random(n) * 0.5
+        G[0] = 0.0
+        K = np.zeros((n, 2))
+        K[rng.permutation(n), 0] = -G
+        for eta in (0.1, 0.3):
+            r = oracle.coverage_profile(to_bf16_bits([1.0, 0.0]), to_bf16_bits(K), scale=1.0,
+                                        eta=[eta], lib=lib)
+            gap, k_eta = r["gap"], int(r["K_eta"][0])
+            assert k_eta <= math.ceil((n - eta) / (1 + eta))
+            if gamma > 1:
+                b = max(0.0, float(np.max(gamma * np.log(j) - gap)))
+                cap = math.ceil((math.exp(b) / ((gamma - 1) * eta)) ** (1 / (gamma - 1)))
+                assert k_eta <= cap, (n, gamma, eta, k_eta, cap)
+            else:
+                b2 = max(0.0, float(np.max(gap - gamma * np.log(j))))
+                floor_ = (1 - eta) * math.exp(-b2) / 2 * n ** (1 - gamma)
+                assert k_eta >= floor_, (n, gamma, eta, k_eta, floor_)
+
+
 def pin_compress_batching(lib=None):
     """The batched pass scores unit (b, l, h) with the observation rows of query
     heads h*G .. h*G+G-1 of the same (b, l) (query head qh reads KV head qh/G)."""

@@ -51,6 +51,11 @@ MUTANTS = {
                                      "sumT += exp(z[j] - zmaxT);"),
     "lift_tail_weights_not_renormalised": ("const double a = p > 0.0 ? A / p : 0.0;",
                                            "const double a = A;"),
+    "coverage_strict_threshold": ("if (c >= 1.0 - eta[e])", "if (c > 1.0 - eta[e])"),
+    "coverage_gap_sign": ("if (gap) gap[r] = z1 - t[r].a;", "if (gap) gap[r] = t[r].a - z1;"),
+    "coverage_relative_count_absolute": ("> rel_eps[e] * A1", "> rel_eps[e]"),
+    "coverage_calibrated_count_unnormalised": ("if (exp(t[r].a - z1) / Z > abs_eps[e])",
+                                               "if (exp(t[r].a - z1) > abs_eps[e])"),
     "bisection_inverted": ("if (total > B_real) lam_lo = lam; else lam_hi = lam;",
                            "if (total > B_real) lam_hi = lam; else lam_lo = lam;"),
     "kept_not_sorted": ("qsort(kept, (size_t)b, sizeof(int32_t), cmp_int32);", ""),
