@@ -289,6 +289,35 @@ int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void*
                            int32_t tail_slot, float* stats, void* workspace,
                            size_t workspace_bytes, void* stream);
 
+/* Coverage profile of realized query rows (an evaluation instrument: §3,
+ * "count sparsity does not imply coverage sparsity", with the ranked gap
+ * profile G(j) = z_(1) - z_(j) and the coverage budget K_eta; the appendix's
+ * gap-profile instrument recomputes the row logits in fp32, as here).  One row
+ * per query head qh of each (sequence, layer), over the n keys of KV head
+ * qh / G: z_j = scale <q, k_j> (fp32), A = softmax(z), pi the order of the
+ * logits, descending, ties by lower index.  Per row r = (b L + l) Hq + qh:
+ *   K_eta[r][e]      = min{k : sum_{j <= k} A_(j) >= 1 - eta[e]}  (int32)
+ *   rel_counts[r][e] = #{j : A_j > rel_eps[e] A_(1)}  (relative-weight count)
+ *   abs_counts[r][e] = #{j : A_j > abs_eps[e]}        (calibrated count k(eps))
+ *   top[r][0] = z_(1), top[r][1] = log sum_j e^{z_j}  (fp32)
+ *   order[r][i] = pi(i + 1), the token at rank i (int32 [rows][n], may be NULL)
+ *   gap[r][i]   = G(i + 1) (fp32 [rows][n], may be NULL)
+ * The ranked mass is summed in float64 in one fixed order from fp32 weights
+ * e^{z_(j) - z_(1)}; the counts compare fp32 logit differences with log eps.
+ * eta, rel_eps, abs_eps: HOST arrays of n_eta, n_rel, n_abs values (each count
+ * 0..CERTKV_COVERAGE_MAX_THRESHOLDS; 0 < eta < 1; eps > 0, finite); an output
+ * array may be NULL when its count is 0.  q bf16 [B][L][Hq][d], K bf16 as for
+ * certkv_compress; scale 0 selects 1/sqrt(d).  Workspace:
+ * certkv_coverage_workspace_bytes(shape) (16 n bytes per row plus the sort's
+ * tile histograms). */
+#define CERTKV_COVERAGE_MAX_THRESHOLDS 16
+size_t certkv_coverage_workspace_bytes(const certkv_shape* shape);
+int certkv_coverage_profile(const certkv_shape* shape, const void* q, const void* K, float scale,
+                            const double* eta, int32_t n_eta, const double* rel_eps,
+                            int32_t n_rel, const double* abs_eps, int32_t n_abs, int32_t* K_eta,
+                            int32_t* rel_counts, int32_t* abs_counts, float* top, int32_t* order,
+                            float* gap, void* workspace, size_t workspace_bytes, void* stream);
+
 /* Decode attention that allocates nothing.  The paper has no counterpart: this
  * entry point exists for callers that cannot hand the library a scratch
  * buffer, for example a plugin that an inference server gives only its input

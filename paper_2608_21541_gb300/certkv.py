@@ -52,7 +52,8 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_read_status", "certkv_strerror", "certkv_trace_enable",
             "certkv_trace_report", "certkv_decode_attn_noalloc", "certkv_host_workspace_bytes",
             "certkv_compress_host", "certkv_decode_certified", "certkv_fixed_row_workspace_bytes",
-            "certkv_fixed_row_stats")
+            "certkv_fixed_row_stats", "certkv_coverage_workspace_bytes",
+            "certkv_coverage_profile")
 
 _lock = threading.Lock()
 _lib = None
@@ -117,6 +118,11 @@ def load_library(path: Optional[str] = None):
         lib.certkv_fixed_row_stats.argtypes = [sp, P, P, P, P, kp, ctypes.c_float, I32, P, P, SZ,
                                                     P]
         lib.certkv_fixed_row_stats.restype = ctypes.c_int
+        lib.certkv_coverage_workspace_bytes.argtypes = [sp]
+        lib.certkv_coverage_workspace_bytes.restype = SZ
+        lib.certkv_coverage_profile.argtypes = [sp, P, P, ctypes.c_float, P, I32, P, I32, P, I32,
+                                                P, P, P, P, P, P, P, SZ, P]
+        lib.certkv_coverage_profile.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -425,6 +431,41 @@ def certkv_fixed_row_stats(q, K, V, packed: Packed, *, scores=None, scale: float
                                                ws.numel(), _stream(stream))
     _check(rc, "certkv_fixed_row_stats")
     return stats
+
+
+def certkv_coverage_profile(q, K, *, eta=(0.1,), rel_eps=(0.1,), abs_eps=(), scale: float = 0.0,
+                            with_order: bool = False, with_gap: bool = False, ws=None,
+                            stream=None) -> dict:
+    """Coverage profile of the decode query rows q [B][L][Hq][d] over the keys K
+    [B][L][H][n][d]: K_eta int32 [B][L][Hq][len(eta)], rel / abs counts int32,
+    top fp32 [B][L][Hq][2] (max logit, log-partition), and optionally order
+    int32 / gap fp32 [B][L][Hq][n] (evaluation instrument; reads all of K)."""
+    _bf16(q, "q"); _bf16(K, "K")
+    B, L, Hq, d = q.shape
+    n = K.shape[3]
+    shape = certkv_shape(B, L, Hq, K.shape[2], n, d, 1)
+    dev = q.device
+
+    def host(x):
+        return (ctypes.c_double * max(len(x), 1))(*[float(v) for v in x])
+
+    def out(cnt, dtype):
+        return torch.empty((B, L, Hq, cnt), dtype=dtype, device=dev) if cnt else None
+
+    K_eta, rel, ab = out(len(eta), torch.int32), out(len(rel_eps), torch.int32), \
+        out(len(abs_eps), torch.int32)
+    top = torch.empty((B, L, Hq, 2), dtype=torch.float32, device=dev)
+    order = out(n, torch.int32) if with_order else None
+    gap = out(n, torch.float32) if with_gap else None
+    if ws is None:
+        ws = workspace(int(load_library().certkv_coverage_workspace_bytes(ctypes.byref(shape))),
+                       dev)
+    rc = load_library().certkv_coverage_profile(
+        ctypes.byref(shape), _ptr(q), _ptr(K), float(scale), host(eta), len(eta), host(rel_eps),
+        len(rel_eps), host(abs_eps), len(abs_eps), _ptr(K_eta), _ptr(rel), _ptr(ab), _ptr(top),
+        _ptr(order), _ptr(gap), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "certkv_coverage_profile")
+    return dict(K_eta=K_eta, rel=rel, abs=ab, top=top, order=order, gap=gap)
 
 
 def certkv_read_status(ws: torch.Tensor, stream=None) -> int:

@@ -523,6 +523,49 @@ int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void*
   return cuda_ok(cudaGetLastError());
 }
 
+size_t certkv_coverage_workspace_bytes(const certkv_shape* shape) {
+  certkv_params prm;
+  certkv_default_params(&prm);
+  Prob p;
+  if (make_prob(shape, &prm, -1, &p)) return 0;
+  return coverage_workspace(p);
+}
+
+namespace {
+bool thresholds_ok(const double* x, int32_t cnt, bool below_one, const void* out) {
+  if (cnt < 0 || cnt > CERTKV_COVERAGE_MAX_THRESHOLDS) return false;
+  if (cnt == 0) return true;
+  if (!x || !out) return false;
+  for (int32_t e = 0; e < cnt; ++e)
+    if (!(x[e] > 0.0) || !isfinite(x[e]) || (below_one && !(x[e] < 1.0))) return false;
+  return true;
+}
+}  // namespace
+
+int certkv_coverage_profile(const certkv_shape* shape, const void* q, const void* K, float scale,
+                            const double* eta, int32_t n_eta, const double* rel_eps,
+                            int32_t n_rel, const double* abs_eps, int32_t n_abs, int32_t* K_eta,
+                            int32_t* rel_counts, int32_t* abs_counts, float* top, int32_t* order,
+                            float* gap, void* workspace, size_t workspace_bytes, void* stream) {
+  certkv_params prm;
+  certkv_default_params(&prm);
+  Prob p;
+  int rc = make_prob(shape, &prm, -1, &p);
+  if (rc) return rc;
+  if (!q || !K || !top || !aligned(q, 16) || !aligned(K, 16)) return CERTKV_EINVAL;
+  if (!thresholds_ok(eta, n_eta, true, K_eta) || !thresholds_ok(rel_eps, n_rel, false, rel_counts) ||
+      !thresholds_ok(abs_eps, n_abs, false, abs_counts))
+    return CERTKV_EINVAL;
+  if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < coverage_workspace(p))
+    return CERTKV_EWORKSPACE;
+  const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
+  launch_coverage(p, q, K, sc, eta, n_eta, rel_eps, n_rel, abs_eps, n_abs, K_eta, rel_counts,
+                  abs_counts, top, order, gap, reinterpret_cast<char*>(workspace),
+                  reinterpret_cast<cudaStream_t>(stream));
+  return cuda_ok(cudaGetLastError());
+}
+
 int certkv_read_status(const void* workspace, void* stream) {
   if (!workspace) return -1;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

@@ -90,6 +90,12 @@ void launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
                    void* out, char* ws, cudaStream_t st);
 size_t decode_workspace(const Prob& p);
 size_t fixed_row_workspace(const Prob& p);
+size_t coverage_workspace(const Prob& p);
+void launch_coverage(const Prob& p, const void* q, const void* K, float scale,
+                     const double* eta, int n_eta, const double* rel_eps, int n_rel,
+                     const double* abs_eps, int n_abs, int32_t* K_eta, int32_t* rel,
+                     int32_t* abs_, float* top, int32_t* order, float* gap, char* ws,
+                     cudaStream_t st);
 void launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V,
                       const float* scores, const int64_t* offsets, const int32_t* counts,
                       const int32_t* positions,

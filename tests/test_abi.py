@@ -139,3 +139,34 @@ def test_host_entry_point_validation(lib):
     assert call(ws=0) == ck.EWORKSPACE
     assert call(ws=257) == ck.EWORKSPACE
     assert call(ws_bytes=need - 1) == ck.EWORKSPACE
+
+
+def test_coverage_profile_validation(lib):
+    s = shape()
+    need = lib.certkv_coverage_workspace_bytes(ctypes.byref(s))
+    assert need > 16 * s.n * s.batch * s.layers * s.hq
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
+
+    def arr(*x):
+        return (ctypes.c_double * max(len(x), 1))(*x)
+
+    def call(eta=(0.1,), rel=(0.1,), ab=(0.01,), out=fake, ws=256, ws_bytes=None, scale=0.0,
+             n_eta=None):
+        return lib.certkv_coverage_profile(
+            ctypes.byref(s), fake, fake, scale, arr(*eta), len(eta) if n_eta is None else n_eta,
+            arr(*rel), len(rel), arr(*ab), len(ab), out, out, out, fake, None, None,
+            ctypes.c_void_p(ws) if ws else None, need if ws_bytes is None else ws_bytes, None)
+
+    assert call(eta=(1.0,)) == ck.EINVAL          # eta must lie in (0, 1)
+    assert call(eta=(0.0,)) == ck.EINVAL
+    assert call(rel=(0.0,)) == ck.EINVAL          # thresholds positive
+    assert call(ab=(float("inf"),)) == ck.EINVAL
+    assert call(out=None) == ck.EINVAL            # an output missing for a nonzero count
+    assert call(n_eta=17) == ck.EINVAL            # at most 16 thresholds per kind
+    assert call(scale=-1.0) == ck.EINVAL
+    assert call(ws=0) == ck.EWORKSPACE
+    assert call(ws_bytes=need - 1) == ck.EWORKSPACE
+    # counts of zero need no arrays
+    assert lib.certkv_coverage_profile(
+        ctypes.byref(s), fake, fake, 0.0, None, 0, None, 0, None, 0, None, None, None, fake,
+        None, None, None, need, None) == ck.EWORKSPACE
