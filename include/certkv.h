@@ -327,10 +327,12 @@ int certkv_coverage_profile(const certkv_shape* shape, const void* q, const void
  * (same kernels, same arguments minus the workspace); its split-K scratch is a
  * fixed array of CERTKV_NOALLOC_SCRATCH_BYTES in the library's own device
  * memory, present on every GPU that loads the library until the process exits.
- *   - Limit: (B * L * H) * G * 16 partial records of 520 bytes must fit in the
- *     array, i.e. (B * L * H) * G <= 2016 (one 32-layer, 8-KV-head, G = 4
- *     sequence per call); larger calls return CERTKV_ETOOLARGE and enqueue
- *     nothing.  Split a larger batch into several calls.
+ *   - Limit: certkv_decode_workspace_bytes(shape) must fit in the array: with
+ *     U = B * L * H, 4 (U + 1) bytes of tile offsets and (U + 1024) * G split
+ *     records of 520 bytes, about (U + 1024) * G <= 32000 (eight 32-layer,
+ *     8-KV-head, G = 4 sequences per call); larger calls return
+ *     CERTKV_ETOOLARGE and enqueue nothing.  Split a larger batch into
+ *     several calls.
  *   - The first call on each device looks up the array's device address (with
  *     that device current); make that first call before any stream capture.
  *   - Every call on a device shares the one array, and each call rewrites every

@@ -14,7 +14,6 @@ constexpr int kHullSeg = 256;    // curve points per hull-filter thread
 constexpr int kGroupSegs = 16;   // hull-filter segments per group
 constexpr int kSortTile = 2048;  // keys per radix-sort tile
 constexpr int kSortThreads = 256;
-constexpr int kDecodeSplits = 16;
 constexpr uint32_t kFull = 0xffffffffu;
 
 // ------------------------------------------------------------ status word --
@@ -210,6 +209,25 @@ __device__ __forceinline__ float key_score(uint32_t k) { return __uint_as_float(
 __device__ __forceinline__ float warp_max(float x) {
 #pragma unroll
   for (int m = 16; m >= 1; m >>= 1) x = fmaxf(x, __shfl_xor_sync(kFull, x, m));
+  return x;
+}
+
+// Eight per-lane partials of rows 0..7 -> every lane l holds the lane sum of
+// row (l & 7).
+__device__ __forceinline__ float reduce8(float (&v)[8], int lane) {
+#pragma unroll
+  for (int o = 4; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const float keep = upper ? v[i + o] : v[i];
+      const float send = upper ? v[i] : v[i + o];
+      v[i] = keep + __shfl_xor_sync(kFull, send, o);
+    }
+  }
+  float x = v[0];
+  x += __shfl_xor_sync(kFull, x, 8);
+  x += __shfl_xor_sync(kFull, x, 16);
   return x;
 }
 

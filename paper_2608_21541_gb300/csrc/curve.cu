@@ -22,24 +22,7 @@ namespace certkv {
 
 namespace {
 
-// Eight per-lane partials of rows 0..7 -> every lane l holds the lane sum of
-// row (l & 7).
-__device__ __forceinline__ float reduce8(float (&v)[8], int lane) {
-#pragma unroll
-  for (int o = 4; o >= 1; o >>= 1) {
-    const bool upper = (lane & o) != 0;
-#pragma unroll
-    for (int i = 0; i < o; ++i) {
-      const float keep = upper ? v[i + o] : v[i];
-      const float send = upper ? v[i] : v[i + o];
-      v[i] = keep + __shfl_xor_sync(kFull, send, o);
-    }
-  }
-  float x = v[0];
-  x += __shfl_xor_sync(kFull, x, 8);
-  x += __shfl_xor_sync(kFull, x, 16);
-  return x;
-}
+// As reduce8 (common.cuh), in double-float.
 __device__ __forceinline__ DF reduce8_df(DF (&v)[8], int lane) {
 #pragma unroll
   for (int o = 4; o >= 1; o >>= 1) {

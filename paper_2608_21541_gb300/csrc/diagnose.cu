@@ -124,30 +124,41 @@ __global__ void __launch_bounds__(128) fixed_row_split_kernel(
       lk[g] += pk[g];
       lt[g] += pt[g];
     }
+    // value rows of the tile, 8 loads in flight per lane; rows past the end
+    // of the unit read as zero and carry zero weight
     const int cnt = min(32, n - t * 32);
-    for (int r = 0; r < cnt; ++r) {
-      const uint2 raw = __ldg(Vu + (size_t)(t * 32 + r) * (kD / 4) + lane);
-      const float v[4] = {bf16lo(raw.x), bf16hi(raw.x), bf16lo(raw.y), bf16hi(raw.y)};
-      float sq = fmaf(v[3], v[3], fmaf(v[2], v[2], fmaf(v[1], v[1], v[0] * v[0])));
+    for (int r0 = 0; r0 < cnt; r0 += 8) {
+      uint2 raw[8];
 #pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) sq += __shfl_xor_sync(kFull, sq, o);
-      vmax = fmaxf(vmax, sqrtf(sq));
+      for (int k = 0; k < 8; ++k)
+        raw[k] = r0 + k < cnt ? __ldg(Vu + (size_t)(t * 32 + r0 + k) * (kD / 4) + lane)
+                              : make_uint2(0u, 0u);
+      float sq[8];
 #pragma unroll
-      for (int g = 0; g < G; ++g) {
-        const float wk = __shfl_sync(kFull, pk[g], r), wt = __shfl_sync(kFull, pt[g], r);
+      for (int k = 0; k < 8; ++k) {
+        const int r = r0 + k;
+        const float v[4] = {bf16lo(raw[k].x), bf16hi(raw[k].x), bf16lo(raw[k].y),
+                            bf16hi(raw[k].y)};
+        sq[k] = fmaf(v[3], v[3], fmaf(v[2], v[2], fmaf(v[1], v[1], v[0] * v[0])));
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          ak[g][i] = fmaf(wk, v[i], ak[g][i]);
-          at[g][i] = fmaf(wt, v[i], at[g][i]);
+        for (int g = 0; g < G; ++g) {
+          const float wk = __shfl_sync(kFull, pk[g], r), wt = __shfl_sync(kFull, pt[g], r);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            ak[g][i] = fmaf(wk, v[i], ak[g][i]);
+            at[g][i] = fmaf(wt, v[i], at[g][i]);
+          }
+        }
+        if (sc != nullptr) {
+          const float ws = __shfl_sync(kFull, sj, r);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) sv[i] = fmaf(ws, v[i], sv[i]);
         }
       }
-      if (sc != nullptr) {
-        const float ws = __shfl_sync(kFull, sj, r);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) sv[i] = fmaf(ws, v[i], sv[i]);
-      }
+      vmax = fmaxf(vmax, sqrtf(reduce8(sq, lane)));  // lane l: row r0 + (l & 7)
     }
   }
+  vmax = warp_max(vmax);
   // combine the 4 warps, one query head at a time
   const int i = threadIdx.x;  // 128 threads = kD dimensions
 #pragma unroll
@@ -346,10 +357,11 @@ FixedRowLayout fixed_row_layout(const Prob& p) {
 
 size_t fixed_row_workspace(const Prob& p) { return fixed_row_layout(p).total; }
 
-void launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V,
-                      const float* scores, const int64_t* offsets, const int32_t* counts,
-                      const int32_t* positions, const void* pk, const void* pv, int tail_slot,
-                      float scale, float* stats, char* ws, cudaStream_t st) {
+bool launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V,
+                      const float* scores, int64_t rows, const int64_t* offsets,
+                      const int32_t* counts, const int32_t* positions, const void* pk,
+                      const void* pv, int tail_slot, float scale, float* stats, char* ws,
+                      cudaStream_t st) {
   const FixedRowLayout ly = fixed_row_layout(p);
   const size_t words = (size_t)(p.n + 31) / 32;
   uint32_t* mask = reinterpret_cast<uint32_t*>(ws + ly.mask);
@@ -359,7 +371,8 @@ void launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V
   float* psv = reinterpret_cast<float*>(ws + ly.sv);
   char* ohat = ws + ly.ohat;
   // the compressed decode's output, for its error against O
-  launch_decode(p, q, pk, pv, offsets, counts, tail_slot, scale, ohat, ws + ly.dec, st);
+  if (!launch_decode(p, q, pk, pv, rows, offsets, counts, tail_slot, scale, ohat, ws + ly.dec, st))
+    return false;
   cudaMemsetAsync(mask, 0, p.units * words * 4, st);
   {
     TraceScope ts_("kept_mask", st);
@@ -381,7 +394,7 @@ void launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V
       case 4: CERTKV_FR_SPLIT(4); break;
       case 8: CERTKV_FR_SPLIT(8); break;
       case 16: CERTKV_FR_SPLIT(16); break;
-      default: return;
+      default: return false;
     }
 #undef CERTKV_FR_SPLIT
   }
@@ -392,6 +405,7 @@ void launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V
         reinterpret_cast<const __nv_bfloat16*>(pk), reinterpret_cast<const __nv_bfloat16*>(pv),
         offsets, counts, tail_slot, sl2, scores, z2, psv, mask, stats);
   }
+  return true;
 }
 
 }  // namespace certkv

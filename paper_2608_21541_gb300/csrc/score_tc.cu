@@ -24,6 +24,7 @@
 #include "../../include/certkv.h"
 #include "common.cuh"
 #include "internal.cuh"
+#include "tma.cuh"
 
 namespace certkv {
 namespace tc {
@@ -34,7 +35,6 @@ namespace tc {
 constexpr int kEpiWarps = 16;  // warp (q, cq): TMEM lane quadrant q, 64-column quarter cq
 constexpr int kThreads = (2 + kEpiWarps) * 32;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kSpinLimit = 1u << 22;
 constexpr uint32_t kStatusTimeout = CERTKV_STATUS_TIMEOUT;
 
 // Shared-memory plan of one pass: Q rows staged once, a ring of K tiles.
@@ -52,49 +52,6 @@ struct Cfg {
 using Pass1 = Cfg<128, 256, 2>;
 // pass 2: all (<= 256) rows of Q, 128-key tiles (M128 x N<=256 MMAs)
 using Pass2 = Cfg<256, 128, CERTKV_TC_STAGES>;
-
-// ------------------------------------------------------------ primitives --
-__device__ __forceinline__ uint32_t saddr(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
-}
-__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t a) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
-}
-__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred P;\n mbarrier.try_wait.parity.shared::cta.b64 P, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, P;\n}\n"
-      : "=r"(ok)
-      : "r"(a), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Bounded wait: false on timeout or when another role has aborted.
-__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, volatile int* abort_flag) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if (mbar_try(a, parity)) return true;
-    if ((i & 255u) == 255u && *abort_flag) return false;
-  }
-  *abort_flag = 1;
-  return false;
-}
-
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
-                                            uint32_t mbar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(mbar)
-      : "memory");
-}
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
 // 128 B, groups of 8 rows 1024 B apart.
@@ -518,9 +475,9 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 2-D view [rows][128] of a bf16 tensor, boxes of {64 dims, box_rows rows},
-// 128-byte swizzle.
-bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {
+}  // namespace
+
+bool make_row_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {128, rows};
@@ -532,16 +489,15 @@ bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t box_ro
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-}  // namespace
-
 bool score_tc_supported(const Prob& p) { return p.R == 128 || p.R == 256; }
 
 bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_part, float* lse2,
                      float* s_part, uint32_t* status, cudaStream_t st) {
   CUtensorMap mk1, mq1, mk2, mq2;
   const uint64_t krows = (uint64_t)p.units * p.n, qrows = (uint64_t)p.units * p.R;
-  if (!make_map(&mk1, K, krows, tc::Pass1::kTileKeys) || !make_map(&mq1, Q, qrows, 128) ||
-      !make_map(&mk2, K, krows, tc::Pass2::kTileKeys) || !make_map(&mq2, Q, qrows, (uint32_t)p.R))
+  if (!make_row_map(&mk1, K, krows, tc::Pass1::kTileKeys) || !make_row_map(&mq1, Q, qrows, 128) ||
+      !make_row_map(&mk2, K, krows, tc::Pass2::kTileKeys) ||
+      !make_row_map(&mq2, Q, qrows, (uint32_t)p.R))
     return false;
   static bool attr = false;
   if (!attr) {

@@ -46,7 +46,7 @@ def test_noalloc_decode_matches_regular_decode_twice():
 
 def test_noalloc_decode_refuses_beyond_its_scratch():
     lib = ck.load_library()
-    shape = ck.certkv_shape(8, 32, 32, 8, 32768, 128, 64)  # (B*L*H)*G = 8192 > 2016
+    shape = ck.certkv_shape(8, 80, 64, 8, 32768, 128, 64)  # (B*L*H + 1024)*G = 49152
     fake = ctypes.c_void_p(1 << 20)
     st = ck.certkv_packed(fake, fake, fake, fake, fake, 1 << 30, None, None)
     rc = lib.certkv_decode_attn_noalloc(ctypes.byref(shape), fake, ctypes.byref(st),
