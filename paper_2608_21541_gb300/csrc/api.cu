@@ -449,7 +449,6 @@ int certkv_decode_attn(const certkv_shape* shape, const void* q, const certkv_pa
     return CERTKV_EINVAL;
   if (!aligned(packed->k, 16) || !aligned(packed->v, 16) || !aligned(q, 16)) return CERTKV_EINVAL;
   if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
-  if (packed->capacity_slots < 1 || packed->capacity_slots > INT32_MAX) return CERTKV_EINVAL;
   if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
   certkv_params prm;
   certkv_default_params(&prm);
@@ -459,9 +458,8 @@ int certkv_decode_attn(const certkv_shape* shape, const void* q, const certkv_pa
     return CERTKV_EWORKSPACE;
   const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (!launch_decode(p, q, packed->k, packed->v, packed->capacity_slots, packed->offsets,
-                     packed->real_counts, tail_slot, sc, out, reinterpret_cast<char*>(workspace),
-                     st))
+  if (!launch_decode(p, q, packed->k, packed->v, packed->offsets, packed->real_counts, tail_slot,
+                     sc, out, reinterpret_cast<char*>(workspace), st))
     return CERTKV_ECUDA;
   return cuda_ok(cudaGetLastError());
 }
@@ -477,7 +475,6 @@ int certkv_decode_certified(const certkv_shape* shape, const void* q, const cert
     return CERTKV_EINVAL;
   if (!aligned(packed->k, 16) || !aligned(packed->v, 16) || !aligned(q, 16)) return CERTKV_EINVAL;
   if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
-  if (packed->capacity_slots < 1 || packed->capacity_slots > INT32_MAX) return CERTKV_EINVAL;
   if (clusters < 1 || clusters > CERTKV_MAX_CLUSTERS) return CERTKV_EINVAL;
   if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
   certkv_params prm;
@@ -488,9 +485,9 @@ int certkv_decode_certified(const certkv_shape* shape, const void* q, const cert
     return CERTKV_EWORKSPACE;
   const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (!launch_decode_certified(p, q, packed->k, packed->v, packed->capacity_slots,
-                               packed->offsets, packed->real_counts, tail_slot, clusters,
-                               packed->cluster_meta, packed->kept_vmax, sc, out, bound, certified,
+  if (!launch_decode_certified(p, q, packed->k, packed->v, packed->offsets,
+                               packed->real_counts, tail_slot, clusters, packed->cluster_meta,
+                               packed->kept_vmax, sc, out, bound, certified,
                                reinterpret_cast<char*>(workspace), st))
     return CERTKV_ECUDA;
   return cuda_ok(cudaGetLastError());
@@ -519,16 +516,14 @@ int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void*
   if (!aligned(q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(packed->k, 16) ||
       !aligned(packed->v, 16) || !aligned(scores, 4))
     return CERTKV_EINVAL;
-  if (packed->capacity_slots < 1 || packed->capacity_slots > INT32_MAX) return CERTKV_EINVAL;
   if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
   if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < fixed_row_workspace(p))
     return CERTKV_EWORKSPACE;
   const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
-  if (!launch_fixed_row(p, q, K, V, scores, packed->capacity_slots, packed->offsets,
-                        packed->real_counts, packed->positions, packed->k, packed->v, tail_slot,
-                        sc, stats, reinterpret_cast<char*>(workspace),
-                        reinterpret_cast<cudaStream_t>(stream)))
+  if (!launch_fixed_row(p, q, K, V, scores, packed->offsets, packed->real_counts,
+                        packed->positions, packed->k, packed->v, tail_slot, sc, stats,
+                        reinterpret_cast<char*>(workspace), reinterpret_cast<cudaStream_t>(stream)))
     return CERTKV_ECUDA;
   return cuda_ok(cudaGetLastError());
 }

@@ -11,14 +11,15 @@
 // work is balanced over the global sequence of 32-slot tiles of all units, not
 // over units: a plan kernel scans the tile counts, then a persistent split
 // kernel gives every CTA an equal contiguous range of that sequence.  In each
-// CTA one thread streams the tiles into a ring of shared-memory stages with
-// the TMA (K through a 2-D tensor map with the 128-byte swizzle, so that a lane
-// reading its own slot's row meets no bank conflict; V as one contiguous bulk
-// copy), and the consumer warps keep online (max, sum, acc) for the G query
-// heads of the current unit; where the range crosses into the next unit they
-// combine their states into one record for (CTA, unit).  Every packed K/V
-// byte is read once per step, in whole tiles.  A merge kernel combines the
-// records of each unit in the log-sum-exp domain.
+// CTA one thread streams the tiles' K and V rows into a ring of shared-memory
+// stages with bulk copies, and the consumer warps keep online (max, sum, acc)
+// for the G query heads of the current unit: for the logits, 2G lanes share a
+// slot and hold their slice of the G queries in registers (so a K row is read
+// once, coalesced, with no per-lane query traffic through shared memory); for
+// the values, a lane owns four dimensions.  Where a CTA's range crosses into
+// the next unit the consumer warps combine their states into one record for
+// (CTA, unit).  Every packed K/V byte is read once per step.  A merge kernel
+// combines the records of each unit in the log-sum-exp domain.
 #include "../../include/certkv.h"
 #include "common.cuh"
 #include "internal.cuh"
@@ -27,10 +28,10 @@
 namespace certkv {
 
 #ifndef CERTKV_DEC_STAGES
-#define CERTKV_DEC_STAGES 5
+#define CERTKV_DEC_STAGES 4
 #endif
 #ifndef CERTKV_DEC_CONSUMERS
-#define CERTKV_DEC_CONSUMERS 5
+#define CERTKV_DEC_CONSUMERS 4
 #endif
 constexpr int kDecTile = 32;
 constexpr int kDecStages = CERTKV_DEC_STAGES;
@@ -43,14 +44,12 @@ constexpr int kDecThreads = (1 + kDecConsumers) * 32;
 // itself waited for that previous phase.
 static_assert(kDecStages % kDecConsumers == 0, "each ring stage must belong to one consumer warp");
 constexpr int kDecMaxBlocks = 1024;  // records are sized for at most this many split CTAs
-constexpr int kDecKBytes = kDecTile * 256;  // two 4 KB boxes of 64 columns
+constexpr int kDecKBytes = kDecTile * 256;
 constexpr int kDecVBytes = kDecTile * 256;
 constexpr int kDecStageBytes = kDecKBytes + kDecVBytes;
-static_assert(kDecKBytes % 1024 == 0 && kDecVBytes % 1024 == 0,
-              "the swizzled K boxes need 1024-B alignment");
 __host__ __device__ constexpr int decode_smem_bytes(int G) {
-  return kDecStages * kDecStageBytes + G * kD * 2 + kDecConsumers * G * (kD + 2) * 4 +
-         kDecConsumers * kDecTile * G * 4 + 2 * kDecStages * 8 + 16 + 1024;
+  return kDecStages * kDecStageBytes + kDecConsumers * G * (kD + 2) * 4 +
+         kDecConsumers * kDecTile * G * 4 + 2 * kDecStages * 8 + 16 + 128;
 }
 // records: one per (CTA b, unit u) that meet, at index b + u (unique, and the
 // records of a unit are consecutive)
@@ -99,33 +98,62 @@ __device__ __forceinline__ void consumers_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(kDecConsumers * 32) : "memory");
 }
 
+// Lane geometry of the logits for G query heads: 2G lanes share one slot, each
+// holding 128 / 2G of the G queries' dimensions in registers, so every K row
+// is read once, coalesced, and a transposing shuffle reduction leaves lane i of
+// the slot's group with the logit of head i mod G.
+template <int G>
+struct DecGeo {
+  static constexpr int LPS = 2 * G;           // lanes per slot
+  static constexpr int SPP = 32 / LPS;        // slots per pass
+  static constexpr int NP = kDecTile / SPP;   // passes per tile
+  static constexpr int DPL = kD / LPS;        // dimensions per lane
+  static constexpr int NPAIR = DPL / 2;       // fp32 pairs per lane and head
+};
+
+// v[h]: this lane's partial dot product for head h.  Returns the full dot
+// product of head (lane mod G) over the 2G lanes of the slot group.
+template <int G>
+__device__ __forceinline__ float reduce_heads(float (&v)[G], int lane) {
+#pragma unroll
+  for (int o = G / 2; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int k = 0; k < o; ++k) {
+      const float keep = upper ? v[k + o] : v[k];
+      const float send = upper ? v[k] : v[k + o];
+      v[k] = keep + __shfl_xor_sync(kFull, send, o);
+    }
+  }
+  return v[0] + __shfl_xor_sync(kFull, v[0], G);
+}
+
 // grid = NB persistent CTAs, block = kDecThreads.  CTA b takes the global
 // tiles [b per, (b + 1) per), per = ceil(T[units] / NB); its k-th tile goes
-// through ring stage k % kDecStages and is consumed by consumer warp
-// k % kDecConsumers.  A consumer lane owns one slot for the logits (its K row
-// read from the swizzled stage, the query broadcast from shared memory) and
-// four dimensions for the value sums.  Every wait is bounded; after a timeout
-// the CTA skips the remaining work but keeps its barrier sequence, and writes
-// NaN records, so the affected query heads read NaN.
+// through ring stage k % kDecStages (K and V rows as bulk copies) and is
+// consumed by consumer warp k % kDecConsumers.  Logits as in DecGeo; the value
+// sums with lane = four dimensions and the weights of a row read as one
+// broadcast.  Every wait is bounded; after a timeout the CTA skips the
+// remaining work but keeps its barrier sequence, and writes NaN records, so
+// the affected query heads read NaN.
 template <int G>
 __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
-    const __grid_constant__ CUtensorMap map_k, Prob p, const __nv_bfloat16* __restrict__ q,
+    Prob p, const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ pk,
     const __nv_bfloat16* __restrict__ pv, const int64_t* __restrict__ offsets,
     const int32_t* __restrict__ counts, const int32_t* __restrict__ T, int tail_slot,
     float scale_log2, float2* __restrict__ rec_ml, float* __restrict__ rec_acc) {
+  using Geo = DecGeo<G>;
   extern __shared__ uint8_t dsm_raw[];
-  uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* kst = sm;                                                    // [stage][2][32][128 B]
-  uint8_t* vst = sm + kDecStages * kDecKBytes;                          // [stage][32][256 B]
-  // every region that is read or written with 16-byte vectors starts on a
-  // 16-byte boundary: qs (256 B per head), wacc (512 B per warp and head) and pw
-  // (128 B per warp and head) come first, the scalar arrays after them
-  uint32_t* qs = reinterpret_cast<uint32_t*>(vst + kDecStages * kDecVBytes);  // [G][kD / 2] bf16 pairs
-  float* wacc = reinterpret_cast<float*>(qs + G * kD / 2);              // [consumers][G][kD]
+  uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)dsm_raw + 127) & ~(uintptr_t)127);
+  uint8_t* kst = sm;                                  // [stage][32 rows][256 B]
+  uint8_t* vst = sm + kDecStages * kDecKBytes;        // [stage][32 rows][256 B]
+  // the regions read or written with 16-byte vectors (wacc: 512 B per warp and
+  // head, pw: 128 B per warp and head) start on 16-byte boundaries
+  float* wacc = reinterpret_cast<float*>(vst + kDecStages * kDecVBytes);  // [consumers][G][kD]
   float* pw = wacc + kDecConsumers * G * kD;  // [consumers][32 slots][G] softmax weights
-  float* wm = pw + kDecConsumers * kDecTile * G;                        // [consumers][G]
-  float* wl = wm + kDecConsumers * G;                                   // [consumers][G]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(wl + kDecConsumers * G);  // full, empty (8-B aligned)
+  float* wm = pw + kDecConsumers * kDecTile * G;                          // [consumers][G]
+  float* wl = wm + kDecConsumers * G;                                     // [consumers][G]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(wl + kDecConsumers * G);   // full, empty
   volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * kDecStages);
   const uint32_t full0 = tc::saddr(bars), empty0 = tc::saddr(bars + kDecStages);
 
@@ -166,12 +194,11 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
           break;
         const int t = gt - T[u];
         const int cnt = min(kDecTile, counts[u] + tail_slot - t * kDecTile);
-        const int64_t row0 = offsets[u] + (int64_t)t * kDecTile;
-        tc::mbar_expect_tx(full0 + 8 * s, (uint32_t)(kDecKBytes + cnt * 256));
-        const uint32_t kd = tc::saddr(kst + s * kDecKBytes);
-        tc::tma_load_2d(kd, &map_k, 0, (int)row0, full0 + 8 * s);
-        tc::tma_load_2d(kd + kDecKBytes / 2, &map_k, 64, (int)row0, full0 + 8 * s);
-        tc::bulk_load(tc::saddr(vst + s * kDecVBytes), pv + row0 * kD, (uint32_t)cnt * 256u,
+        const size_t e0 = (size_t)(offsets[u] + (int64_t)t * kDecTile) * kD;
+        tc::mbar_expect_tx(full0 + 8 * s, (uint32_t)cnt * 512u);
+        tc::bulk_load(tc::saddr(kst + s * kDecKBytes), pk + e0, (uint32_t)cnt * 256u,
+                      full0 + 8 * s);
+        tc::bulk_load(tc::saddr(vst + s * kDecVBytes), pv + e0, (uint32_t)cnt * 256u,
                       full0 + 8 * s);
         issued = k + 1;
       }
@@ -183,27 +210,37 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
     }
   } else {  // consumers: one segment per unit met
     const int cw = warp - 1, ct = threadIdx.x - 32;
-    const uint4* q4 = reinterpret_cast<const uint4*>(qs);  // 8 bf16 dimensions per load
+    const int gi = lane % Geo::LPS;  // lane within its slot group
+    const int gs = lane / Geo::LPS;  // slot group: slot = pass * SPP + gs
+    const int myg = gi & (G - 1);    // head of the logits this lane ends with
+    float* pwarp = pw + cw * kDecTile * G;
     for (int u = u_first; u < units && T[u] < g1; ++u) {
       const int ka = max(g0, T[u]) - g0, kb = min(g1, T[u + 1]) - g0;
       if (ka >= kb) continue;  // a unit without tiles (uniform over the consumers)
       const int bl = u / p.H, h = u - bl * p.H;
-      // the group's queries as their bf16 pairs (the scale is applied to the dot
-      // products)
-      const uint32_t* qu =
-          reinterpret_cast<const uint32_t*>(q + ((size_t)bl * p.Hq + (size_t)h * G) * kD);
-      for (int i = ct; i < G * kD / 2; i += kDecConsumers * 32) qs[i] = qu[i];
-      consumers_sync();
+      // this lane's dimensions of the group's queries, as fp32 pairs:
+      // G <= 8: the 16-byte chunks gi + LPS t of the row; G = 16: dims 4 gi .. 4 gi + 3
+      float2 qr[Geo::NPAIR][G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const uint32_t* qg = reinterpret_cast<const uint32_t*>(
+            q + ((size_t)bl * p.Hq + (size_t)h * G + g) * kD);
+#pragma unroll
+        for (int j = 0; j < Geo::NPAIR; ++j) {
+          const int dim = Geo::DPL >= 8 ? 8 * (gi + Geo::LPS * (j / 4)) + 2 * (j % 4)
+                                        : Geo::DPL * gi + 2 * j;
+          const uint32_t w = __ldg(qg + dim / 2);
+          qr[j][g] = make_float2(bf16lo(w), bf16hi(w));
+        }
+      }
       const int slots = counts[u] + tail_slot;
-      float m[G], l[G];
+      float m[G], l_own = 0.f;
       float2 acc[G][2];  // dimensions (4 lane, 4 lane + 1), (4 lane + 2, 4 lane + 3)
 #pragma unroll
       for (int g = 0; g < G; ++g) {
         m[g] = -INFINITY;
-        l[g] = 0.f;
         acc[g][0] = acc[g][1] = make_float2(0.f, 0.f);
       }
-      float* pwarp = pw + cw * kDecTile * G;
       for (int k = ka + ((cw - ka % kDecConsumers) + kDecConsumers) % kDecConsumers; k < kb;
            k += kDecConsumers) {
         const int s = k % kDecStages;
@@ -215,43 +252,70 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
         if (skip) continue;
         const int t = g0 + k - T[u];
         const int cnt = min(kDecTile, slots - t * kDecTile);
-        const bool ok = lane < cnt;
-        // logits: lane = slot; chunk c of the row sits at chunk (c ^ (row & 7))
-        // of its 128-byte box row; even and odd dimensions in the two halves of
-        // a packed f32x2 accumulator
-        const uint8_t* krow = kst + s * kDecKBytes + lane * 128;
-        float2 x2[G];
+        // logits of (slot pass * SPP + gs, head myg); rows past cnt were not
+        // copied and are masked below
+        const uint8_t* kt = kst + s * kDecKBytes;
+        float xl[Geo::NP];
 #pragma unroll
-        for (int g = 0; g < G; ++g) x2[g] = make_float2(0.f, 0.f);
+        for (int ps = 0; ps < Geo::NP; ++ps) {
+          const uint8_t* row = kt + (ps * Geo::SPP + gs) * 256;
+          float2 x2[G];
 #pragma unroll
-        for (int c = 0; c < 16; ++c) {
-          const uint4 raw = *reinterpret_cast<const uint4*>(krow + (c >> 3) * (kDecKBytes / 2) +
-                                                            (((c & 7) ^ (lane & 7)) << 4));
-          const float2 k0 = make_float2(bf16lo(raw.x), bf16hi(raw.x));
-          const float2 k1 = make_float2(bf16lo(raw.y), bf16hi(raw.y));
-          const float2 k2 = make_float2(bf16lo(raw.z), bf16hi(raw.z));
-          const float2 k3 = make_float2(bf16lo(raw.w), bf16hi(raw.w));
+          for (int g = 0; g < G; ++g) x2[g] = make_float2(0.f, 0.f);
+          if constexpr (Geo::DPL >= 8) {
 #pragma unroll
-          for (int g = 0; g < G; ++g) {
-            const uint4 qq = q4[g * (kD / 8) + c];
-            x2[g] = ffma2(make_float2(bf16lo(qq.x), bf16hi(qq.x)), k0, x2[g]);
-            x2[g] = ffma2(make_float2(bf16lo(qq.y), bf16hi(qq.y)), k1, x2[g]);
-            x2[g] = ffma2(make_float2(bf16lo(qq.z), bf16hi(qq.z)), k2, x2[g]);
-            x2[g] = ffma2(make_float2(bf16lo(qq.w), bf16hi(qq.w)), k3, x2[g]);
+            for (int c = 0; c < Geo::DPL / 8; ++c) {
+              const uint4 raw = *reinterpret_cast<const uint4*>(row + (gi + Geo::LPS * c) * 16);
+              const float2 kp[4] = {make_float2(bf16lo(raw.x), bf16hi(raw.x)),
+                                    make_float2(bf16lo(raw.y), bf16hi(raw.y)),
+                                    make_float2(bf16lo(raw.z), bf16hi(raw.z)),
+                                    make_float2(bf16lo(raw.w), bf16hi(raw.w))};
+#pragma unroll
+              for (int e = 0; e < 4; ++e)
+#pragma unroll
+                for (int g = 0; g < G; ++g) x2[g] = ffma2(qr[4 * c + e][g], kp[e], x2[g]);
+            }
+          } else {
+            const uint2 raw = *reinterpret_cast<const uint2*>(row + gi * 8);
+            const float2 kp[2] = {make_float2(bf16lo(raw.x), bf16hi(raw.x)),
+                                  make_float2(bf16lo(raw.y), bf16hi(raw.y))};
+#pragma unroll
+            for (int e = 0; e < 2; ++e)
+#pragma unroll
+              for (int g = 0; g < G; ++g) x2[g] = ffma2(qr[e][g], kp[e], x2[g]);
           }
+          float v[G];
+#pragma unroll
+          for (int g = 0; g < G; ++g) v[g] = x2[g].x + x2[g].y;
+          xl[ps] = reduce_heads<G>(v, lane) * scale_log2;
         }
+        // tile maximum of head myg, then every head's maximum on every lane
+        float tm = -INFINITY;
+#pragma unroll
+        for (int ps = 0; ps < Geo::NP; ++ps)
+          if (ps * Geo::SPP + gs < cnt) tm = fmaxf(tm, xl[ps]);
+#pragma unroll
+        for (int o = Geo::LPS; o < 32; o <<= 1) tm = fmaxf(tm, __shfl_xor_sync(kFull, tm, o));
+        float m_own = 0.f, c_own = 0.f;
 #pragma unroll
         for (int g = 0; g < G; ++g) {
-          const float xv = ok ? (x2[g].x + x2[g].y) * scale_log2 : -INFINITY;
-          const float nm = fmaxf(m[g], warp_max(xv));
+          const float nm = fmaxf(m[g], __shfl_sync(kFull, tm, g));  // lane g holds head g
           const float corr = exp2f(m[g] - nm);
           m[g] = nm;
-          l[g] *= corr;
           acc[g][0] = fmul2(acc[g][0], make_float2(corr, corr));
           acc[g][1] = fmul2(acc[g][1], make_float2(corr, corr));
-          const float pe = ok ? exp2f(xv - nm) : 0.f;
-          l[g] += pe;
-          pwarp[lane * G + g] = pe;
+          if (g == myg) {
+            m_own = nm;
+            c_own = corr;
+          }
+        }
+        l_own *= c_own;
+#pragma unroll
+        for (int ps = 0; ps < Geo::NP; ++ps) {
+          const int slot = ps * Geo::SPP + gs;
+          const float pe = slot < cnt ? exp2f(xl[ps] - m_own) : 0.f;
+          l_own += pe;
+          if (gi < G) pwarp[slot * G + gi] = pe;
         }
         __syncwarp();
         // values: lane = 4 dimensions; only the tile's cnt rows were copied; the
@@ -286,13 +350,14 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(empty0 + 8 * s);
       }
-      // the unit's record for this CTA: combine the consumer warps
+      // the unit's record for this CTA: combine the consumer warps.  The sum of
+      // head g: lanes gi = g of every slot group (lanes gi = g + G repeat them).
+      float lt = gi < G ? l_own : 0.f;
+#pragma unroll
+      for (int o = Geo::LPS; o < 32; o <<= 1) lt += __shfl_xor_sync(kFull, lt, o);
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        float lt = l[g];
-#pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) lt += __shfl_xor_sync(kFull, lt, o);
-        if (lane == 0) {
+        if (lane == g) {
           wm[cw * G + g] = m[g];
           wl[cw * G + g] = lt;
         }
@@ -323,7 +388,7 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
         rec_acc[(rec * G + g) * kD + i] = A;
         if (i == 0) rec_ml[rec * G + g] = make_float2(M, L);
       }
-      consumers_sync();  // wm / wl / wacc and qs are reused by the next unit
+      consumers_sync();  // wm / wl / wacc are reused by the next unit
     }
   }
   __syncthreads();
@@ -491,7 +556,7 @@ int split_blocks() {
 }
 
 template <int G>
-int launch_split(const Prob& p, const CUtensorMap& map_k, const __nv_bfloat16* q,
+int launch_split(const Prob& p, const __nv_bfloat16* q, const __nv_bfloat16* pk,
                  const __nv_bfloat16* pv, const int64_t* offsets, const int32_t* counts,
                  const int32_t* T, int tail_slot, float sl2, float2* ml, float* acc,
                  cudaStream_t st) {
@@ -499,17 +564,14 @@ int launch_split(const Prob& p, const CUtensorMap& map_k, const __nv_bfloat16* q
   if (nb < 1) return 0;
   TraceScope ts_("decode_split", st);
   decode_split_kernel<G><<<nb, kDecThreads, decode_smem_bytes(G), st>>>(
-      map_k, p, q, pv, offsets, counts, T, tail_slot, sl2, ml, acc);
+      p, q, pk, pv, offsets, counts, T, tail_slot, sl2, ml, acc);
   return nb;
 }
 
 // plan + split kernels; returns the number of split CTAs (0: nothing launched)
-int run_splits(const Prob& p, const void* q, const void* pk, const void* pv, int64_t rows,
+int run_splits(const Prob& p, const void* q, const void* pk, const void* pv,
                const int64_t* offsets, const int32_t* counts, int tail_slot, float scale,
                char* ws, cudaStream_t st) {
-  CUtensorMap map_k;
-  if (rows < 1 || rows > INT32_MAX || !make_row_map(&map_k, pk, (uint64_t)rows, kDecTile))
-    return 0;
   const DecodeLayout ly = decode_layout(p);
   int32_t* T = reinterpret_cast<int32_t*>(ws + ly.T);
   float2* ml = reinterpret_cast<float2*>(ws + ly.ml);
@@ -520,13 +582,14 @@ int run_splits(const Prob& p, const void* q, const void* pk, const void* pv, int
   }
   const float sl2 = scale * 1.4426950408889634f;
   const __nv_bfloat16* qb = reinterpret_cast<const __nv_bfloat16*>(q);
+  const __nv_bfloat16* kb = reinterpret_cast<const __nv_bfloat16*>(pk);
   const __nv_bfloat16* vb = reinterpret_cast<const __nv_bfloat16*>(pv);
   switch (p.G) {
-    case 1: return launch_split<1>(p, map_k, qb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
-    case 2: return launch_split<2>(p, map_k, qb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
-    case 4: return launch_split<4>(p, map_k, qb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
-    case 8: return launch_split<8>(p, map_k, qb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
-    case 16: return launch_split<16>(p, map_k, qb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    case 1: return launch_split<1>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    case 2: return launch_split<2>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    case 4: return launch_split<4>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    case 8: return launch_split<8>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    case 16: return launch_split<16>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
     default: return 0;
   }
 }
@@ -534,10 +597,10 @@ int run_splits(const Prob& p, const void* q, const void* pk, const void* pv, int
 
 size_t decode_workspace(const Prob& p) { return decode_layout(p).total; }
 
-bool launch_decode(const Prob& p, const void* q, const void* pk, const void* pv, int64_t rows,
+bool launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
                    const int64_t* offsets, const int32_t* counts, int tail_slot, float scale,
                    void* out, char* ws, cudaStream_t st) {
-  const int nb = run_splits(p, q, pk, pv, rows, offsets, counts, tail_slot, scale, ws, st);
+  const int nb = run_splits(p, q, pk, pv, offsets, counts, tail_slot, scale, ws, st);
   if (nb < 1) return false;
   const DecodeLayout ly = decode_layout(p);
   {
@@ -551,12 +614,12 @@ bool launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
 }
 
 bool launch_decode_certified(const Prob& p, const void* q, const void* pk, const void* pv,
-                             int64_t rows, const int64_t* offsets, const int32_t* counts,
-                             int tail_slot, int clusters, const float* cluster_meta,
-                             const float* kept_vmax, float scale, void* out, float* bound,
-                             int32_t* certified, char* ws, cudaStream_t st) {
+                             const int64_t* offsets, const int32_t* counts, int tail_slot,
+                             int clusters, const float* cluster_meta, const float* kept_vmax,
+                             float scale, void* out, float* bound, int32_t* certified, char* ws,
+                             cudaStream_t st) {
   // the real slots only: the splits see no tail slot
-  const int nb = run_splits(p, q, pk, pv, rows, offsets, counts, 0, scale, ws, st);
+  const int nb = run_splits(p, q, pk, pv, offsets, counts, 0, scale, ws, st);
   if (nb < 1) return false;
   const DecodeLayout ly = decode_layout(p);
   {

@@ -358,10 +358,9 @@ FixedRowLayout fixed_row_layout(const Prob& p) {
 size_t fixed_row_workspace(const Prob& p) { return fixed_row_layout(p).total; }
 
 bool launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V,
-                      const float* scores, int64_t rows, const int64_t* offsets,
-                      const int32_t* counts, const int32_t* positions, const void* pk,
-                      const void* pv, int tail_slot, float scale, float* stats, char* ws,
-                      cudaStream_t st) {
+                      const float* scores, const int64_t* offsets, const int32_t* counts,
+                      const int32_t* positions, const void* pk, const void* pv, int tail_slot,
+                      float scale, float* stats, char* ws, cudaStream_t st) {
   const FixedRowLayout ly = fixed_row_layout(p);
   const size_t words = (size_t)(p.n + 31) / 32;
   uint32_t* mask = reinterpret_cast<uint32_t*>(ws + ly.mask);
@@ -371,7 +370,7 @@ bool launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V
   float* psv = reinterpret_cast<float*>(ws + ly.sv);
   char* ohat = ws + ly.ohat;
   // the compressed decode's output, for its error against O
-  if (!launch_decode(p, q, pk, pv, rows, offsets, counts, tail_slot, scale, ohat, ws + ly.dec, st))
+  if (!launch_decode(p, q, pk, pv, offsets, counts, tail_slot, scale, ohat, ws + ly.dec, st))
     return false;
   cudaMemsetAsync(mask, 0, p.units * words * 4, st);
   {

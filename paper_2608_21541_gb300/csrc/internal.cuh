@@ -85,10 +85,9 @@ void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const
                  double* tail_mass, float* cluster_meta, float* kept_vmax, cudaStream_t st);
 void launch_export_curves(const Prob& p, const Layout& ly, char* ws, int32_t* perm_out,
                           double* c_out, cudaStream_t st);
-// Decode launchers: `rows` = rows of the packed k and v arrays that the
-// kernels may read (the packed capacity; at most INT32_MAX).  False if the
-// K tensor map cannot be built (nothing launched).
-bool launch_decode(const Prob& p, const void* q, const void* pk, const void* pv, int64_t rows,
+// Decode launchers: false if nothing could be launched (the device query of
+// the persistent grid failed).
+bool launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
                    const int64_t* offsets, const int32_t* counts, int tail_slot, float scale,
                    void* out, char* ws, cudaStream_t st);
 size_t decode_workspace(const Prob& p);
@@ -100,15 +99,15 @@ void launch_coverage(const Prob& p, const void* q, const void* K, float scale,
                      int32_t* abs_, float* top, int32_t* order, float* gap, char* ws,
                      cudaStream_t st);
 bool launch_fixed_row(const Prob& p, const void* q, const void* K, const void* V,
-                      const float* scores, int64_t rows, const int64_t* offsets,
-                      const int32_t* counts, const int32_t* positions,
+                      const float* scores, const int64_t* offsets, const int32_t* counts,
+                      const int32_t* positions,
                       const void* pk, const void* pv, int tail_slot, float scale, float* stats,
                       char* ws, cudaStream_t st);
 bool launch_decode_certified(const Prob& p, const void* q, const void* pk, const void* pv,
-                             int64_t rows, const int64_t* offsets, const int32_t* counts,
-                             int tail_slot, int clusters, const float* cluster_meta,
-                             const float* kept_vmax, float scale, void* out, float* bound,
-                             int32_t* certified, char* ws, cudaStream_t st);
+                             const int64_t* offsets, const int32_t* counts, int tail_slot,
+                             int clusters, const float* cluster_meta, const float* kept_vmax,
+                             float scale, void* out, float* bound, int32_t* certified, char* ws,
+                             cudaStream_t st);
 
 // ---- optional kernel timing (off by default) ------------------------------
 // When enabled with certkv_trace_enable(), every kernel launch is bracketed

@@ -41,7 +41,6 @@ extern "C" int certkv_decode_attn_noalloc(const certkv_shape* shape, const void*
     return CERTKV_EINVAL;
   if (((uintptr_t)packed->k | (uintptr_t)packed->v | (uintptr_t)q) % 16 != 0) return CERTKV_EINVAL;
   if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
-  if (packed->capacity_slots < 1 || packed->capacity_slots > INT32_MAX) return CERTKV_EINVAL;
   if (!(scale >= 0.0f) || scale > 3.0e38f) return CERTKV_EINVAL;
 
   Prob p = {};
@@ -70,8 +69,8 @@ extern "C" int certkv_decode_attn_noalloc(const certkv_shape* shape, const void*
     scratch = g_scratch_ptr[dev];
   }
   const float sc = scale > 0.0f ? scale : 0.08838834764831845f;  // 1/sqrt(128)
-  if (!launch_decode(p, q, packed->k, packed->v, packed->capacity_slots, packed->offsets,
-                     packed->real_counts, tail_slot, sc, out, reinterpret_cast<char*>(scratch),
+  if (!launch_decode(p, q, packed->k, packed->v, packed->offsets, packed->real_counts, tail_slot,
+                     sc, out, reinterpret_cast<char*>(scratch),
                      reinterpret_cast<cudaStream_t>(stream)))
     return CERTKV_ECUDA;
   return cudaGetLastError() == cudaSuccess ? CERTKV_OK : CERTKV_ECUDA;
