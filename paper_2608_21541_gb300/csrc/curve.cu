@@ -77,7 +77,7 @@ __device__ __forceinline__ void cp_async_commit() {
 }
 
 constexpr int kEvalGroup = 8;                  // V rows per staged group
-constexpr int kEvalAhead = 3;                  // groups in flight ahead of the one in use
+constexpr int kEvalAhead = 2;                  // groups in flight ahead of the one in use
 constexpr int kEvalRing = kEvalAhead + 1;
 constexpr int kEvalGroupBytes = kEvalGroup * kD * 2;
 
