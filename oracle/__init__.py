@@ -69,6 +69,8 @@ def _bind(lib):
     lib.oracle_future_query_lift.restype = None
     lib.oracle_coverage_profile.argtypes = [P, P, I, I, D, P, I, P, I, P, I, P, P, P, P, P, P]
     lib.oracle_coverage_profile.restype = None
+    lib.oracle_sampled_compensation.argtypes = [P, P, P, P, I, I, D, I, P, P, P, P]
+    lib.oracle_sampled_compensation.restype = None
     lib.oracle_compress.restype = I
     lib.oracle_decode.argtypes = [P, D, P, P, P, P, P, I, P]
     lib.oracle_decode.restype = None
@@ -343,6 +345,28 @@ def coverage_profile(q, K, *, scale: float, eta=(0.1,), rel_eps=(0.1,), abs_eps=
         _ptr(top))
     return dict(order=order, gap=gap, K_eta=K_eta[:len(eta)], rel=rel[:len(rel_eps)],
                 abs=ab[:len(abs_eps)], top=top)
+
+
+def sampled_compensation(q, K, V, kept, u, *, scale: float, m: int, forced_idx=None,
+                         lib=None):
+    """Sampled tail compensation of one query row (see
+    oracle_sampled_compensation): q uint16 [d], K, V uint16 [n][d], kept bool
+    [n], u float32 [2m] uniforms in [0, 1), forced_idx int32 [2m] or None.
+    Returns (idx int32 [2m], stats [8])."""
+    q = _u16(q); K = _u16(K); V = _u16(V)
+    n, d = K.shape
+    kept = np.ascontiguousarray(kept, dtype=np.uint8)
+    if (~kept.astype(bool)).sum() < m:
+        raise ValueError("m exceeds the tail")
+    u = np.ascontiguousarray(u, dtype=np.float32)
+    assert u.shape == (2 * m,)
+    f = None if forced_idx is None else np.ascontiguousarray(forced_idx, dtype=np.int32)
+    idx = np.zeros(2 * m, np.int32)
+    st = np.zeros(8)
+    (lib or _load()).oracle_sampled_compensation(
+        _ptr(q), _ptr(K), _ptr(V), _ptr(kept), n, d, float(scale), int(m), _ptr(u),
+        _ptr(f) if f is not None else None, _ptr(idx), _ptr(st))
+    return idx, st
 
 
 def decode(q, pk, pv, offsets, counts, *, B: int, L: int, Hq: int, H: int, d: int,

@@ -944,3 +944,127 @@ void oracle_future_query_lift(const uint16_t* q, const uint16_t* K, const uint16
   free(mix);
   free(z);
 }
+
+/*
+ * Sampled tail compensation (appendix: proposition on sampled tail
+ * compensation) for one realized query row over all n original tokens of a
+ * unit.  A = softmax(scale <q, k_j>), S = tokens with kept[j] != 0, T the
+ * others (|T| = N >= 1), p_S = A(S), u* = sum_T A_j v_j, Q_T = sum_T A_j^2.
+ * Two estimators of u* from m tail tokens, with the 2m uniforms u[0..2m-1] in
+ * [0, 1) as the only randomness:
+ *   weight-proportional: for r < m, j_r = the first tail token (in index
+ *     order) whose cumulative tail weight exceeds u[r] * A(T);
+ *     u_w = (1 - p_S)/m sum_r v_{j_r}
+ *   uniform m-subset (Floyd's algorithm, m <= N): for i = N - m .. N - 1,
+ *     t = floor(u[m + i - (N - m)] * (i + 1)); take tail rank t unless already
+ *     taken, else rank i; u_u = (1 - p_S)/m sum over the subset of v_j
+ *     (tail rank t = the t-th tail token in index order)
+ * forced_idx (2m token indices, or NULL) replaces both draws.  Writes the
+ * sampled token indices to idx[2m] and stats[8]:
+ *   0 p_S   1 Q_T   2 ||u*||   3 ||u_w - u*||   4 ||u_u - u*||
+ *   5 sqrt(d s2 (1 - p_S)^2 / m (1 - Q_T / (1 - p_S)^2))       (part (i))
+ *   6 sqrt(d s2 (1 - p_S)^2 (1/m - 2/N + Q_T / (1 - p_S)^2))  (part (ii))
+ *   7 s2 = sum_T ||v_j - vbar_T||^2 / (d N), the per-coordinate variance of
+ *     the tail values (unweighted mean vbar_T), which stands for sigma_V^2
+ */
+void oracle_sampled_compensation(const uint16_t* q, const uint16_t* K, const uint16_t* V,
+                                 const uint8_t* kept, int n, int d, double scale, int m,
+                                 const float* u, const int32_t* forced_idx, int32_t* idx,
+                                 double* stats) {
+  double* w = (double*)malloc((size_t)n * sizeof(double));
+  int32_t* tail = (int32_t*)malloc((size_t)n * sizeof(int32_t));
+  double* ustar = (double*)calloc((size_t)d, sizeof(double));
+  double* uw = (double*)calloc((size_t)d, sizeof(double));
+  double* uu = (double*)calloc((size_t)d, sizeof(double));
+  double* vbar = (double*)calloc((size_t)d, sizeof(double));
+  double zmax = -INFINITY;
+  for (int j = 0; j < n; ++j) {
+    double dot = 0.0;
+    for (int i = 0; i < d; ++i) dot += bf16_to_f64(q[i]) * bf16_to_f64(K[(size_t)j * d + i]);
+    w[j] = scale * dot;
+    if (w[j] > zmax) zmax = w[j];
+  }
+  double Z = 0.0;
+  for (int j = 0; j < n; ++j) {
+    w[j] = exp(w[j] - zmax);
+    Z += w[j];
+  }
+  int N = 0;
+  double pT = 0.0, QT = 0.0;
+  for (int j = 0; j < n; ++j) {
+    w[j] /= Z; /* A_j */
+    if (!kept[j]) {
+      tail[N++] = j;
+      pT += w[j];
+      QT += w[j] * w[j];
+      for (int i = 0; i < d; ++i) {
+        const double v = bf16_to_f64(V[(size_t)j * d + i]);
+        ustar[i] += w[j] * v;
+        vbar[i] += v;
+      }
+    }
+  }
+  const double pS = 1.0 - pT;
+  /* weight-proportional draws by the inverse of the cumulative tail weight */
+  for (int r = 0; r < m; ++r) {
+    if (forced_idx) {
+      idx[r] = forced_idx[r];
+      continue;
+    }
+    const double target = (double)u[r] * pT;
+    double c = 0.0;
+    int pick = tail[N - 1];
+    for (int t = 0; t < N; ++t) {
+      c += w[tail[t]];
+      if (c > target) { pick = tail[t]; break; }
+    }
+    idx[r] = pick;
+  }
+  /* uniform m-subset of the tail ranks, Floyd's algorithm */
+  for (int s = 0; s < m; ++s) {
+    if (forced_idx) {
+      idx[m + s] = forced_idx[m + s];
+      continue;
+    }
+    const int i = N - m + s;
+    int t = (int)floor((double)u[m + s] * (double)(i + 1));
+    if (t > i) t = i;
+    int taken = 0;
+    for (int e = 0; e < s; ++e)
+      if (idx[m + e] == tail[t]) taken = 1;
+    idx[m + s] = taken ? tail[i] : tail[t];
+  }
+  for (int r = 0; r < m; ++r)
+    for (int i = 0; i < d; ++i) {
+      uw[i] += bf16_to_f64(V[(size_t)idx[r] * d + i]);
+      uu[i] += bf16_to_f64(V[(size_t)idx[m + r] * d + i]);
+    }
+  double nu = 0.0, ew = 0.0, eu = 0.0, var = 0.0;
+  for (int i = 0; i < d; ++i) {
+    vbar[i] /= N;
+    uw[i] *= (1.0 - pS) / m;
+    uu[i] *= (1.0 - pS) / m;
+    nu += ustar[i] * ustar[i];
+    ew += (uw[i] - ustar[i]) * (uw[i] - ustar[i]);
+    eu += (uu[i] - ustar[i]) * (uu[i] - ustar[i]);
+  }
+  for (int t = 0; t < N; ++t)
+    for (int i = 0; i < d; ++i) {
+      const double e = bf16_to_f64(V[(size_t)tail[t] * d + i]) - vbar[i];
+      var += e * e;
+    }
+  const double s2 = var / ((double)d * N);
+  const double omp2 = (1.0 - pS) * (1.0 - pS);
+  const double imb = omp2 > 0.0 ? QT / omp2 : 0.0;
+  const double mse_w = d * s2 * omp2 / m * (1.0 - imb);
+  const double mse_u = d * s2 * omp2 * (1.0 / m - 2.0 / N + imb);
+  stats[0] = pS;
+  stats[1] = QT;
+  stats[2] = sqrt(nu);
+  stats[3] = sqrt(ew);
+  stats[4] = sqrt(eu);
+  stats[5] = sqrt(mse_w > 0.0 ? mse_w : 0.0);
+  stats[6] = sqrt(mse_u > 0.0 ? mse_u : 0.0);
+  stats[7] = s2;
+  free(w); free(tail); free(ustar); free(uw); free(uu); free(vbar);
+}

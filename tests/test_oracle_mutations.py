@@ -56,6 +56,10 @@ MUTANTS = {
     "coverage_relative_count_absolute": ("> rel_eps[e] * A1", "> rel_eps[e]"),
     "coverage_calibrated_count_unnormalised": ("if (exp(t[r].a - z1) / Z > abs_eps[e])",
                                                "if (exp(t[r].a - z1) > abs_eps[e])"),
+    "sampled_draws_ignore_weights": ("      c += w[tail[t]];", "      c += pT / N;"),
+    "sampled_estimate_without_tail_mass": ("    uw[i] *= (1.0 - pS) / m;", "    uw[i] *= 1.0 / m;"),
+    "sampled_subset_repeats": ("    idx[m + s] = taken ? tail[i] : tail[t];", "    idx[m + s] = tail[t];"),
+    "sampled_qt_is_mass": ("      QT += w[j] * w[j];", "      QT += w[j];"),
     "bisection_inverted": ("if (total > B_real) lam_lo = lam; else lam_hi = lam;",
                            "if (total > B_real) lam_hi = lam; else lam_lo = lam;"),
     "kept_not_sorted": ("qsort(kept, (size_t)b, sizeof(int32_t), cmp_int32);", ""),
