@@ -289,6 +289,34 @@ int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void*
                            int32_t tail_slot, float* stats, void* workspace,
                            size_t workspace_bytes, void* stream);
 
+/* Sampled tail compensation (an evaluation tool over the full K and V; appendix:
+ * proposition on sampled tail compensation).  For every query head qh of unit
+ * u with its decode query q, the realized softmax row A over all n original
+ * tokens, S = the real tokens kept in `packed` and T the N evicted ones, the
+ * fixed-row correction u* = sum_T A_j v_j is estimated from m tail tokens:
+ *   weight-proportional: token j_r (r < m) is the first evicted token, in
+ *     index order, whose cumulative tail weight exceeds unif[r] * A(T) (the
+ *     cumulative weight summed in float64); u_w = (1 - p_S)/m sum_r v_{j_r}
+ *   uniform subset: Floyd's algorithm over the tail ranks, for i = N - m .. N - 1
+ *     rank floor(unif[m + i - N + m] * (i + 1)) unless already taken, else i
+ *     (float64 products); u_u = (1 - p_S)/m sum of the subset's values.
+ * unif: fp32 [B][L][Hq][2m] uniforms in [0, 1) (device); idx_out: int32
+ * [B][L][Hq][2m] the drawn token indices (may be NULL); stats fp32
+ * [B][L][Hq][8]: 0 p_S, 1 Q_T = sum_T A_j^2, 2 ||u*||, 3 ||u_w - u*||,
+ * 4 ||u_u - u*||, 5 the proposition's root-mean-square error of u_w,
+ * sqrt(d s2 (1 - p_S)^2/m (1 - Q_T/(1 - p_S)^2)), 6 that of u_u,
+ * sqrt(d s2 (1 - p_S)^2 (1/m - 2/N + Q_T/(1 - p_S)^2)), 7 s2 = the evicted
+ * values' per-coordinate variance (standing for sigma_V^2).  1 <= m <=
+ * CERTKV_MAX_SAMPLES; a head with fewer than m evicted tokens gets NaN stats
+ * and -1 indices.  q bf16 [B][L][Hq][d]; K, V as for certkv_compress;
+ * workspace: certkv_sampled_workspace_bytes(shape). */
+#define CERTKV_MAX_SAMPLES 64
+size_t certkv_sampled_workspace_bytes(const certkv_shape* shape);
+int certkv_sampled_compensation(const certkv_shape* shape, const void* q, const void* K,
+                                const void* V, const certkv_packed* packed, float scale,
+                                int32_t m, const float* unif, int32_t* idx_out, float* stats,
+                                void* workspace, size_t workspace_bytes, void* stream);
+
 /* Coverage profile of realized query rows (an evaluation instrument: §3,
  * "count sparsity does not imply coverage sparsity", with the ranked gap
  * profile G(j) = z_(1) - z_(j) and the coverage budget K_eta; the appendix's

@@ -53,7 +53,8 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_trace_report", "certkv_decode_attn_noalloc", "certkv_host_workspace_bytes",
             "certkv_compress_host", "certkv_decode_certified", "certkv_fixed_row_workspace_bytes",
             "certkv_fixed_row_stats", "certkv_coverage_workspace_bytes",
-            "certkv_coverage_profile")
+            "certkv_coverage_profile", "certkv_sampled_workspace_bytes",
+            "certkv_sampled_compensation")
 
 _lock = threading.Lock()
 _lib = None
@@ -123,6 +124,11 @@ def load_library(path: Optional[str] = None):
         lib.certkv_coverage_profile.argtypes = [sp, P, P, ctypes.c_float, P, I32, P, I32, P, I32,
                                                 P, P, P, P, P, P, P, SZ, P]
         lib.certkv_coverage_profile.restype = ctypes.c_int
+        lib.certkv_sampled_workspace_bytes.argtypes = [sp]
+        lib.certkv_sampled_workspace_bytes.restype = SZ
+        lib.certkv_sampled_compensation.argtypes = [sp, P, P, P, kp, ctypes.c_float, I32, P, P, P,
+                                                    P, SZ, P]
+        lib.certkv_sampled_compensation.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -466,6 +472,35 @@ def certkv_coverage_profile(q, K, *, eta=(0.1,), rel_eps=(0.1,), abs_eps=(), sca
         _ptr(order), _ptr(gap), _ptr(ws), ws.numel(), _stream(stream))
     _check(rc, "certkv_coverage_profile")
     return dict(K_eta=K_eta, rel=rel, abs=ab, top=top, order=order, gap=gap)
+
+
+SAMPLED_FIELDS = ("kept_mass", "q_tail", "norm_correction", "err_weighted", "err_uniform",
+                  "rmse_weighted", "rmse_uniform", "tail_value_variance")
+
+
+def certkv_sampled_compensation(q, K, V, packed: Packed, unif, m: int, *, scale: float = 0.0,
+                                stats=None, idx=None, ws=None, stream=None):
+    """Sampled tail compensation per query head (evaluation tool; reads the full
+    K and V): unif fp32 [B][L][Hq][2m] uniforms in [0, 1).  Returns (stats fp32
+    [B][L][Hq][8] in the order of SAMPLED_FIELDS, idx int32 [B][L][Hq][2m])."""
+    _bf16(q, "q"); _bf16(K, "K"); _bf16(V, "V")
+    B, L, Hq, d = q.shape
+    shape = certkv_shape(B, L, Hq, K.shape[2], K.shape[3], d, 1)
+    if unif.dtype != torch.float32 or not unif.is_contiguous() or unif.numel() != B * L * Hq * 2 * m:
+        raise ValueError("unif must be contiguous fp32 [B][L][Hq][2m]")
+    if stats is None:
+        stats = torch.empty((B, L, Hq, 8), dtype=torch.float32, device=q.device)
+    if idx is None:
+        idx = torch.empty((B, L, Hq, 2 * m), dtype=torch.int32, device=q.device)
+    if ws is None:
+        ws = workspace(int(load_library().certkv_sampled_workspace_bytes(ctypes.byref(shape))),
+                       q.device)
+    st = packed.struct()
+    rc = load_library().certkv_sampled_compensation(
+        ctypes.byref(shape), _ptr(q), _ptr(K), _ptr(V), ctypes.byref(st), float(scale), int(m),
+        _ptr(unif), _ptr(idx), _ptr(stats), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "certkv_sampled_compensation")
+    return stats, idx
 
 
 def certkv_read_status(ws: torch.Tensor, stream=None) -> int:

@@ -528,6 +528,39 @@ int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void*
   return cuda_ok(cudaGetLastError());
 }
 
+size_t certkv_sampled_workspace_bytes(const certkv_shape* shape) {
+  certkv_params prm;
+  certkv_default_params(&prm);
+  Prob p;
+  if (make_prob(shape, &prm, -1, &p)) return 0;
+  return sampled_workspace(p);
+}
+
+int certkv_sampled_compensation(const certkv_shape* shape, const void* q, const void* K,
+                                const void* V, const certkv_packed* packed, float scale,
+                                int32_t m, const float* unif, int32_t* idx_out, float* stats,
+                                void* workspace, size_t workspace_bytes, void* stream) {
+  certkv_params prm;
+  certkv_default_params(&prm);
+  Prob p;
+  int rc = make_prob(shape, &prm, -1, &p);
+  if (rc) return rc;
+  if (!q || !K || !V || !packed || !packed->offsets || !packed->real_counts ||
+      !packed->positions || !unif || !stats)
+    return CERTKV_EINVAL;
+  if (!aligned(q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(unif, 4)) return CERTKV_EINVAL;
+  if (m < 1 || m > CERTKV_MAX_SAMPLES) return CERTKV_EINVAL;
+  if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < sampled_workspace(p))
+    return CERTKV_EWORKSPACE;
+  const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
+  if (!launch_sampled(p, q, K, V, packed->offsets, packed->real_counts, packed->positions, m, unif,
+                      idx_out, sc, stats, reinterpret_cast<char*>(workspace),
+                      reinterpret_cast<cudaStream_t>(stream)))
+    return CERTKV_EINVAL;
+  return cuda_ok(cudaGetLastError());
+}
+
 size_t certkv_coverage_workspace_bytes(const certkv_shape* shape) {
   certkv_params prm;
   certkv_default_params(&prm);

@@ -93,6 +93,11 @@ bool launch_decode(const Prob& p, const void* q, const void* pk, const void* pv,
 size_t decode_workspace(const Prob& p);
 size_t fixed_row_workspace(const Prob& p);
 size_t coverage_workspace(const Prob& p);
+size_t sampled_workspace(const Prob& p);
+bool launch_sampled(const Prob& p, const void* q, const void* K, const void* V,
+                    const int64_t* offsets, const int32_t* counts, const int32_t* positions,
+                    int m, const float* unif, int32_t* idx_out, float scale, float* stats,
+                    char* ws, cudaStream_t st);
 void launch_coverage(const Prob& p, const void* q, const void* K, float scale,
                      const double* eta, int n_eta, const double* rel_eps, int n_rel,
                      const double* abs_eps, int n_abs, int32_t* K_eta, int32_t* rel,

@@ -170,3 +170,24 @@ def test_coverage_profile_validation(lib):
     assert lib.certkv_coverage_profile(
         ctypes.byref(s), fake, fake, 0.0, None, 0, None, 0, None, 0, None, None, None, fake,
         None, None, None, need, None) == ck.EWORKSPACE
+
+
+def test_sampled_compensation_validation(lib):
+    s = shape()
+    need = lib.certkv_sampled_workspace_bytes(ctypes.byref(s))
+    assert need > lib.certkv_fixed_row_workspace_bytes(ctypes.byref(s))
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
+    packed = ck.certkv_packed(fake, fake, fake, fake, fake, 1 << 40, None, None)
+
+    def call(m=4, unif=fake, ws=256, ws_bytes=None, scale=0.0):
+        return lib.certkv_sampled_compensation(ctypes.byref(s), fake, fake, fake,
+                                               ctypes.byref(packed), scale, m, unif, None, fake,
+                                               ctypes.c_void_p(ws) if ws else None,
+                                               need if ws_bytes is None else ws_bytes, None)
+
+    assert call(m=0) == ck.EINVAL
+    assert call(m=65) == ck.EINVAL  # at most CERTKV_MAX_SAMPLES
+    assert call(unif=None) == ck.EINVAL
+    assert call(scale=float("nan")) == ck.EINVAL
+    assert call(ws=0) == ck.EWORKSPACE
+    assert call(ws_bytes=need - 1) == ck.EWORKSPACE
