@@ -149,8 +149,33 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   const int b0 = p.b_min + seg * kHullSeg;
   const int b1 = min(n, b0 + kHullSeg);
   const Shear sh = make_shear(cu, b0, b1 - 1);
-  int32_t st[kHullSeg];  // thread-private (L1-resident) chain stack
-  const int top = tolerant_chain(sh, b1 - b0, [&](int i) { return b0 + i; }, st);
+  // the tolerant chain of tolerant_chain, with the sheared values of eight
+  // consecutive points evaluated ahead (their curve loads in flight together)
+  // and kept on the thread-private stack next to b, so that a pop needs no
+  // reload
+  int32_t st[kHullSeg];
+  float sty[kHullSeg], std_[kHullSeg];
+  int top = 0;
+  const int count = b1 - b0;
+  for (int i0 = 0; i0 < count; i0 += 8) {
+    float yv[8], dv[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (i0 + k < count) sh.at(b0 + i0 + k, yv[k], dv[k]);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (i0 + k >= count) break;
+      const int b = b0 + i0 + k;
+      while (top >= 2 && clearly_above(st[top - 2], sty[top - 2], st[top - 1], sty[top - 1], b,
+                                       yv[k],
+                                       fmaxf(fmaxf(std_[top - 2], std_[top - 1]), dv[k])))
+        --top;
+      st[top] = b;
+      sty[top] = yv[k];
+      std_[top] = dv[k];
+      ++top;
+    }
+  }
   for (int i = 0; i < top; ++i) out[i] = st[i];
   ncand[(size_t)u * ncand_stride(p) + seg] = top;
 }

@@ -14,6 +14,7 @@
 #include "../../include/certkv.h"
 #include "common.cuh"
 #include "internal.cuh"
+#include "headlogits.cuh"
 
 namespace certkv {
 
@@ -33,48 +34,34 @@ __device__ __forceinline__ float key_logit(uint32_t key) {
   return __uint_as_float((ord & 0x80000000u) ? (ord & 0x7fffffffu) : ~ord);
 }
 
-// grid = (units, kCovSplits), block = 128: lane = token; the G query heads of
-// the unit's group share each K row.  keys/vals [u * G + g][n].
+// grid = (units, kCovSplits), block = 128: each warp takes 32-token tiles; the
+// G query heads of the unit's group are dotted with each K row by 2G lanes
+// (coalesced), then lane = token writes its keys.  keys/vals [u * G + g][n].
 template <int G>
 __global__ void __launch_bounds__(128) coverage_logits_kernel(
     Prob p, const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ K,
     float scale, uint32_t* __restrict__ keys, int32_t* __restrict__ vals) {
-  __shared__ __align__(16) float qs[G][kD];
+  __shared__ float xs[4][32 * G];
   const int u = blockIdx.x, split = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bl = u / p.H, h = u - bl * p.H;
   const int n = p.n;
-  const __nv_bfloat16* qu = q + ((size_t)bl * p.Hq + (size_t)h * G) * kD;
-  for (int i = threadIdx.x; i < G * kD; i += blockDim.x)
-    (&qs[0][0])[i] = __bfloat162float(qu[i]);
-  __syncthreads();
-  const uint4* Ku = reinterpret_cast<const uint4*>(K + (size_t)u * n * kD);
+  float2 qr[DecGeo<G>::NPAIR][G];
+  load_query_slice<G>(q + ((size_t)bl * p.Hq + (size_t)h * G) * kD, lane, qr);
+  const __nv_bfloat16* Ku = K + (size_t)u * n * kD;
   const int ntiles = (n + 31) / 32;
   for (int t = split * 4 + warp; t < ntiles; t += kCovSplits * 4) {
+    tile_head_logits<G>(Ku + (size_t)t * 32 * kD, min(32, n - t * 32), qr, lane, xs[warp]);
     const int j = t * 32 + lane;
-    if (j >= n) continue;
-    uint4 krow[16];
+    if (j < n) {
 #pragma unroll
-    for (int c = 0; c < 16; ++c) krow[c] = __ldg(Ku + (size_t)j * 16 + c);
-    float x[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) x[g] = 0.f;
-#pragma unroll
-    for (int c = 0; c < 16; ++c) {
-      const uint4 raw = krow[c];
-      const float kf[8] = {bf16lo(raw.x), bf16hi(raw.x), bf16lo(raw.y), bf16hi(raw.y),
-                           bf16lo(raw.z), bf16hi(raw.z), bf16lo(raw.w), bf16hi(raw.w)};
-#pragma unroll
-      for (int g = 0; g < G; ++g)
-#pragma unroll
-        for (int e = 0; e < 8; ++e) x[g] = fmaf(qs[g][c * 8 + e], kf[e], x[g]);
+      for (int g = 0; g < G; ++g) {
+        const size_t o = ((size_t)u * G + g) * n + j;
+        keys[o] = desc_key(xs[warp][lane * G + g] * scale);
+        vals[o] = j;
+      }
     }
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const size_t o = ((size_t)u * G + g) * n + j;
-      keys[o] = desc_key(x[g] * scale);
-      vals[o] = j;
-    }
+    __syncwarp();  // xs is rewritten by the next tile
   }
 }
 

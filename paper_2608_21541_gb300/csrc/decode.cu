@@ -24,6 +24,7 @@
 #include "common.cuh"
 #include "internal.cuh"
 #include "tma.cuh"
+#include "headlogits.cuh"
 
 namespace certkv {
 
@@ -96,36 +97,6 @@ __global__ void __launch_bounds__(1024) decode_plan_kernel(int units,
 
 __device__ __forceinline__ void consumers_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(kDecConsumers * 32) : "memory");
-}
-
-// Lane geometry of the logits for G query heads: 2G lanes share one slot, each
-// holding 128 / 2G of the G queries' dimensions in registers, so every K row
-// is read once, coalesced, and a transposing shuffle reduction leaves lane i of
-// the slot's group with the logit of head i mod G.
-template <int G>
-struct DecGeo {
-  static constexpr int LPS = 2 * G;           // lanes per slot
-  static constexpr int SPP = 32 / LPS;        // slots per pass
-  static constexpr int NP = kDecTile / SPP;   // passes per tile
-  static constexpr int DPL = kD / LPS;        // dimensions per lane
-  static constexpr int NPAIR = DPL / 2;       // fp32 pairs per lane and head
-};
-
-// v[h]: this lane's partial dot product for head h.  Returns the full dot
-// product of head (lane mod G) over the 2G lanes of the slot group.
-template <int G>
-__device__ __forceinline__ float reduce_heads(float (&v)[G], int lane) {
-#pragma unroll
-  for (int o = G / 2; o >= 1; o >>= 1) {
-    const bool upper = (lane & o) != 0;
-#pragma unroll
-    for (int k = 0; k < o; ++k) {
-      const float keep = upper ? v[k + o] : v[k];
-      const float send = upper ? v[k] : v[k + o];
-      v[k] = keep + __shfl_xor_sync(kFull, send, o);
-    }
-  }
-  return v[0] + __shfl_xor_sync(kFull, v[0], G);
 }
 
 // grid = NB persistent CTAs, block = kDecThreads.  CTA b takes the global
@@ -221,18 +192,7 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
       // this lane's dimensions of the group's queries, as fp32 pairs:
       // G <= 8: the 16-byte chunks gi + LPS t of the row; G = 16: dims 4 gi .. 4 gi + 3
       float2 qr[Geo::NPAIR][G];
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        const uint32_t* qg = reinterpret_cast<const uint32_t*>(
-            q + ((size_t)bl * p.Hq + (size_t)h * G + g) * kD);
-#pragma unroll
-        for (int j = 0; j < Geo::NPAIR; ++j) {
-          const int dim = Geo::DPL >= 8 ? 8 * (gi + Geo::LPS * (j / 4)) + 2 * (j % 4)
-                                        : Geo::DPL * gi + 2 * j;
-          const uint32_t w = __ldg(qg + dim / 2);
-          qr[j][g] = make_float2(bf16lo(w), bf16hi(w));
-        }
-      }
+      load_query_slice<G>(q + ((size_t)bl * p.Hq + (size_t)h * G) * kD, lane, qr);
       const int slots = counts[u] + tail_slot;
       float m[G], l_own = 0.f;
       float2 acc[G][2];  // dimensions (4 lane, 4 lane + 1), (4 lane + 2, 4 lane + 3)
