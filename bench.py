@@ -42,6 +42,9 @@ def parse():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: compress this many layers instead of the workload's")
+    ap.add_argument("--decode-steps", type=int, default=1,
+                    help="decode steps per step after the compression, each with fresh queries "
+                         "(the C4 configuration decodes 256)")
     return ap.parse_args()
 
 
@@ -125,7 +128,7 @@ def kernel_work(wl, B_live, name):
     if name == "curve_eval":
         return dict(bytes=kbytes, flops=0)           # V rows gathered again
     if name == "sort_scatter":
-        return dict(bytes=U * n * 16, flops=0)       # key + value in and out
+        return dict(bytes=U * n * 16, flops=0)       # one digit pass: key + value in and out
     if name == "copy_rows":
         slots = wl.B * wl.L * (B_live - wl.H)
         return dict(bytes=slots * d * 2 * 2 * 2, flops=0)
@@ -252,7 +255,9 @@ def run_ours(args, wl, rank, world):
     peaks = load_peaks()
     B_live = wl.B_live
     K, V, Q = W.draw(wl, seed=args.seed + rank, device=dev)
-    q = W.draw_decode_queries(wl, 0, seed=args.seed + rank, device=dev)
+    nd = max(1, args.decode_steps)
+    qs = [W.draw_decode_queries(wl, i, seed=args.seed + rank, device=dev) for i in range(nd)]
+    q = qs[0]
     params = ck.certkv_default_params()
     shape = ck.shape_of(K, Q)
     ws = ck.workspace(ck.certkv_workspace_bytes(shape, params), dev)
@@ -264,7 +269,8 @@ def run_ours(args, wl, rank, world):
 
     def step():
         ck.certkv_compress(K, V, Q, B_live, params, out=packed, ws=ws, stream=stream)
-        ck.certkv_decode_attn(q, packed, hkv=wl.H, out=out, ws=dws, stream=stream)
+        for qi in qs:
+            ck.certkv_decode_attn(qi, packed, hkv=wl.H, out=out, ws=dws, stream=stream)
 
     for _ in range(args.warmup):
         step()
@@ -311,15 +317,14 @@ def run_ours(args, wl, rank, world):
         if work:
             per_launch_ms = trace[name][1] / trace[name][0]
             launches_per_step = trace[name][0] / args.steps
-            w1 = {k: v / launches_per_step for k, v in work.items()}
-            roof_all[name] = roofline_for(name, w1, per_launch_ms, peaks,
+            roof_all[name] = roofline_for(name, work, per_launch_ms, peaks,
                                           measured_traffic(name, wl, launches_per_step))
     dominant = next(iter(kernels))
     roof = roof_all.get(dominant) or next(iter(roof_all.values()))
 
     decode_ms = kernels.get("decode_split", {}).get("ms_per_step", 0) + \
         kernels.get("decode_merge", {}).get("ms_per_step", 0)
-    decode_bytes = wl.B * wl.L * B_live * wl.d * 2 * 2
+    decode_bytes = nd * wl.B * wl.L * B_live * wl.d * 2 * 2  # per step, all decode steps
     compress_ms = ms - decode_ms
     roof_bytes = wl.B * wl.L * (wl.H * wl.n * wl.d * 2 * 2 + B_live * wl.d * 2 * 2)
 
@@ -327,7 +332,7 @@ def run_ours(args, wl, rank, world):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": config_dict(wl, B_live),
+        "config": dict(config_dict(wl, B_live), decode_steps=nd),
         "compress_ms": compress_ms,
         "compress_hbm_roofline": {
             "bytes": roof_bytes, "achieved_GBps": round(roof_bytes / (compress_ms / 1e3) / 1e9, 1),
@@ -341,7 +346,7 @@ def run_ours(args, wl, rank, world):
     }
 
     if not args.no_e2e:
-        line["e2e"] = run_e2e(args, wl, K, V, Q, q, params, ws, dws, dev, stream, world, B_live)
+        line["e2e"] = run_e2e(args, wl, K, V, Q, qs, params, ws, dws, dev, stream, world, B_live)
     del K, V, Q
     torch.cuda.empty_cache()
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -356,7 +361,7 @@ def run_ours(args, wl, rank, world):
         print(json.dumps(line), flush=True)
 
 
-def run_e2e(args, wl, K, V, Q, q, params, ws, dws, dev, stream, world, B_live):
+def run_e2e(args, wl, K, V, Q, qs, params, ws, dws, dev, stream, world, B_live):
     """Same metric through the public API with host buffers: pinned host ->
     device copies of the step's inputs, compress, decode, and the packed cache
     and decode output copied back, all inside the timed region."""
@@ -366,8 +371,9 @@ def run_e2e(args, wl, K, V, Q, q, params, ws, dws, dev, stream, world, B_live):
     hK = K.cpu().pin_memory()
     hV = V.cpu().pin_memory()
     hQ = Q.cpu().pin_memory()
-    hq = q.cpu().pin_memory()
-    dq = torch.empty_like(q)
+    q = qs[0]
+    hq = torch.stack(qs).cpu().pin_memory()  # the step's decode queries
+    dq = torch.empty_like(hq, device=dev)
     packed = ck.Packed.empty(wl.B, wl.L, wl.H, wl.d, B_live, dev)
     out = torch.empty_like(q)
     host_out = dict(k=torch.empty(packed.k.shape, dtype=torch.bfloat16, pin_memory=True),
@@ -385,7 +391,8 @@ def run_e2e(args, wl, K, V, Q, q, params, ws, dws, dev, stream, world, B_live):
     def step():
         ck.certkv_compress_host(hK, hV, hQ, B_live, params, out=packed, ws=hws, stream=stream)
         dq.copy_(hq, non_blocking=True)
-        ck.certkv_decode_attn(dq, packed, hkv=wl.H, out=out, ws=dws, stream=stream)
+        for i in range(dq.shape[0]):
+            ck.certkv_decode_attn(dq[i], packed, hkv=wl.H, out=out, ws=dws, stream=stream)
         host_out["k"].copy_(packed.k, non_blocking=True)
         host_out["v"].copy_(packed.v, non_blocking=True)
         host_out["pos"].copy_(packed.positions, non_blocking=True)

@@ -1,0 +1,32 @@
+"""bench.py's roofline arithmetic on the CPU: the algorithmic work of a kernel
+is per launch (one radix digit pass, one decode step), and the achieved rate is
+that work over the average launch time."""
+import bench
+from paper_2608_21541_gb300 import workloads as W
+
+PEAKS = dict(hbm=6768.8, tensor=1732.7, source="measured")
+
+
+def test_sort_pass_work_is_per_launch():
+    wl = W.WORKLOADS["C3"]
+    work = bench.kernel_work(wl, wl.B_live, "sort_scatter")
+    assert work["bytes"] == wl.units * wl.n * 16  # keys and indices, read and written once
+    r = bench.roofline_for("sort_scatter", work, 0.25, PEAKS)
+    assert r["bound"] == "hbm"
+    assert abs(r["achieved"] - work["bytes"] / 0.25e-3 / 1e9) < 0.1
+
+
+def test_decode_work_is_one_step():
+    wl = W.WORKLOADS["C4"]
+    work = bench.kernel_work(wl, wl.B_live, "decode_split")
+    assert work["bytes"] == wl.B * wl.L * wl.B_live * wl.d * 2 * 2
+    r = bench.roofline_for("decode_split", work, 0.6, PEAKS)
+    assert abs(r["frac"] - work["bytes"] / 0.6e-3 / 1e9 / PEAKS["hbm"]) < 1e-4
+
+
+def test_score_passes_are_tensor_bound_at_full_size():
+    wl = W.WORKLOADS["C3"]
+    work = bench.kernel_work(wl, wl.B_live, "score_pass1")
+    assert work["flops"] == 2.0 * wl.G * wl.w * wl.d * wl.n * wl.units
+    r = bench.roofline_for("score_pass1", work, 1.8, PEAKS)
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
