@@ -2,7 +2,7 @@
 //
 // The same two passes as score.cu (§4 observation-window score; the log-sum-
 // exp of every observation row is needed before any column sum), for the
-// observation-row counts R in {128, 256} that fit one MMA instruction:
+// observation-row counts R that are multiples of 128 (of 256 above 256):
 //   pass 1  D[rows x keys] = Q K^T.  Each epilogue thread owns one row and
 //           keeps its online (max, sum) over the CTA's keys without shuffles.
 //   pass 2  D[keys x rows] = K Q^T.  Each epilogue thread owns one key and sums
@@ -388,35 +388,42 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
   extern __shared__ char smem_raw[];
   const Shared<C> sh = shared_layout<C>(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int u = blockIdx.x / p.key_splits, split = blockIdx.x % p.key_splits;
+  // rows come in groups of RG <= 256 (one MMA's N); adjacent CTAs are the
+  // groups of one key range and stream the same K tiles
   const int n = p.n, R = p.R;
+  const int RG = R < 256 ? R : 256;
+  const int groups = R / RG;
+  const int grp = blockIdx.x % groups, item = blockIdx.x / groups;
+  const int u = item / p.key_splits, split = item % p.key_splits;
+  const int rg0 = grp * RG;
   const int j_begin = split * kKeysPerItemTc;
   const int j_end = min(n, j_begin + kKeysPerItemTc);
   const int ntiles = (j_end - j_begin + C::kTileKeys - 1) / C::kTileKeys;
-  for (int r = threadIdx.x; r < R; r += blockDim.x) sh.lse()[r] = lse2[(size_t)u * R + r];
+  for (int r = threadIdx.x; r < RG; r += blockDim.x) sh.lse()[r] = lse2[(size_t)u * R + rg0 + r];
   const uint32_t tmem = setup<C>(sh, warp);
   volatile int* ab = sh.abort_flag();
 
   if (warp == 0) {
-    if (lane == 0) produce<C>(sh, &tmK, &tmQ, u * R, R, (long)u * n + j_begin, ntiles);
+    if (lane == 0) produce<C>(sh, &tmK, &tmQ, u * R + rg0, RG, (long)u * n + j_begin, ntiles);
   } else if (warp == 1) {
     if (lane == 0)
       issue_mmas<C>(
-          sh, tmem, idesc_bf16(C::kTileKeys, R), ntiles,
+          sh, tmem, idesc_bf16(C::kTileKeys, RG), ntiles,
           [&](int s, uint32_t kh, uint32_t koff) {
             return sh.kst(s) + kh * (C::kStageBytes / 2) + koff;
           },
           [&](int, uint32_t kh, uint32_t koff) { return sh.q() + kh * (C::kQBytes / 2) + koff; });
   } else {
     // every warp takes every tile: warp (q, cq) owns keys q*32.. of the tile
-    // (its TMEM lane quadrant) and rows cq*64 .. cq*64+63, summed into row
-    // block cq.  It releases the accumulator as soon as its columns are read.
+    // (its TMEM lane quadrant) and rows rg0 + cq*64 .. +63, summed into row
+    // block grp*4 + cq.  It releases the accumulator as soon as its columns
+    // are read.
     const int ew = warp - 2, q = warp & 3, cq = ew >> 2;
     const int key = q * 32 + lane;
-    const bool rows_here = cq * 64 < R;
+    const bool rows_here = cq * 64 < RG;
     const float sl2 = p.scale_log2;
     const int nw = n - p.w;
-    float* out = s_part + ((size_t)u * p.row_blocks + cq) * n;
+    float* out = s_part + ((size_t)u * p.row_blocks + grp * 4 + cq) * n;
     const int r0 = cq * 64;
     const float4* L4 = reinterpret_cast<const float4*>(sh.lse() + r0);
     for (int t = 0; t < ntiles; ++t) {
@@ -446,8 +453,8 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
       } else {
 #pragma unroll
         for (int i = 0; i < 64; ++i) {
-          const int r = r0 + i;
-          if (j < j_end && j <= nw + (r % p.w)) acc[0] += ex2(fmaf(v[i], sl2, -sh.lse()[r]));
+          const int r = r0 + i;  // row of the group; rg0 + r of the unit
+          if (j < j_end && j <= nw + ((rg0 + r) % p.w)) acc[0] += ex2(fmaf(v[i], sl2, -sh.lse()[r]));
         }
       }
       if (j < j_end)
@@ -489,7 +496,11 @@ bool make_row_map(CUtensorMap* map, const void* base, uint64_t rows, uint32_t bo
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-bool score_tc_supported(const Prob& p) { return p.R == 128 || p.R == 256; }
+// R = G w observation rows per KV head: pass 1 takes 128-row halves, pass 2
+// groups of min(R, 256) rows (one MMA's N each).
+bool score_tc_supported(const Prob& p) {
+  return p.R >= 128 && p.R % 128 == 0 && (p.R <= 256 || p.R % 256 == 0);
+}
 
 bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_part, float* lse2,
                      float* s_part, uint32_t* status, cudaStream_t st) {
@@ -497,7 +508,7 @@ bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_pa
   const uint64_t krows = (uint64_t)p.units * p.n, qrows = (uint64_t)p.units * p.R;
   if (!make_row_map(&mk1, K, krows, tc::Pass1::kTileKeys) || !make_row_map(&mq1, Q, qrows, 128) ||
       !make_row_map(&mk2, K, krows, tc::Pass2::kTileKeys) ||
-      !make_row_map(&mq2, Q, qrows, (uint32_t)p.R))
+      !make_row_map(&mq2, Q, qrows, (uint32_t)(p.R < 256 ? p.R : 256)))
     return false;
   static bool attr = false;
   if (!attr) {
@@ -520,8 +531,9 @@ bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_pa
   }
   {
     TraceScope ts_("score_pass2", st);
-    tc::colsum_tc_kernel<<<items, tc::kThreads, tc::Pass2::kSmemBytes, st>>>(mk2, mq2, p, lse2,
-                                                                             s_part, status);
+    const unsigned groups = (unsigned)(p.R < 256 ? 1 : p.R / 256);
+    tc::colsum_tc_kernel<<<items * groups, tc::kThreads, tc::Pass2::kSmemBytes, st>>>(
+        mk2, mq2, p, lse2, s_part, status);
   }
   return true;
 }

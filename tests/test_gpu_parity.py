@@ -29,6 +29,11 @@ CASES = {
                                    kind="student_t"),
     "zipf_long": W.Workload("Z", B=1, L=1, Hq=8, H=2, n=9000, d=128, w=64, keep=(1, 10),
                             kind="zipf"),
+    # R = G w = 512 and 768: the tcgen05 pass 2 in two and three 256-row groups
+    "rows512_zipf": W.Workload("Z5", B=1, L=2, Hq=16, H=2, n=4100, d=128, w=64, keep=(1, 10),
+                               kind="zipf"),
+    "rows768_planted": W.Workload("P7", B=1, L=1, Hq=32, H=2, n=3333, d=128, w=48, keep=(1, 8),
+                                  kind="planted"),
 }
 
 _cache = {}
