@@ -42,6 +42,10 @@ def parse():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: compress this many layers instead of the workload's")
+    ap.add_argument("--rows", action="store_true",
+                    help="time the evaluation instruments and variants (fixed-row and lift "
+                         "diagnostics, coverage profile, sampled compensation, clustered "
+                         "summaries with the certified decode) instead of the hot path")
     ap.add_argument("--decode-steps", type=int, default=1,
                     help="decode steps per step after the compression, each with fresh queries "
                          "(the C4 configuration decodes 256)")
@@ -224,6 +228,110 @@ def run_reference(args, wl, rank):
                                    "cycled, float64, all host threads"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
+    print(json.dumps(line), flush=True)
+
+
+def run_rows(args, wl):
+    """The evaluation instruments and method variants beyond the hot path on the
+    full workload: the GPU time of each entry point (CUDA events, inputs
+    resident), its bytes of K and V against the HBM roof, and the float64
+    oracle timed on two sampled query heads of layer 0 (one host thread each,
+    extrapolated to every head).  Prints one JSON line."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2608_21541_gb300 import build as B
+    from paper_2608_21541_gb300 import certkv as ck
+    from paper_2608_21541_gb300 import workloads as W
+
+    B.build()
+    dev = torch.device("cuda", 0)
+    peaks = load_peaks()
+    K, V, Q = W.draw(wl, seed=args.seed, device=dev)
+    q = W.draw_decode_queries(wl, 0, seed=args.seed, device=dev)
+    plain = ck.certkv_default_params()
+    clus = ck.certkv_default_params(tail_clusters=4)
+    packed = ck.certkv_compress(K, V, Q, wl.B_live, plain)
+    packed_c = ck.certkv_compress(K, V, Q, wl.B_live, clus)
+    a = ck.certkv_score(K, Q, plain)
+    m = 32
+    g = torch.Generator().manual_seed(args.seed)
+    unif = torch.rand((wl.B, wl.L, wl.Hq, 2 * m), generator=g).to(dev)
+    heads = wl.B * wl.L * wl.Hq
+
+    def timed(fn, reps=3):
+        fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    kv = K.numel() * 2 * 2
+    entries = {
+        "fixed_row_stats": dict(ms=timed(lambda: ck.certkv_fixed_row_stats(q, K, V, packed,
+                                                                           scores=a)), bytes=kv),
+        "coverage_profile": dict(ms=timed(lambda: ck.certkv_coverage_profile(
+            q, K, eta=(0.5, 0.1, 0.05), rel_eps=(0.1,), abs_eps=(1e-4,))), bytes=kv // 2),
+        "sampled_compensation": dict(ms=timed(lambda: ck.certkv_sampled_compensation(
+            q, K, V, packed, unif, m)), bytes=kv),
+        "decode_certified": dict(ms=timed(lambda: ck.certkv_decode_certified(q, packed_c,
+                                                                             hkv=wl.H)),
+                                 bytes=packed_c.k.numel() * 2 * 2),
+    }
+    t_plain = timed(lambda: ck.certkv_compress(K, V, Q, wl.B_live, plain, out=packed))
+    t_clus = timed(lambda: ck.certkv_compress(K, V, Q, wl.B_live, clus, out=packed_c))
+    entries["compress_with_4_clusters"] = dict(ms=t_clus, bytes=kv, plain_ms=t_plain)
+    for e in entries.values():
+        e["GBps"] = round(e["bytes"] / (e["ms"] / 1e3) / 1e9, 1)
+        e["frac_of_hbm"] = round(e["GBps"] / peaks["hbm"], 4)
+        e["ms"] = round(e["ms"], 3)
+
+    # the float64 oracle on query heads 0 and Hq - 1 of layer 0 (KV heads 0 and H - 1)
+    Kb = W.bf16_bits(K[0, 0].cpu())
+    Vb = W.bf16_bits(V[0, 0].cpu())
+    qb = W.bf16_bits(q[0, 0].cpu())
+    a0 = a[:wl.H].cpu().numpy()
+    pos, offs, cnts = (x.cpu().numpy() for x in (packed.positions, packed.offsets,
+                                                  packed.real_counts))
+    pk, pvb = W.bf16_bits(packed.k[:offs[wl.H]].cpu()), W.bf16_bits(packed.v[:offs[wl.H]].cpu())
+    un = unif[0, 0].cpu().numpy()
+    scale = 1.0 / np.sqrt(wl.d)
+    G = wl.Hq // wl.H
+    cost = {"fixed_row_stats": 0.0, "coverage_profile": 0.0, "sampled_compensation": 0.0}
+    sample = [0, wl.Hq - 1]
+    for qh in sample:
+        h = qh // G
+        kept = np.zeros(wl.n, bool)
+        kept[pos[offs[h]:offs[h] + cnts[h]]] = True
+        slot = offs[h] + cnts[h]
+        t0 = time.perf_counter()
+        oracle.fixed_row(qb[qh], Kb[h], Vb[h], kept, scale=scale)
+        oracle.future_query_lift(qb[qh], Kb[h], Vb[h], kept, a0[h], scale=scale, kstar=pk[slot],
+                                 vstar=pvb[slot])
+        t1 = time.perf_counter()
+        oracle.coverage_profile(qb[qh], Kb[h], scale=scale, eta=(0.5, 0.1, 0.05), rel_eps=(0.1,),
+                                abs_eps=(1e-4,))
+        t2 = time.perf_counter()
+        oracle.sampled_compensation(qb[qh], Kb[h], Vb[h], kept, un[qh], scale=scale, m=m)
+        t3 = time.perf_counter()
+        cost["fixed_row_stats"] += t1 - t0
+        cost["coverage_profile"] += t2 - t1
+        cost["sampled_compensation"] += t3 - t2
+    for name, c in cost.items():
+        entries[name]["oracle"] = {"ms_per_head": round(c / len(sample) * 1e3, 2),
+                                   "ms_all_heads_one_thread": round(c / len(sample) * heads * 1e3,
+                                                                    1),
+                                   "sample": f"query heads {sample} of layer 0"}
+    line = {"metric": "evaluation instruments and variants beyond the hot path",
+            "unit": "ms per call over every query head (events, inputs resident)",
+            "config": dict(config_dict(wl, wl.B_live), query_heads=heads, samples_m=m,
+                           clusters=4),
+            "peak_hbm_GBps": peaks["hbm"], "rows": entries}
     print(json.dumps(line), flush=True)
 
 
@@ -430,7 +538,10 @@ def main():
         import torch.distributed as dist
         backend = "nccl" if torch.cuda.is_available() else "gloo"
         dist.init_process_group(backend)
-    if args.impl == "reference":
+    if args.rows:
+        if rank == 0:
+            run_rows(args, wl)
+    elif args.impl == "reference":
         run_reference(args, wl, rank)
     else:
         run_ours(args, wl, rank, world)
