@@ -272,12 +272,24 @@ __global__ void __launch_bounds__(256) score_pool_kernel(Prob p, const float* __
   const float invR = 1.0f / (float)p.R;
   const float invPool = 1.0f / (float)p.pool;
   const int lo = j0 - half, cnt = (j1 + half) - lo;
-  for (int t = threadIdx.x; t < cnt; t += blockDim.x) {
-    const int i = lo + t;
-    float s = 0.f;
-    if (i >= 0 && i < n)
-      for (int rb = 0; rb < p.row_blocks; ++rb) s += s_part[((size_t)u * p.row_blocks + rb) * n + i];
-    s_win[t] = s * invR;
+  // the row-block partials summed in row-block order; four window positions
+  // per thread and iteration, so that their loads are in flight together
+  const float* sb = s_part + (size_t)u * p.row_blocks * n;
+  for (int t0 = threadIdx.x; t0 < cnt; t0 += 4 * blockDim.x) {
+    float s[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int rb = 0; rb < p.row_blocks; ++rb) {
+      float x[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int i = lo + t0 + e * (int)blockDim.x;
+        x[e] = (t0 + e * (int)blockDim.x < cnt && i >= 0 && i < n) ? sb[(size_t)rb * n + i] : 0.f;
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e) s[e] += x[e];
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      if (t0 + e * (int)blockDim.x < cnt) s_win[t0 + e * blockDim.x] = s[e] * invR;
   }
   __syncthreads();
   float* sp = s_pool + (size_t)u * n;
@@ -347,14 +359,24 @@ __global__ void __launch_bounds__(256) score_scale_kernel(Prob p, const float* _
   const float* sp = s_pool + (size_t)u * n;
   float* au = a_out + (size_t)u * n;
   const int j0 = slice * kFinSpan, j1 = min(n, j0 + kFinSpan);
-  for (int j = j0 + threadIdx.x; j < j1; j += blockDim.x) {
-    float v = (j >= nw && p.protect) ? smax : sp[j];
-    v = v > 0.f ? v : 0.f;
-    const float a = __fdiv_rn(v, total);
-    au[j] = a;
-    if (keys) {
-      keys[(size_t)u * n + j] = score_key(a);
-      vals[(size_t)u * n + j] = j;
+  for (int jb = j0 + threadIdx.x; jb < j1; jb += 4 * blockDim.x) {
+    float v[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {  // four loads in flight
+      const int j = jb + e * (int)blockDim.x;
+      v[e] = j < j1 ? ((j >= nw && p.protect) ? smax : sp[j]) : 0.f;
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = jb + e * (int)blockDim.x;
+      if (j >= j1) break;
+      const float x = v[e] > 0.f ? v[e] : 0.f;
+      const float a = __fdiv_rn(x, total);
+      au[j] = a;
+      if (keys) {
+        keys[(size_t)u * n + j] = score_key(a);
+        vals[(size_t)u * n + j] = j;
+      }
     }
   }
 }

@@ -379,6 +379,7 @@ __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_consta
 
 // Pass 2.  grid = units * key_splits.  D[128 keys x R rows]; epilogue thread
 // = one key, summing exp(l - LSE_row) over a 64-row quarter of its TMEM lane.
+template <bool kGrouped>  // R > 256: the rows come in groups of 256, one per CTA
 __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_constant__ CUtensorMap tmK,
                                                                 const __grid_constant__ CUtensorMap tmQ,
                                                                 Prob p, const float* __restrict__ lse2,
@@ -391,9 +392,10 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
   // rows come in groups of RG <= 256 (one MMA's N); adjacent CTAs are the
   // groups of one key range and stream the same K tiles
   const int n = p.n, R = p.R;
-  const int RG = R < 256 ? R : 256;
-  const int groups = R / RG;
-  const int grp = blockIdx.x % groups, item = blockIdx.x / groups;
+  const int RG = kGrouped ? 256 : R;
+  const int groups = kGrouped ? R / 256 : 1;
+  const int grp = kGrouped ? (int)(blockIdx.x % groups) : 0;
+  const unsigned item = kGrouped ? blockIdx.x / groups : blockIdx.x;
   const int u = item / p.key_splits, split = item % p.key_splits;
   const int rg0 = grp * RG;
   const int j_begin = split * kKeysPerItemTc;
@@ -514,7 +516,9 @@ bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_pa
   if (!attr) {
     cudaFuncSetAttribute(tc::lse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          tc::Pass1::kSmemBytes);
-    cudaFuncSetAttribute(tc::colsum_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(tc::colsum_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         tc::Pass2::kSmemBytes);
+    cudaFuncSetAttribute(tc::colsum_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          tc::Pass2::kSmemBytes);
     attr = true;
   }
@@ -531,9 +535,12 @@ bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_pa
   }
   {
     TraceScope ts_("score_pass2", st);
-    const unsigned groups = (unsigned)(p.R < 256 ? 1 : p.R / 256);
-    tc::colsum_tc_kernel<<<items * groups, tc::kThreads, tc::Pass2::kSmemBytes, st>>>(
-        mk2, mq2, p, lse2, s_part, status);
+    if (p.R <= 256)
+      tc::colsum_tc_kernel<false><<<items, tc::kThreads, tc::Pass2::kSmemBytes, st>>>(
+          mk2, mq2, p, lse2, s_part, status);
+    else
+      tc::colsum_tc_kernel<true><<<items * (p.R / 256), tc::kThreads, tc::Pass2::kSmemBytes, st>>>(
+          mk2, mq2, p, lse2, s_part, status);
   }
   return true;
 }
