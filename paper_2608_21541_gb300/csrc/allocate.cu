@@ -151,10 +151,14 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   const Shear sh = make_shear(cu, b0, b1 - 1);
   // the tolerant chain of tolerant_chain, with the sheared values of eight
   // consecutive points evaluated ahead (their curve loads in flight together)
-  // and kept on the thread-private stack next to b, so that a pop needs no
-  // reload
-  int32_t st[kHullSeg];
-  float sty[kHullSeg], std_[kHullSeg];
+  // and kept on the thread-private stack next to b (as its offset in the
+  // segment), so that a pop needs no reload.  Each test takes the largest
+  // error bound of the points seen so far, at least that of its own three
+  // points: the filter can only keep more.
+  static_assert(kHullSeg <= 256, "segment offsets are stored in one byte");
+  uint8_t st[kHullSeg];
+  float sty[kHullSeg];
+  float dmax = 0.f;
   int top = 0;
   const int count = b1 - b0;
   for (int i0 = 0; i0 < count; i0 += 8) {
@@ -165,18 +169,17 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       if (i0 + k >= count) break;
-      const int b = b0 + i0 + k;
-      while (top >= 2 && clearly_above(st[top - 2], sty[top - 2], st[top - 1], sty[top - 1], b,
-                                       yv[k],
-                                       fmaxf(fmaxf(std_[top - 2], std_[top - 1]), dv[k])))
+      const int i = i0 + k;
+      dmax = fmaxf(dmax, dv[k]);
+      while (top >= 2 && clearly_above(st[top - 2], sty[top - 2], st[top - 1], sty[top - 1], i,
+                                       yv[k], dmax))
         --top;
-      st[top] = b;
+      st[top] = (uint8_t)i;
       sty[top] = yv[k];
-      std_[top] = dv[k];
       ++top;
     }
   }
-  for (int i = 0; i < top; ++i) out[i] = st[i];
+  for (int i = 0; i < top; ++i) out[i] = b0 + st[i];
   ncand[(size_t)u * ncand_stride(p) + seg] = top;
 }
 

@@ -142,10 +142,10 @@ int cuda_ok(cudaError_t e) { return e == cudaSuccess ? CERTKV_OK : CERTKV_ECUDA;
 
 bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
 
-// key-init for caller-given scores: keys0 = ~bits(a), vals0 = index; flags
-// negative or non-finite scores.
+// key-init for caller-given scores: keys0 = ~bits(a) (the sort's first pass
+// takes the indices as its values); flags negative or non-finite scores.
 __global__ void key_init_kernel(Prob p, const float* __restrict__ a, uint32_t* __restrict__ keys,
-                                int32_t* __restrict__ vals, uint32_t* status) {
+                                uint32_t* status) {
   const size_t total = (size_t)p.units * p.n;
   bool bad = false;
   for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
@@ -153,7 +153,6 @@ __global__ void key_init_kernel(Prob p, const float* __restrict__ a, uint32_t* _
     const float x = a[i];
     if (!(x >= 0.0f && x <= 3.0e38f)) bad = true;
     keys[i] = score_key(x > 0.0f ? x : 0.0f);
-    vals[i] = (int32_t)(i % (size_t)p.n);
   }
   if (bad) raise_status(status, CERTKV_STATUS_NONFINITE);
 }
@@ -257,7 +256,6 @@ int certkv_curves(const certkv_shape* shape, const void* V, const float* a,
   {
     TraceScope ts_("key_init", st);
     key_init_kernel<<<1024, 256, 0, st>>>(p, a, reinterpret_cast<uint32_t*>(ws + ly.keys0),
-                                          reinterpret_cast<int32_t*>(ws + ly.vals0),
                                           reinterpret_cast<uint32_t*>(ws + ly.status));
   }
   launch_sort(p, ly, ws, a, st);
@@ -285,7 +283,6 @@ int certkv_compress_scored(const certkv_shape* shape, const void* K, const void*
   {
     TraceScope ts_("key_init", st);
     key_init_kernel<<<1024, 256, 0, st>>>(p, a, reinterpret_cast<uint32_t*>(ws + ly.keys0),
-                                          reinterpret_cast<int32_t*>(ws + ly.vals0),
                                           reinterpret_cast<uint32_t*>(ws + ly.status));
   }
   return run_scored(p, ly, ws, K, V, a, out, st);

@@ -36,11 +36,12 @@ __device__ __forceinline__ float key_logit(uint32_t key) {
 
 // grid = (units, kCovSplits), block = 128: each warp takes 32-token tiles; the
 // G query heads of the unit's group are dotted with each K row by 2G lanes
-// (coalesced), then lane = token writes its keys.  keys/vals [u * G + g][n].
+// (coalesced), then lane = token writes its keys, [u * G + g][n] (the sort's
+// first pass takes the token indices as its values).
 template <int G>
 __global__ void __launch_bounds__(128) coverage_logits_kernel(
     Prob p, const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ K,
-    float scale, uint32_t* __restrict__ keys, int32_t* __restrict__ vals) {
+    float scale, uint32_t* __restrict__ keys) {
   __shared__ float xs[4][32 * G];
   const int u = blockIdx.x, split = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -55,11 +56,8 @@ __global__ void __launch_bounds__(128) coverage_logits_kernel(
     const int j = t * 32 + lane;
     if (j < n) {
 #pragma unroll
-      for (int g = 0; g < G; ++g) {
-        const size_t o = ((size_t)u * G + g) * n + j;
-        keys[o] = desc_key(xs[warp][lane * G + g] * scale);
-        vals[o] = j;
-      }
+      for (int g = 0; g < G; ++g)
+        keys[((size_t)u * G + g) * n + j] = desc_key(xs[warp][lane * G + g] * scale);
     }
     __syncwarp();  // xs is rewritten by the next tile
   }
@@ -204,7 +202,7 @@ void launch_coverage(const Prob& p, const void* q, const void* K, float scale,
   {
     TraceScope ts_("coverage_logits", st);
 #define CERTKV_COV_LOGITS(GG) \
-  coverage_logits_kernel<GG><<<grid, 128, 0, st>>>(p, qb, kb, scale, k0, v0)
+  coverage_logits_kernel<GG><<<grid, 128, 0, st>>>(p, qb, kb, scale, k0)
     switch (p.G) {
       case 1: CERTKV_COV_LOGITS(1); break;
       case 2: CERTKV_COV_LOGITS(2); break;

@@ -209,46 +209,65 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
   if (lane == 0) agg_mq[ci] = make_float4(m.hi, m.lo, q.hi, q.lo);
 }
 
-// grid = units, block = 128 (one thread per dimension): exclusive suffix sums
-// over chunks, in double-float, folded from the last chunk down.  The chunk
-// sums are loaded kPrefixBlock chunks at a time so that the loads overlap.
-constexpr int kPrefixBlock = 16;
-__global__ void __launch_bounds__(128) curve_prefix_kernel(Prob p, const float4* __restrict__ agg_mq,
+// grid = (units, need_k ? 2 : 1), block = 160: exclusive suffix sums over
+// chunks in double-float, folded from the last chunk down in chunk order.
+// Threads 0..127 take one dimension of the V sums (blockIdx.y = 0) or of the K
+// sums (blockIdx.y = 1), with the next kPrefixBlock chunks' loads in flight
+// while the current ones are folded; warp 4 of the V block takes the scalar
+// sums m and Q, one chunk per lane per round.
+constexpr int kPrefixBlock = 32;
+__global__ void __launch_bounds__(160) curve_prefix_kernel(Prob p, const float4* __restrict__ agg_mq,
                                                            const float* __restrict__ agg_v,
                                                            const float* __restrict__ agg_k,
-                                                           bool need_k, float4* __restrict__ base_mq,
+                                                           float4* __restrict__ base_mq,
                                                            float2* __restrict__ base_v,
                                                            float2* __restrict__ base_k) {
-  const int u = blockIdx.x, i = threadIdx.x;
-  const size_t c0 = (size_t)u * p.chunks;
-  DF rv = df_make(0.f), rk = df_make(0.f), rm = df_make(0.f), rq = df_make(0.f);
-  for (int top = p.chunks - 1; top >= 0; top -= kPrefixBlock) {
-    float cv[kPrefixBlock], ck[kPrefixBlock];
-    float4 cmq[kPrefixBlock];
+  const int u = blockIdx.x;
+  const int chunks = p.chunks;
+  const size_t c0 = (size_t)u * chunks;
+  if (threadIdx.x >= kD) {
+    if (blockIdx.y != 0) return;
+    const int lane = threadIdx.x & 31;
+    DF rm = df_make(0.f), rq = df_make(0.f);
+    float4 nxt = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (chunks - 1 - lane >= 0) nxt = agg_mq[c0 + chunks - 1 - lane];
+    for (int top = chunks - 1; top >= 0; top -= 32) {
+      const float4 cur = nxt;
+      if (top - 32 - lane >= 0) nxt = agg_mq[c0 + top - 32 - lane];
+      for (int e = 0; e < 32 && top - e >= 0; ++e) {
+        if (lane == e) base_mq[c0 + top - e] = make_float4(rm.hi, rm.lo, rq.hi, rq.lo);
+        const float mh = __shfl_sync(kFull, cur.x, e), ml = __shfl_sync(kFull, cur.y, e);
+        const float qh = __shfl_sync(kFull, cur.z, e), ql = __shfl_sync(kFull, cur.w, e);
+        rm = df_add(rm, DF{mh, ml});
+        rq = df_add(rq, DF{qh, ql});
+      }
+    }
+    return;
+  }
+  const int i = threadIdx.x;
+  const float* src = (blockIdx.y == 0 ? agg_v : agg_k) + c0 * kD + i;
+  float2* dst = (blockIdx.y == 0 ? base_v : base_k) + c0 * kD + i;
+  DF r = df_make(0.f);
+  float nxt[kPrefixBlock];
+#pragma unroll
+  for (int e = 0; e < kPrefixBlock; ++e) {
+    const int c = chunks - 1 - e;
+    nxt[e] = c >= 0 ? src[(size_t)c * kD] : 0.f;
+  }
+  for (int top = chunks - 1; top >= 0; top -= kPrefixBlock) {
+    float cur[kPrefixBlock];
 #pragma unroll
     for (int e = 0; e < kPrefixBlock; ++e) {
-      const int c = top - e;
-      cv[e] = ck[e] = 0.f;
-      cmq[e] = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (c >= 0) {
-        cv[e] = agg_v[(c0 + c) * kD + i];
-        if (need_k) ck[e] = agg_k[(c0 + c) * kD + i];
-        if (i == 0) cmq[e] = agg_mq[c0 + c];
-      }
+      cur[e] = nxt[e];
+      const int c = top - kPrefixBlock - e;
+      nxt[e] = c >= 0 ? src[(size_t)c * kD] : 0.f;
     }
 #pragma unroll
     for (int e = 0; e < kPrefixBlock; ++e) {
       const int c = top - e;
       if (c < 0) break;
-      base_v[(c0 + c) * kD + i] = make_float2(rv.hi, rv.lo);
-      if (need_k) base_k[(c0 + c) * kD + i] = make_float2(rk.hi, rk.lo);
-      if (i == 0) base_mq[c0 + c] = make_float4(rm.hi, rm.lo, rq.hi, rq.lo);
-      rv = df_add_f(rv, cv[e]);
-      if (need_k) rk = df_add_f(rk, ck[e]);
-      if (i == 0) {
-        rm = df_add(rm, DF{cmq[e].x, cmq[e].y});
-        rq = df_add(rq, DF{cmq[e].z, cmq[e].w});
-      }
+      dst[(size_t)c * kD] = make_float2(r.hi, r.lo);
+      r = df_add_f(r, cur[e]);
     }
   }
 }
@@ -495,8 +514,8 @@ void launch_curves(const Prob& p, const Layout& ly, char* ws, const void* K, con
   }
   {
     TraceScope ts_("curve_prefix", st);
-    curve_prefix_kernel<<<p.units, 128, 0, st>>>(p, agg_mq, agg_v, agg_k, need_k, base_mq, base_v,
-                                                 base_k);
+    curve_prefix_kernel<<<dim3(p.units, need_k ? 2 : 1), 160, 0, st>>>(p, agg_mq, agg_v, agg_k,
+                                                                        base_mq, base_v, base_k);
   }
   {
     TraceScope ts_("curve_eval", st);

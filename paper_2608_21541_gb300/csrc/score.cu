@@ -340,7 +340,6 @@ __global__ void __launch_bounds__(256) score_scale_kernel(Prob p, const float* _
                                                           const float4* __restrict__ fin_part,
                                                           float* __restrict__ a_out,
                                                           uint32_t* __restrict__ keys,
-                                                          int32_t* __restrict__ vals,
                                                           uint32_t* status) {
   const int slice = blockIdx.x, u = blockIdx.y;
   const int n = p.n, nw = n - p.w;
@@ -373,10 +372,7 @@ __global__ void __launch_bounds__(256) score_scale_kernel(Prob p, const float* _
       const float x = v[e] > 0.f ? v[e] : 0.f;
       const float a = __fdiv_rn(x, total);
       au[j] = a;
-      if (keys) {
-        keys[(size_t)u * n + j] = score_key(a);
-        vals[(size_t)u * n + j] = j;
-      }
+      if (keys) keys[(size_t)u * n + j] = score_key(a);
     }
   }
 }
@@ -428,8 +424,7 @@ void launch_score(const Prob& p, const Layout& ly, char* ws, const void* K, cons
   {
     TraceScope ts_("score_scale", st);
     score_scale_kernel<<<fgrid, 256, 0, st>>>(
-        p, s_pool, fin_part, a_out, reinterpret_cast<uint32_t*>(ws + ly.keys0),
-        reinterpret_cast<int32_t*>(ws + ly.vals0), status);
+        p, s_pool, fin_part, a_out, reinterpret_cast<uint32_t*>(ws + ly.keys0), status);
   }
 }
 

@@ -4,8 +4,9 @@
 // Segmented LSD radix sort over all units at once: 32-bit keys
 // (~bits(a), ascending = a descending), 8-bit digits, 4 passes.  Each pass is
 // histogram -> per-unit exclusive scan in (digit, tile) order -> stable
-// scatter.  The input of pass 0 is in index order, so stability yields the
-// lower-index tie-break.
+// scatter.  The input of pass 0 is in index order and its values are the
+// indices themselves (not read), so stability yields the lower-index
+// tie-break.
 #include "common.cuh"
 #include "internal.cuh"
 
@@ -93,7 +94,8 @@ __global__ void __launch_bounds__(1024) radix_scan_kernel(uint32_t* __restrict__
 // grid = (tiles, units): stable scatter of one tile.  The tile is first
 // ordered by digit in shared memory (stable ranks from per-warp counts), then
 // written out so that consecutive threads store consecutive positions of a
-// digit's run.
+// digit's run.  kFirst: the values are the key indices (vin is not read).
+template <bool kFirst>
 __global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
     const uint32_t* __restrict__ kin, const int32_t* __restrict__ vin, uint32_t* __restrict__ kout,
     int32_t* __restrict__ vout, int n, int tiles, int shift, const uint32_t* __restrict__ hist) {
@@ -119,7 +121,7 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
     int j = wbase + i * 32 + lane;
     bool ok = j < n;
     key[i] = ok ? ku[j] : 0u;
-    val[i] = ok ? vu[j] : 0;
+    val[i] = kFirst ? j : (ok ? vu[j] : 0);
   }
   const uint32_t lt = (1u << lane) - 1u;
   // 1. per-warp digit counts; peers[i] = lanes holding the same digit
@@ -216,8 +218,12 @@ void launch_sort(const Prob& p, const Layout& ly, char* ws, const float* /*a*/, 
     }
     {
       TraceScope ts_("sort_scatter", st);
-      radix_scatter_kernel<<<grid, kSortThreads, 0, st>>>(kin, vin, kout, vout, p.n, p.sort_tiles,
-                                                           shift, hist);
+      if (pass == 0)
+        radix_scatter_kernel<true><<<grid, kSortThreads, 0, st>>>(kin, vin, kout, vout, p.n,
+                                                                  p.sort_tiles, shift, hist);
+      else
+        radix_scatter_kernel<false><<<grid, kSortThreads, 0, st>>>(kin, vin, kout, vout, p.n,
+                                                                   p.sort_tiles, shift, hist);
     }
   }
   // after 4 passes the sorted keys / permutation are back in keys0 / vals0
