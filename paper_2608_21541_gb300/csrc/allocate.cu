@@ -228,8 +228,11 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
                                                             int64_t* __restrict__ offsets) {
   __shared__ int bsel[32];
   __shared__ int coff[33];
+  __shared__ int htot[32];
+  __shared__ int klo[32], khi[32];  // per head: staged index range that holds b_h(lambda)
+  __shared__ int blo[32], bhi[32];  // the same range as values of b
   __shared__ DF wbest_f[32];  // per-warp argmin, combined per head
-  __shared__ int wbest_b[32];
+  __shared__ int wbest_b[32], wbest_k[32];
   __shared__ double lam_sh[2];
   __shared__ DF lam_df;  // the step's multiplier as double-float, for every warp
   __shared__ float2 win[32][64];
@@ -245,6 +248,36 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
   const int groups = groups_of(p);
   const size_t stride = ncand_stride(p);
 
+  const bool lagrangian = p.allocator == CERTKV_ALLOC_LAGRANGIAN;  // the hull filter ran only for it
+  // Candidate offsets: warp h scans head h's group counts into gpre[h][g]
+  // (exclusive, gpre[h][groups] = the head's total), kept in the repair's
+  // scan buffer, which is free until the repair.
+  int* gpre = reinterpret_cast<int*>(scanbuf);
+  const int gstride = groups + 1;
+  const bool gfit = H * gstride <= (int)(sizeof(scanbuf) / sizeof(int));
+  if (lagrangian && gfit) {
+    for (int h = warp; h < H; h += nwarps) {
+      const int32_t* nc = ncand + (size_t)(bl * H + h) * stride + p.hull_segs;
+      int carry = 0;
+      for (int g0 = 0; g0 < groups; g0 += 32) {
+        const int g = g0 + lane;
+        const int v = g < groups ? nc[g] : 0;
+        int x = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(kFull, x, o);
+          if (lane >= o) x += y;
+        }
+        if (g < groups) gpre[h * gstride + g] = carry + x - v;
+        carry += __shfl_sync(kFull, x, 31);
+      }
+      if (lane == 0) {
+        gpre[h * gstride + groups] = carry;
+        htot[h] = carry;
+      }
+    }
+  }
+  __syncthreads();
   if (threadIdx.x == 0) {
     double mx = 0.0;
     int acc = 0;
@@ -252,107 +285,161 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
       const double v = df_to_double(df_from_order_key(cmax[(size_t)bl * H + h]));
       mx = v > mx ? v : mx;
       coff[h] = acc;
-      const int32_t* nc = ncand + (size_t)(bl * H + h) * stride + p.hull_segs;
-      if (p.allocator == CERTKV_ALLOC_LAGRANGIAN)  // the hull filter ran only for it
-        for (int g = 0; g < groups; ++g) acc += nc[g];
+      if (lagrangian) {
+        if (gfit) {
+          acc += htot[h];
+        } else {
+          const int32_t* nc = ncand + (size_t)(bl * H + h) * stride + p.hull_segs;
+          for (int g = 0; g < groups; ++g) acc += nc[g];
+        }
+      }
     }
     coff[H] = acc;
     lam_sh[0] = 0.0;
     lam_sh[1] = __dadd_rn(__dmul_rn(2.0, mx), 1.0);
   }
+  if (threadIdx.x < H) {
+    blo[threadIdx.x] = 0;
+    bhi[threadIdx.x] = INT_MAX;
+  }
   __syncthreads();
-  const bool lagrangian = p.allocator == CERTKV_ALLOC_LAGRANGIAN;
-  const bool staged = lagrangian && coff[H] <= kCandCap;
-  if (staged) {  // gather the group survivors of every head, in order; warp per (head, group)
-    for (int hg = warp; hg < H * groups; hg += nwarps) {
-      const int h = hg / groups, g = hg - h * groups;
-      const int u = bl * H + h;
-      const int32_t* nc = ncand + (size_t)u * stride + p.hull_segs;
-      const int32_t* cl = cand + (size_t)u * n;
-      int acc = coff[h];
-      for (int g2 = 0; g2 < g; ++g2) acc += nc[g2];
-      const int cnt = nc[g];
-      for (int k = lane; k < cnt; k += 32) {
-        const int b = cl[(size_t)g * kGroupSegs * kHullSeg + k];
-        cb_[acc + k] = b;
-        cy[acc + k] = curve[(size_t)u * n + b];
+  const bool staged = lagrangian && gfit && coff[H] <= kCandCap;
+  if (staged) {
+    // gather the group survivors of every head, in order: one thread per
+    // candidate finds its head and group and loads b and c(b)
+    for (int k = threadIdx.x; k < coff[H]; k += blockDim.x) {
+      int h = 0;
+      while (coff[h + 1] <= k) ++h;
+      const int r = k - coff[h];
+      const int* gp = gpre + h * gstride;
+      int lo = 0, hi = groups - 1;  // the last group g with gp[g] <= r
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (gp[mid] <= r) lo = mid; else hi = mid - 1;
       }
+      const int u = bl * H + h;
+      const int b = cand[(size_t)u * n + (size_t)lo * kGroupSegs * kHullSeg + (r - gp[lo])];
+      cb_[k] = b;
+      cy[k] = curve[(size_t)u * n + b];
     }
+  }
+  if (threadIdx.x < H) {
+    klo[threadIdx.x] = coff[threadIdx.x];
+    khi[threadIdx.x] = coff[threadIdx.x + 1] - 1;
   }
   __syncthreads();
 
   // Head h is scanned by warps h * wph .. h * wph + wph - 1 (wph = warps per
   // head); the lexicographic (value, b) minimum does not depend on the split.
+  // The smallest minimiser of c(b) + lambda b does not increase with lambda,
+  // so for lambda inside the bracket (lo, hi) it lies between the minimisers
+  // found at hi and at lo: each head scans only that range of its candidates
+  // (blo..bhi, as staged indices klo..khi).
   const int wph = nwarps / H;  // >= 1 since H <= 32
-  auto argmin_heads = [&]() {
+  auto scan_heads = [&]() {
     const DF ld = lam_df;
     const int h = warp / wph, sub = warp - h * wph;
     if (h < H) {
       const int u = bl * H + h;
       DF bf{INFINITY, 0.f};
-      int bb = INT_MAX;
-      auto consider = [&](int b, float2 c) {
+      int bb = INT_MAX, bk = -1;
+      auto consider = [&](int b, float2 c, int k) {
         const DF f = df_add(DF{c.x, c.y}, df_mul_f(ld, (float)b));
         if (df_less(f, bf) || (f.hi == bf.hi && f.lo == bf.lo && b < bb)) {
           bf = f;
           bb = b;
+          bk = k;
         }
       };
       if (staged) {
-        for (int k = coff[h] + sub * 32 + lane; k < coff[h + 1]; k += wph * 32) consider(cb_[k], cy[k]);
+        const int k1 = khi[h];
+        for (int k = klo[h] + sub * 32 + lane; k <= k1; k += wph * 32) consider(cb_[k], cy[k], k);
       } else {
         const int32_t* nc = ncand + (size_t)u * stride + p.hull_segs;
         const int32_t* cl = cand + (size_t)u * n;
+        const int b_lo = blo[h], b_hi = bhi[h];
         for (int g = 0; g < groups; ++g)
           for (int k = sub * 32 + lane; k < nc[g]; k += wph * 32) {
             const int b = cl[(size_t)g * kGroupSegs * kHullSeg + k];
-            consider(b, curve[(size_t)u * n + b]);
+            if (b >= b_lo && b <= b_hi) consider(b, curve[(size_t)u * n + b], -1);
           }
       }
+      const int own_b = bb, own_k = bk;
       warp_argmin_df(bf, bb);
+      // b is unique within a head: the winner's index is held by the lane
+      // whose own best was bb
+      const unsigned holder = __ballot_sync(kFull, bb != INT_MAX && own_b == bb);
+      const int kw = holder ? __shfl_sync(kFull, own_k, __ffs(holder) - 1) : -1;
       if (lane == 0) {
         wbest_f[warp] = bf;
         wbest_b[warp] = bb;
+        wbest_k[warp] = kw;
       }
     }
-    __syncthreads();
-    if (threadIdx.x < H) {
-      const int hh = threadIdx.x;
-      DF bf = wbest_f[hh * wph];
-      int bb = wbest_b[hh * wph];
-      for (int w = 1; w < wph; ++w) {
-        const DF f = wbest_f[hh * wph + w];
-        const int b = wbest_b[hh * wph + w];
+  };
+  // warp 0, lane = head, after the scan: the head's minimiser b (b_min when it
+  // has no candidate) and its staged index k (-2: no candidate; -1: not staged)
+  auto combine = [&](int& b_out, int& k_out) {
+    DF bf{INFINITY, 0.f};
+    int bb = INT_MAX, kk = -2;
+    if (lane < H) {
+      for (int w = 0; w < wph; ++w) {
+        const DF f = wbest_f[lane * wph + w];
+        const int b = wbest_b[lane * wph + w];
         if (df_less(f, bf) || (f.hi == bf.hi && f.lo == bf.lo && b < bb)) {
           bf = f;
           bb = b;
+          kk = wbest_k[lane * wph + w];
         }
       }
-      bsel[hh] = (bb == INT_MAX) ? p.b_min : bb;
     }
+    b_out = (bb == INT_MAX) ? p.b_min : bb;
+    k_out = (bb == INT_MAX) ? -2 : kk;
   };
 
-  // float64 bisection of the multiplier, by one thread; the argmin runs in
-  // double-float on every warp
-  if (threadIdx.x == 0) lam_df = df_from_double(__dmul_rn(__dadd_rn(lam_sh[0], lam_sh[1]), 0.5));
+  // float64 bisection of the multiplier in warp 0 (every lane holds the same
+  // bracket); the argmin runs in double-float on every warp
+  double lam_lo = lam_sh[0], lam_hi = lam_sh[1];
+  if (threadIdx.x == 0) lam_df = df_from_double(__dmul_rn(__dadd_rn(lam_lo, lam_hi), 0.5));
   __syncthreads();
   for (int t = 0; lagrangian && t < p.T; ++t) {
-    argmin_heads();
+    scan_heads();
     __syncthreads();
-    if (threadIdx.x == 0) {
-      const double lam = __dmul_rn(__dadd_rn(lam_sh[0], lam_sh[1]), 0.5);
-      int64_t tot = 0;
-      for (int h = 0; h < H; ++h) tot += bsel[h];
-      if (tot > B_real) lam_sh[0] = lam; else lam_sh[1] = lam;
-      lam_df = (t + 1 < p.T) ? df_from_double(__dmul_rn(__dadd_rn(lam_sh[0], lam_sh[1]), 0.5))
-                             : df_from_double(lam_sh[1]);
+    if (warp == 0) {
+      int bh, kh;
+      combine(bh, kh);
+      long long tot = lane < H ? bh : 0;
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) tot += __shfl_xor_sync(kFull, tot, o);
+      const double lam = __dmul_rn(__dadd_rn(lam_lo, lam_hi), 0.5);
+      const bool up = tot > B_real;
+      if (up) lam_lo = lam; else lam_hi = lam;
+      // the new bracket end's minimisers bound the next scans
+      if (lane < H && kh != -2) {
+        if (up) {
+          bhi[lane] = bh;
+          if (staged) khi[lane] = kh;
+        } else {
+          blo[lane] = bh;
+          if (staged) klo[lane] = kh;
+        }
+      }
+      if (lane == 0)
+        lam_df = (t + 1 < p.T) ? df_from_double(__dmul_rn(__dadd_rn(lam_lo, lam_hi), 0.5))
+                               : df_from_double(lam_hi);
     }
     __syncthreads();
   }
-  if (p.T == 0 && threadIdx.x == 0) lam_df = df_from_double(lam_sh[1]);
+  if (p.T == 0 && threadIdx.x == 0) lam_df = df_from_double(lam_hi);
   __syncthreads();
   if (lagrangian) {
-    argmin_heads();
+    scan_heads();
+    __syncthreads();
+    if (warp == 0) {
+      int bh, kh;
+      combine(bh, kh);
+      if (lane < H) bsel[lane] = bh;
+    }
   } else if (threadIdx.x < H) {  // the allocator ablations' starting points
     const int h = threadIdx.x;
     bsel[h] = (p.allocator == CERTKV_ALLOC_UNIFORM)

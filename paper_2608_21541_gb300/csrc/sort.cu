@@ -107,10 +107,8 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
   __shared__ int32_t sval[kSortTile];
   const int tile = blockIdx.x, u = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int i = threadIdx.x; i < kWarps * 256; i += kSortThreads) (&wcnt[0][0])[i] = 0;
-  gbase[threadIdx.x] = hist[((size_t)u * 256 + threadIdx.x) * tiles + tile];
-  __syncthreads();
-
+  // the tile's keys and values, its digit offsets and the counter reset all
+  // in flight together
   const uint32_t* ku = kin + (size_t)u * n;
   const int32_t* vu = vin + (size_t)u * n;
   const int wbase = tile * kSortTile + warp * (kSortTile / kWarps);
@@ -123,6 +121,9 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
     key[i] = ok ? ku[j] : 0u;
     val[i] = kFirst ? j : (ok ? vu[j] : 0);
   }
+  gbase[threadIdx.x] = hist[((size_t)u * 256 + threadIdx.x) * tiles + tile];
+  for (int i = threadIdx.x; i < kWarps * 256; i += kSortThreads) (&wcnt[0][0])[i] = 0;
+  __syncthreads();
   const uint32_t lt = (1u << lane) - 1u;
   // 1. per-warp digit counts; peers[i] = lanes holding the same digit
   uint32_t peers[kPerLane];
