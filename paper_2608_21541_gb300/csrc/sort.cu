@@ -53,41 +53,62 @@ __global__ void __launch_bounds__(kSortThreads) radix_hist_kernel(const uint32_t
   hist[((size_t)u * 256 + threadIdx.x) * tiles + tile] = cnt[threadIdx.x];
 }
 
-// grid = units: exclusive scan of the unit's 256 * tiles counters.
+// grid = units, block = 1024: exclusive scan of the unit's 256 * tiles
+// counters, 16 consecutive counters per thread per round (four 16-byte loads;
+// 256 * tiles is a multiple of 16).
+constexpr int kScanPer = 16;
 __global__ void __launch_bounds__(1024) radix_scan_kernel(uint32_t* __restrict__ hist, int tiles) {
   __shared__ uint32_t warp_tot[32];
-  __shared__ uint32_t carry;
   uint32_t* h = hist + (size_t)blockIdx.x * 256 * tiles;
   const int total = 256 * tiles;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) carry = 0;
-  __syncthreads();
-  for (int base = 0; base < total; base += blockDim.x) {
-    int i = base + threadIdx.x;
-    uint32_t v = i < total ? h[i] : 0u;
-    uint32_t x = v;
+  uint32_t carry = 0;
+  for (int base = 0; base < total; base += kScanPer * 1024) {
+    const int i0 = base + kScanPer * (int)threadIdx.x;
+    const bool mine = i0 < total;
+    uint4 v[kScanPer / 4];
+#pragma unroll
+    for (int e = 0; e < kScanPer / 4; ++e)
+      v[e] = mine ? reinterpret_cast<const uint4*>(h + i0)[e] : make_uint4(0u, 0u, 0u, 0u);
+    uint32_t s = 0;
+#pragma unroll
+    for (int e = 0; e < kScanPer / 4; ++e) s += v[e].x + v[e].y + v[e].z + v[e].w;
+    uint32_t x = s;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      uint32_t y = __shfl_up_sync(kFull, x, o);
+      const uint32_t y = __shfl_up_sync(kFull, x, o);
       if (lane >= o) x += y;
     }
     if (lane == 31) warp_tot[warp] = x;
     __syncthreads();
     if (warp == 0) {
-      uint32_t t = lane < (int)(blockDim.x >> 5) ? warp_tot[lane] : 0u;
+      uint32_t t = warp_tot[lane];
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        uint32_t y = __shfl_up_sync(kFull, t, o);
+        const uint32_t y = __shfl_up_sync(kFull, t, o);
         if (lane >= o) t += y;
       }
       warp_tot[lane] = t;  // inclusive
     }
     __syncthreads();
-    uint32_t excl = carry + (warp > 0 ? warp_tot[warp - 1] : 0u) + x - v;
-    if (i < total) h[i] = excl;
-    __syncthreads();
-    if (threadIdx.x == 0) carry += warp_tot[(blockDim.x >> 5) - 1];
-    __syncthreads();
+    uint32_t run = carry + (warp > 0 ? warp_tot[warp - 1] : 0u) + x - s;
+    if (mine) {
+#pragma unroll
+      for (int e = 0; e < kScanPer / 4; ++e) {
+        uint4 o;
+        o.x = run;
+        run += v[e].x;
+        o.y = run;
+        run += v[e].y;
+        o.z = run;
+        run += v[e].z;
+        o.w = run;
+        run += v[e].w;
+        reinterpret_cast<uint4*>(h + i0)[e] = o;
+      }
+    }
+    carry += warp_tot[31];
+    __syncthreads();  // warp_tot is rewritten by the next round
   }
 }
 
@@ -95,8 +116,8 @@ __global__ void __launch_bounds__(1024) radix_scan_kernel(uint32_t* __restrict__
 // ordered by digit in shared memory (stable ranks from per-warp counts), then
 // written out so that consecutive threads store consecutive positions of a
 // digit's run.  kFirst: the values are the key indices (vin is not read).
-template <bool kFirst>
-__global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(
+template <bool kFirst>  // at most 48 registers: five CTAs per SM to hide the load latency
+__global__ void __launch_bounds__(kSortThreads, 5) radix_scatter_kernel(
     const uint32_t* __restrict__ kin, const int32_t* __restrict__ vin, uint32_t* __restrict__ kout,
     int32_t* __restrict__ vout, int n, int tiles, int shift, const uint32_t* __restrict__ hist) {
   __shared__ uint32_t wcnt[kWarps][256];
