@@ -74,39 +74,6 @@ __device__ __forceinline__ Shear make_shear(const float2* cu, int b0, int b1) {
   return s;
 }
 
-// Tolerant monotone chain over the points produced by `next(i)` for
-// i = 0..count-1 (in increasing b); the stack lives in `st` (it may alias the
-// input region as long as it never overtakes it).  Returns the stack size.
-template <typename Next>
-__device__ __forceinline__ int tolerant_chain(const Shear& sh, int count, Next next, int32_t* st) {
-  int top = 0;
-  int xa = 0, xb = 0;
-  float ya = 0.f, yb = 0.f, da = 0.f, db = 0.f;
-  for (int i = 0; i < count; ++i) {
-    const int b = next(i);
-    float y, dy;
-    sh.at(b, y, dy);
-    while (top >= 2 && clearly_above(xa, ya, xb, yb, b, y, fmaxf(fmaxf(da, db), dy))) {
-      --top;
-      xb = xa;
-      yb = ya;
-      db = da;
-      if (top >= 2) {
-        xa = st[top - 2];
-        sh.at(xa, ya, da);
-      }
-    }
-    st[top++] = b;
-    xa = xb;
-    ya = yb;
-    da = db;
-    xb = b;
-    yb = y;
-    db = dy;
-  }
-  return top;
-}
-
 // Candidate counts per unit: [hull_segs] segment counts, then [groups] group
 // counts (see Layout::ncand).
 __device__ __forceinline__ int groups_of(const Prob& p) {
@@ -149,8 +116,9 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   const int b0 = p.b_min + seg * kHullSeg;
   const int b1 = min(n, b0 + kHullSeg);
   const Shear sh = make_shear(cu, b0, b1 - 1);
-  // the tolerant chain of tolerant_chain, with the sheared values of eight
-  // consecutive points evaluated ahead (their curve loads in flight together)
+  // tolerant monotone chain (a point is dropped only when clearly_above says
+  // so), with the sheared values of eight consecutive points evaluated ahead
+  // (their curve loads in flight together)
   // and kept on the thread-private stack next to b (as its offset in the
   // segment), so that a pop needs no reload.  Each test takes the largest
   // error bound of the points seen so far, at least that of its own three
@@ -183,7 +151,12 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   ncand[(size_t)u * ncand_stride(p) + seg] = top;
 }
 
-// grid = (ceil(groups / 128), units), one thread per group of segments.
+// grid = (ceil(groups / 128), units), one thread per group of segments.  The
+// tolerant chain over the segment survivors in order, eight points at a time:
+// their b, then their sheared values, each batch of loads in flight together.
+// The stack is the group's own candidate list (it never overtakes the read
+// position); a pop reloads the sheared value of the new top.  Each test takes
+// the largest error bound seen so far (the filter can only keep more).
 __global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* __restrict__ curve,
                                                          int32_t* __restrict__ cand,
                                                          int32_t* __restrict__ ncand) {
@@ -198,18 +171,44 @@ __global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* _
   const int b0 = p.b_min + s0 * kHullSeg;
   const int b1 = min(n, p.b_min + s1 * kHullSeg) - 1;
   const Shear sh = make_shear(cu, b0, b1);
-  int total = 0;
-  for (int s = s0; s < s1; ++s) total += nc[s];
-  // walk the segment survivors in order; the output compacts to the group start
-  int s = s0, i = 0;
-  auto next = [&](int) {
-    while (i >= nc[s]) {
-      ++s;
-      i = 0;
+  int32_t* st = cl + (size_t)s0 * kHullSeg;
+  int top = 0;
+  int xa = 0, xb = 0;
+  float ya = 0.f, yb = 0.f, dmax = 0.f;
+  for (int s = s0; s < s1; ++s) {
+    const int cnt = nc[s];
+    const int32_t* src = cl + (size_t)s * kHullSeg;
+    for (int i0 = 0; i0 < cnt; i0 += 8) {
+      int bv[8];
+      float yv[8], dv[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) bv[k] = (i0 + k < cnt) ? src[i0 + k] : 0;
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (i0 + k < cnt) sh.at(bv[k], yv[k], dv[k]);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (i0 + k >= cnt) break;
+        const int b = bv[k];
+        dmax = fmaxf(dmax, dv[k]);
+        while (top >= 2 && clearly_above(xa, ya, xb, yb, b, yv[k], dmax)) {
+          --top;
+          xb = xa;
+          yb = ya;
+          if (top >= 2) {
+            xa = st[top - 2];
+            float d;
+            sh.at(xa, ya, d);
+          }
+        }
+        st[top++] = b;  // top <= the points read so far: never past the read position
+        xa = xb;
+        ya = yb;
+        xb = b;
+        yb = yv[k];
+      }
     }
-    return cl[(size_t)s * kHullSeg + i++];
-  };
-  const int top = tolerant_chain(sh, total, next, cl + (size_t)s0 * kHullSeg);
+  }
   nc[p.hull_segs + g] = top;
 }
 
@@ -219,6 +218,7 @@ __global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* _
 // shared memory, refilled by the whole warp.
 constexpr int kCandCap = 12288;  // staged candidates: 96 KB of values + 48 KB of b (dynamic smem)
 constexpr int kScan = 2048;      // curve values per round of a block extension (16 KB)
+constexpr float kFilterTol = 9.5367432e-7f;  // 2^-20, eight times the fp32 error bound of f
 
 __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float2* __restrict__ curve,
                                                             const int32_t* __restrict__ cand,
@@ -234,7 +234,7 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
   __shared__ DF wbest_f[32];  // per-warp argmin, combined per head
   __shared__ int wbest_b[32], wbest_k[32];
   __shared__ double lam_sh[2];
-  __shared__ DF lam_df;  // the step's multiplier as double-float, for every warp
+  __shared__ DF lam_node[7];  // a round's multipliers as double-float, for every warp
   __shared__ float2 win[32][64];
   __shared__ float2 scanbuf[kScan];
   extern __shared__ __align__(16) char dyn[];
@@ -335,11 +335,20 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
   // so for lambda inside the bracket (lo, hi) it lies between the minimisers
   // found at hi and at lo: each head scans only that range of its candidates
   // (blo..bhi, as staged indices klo..khi).
-  const int wph = nwarps / H;  // >= 1 since H <= 32
-  auto scan_heads = [&]() {
-    const DF ld = lam_df;
-    const int h = warp / wph, sub = warp - h * wph;
-    if (h < H) {
+  // Each round evaluates the next `levels` bisection steps at once: the
+  // 2^levels - 1 midpoints they can visit (node 0 the bracket's midpoint, the
+  // children of node j the midpoints of its two half-brackets), computed from
+  // the round's bracket by the same float64 operations as one step at a time;
+  // warp 0 then follows the decisions down the tree.  Warps are shared out
+  // over (node, head) pairs, wpp warps per pair.
+  int max_levels = 1;
+  while (max_levels < 3 && ((2 << max_levels) - 1) * H <= nwarps) ++max_levels;
+  auto scan_heads = [&](int nodes) {
+    const int pairs = nodes * H, wpp = nwarps / pairs;
+    const int pi = warp / wpp, sub = warp - pi * wpp;
+    if (pi < pairs) {
+      const int node = pi / H, h = pi - node * H;
+      const DF ld = lam_node[node];
       const int u = bl * H + h;
       DF bf{INFINITY, 0.f};
       int bb = INT_MAX, bk = -1;
@@ -352,14 +361,26 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
         }
       };
       if (staged) {
-        const int k1 = khi[h];
-        for (int k = klo[h] + sub * 32 + lane; k <= k1; k += wph * 32) consider(cb_[k], cy[k], k);
+        // f = c(b) + lambda b >= 0; fp32 of the high parts is within 2^-23 f
+        // of it, so only candidates whose fp32 lower bound reaches the
+        // warp's least fp32 upper bound can be the warp's minimiser
+        const int k0 = klo[h] + sub * 32 + lane, k1 = khi[h];
+        float ub = INFINITY;
+        for (int k = k0; k <= k1; k += wpp * 32)
+          ub = fminf(ub, fmaf(ld.hi, (float)cb_[k], cy[k].x) * (1.0f + kFilterTol));
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) ub = fminf(ub, __shfl_xor_sync(kFull, ub, o));
+        for (int k = k0; k <= k1; k += wpp * 32) {
+          const int b = cb_[k];
+          const float2 c = cy[k];
+          if (fmaf(ld.hi, (float)b, c.x) * (1.0f - kFilterTol) <= ub) consider(b, c, k);
+        }
       } else {
         const int32_t* nc = ncand + (size_t)u * stride + p.hull_segs;
         const int32_t* cl = cand + (size_t)u * n;
         const int b_lo = blo[h], b_hi = bhi[h];
         for (int g = 0; g < groups; ++g)
-          for (int k = sub * 32 + lane; k < nc[g]; k += wph * 32) {
+          for (int k = sub * 32 + lane; k < nc[g]; k += wpp * 32) {
             const int b = cl[(size_t)g * kGroupSegs * kHullSeg + k];
             if (b >= b_lo && b <= b_hi) consider(b, curve[(size_t)u * n + b], -1);
           }
@@ -377,67 +398,88 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
       }
     }
   };
-  // warp 0, lane = head, after the scan: the head's minimiser b (b_min when it
-  // has no candidate) and its staged index k (-2: no candidate; -1: not staged)
-  auto combine = [&](int& b_out, int& k_out) {
+  // warp 0, lane = head, after a scan: the head's minimiser b at node `node`
+  // (b_min when it has no candidate) and its staged index k (-2: no
+  // candidate; -1: not staged)
+  auto combine = [&](int nodes, int node, int& b_out, int& k_out) {
+    const int wpp = nwarps / (nodes * H);
     DF bf{INFINITY, 0.f};
     int bb = INT_MAX, kk = -2;
     if (lane < H) {
-      for (int w = 0; w < wph; ++w) {
-        const DF f = wbest_f[lane * wph + w];
-        const int b = wbest_b[lane * wph + w];
+      const int w0 = (node * H + lane) * wpp;
+      for (int w = w0; w < w0 + wpp; ++w) {
+        const DF f = wbest_f[w];
+        const int b = wbest_b[w];
         if (df_less(f, bf) || (f.hi == bf.hi && f.lo == bf.lo && b < bb)) {
           bf = f;
           bb = b;
-          kk = wbest_k[lane * wph + w];
+          kk = wbest_k[w];
         }
       }
     }
     b_out = (bb == INT_MAX) ? p.b_min : bb;
     k_out = (bb == INT_MAX) ? -2 : kk;
   };
+  auto mid = [](double x, double y) { return __dmul_rn(__dadd_rn(x, y), 0.5); };
 
-  // float64 bisection of the multiplier in warp 0 (every lane holds the same
-  // bracket); the argmin runs in double-float on every warp
+  // the bracket lives in warp 0 (every lane holds the same values)
   double lam_lo = lam_sh[0], lam_hi = lam_sh[1];
-  if (threadIdx.x == 0) lam_df = df_from_double(__dmul_rn(__dadd_rn(lam_lo, lam_hi), 0.5));
-  __syncthreads();
-  for (int t = 0; lagrangian && t < p.T; ++t) {
-    scan_heads();
-    __syncthreads();
+  double node_lam[7];
+  for (int t = 0; lagrangian && t < p.T;) {
+    const int levels = min(max_levels, p.T - t);
+    const int nodes = (1 << levels) - 1;
     if (warp == 0) {
-      int bh, kh;
-      combine(bh, kh);
-      long long tot = lane < H ? bh : 0;
-#pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) tot += __shfl_xor_sync(kFull, tot, o);
-      const double lam = __dmul_rn(__dadd_rn(lam_lo, lam_hi), 0.5);
-      const bool up = tot > B_real;
-      if (up) lam_lo = lam; else lam_hi = lam;
-      // the new bracket end's minimisers bound the next scans
-      if (lane < H && kh != -2) {
-        if (up) {
-          bhi[lane] = bh;
-          if (staged) khi[lane] = kh;
-        } else {
-          blo[lane] = bh;
-          if (staged) klo[lane] = kh;
-        }
+      node_lam[0] = mid(lam_lo, lam_hi);
+      if (levels >= 2) {
+        node_lam[1] = mid(lam_lo, node_lam[0]);
+        node_lam[2] = mid(node_lam[0], lam_hi);
+      }
+      if (levels >= 3) {
+        node_lam[3] = mid(lam_lo, node_lam[1]);
+        node_lam[4] = mid(node_lam[1], node_lam[0]);
+        node_lam[5] = mid(node_lam[0], node_lam[2]);
+        node_lam[6] = mid(node_lam[2], lam_hi);
       }
       if (lane == 0)
-        lam_df = (t + 1 < p.T) ? df_from_double(__dmul_rn(__dadd_rn(lam_lo, lam_hi), 0.5))
-                               : df_from_double(lam_hi);
+        for (int j = 0; j < nodes; ++j) lam_node[j] = df_from_double(node_lam[j]);
     }
     __syncthreads();
+    scan_heads(nodes);
+    __syncthreads();
+    if (warp == 0) {
+      int j = 0;
+      for (int l = 0; l < levels; ++l) {
+        int bh, kh;
+        combine(nodes, j, bh, kh);
+        long long tot = lane < H ? bh : 0;
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) tot += __shfl_xor_sync(kFull, tot, o);
+        const bool up = tot > B_real;
+        if (up) lam_lo = node_lam[j]; else lam_hi = node_lam[j];
+        // the new bracket end's minimisers bound the next scans
+        if (lane < H && kh != -2) {
+          if (up) {
+            bhi[lane] = bh;
+            if (staged) khi[lane] = kh;
+          } else {
+            blo[lane] = bh;
+            if (staged) klo[lane] = kh;
+          }
+        }
+        j = 2 * j + (up ? 2 : 1);
+      }
+    }
+    t += levels;
+    __syncthreads();
   }
-  if (p.T == 0 && threadIdx.x == 0) lam_df = df_from_double(lam_hi);
-  __syncthreads();
-  if (lagrangian) {
-    scan_heads();
+  if (lagrangian) {  // the minimisers at lambda_hi
+    if (threadIdx.x == 0) lam_node[0] = df_from_double(lam_hi);
+    __syncthreads();
+    scan_heads(1);
     __syncthreads();
     if (warp == 0) {
       int bh, kh;
-      combine(bh, kh);
+      combine(1, 0, bh, kh);
       if (lane < H) bsel[lane] = bh;
     }
   } else if (threadIdx.x < H) {  // the allocator ablations' starting points
@@ -553,29 +595,32 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
       while (more) {  // warp-cooperative scan, kScan values per round
         extended = true;
         __syncwarp();
-        for (int k = lane; k < kScan; k += 32)
-          scanbuf[k] = (bw + 1 + k < n) ? ch[bw + 1 + k] : make_float2(0.f, 0.f);
+        // every value of the round in flight at once (8-byte asynchronous copies)
+        const uint32_t sbuf = (uint32_t)__cvta_generic_to_shared(scanbuf);
+        for (int k = lane; k < kScan; k += 32) {
+          if (bw + 1 + k < n)
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(sbuf + (uint32_t)k * 8u),
+                         "l"(ch + bw + 1 + k)
+                         : "memory");
+          else
+            scanbuf[k] = make_float2(0.f, 0.f);
+        }
+        asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
         __syncwarp();
-        // lane L checks positions e = 64 L .. 64 L + 63: marginal c(bw+e+1) - c(bw+e)
-        int first = 64;
-        for (int i = 0; i < 64; ++i) {
-          const int e = lane * 64 + i;
+        // positions e = 32 i + lane in order, 32 per ballot, up to the first
+        // marginal c(bw+e+1) - c(bw+e) that is not below the front
+        int run = kScan;
+        for (int i = 0; i < kScan / 32; ++i) {
+          const int e = i * 32 + lane;
           const float2 pv = (e == 0) ? make_float2(cw.hi, cw.lo) : scanbuf[e - 1];
           const float2 nv = scanbuf[e];
           const DF d = df_add(DF{nv.x, nv.y}, df_neg(DF{pv.x, pv.y}));
           const bool stop = (bw + e >= n - 1) || !df_less(d, mg);
-          if (stop) {
-            first = i;
+          const unsigned stops = __ballot_sync(kFull, stop);
+          if (stops) {
+            run = i * 32 + __ffs(stops) - 1;
             break;
           }
-        }
-        const unsigned stops = __ballot_sync(kFull, first < 64);
-        int run = kScan;
-        if (stops) {
-          const int L = __ffs(stops) - 1;
-          run = L * 64 + __shfl_sync(kFull, first, L);
-        } else {
-          __shfl_sync(kFull, first, 0);
         }
         const int64_t room = B_real - tot;
         if ((int64_t)run > room) run = (int)room;
