@@ -129,10 +129,11 @@ def kernel_work(wl, B_live, name):
         return dict(bytes=kbytes if name == "score_pass1" else 0, flops=flops)
     if name == "curve_agg":
         return dict(bytes=2 * kbytes, flops=0)       # K and V rows gathered by rank
-    if name == "curve_eval":
-        return dict(bytes=kbytes, flops=0)           # V rows gathered again
-    if name == "sort_scatter":
-        return dict(bytes=U * n * 16, flops=0)       # one digit pass: key + value in and out
+    if name == "curve_eval":                         # V rows gathered again, every chunk
+        last = n - ((n - 1) // 128) * 128            # of 128 ranks but the last (its own launch)
+        return dict(bytes=U * (n - last) * d * 2, flops=0)
+    if name == "sort_scatter":                       # a digit pass: key + value in and out,
+        return dict(bytes=U * n * 15, flops=0)       # pass 0 reads no values (mean of 4 passes)
     if name == "copy_rows":
         slots = wl.B * wl.L * (B_live - wl.H)
         return dict(bytes=slots * d * 2 * 2 * 2, flops=0)

@@ -209,20 +209,256 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
   if (lane == 0) agg_mq[ci] = make_float4(m.hi, m.lo, q.hi, q.lo);
 }
 
-// grid = (units, need_k ? 2 : 1), block = 160: exclusive suffix sums over
-// chunks in double-float, folded from the last chunk down in chunk order.
+// One warp evaluates chunk `chunk` of unit u.  The V rows of the chunk are
+// staged in groups of 8 ranks (descending) through the warp's ring in shared
+// memory (ring_w, kEvalRing groups), kEvalAhead groups ahead of the
+// evaluation; sa, sj, sy hold the chunk's scores, token indices and ||v||^2.
+// kLast: the unit's last chunk (W_base = 0), in double-float.
+struct EvalArgs {
+  const uint32_t* keys;
+  const int32_t* perm;
+  const __nv_bfloat16* V;
+  const float2* yrank;
+  const float4* base_mq;
+  const float2* base_v;
+  float2* curve;
+  unsigned long long* cmax;
+  uint32_t* status;
+};
+template <bool kLast>
+__device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, int chunk, int u,
+                                           int lane, unsigned char* ring_w, float* sa, int* sj,
+                                           float2* sy) {
+  const uint32_t* __restrict__ keys = ea.keys;
+  const int32_t* __restrict__ perm = ea.perm;
+  const __nv_bfloat16* __restrict__ V = ea.V;
+  const float2* __restrict__ yrank = ea.yrank;
+  const float4* __restrict__ base_mq = ea.base_mq;
+  const float2* __restrict__ base_v = ea.base_v;
+  float2* __restrict__ curve = ea.curve;
+  unsigned long long* __restrict__ cmax = ea.cmax;
+  uint32_t* status = ea.status;
+  const int n = p.n;
+  const int r0 = chunk * kChunk, r1 = min(n, r0 + kChunk);
+  const uint32_t* ku = keys + (size_t)u * n;
+  const int32_t* pu = perm + (size_t)u * n;
+  const unsigned char* Vu = reinterpret_cast<const unsigned char*>(V + (size_t)u * n * kD);
+  const size_t ci = (size_t)u * p.chunks + chunk;
+  const uint32_t ring = (uint32_t)__cvta_generic_to_shared(ring_w);
+
+  // per-rank scalars of the whole chunk (zero past the end)
+#pragma unroll
+  for (int e = 0; e < kChunk / 32; ++e) {
+    const int r = r0 + e * 32 + lane;
+    const bool ok = r < r1;
+    sa[e * 32 + lane] = ok ? key_score(ku[r]) : 0.f;
+    sj[e * 32 + lane] = ok ? pu[r] : 0;
+    sy[e * 32 + lane] = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
+  }
+  __syncwarp();
+  const int nb = (r1 - r0 + 31) / 32;
+  const int ngroups = nb * 4;  // group g: ranks r0 + 32*(nb-1-g/4) + 24 - 8*(g%4) + 0..7
+  // lane l copies 16-byte piece (l & 15) of rows (l >> 4) + 2k, k = 0..3
+  auto stage = [&](int g) {
+    if (g < ngroups) {
+      const int rl = 32 * (nb - 1 - g / 4) + 24 - 8 * (g % 4);  // first rank of the group, chunk-local
+      const uint32_t dst = ring + (uint32_t)((g % kEvalRing) * kEvalGroupBytes);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int t = (lane >> 4) + 2 * k;
+        if (r0 + rl + t < r1)
+          cp_async16(dst + t * (kD * 2) + (lane & 15) * 16,
+                     Vu + (size_t)sj[rl + t] * (kD * 2) + (lane & 15) * 16);
+      }
+    }
+    cp_async_commit();
+  };
+#pragma unroll
+  for (int g = 0; g < kEvalAhead; ++g) stage(g);
+
+  // the sums over the ranks after the chunk (zero after the last chunk, which
+  // runs alongside the kernel that writes them and so must not read them)
+  const float4 bmq = kLast ? make_float4(0.f, 0.f, 0.f, 0.f) : base_mq[ci];
+  const DF M0{bmq.x, bmq.y}, Q0{bmq.z, bmq.w};
+  float wb2x[4] = {0.f, 0.f, 0.f, 0.f};
+  DF wb2 = df_make(0.f);
+  if constexpr (!kLast) {
+    const float4* bv = reinterpret_cast<const float4*>(base_v + ci * kD) + lane * 2;
+    float4 x0 = bv[0], x1 = bv[1];
+    const float hi[4] = {x0.x, x0.z, x1.x, x1.z}, lo[4] = {x0.y, x0.w, x1.y, x1.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      wb2x[i] = 2.0f * hi[i];
+      DF sq = two_prod(hi[i], hi[i]);
+      sq = df_add_f(sq, 2.0f * hi[i] * lo[i]);
+      wb2 = df_add(wb2, sq);
+    }
+    wb2 = warp_sum_df(wb2);
+  }
+  // The last chunk has W_base = 0 and a vanishing tail, so c(b)^2 there is a
+  // small difference of small terms: its partial sums run in double-float.
+  constexpr bool exact = kLast;  // the last chunk: W_base = 0, in double-float
+  float P[4] = {0.f, 0.f, 0.f, 0.f};
+  DF Pd[4] = {df_make(0.f), df_make(0.f), df_make(0.f), df_make(0.f)};
+  DF base_m = M0, base_q = Q0;  // sums over the ranks after the current batch
+  unsigned long long best = 0ull;
+  bool bad = false;
+  DF xt = df_make(0.f);  // lane r: ||W_base + P(b)||^2 - ||W_base||^2 for rank r of the batch
+  DF yt = df_make(0.f);  // lane r: ||v||^2 of rank r of the batch (last chunk only)
+  for (int g = 0; g < ngroups; ++g) {
+    stage(g + kEvalAhead);
+    asm volatile("cp.async.wait_group %0;" ::"n"(kEvalAhead) : "memory");
+    __syncwarp();
+    const int bi = nb - 1 - g / 4;
+    const int s0 = 24 - 8 * (g % 4);
+    const int rl = 32 * bi + s0;
+    const int cnt = r1 - (r0 + rl);  // rows of the group that exist (may exceed 8)
+    const unsigned char* rows = ring_w + (g % kEvalRing) * kEvalGroupBytes;
+    if constexpr (!exact) {
+      // dimension pairs (0,1) and (2,3) of this lane in two-wide arithmetic
+      float2 P01 = make_float2(P[0], P[1]), P23 = make_float2(P[2], P[3]);
+      const float2 W01 = make_float2(wb2x[0], wb2x[1]), W23 = make_float2(wb2x[2], wb2x[3]);
+      float xg[8];
+#pragma unroll
+      for (int t = 7; t >= 0; --t) {
+        const float as = sa[rl + t];
+        uint2 raw = make_uint2(0u, 0u);
+        if (t < cnt) raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
+        const float2 a2 = make_float2(as, as);
+        P01 = ffma2(a2, make_float2(bf16lo(raw.x), bf16hi(raw.x)), P01);
+        P23 = ffma2(a2, make_float2(bf16lo(raw.y), bf16hi(raw.y)), P23);
+        const float2 acc = ffma2(fadd2(W23, P23), P23, fmul2(fadd2(W01, P01), P01));
+        xg[t] = (t < cnt) ? acc.x + acc.y : 0.f;
+      }
+      P[0] = P01.x;
+      P[1] = P01.y;
+      P[2] = P23.x;
+      P[3] = P23.y;
+      const float x = reduce8(xg, lane);
+      if ((lane >> 3) == (s0 >> 3)) xt = df_make(x);
+    } else {
+      // ||v||^2 is also recomputed here in double-float (the per-rank values
+      // of curve_agg sum each lane's four squares in fp32, which rounds when
+      // their magnitudes spread over more than 24 bits): near b = n - 1 the
+      // tail holds a few tokens and m Q - ||W||^2 cancels to ~0, so Q and W
+      // must see the same ||v||^2
+      DF xg[8], yg[8];
+#pragma unroll
+      for (int t = 7; t >= 0; --t) {
+        const float as = sa[rl + t];
+        xg[t] = df_make(0.f);
+        yg[t] = df_make(0.f);
+        if (t < cnt) {
+          const uint2 raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
+          const float v[4] = {bf16lo(raw.x), bf16hi(raw.x), bf16lo(raw.y), bf16hi(raw.y)};
+          DF acc = df_make(0.f);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            Pd[i] = df_add(Pd[i], two_prod(as, v[i]));
+            acc = df_add(acc, df_mul(Pd[i], Pd[i]));
+          }
+          xg[t] = acc;
+          // squares of bf16 values are exact in fp32
+          yg[t] = df_add(two_sum(v[0] * v[0], v[1] * v[1]), two_sum(v[2] * v[2], v[3] * v[3]));
+        }
+      }
+      const DF x = reduce8_df(xg, lane);
+      const DF y = reduce8_df(yg, lane);
+      if ((lane >> 3) == (s0 >> 3)) {
+        xt = x;
+        yt = y;
+      }
+    }
+    __syncwarp();  // the ring slot of group g is free once every lane has read it
+    if (s0 != 0) continue;
+
+    // ---- end of batch bi: the curve at its 32 ranks ----
+    const int r = r0 + 32 * bi + lane;
+    const bool ok = r < r1;
+    const float at = sa[32 * bi + lane];
+    const float2 yv = sy[32 * bi + lane];
+    // in-batch inclusive suffix sums over lanes >= t (a and a||v||^2 are
+    // non-negative: same-sign double-float additions)
+    DF sm = df_make(at);
+    DF sq = ok ? df_mul_f(exact ? yt : DF{yv.x, yv.y}, at) : df_make(0.f);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      DF om{__shfl_down_sync(kFull, sm.hi, o), __shfl_down_sync(kFull, sm.lo, o)};
+      DF oq{__shfl_down_sync(kFull, sq.hi, o), __shfl_down_sync(kFull, sq.lo, o)};
+      if (lane + o < 32) {
+        sm = df_add_same_sign(sm, om);
+        sq = df_add_same_sign(sq, oq);
+      }
+    }
+    const DF Mt = df_add_same_sign(base_m, sm);
+    const DF Qt = df_add_same_sign(base_q, sq);
+    DF c;
+    if (p.statistic == 2) {
+      c = Mt;
+    } else if (p.statistic == 1) {
+      c = df_sqrt_newton(df_mul(Mt, Qt));
+    } else {
+      const DF W2 = df_add(wb2, xt);
+      c = df_sqrt_newton(df_add(df_mul(Mt, Qt), df_neg(W2)));
+    }
+    if (ok) {
+      curve[(size_t)u * n + r] = make_float2(c.hi, c.lo);
+      if (!(c.hi <= 3.0e38f)) bad = true;
+      unsigned long long k = df_order_key(c);
+      best = k > best ? k : best;
+    }
+    base_m = df_add_same_sign(base_m, shfl_df(sm, 0));
+    base_q = df_add_same_sign(base_q, shfl_df(sq, 0));
+  }
+  asm volatile("cp.async.wait_all;" ::: "memory");
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    unsigned long long other = __shfl_xor_sync(kFull, best, o);
+    best = other > best ? other : best;
+  }
+  if (lane == 0) atomicMax(cmax + u, best);
+  if (__any_sync(kFull, bad) && lane == 0) raise_status(status, 1u);
+}
+
+// grid = (ceil(chunks / 4), units), block = 128: warp w of block x takes chunk
+// 4x + w, every chunk but the last (curve_prefix_kernel takes the last ones).
+__global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, EvalArgs ea) {
+  __shared__ __align__(16) unsigned char s_ring[4][kEvalRing][kEvalGroupBytes];
+  __shared__ float s_a[4][kChunk];
+  __shared__ int s_j[4][kChunk];
+  __shared__ float2 s_y[4][kChunk];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int chunk = blockIdx.x * 4 + warp;
+  if (chunk >= p.chunks - 1) return;
+  eval_chunk<false>(p, ea, chunk, blockIdx.y, lane, s_ring[warp][0], s_a[warp], s_j[warp],
+                    s_y[warp]);
+}
+
+// grid = (units, (need_k ? 2 : 1) + 1), block = 160: exclusive suffix sums
+// over chunks in double-float, folded from the last chunk down in chunk order.
 // Threads 0..127 take one dimension of the V sums (blockIdx.y = 0) or of the K
 // sums (blockIdx.y = 1), with the next kPrefixBlock chunks' loads in flight
 // while the current ones are folded; warp 4 of the V block takes the scalar
-// sums m and Q, one chunk per lane per round.
+// sums m and Q, one chunk per lane per round.  In the last y slice, warp 0
+// evaluates the unit's last chunk of ranks instead (its W_base, m and Q bases
+// are zero, so it needs none of these sums), in double-float, alongside.
 constexpr int kPrefixBlock = 32;
 __global__ void __launch_bounds__(160) curve_prefix_kernel(Prob p, const float4* __restrict__ agg_mq,
                                                            const float* __restrict__ agg_v,
                                                            const float* __restrict__ agg_k,
                                                            float4* __restrict__ base_mq,
                                                            float2* __restrict__ base_v,
-                                                           float2* __restrict__ base_k) {
+                                                           float2* __restrict__ base_k,
+                                                           EvalArgs ea) {
   const int u = blockIdx.x;
+  if (blockIdx.y == gridDim.y - 1) {
+    __shared__ __align__(16) unsigned char l_ring[kEvalRing][kEvalGroupBytes];
+    __shared__ float l_a[kChunk];
+    __shared__ int l_j[kChunk];
+    __shared__ float2 l_y[kChunk];
+    if (threadIdx.x < 32) eval_chunk<true>(p, ea, p.chunks - 1, u, threadIdx.x, l_ring[0], l_a, l_j, l_y);
+    return;
+  }
   const int chunks = p.chunks;
   const size_t c0 = (size_t)u * chunks;
   if (threadIdx.x >= kD) {
@@ -270,196 +506,6 @@ __global__ void __launch_bounds__(160) curve_prefix_kernel(Prob p, const float4*
       r = df_add_f(r, cur[e]);
     }
   }
-}
-
-// grid = (ceil(chunks / 4), units), block = 128 (one warp per chunk).  The V
-// rows of a chunk are staged in groups of 8 ranks (descending) through a
-// per-warp ring in shared memory, kEvalAhead groups ahead of the evaluation.
-__global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, const uint32_t* __restrict__ keys,
-                                                         const int32_t* __restrict__ perm,
-                                                         const __nv_bfloat16* __restrict__ V,
-                                                         const float2* __restrict__ yrank,
-                                                         const float4* __restrict__ base_mq,
-                                                         const float2* __restrict__ base_v,
-                                                         float2* __restrict__ curve,
-                                                         unsigned long long* __restrict__ cmax,
-                                                         uint32_t* status) {
-  __shared__ __align__(16) unsigned char s_ring[4][kEvalRing][kEvalGroupBytes];
-  __shared__ float s_a[4][kChunk];
-  __shared__ int s_j[4][kChunk];
-  __shared__ float2 s_y[4][kChunk];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int chunk = blockIdx.x * 4 + warp;
-  const int u = blockIdx.y;
-  if (chunk >= p.chunks) return;
-  const int n = p.n;
-  const int r0 = chunk * kChunk, r1 = min(n, r0 + kChunk);
-  const uint32_t* ku = keys + (size_t)u * n;
-  const int32_t* pu = perm + (size_t)u * n;
-  const unsigned char* Vu = reinterpret_cast<const unsigned char*>(V + (size_t)u * n * kD);
-  const size_t ci = (size_t)u * p.chunks + chunk;
-  float* sa = s_a[warp];
-  int* sj = s_j[warp];
-  float2* sy = s_y[warp];
-  const uint32_t ring = (uint32_t)__cvta_generic_to_shared(s_ring[warp][0]);
-
-  // per-rank scalars of the whole chunk (zero past the end)
-#pragma unroll
-  for (int e = 0; e < kChunk / 32; ++e) {
-    const int r = r0 + e * 32 + lane;
-    const bool ok = r < r1;
-    sa[e * 32 + lane] = ok ? key_score(ku[r]) : 0.f;
-    sj[e * 32 + lane] = ok ? pu[r] : 0;
-    sy[e * 32 + lane] = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
-  }
-  __syncwarp();
-  const int nb = (r1 - r0 + 31) / 32;
-  const int ngroups = nb * 4;  // group g: ranks r0 + 32*(nb-1-g/4) + 24 - 8*(g%4) + 0..7
-  // lane l copies 16-byte piece (l & 15) of rows (l >> 4) + 2k, k = 0..3
-  auto stage = [&](int g) {
-    if (g < ngroups) {
-      const int rl = 32 * (nb - 1 - g / 4) + 24 - 8 * (g % 4);  // first rank of the group, chunk-local
-      const uint32_t dst = ring + (uint32_t)((g % kEvalRing) * kEvalGroupBytes);
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int t = (lane >> 4) + 2 * k;
-        if (r0 + rl + t < r1)
-          cp_async16(dst + t * (kD * 2) + (lane & 15) * 16,
-                     Vu + (size_t)sj[rl + t] * (kD * 2) + (lane & 15) * 16);
-      }
-    }
-    cp_async_commit();
-  };
-#pragma unroll
-  for (int g = 0; g < kEvalAhead; ++g) stage(g);
-
-  const float4 bmq = base_mq[ci];
-  const DF M0{bmq.x, bmq.y}, Q0{bmq.z, bmq.w};
-  float wb2x[4];
-  DF wb2 = df_make(0.f);
-  {
-    const float4* bv = reinterpret_cast<const float4*>(base_v + ci * kD) + lane * 2;
-    float4 x0 = bv[0], x1 = bv[1];
-    const float hi[4] = {x0.x, x0.z, x1.x, x1.z}, lo[4] = {x0.y, x0.w, x1.y, x1.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      wb2x[i] = 2.0f * hi[i];
-      DF sq = two_prod(hi[i], hi[i]);
-      sq = df_add_f(sq, 2.0f * hi[i] * lo[i]);
-      wb2 = df_add(wb2, sq);
-    }
-    wb2 = warp_sum_df(wb2);
-  }
-  // The last chunk has W_base = 0 and a vanishing tail, so c(b)^2 there is a
-  // small difference of small terms: its partial sums run in double-float.
-  const bool exact = (chunk == p.chunks - 1);
-  float P[4] = {0.f, 0.f, 0.f, 0.f};
-  DF Pd[4] = {df_make(0.f), df_make(0.f), df_make(0.f), df_make(0.f)};
-  DF base_m = M0, base_q = Q0;  // sums over the ranks after the current batch
-  unsigned long long best = 0ull;
-  bool bad = false;
-  DF xt = df_make(0.f);  // lane r: ||W_base + P(b)||^2 - ||W_base||^2 for rank r of the batch
-  for (int g = 0; g < ngroups; ++g) {
-    stage(g + kEvalAhead);
-    asm volatile("cp.async.wait_group %0;" ::"n"(kEvalAhead) : "memory");
-    __syncwarp();
-    const int bi = nb - 1 - g / 4;
-    const int s0 = 24 - 8 * (g % 4);
-    const int rl = 32 * bi + s0;
-    const int cnt = r1 - (r0 + rl);  // rows of the group that exist (may exceed 8)
-    const unsigned char* rows = s_ring[warp][g % kEvalRing];
-    if (!exact) {
-      // dimension pairs (0,1) and (2,3) of this lane in two-wide arithmetic
-      float2 P01 = make_float2(P[0], P[1]), P23 = make_float2(P[2], P[3]);
-      const float2 W01 = make_float2(wb2x[0], wb2x[1]), W23 = make_float2(wb2x[2], wb2x[3]);
-      float xg[8];
-#pragma unroll
-      for (int t = 7; t >= 0; --t) {
-        const float as = sa[rl + t];
-        uint2 raw = make_uint2(0u, 0u);
-        if (t < cnt) raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
-        const float2 a2 = make_float2(as, as);
-        P01 = ffma2(a2, make_float2(bf16lo(raw.x), bf16hi(raw.x)), P01);
-        P23 = ffma2(a2, make_float2(bf16lo(raw.y), bf16hi(raw.y)), P23);
-        const float2 acc = ffma2(fadd2(W23, P23), P23, fmul2(fadd2(W01, P01), P01));
-        xg[t] = (t < cnt) ? acc.x + acc.y : 0.f;
-      }
-      P[0] = P01.x;
-      P[1] = P01.y;
-      P[2] = P23.x;
-      P[3] = P23.y;
-      const float x = reduce8(xg, lane);
-      if ((lane >> 3) == (s0 >> 3)) xt = df_make(x);
-    } else {
-      DF xg[8];
-#pragma unroll
-      for (int t = 7; t >= 0; --t) {
-        const float as = sa[rl + t];
-        xg[t] = df_make(0.f);
-        if (t < cnt) {
-          const uint2 raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
-          const float v[4] = {bf16lo(raw.x), bf16hi(raw.x), bf16lo(raw.y), bf16hi(raw.y)};
-          DF acc = df_make(0.f);
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            Pd[i] = df_add(Pd[i], two_prod(as, v[i]));
-            acc = df_add(acc, df_mul(Pd[i], Pd[i]));
-          }
-          xg[t] = acc;
-        }
-      }
-      const DF x = reduce8_df(xg, lane);
-      if ((lane >> 3) == (s0 >> 3)) xt = x;
-    }
-    __syncwarp();  // the ring slot of group g is free once every lane has read it
-    if (s0 != 0) continue;
-
-    // ---- end of batch bi: the curve at its 32 ranks ----
-    const int r = r0 + 32 * bi + lane;
-    const bool ok = r < r1;
-    const float at = sa[32 * bi + lane];
-    const float2 yv = sy[32 * bi + lane];
-    // in-batch inclusive suffix sums over lanes >= t (a and a||v||^2 are
-    // non-negative: same-sign double-float additions)
-    DF sm = df_make(at);
-    DF sq = ok ? df_mul_f(DF{yv.x, yv.y}, at) : df_make(0.f);
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      DF om{__shfl_down_sync(kFull, sm.hi, o), __shfl_down_sync(kFull, sm.lo, o)};
-      DF oq{__shfl_down_sync(kFull, sq.hi, o), __shfl_down_sync(kFull, sq.lo, o)};
-      if (lane + o < 32) {
-        sm = df_add_same_sign(sm, om);
-        sq = df_add_same_sign(sq, oq);
-      }
-    }
-    const DF Mt = df_add_same_sign(base_m, sm);
-    const DF Qt = df_add_same_sign(base_q, sq);
-    DF c;
-    if (p.statistic == 2) {
-      c = Mt;
-    } else if (p.statistic == 1) {
-      c = df_sqrt_newton(df_mul(Mt, Qt));
-    } else {
-      const DF W2 = df_add(wb2, xt);
-      c = df_sqrt_newton(df_add(df_mul(Mt, Qt), df_neg(W2)));
-    }
-    if (ok) {
-      curve[(size_t)u * n + r] = make_float2(c.hi, c.lo);
-      if (!(c.hi <= 3.0e38f)) bad = true;
-      unsigned long long k = df_order_key(c);
-      best = k > best ? k : best;
-    }
-    base_m = df_add_same_sign(base_m, shfl_df(sm, 0));
-    base_q = df_add_same_sign(base_q, shfl_df(sq, 0));
-  }
-  asm volatile("cp.async.wait_all;" ::: "memory");
-#pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) {
-    unsigned long long other = __shfl_xor_sync(kFull, best, o);
-    best = other > best ? other : best;
-  }
-  if (lane == 0) atomicMax(cmax + u, best);
-  if (__any_sync(kFull, bad) && lane == 0) raise_status(status, 1u);
 }
 
 __global__ void cmax_clear_kernel(unsigned long long* cmax, int units) {
@@ -512,15 +558,16 @@ void launch_curves(const Prob& p, const Layout& ly, char* ws, const void* K, con
     curve_agg_kernel<<<grid, 128, kAggSmemBytes, st>>>(p, keys, perm, Kb, Vb, need_k, agg_mq, agg_v, agg_k,
                                            yrank);
   }
+  const EvalArgs ea{keys,    perm,  Vb,   yrank, base_mq, base_v,
+                    curve,   cmax,  reinterpret_cast<uint32_t*>(ws + ly.status)};
   {
     TraceScope ts_("curve_prefix", st);
-    curve_prefix_kernel<<<dim3(p.units, need_k ? 2 : 1), 160, 0, st>>>(p, agg_mq, agg_v, agg_k,
-                                                                        base_mq, base_v, base_k);
+    curve_prefix_kernel<<<dim3(p.units, (need_k ? 2 : 1) + 1), 160, 0, st>>>(
+        p, agg_mq, agg_v, agg_k, base_mq, base_v, base_k, ea);
   }
   {
     TraceScope ts_("curve_eval", st);
-    curve_eval_kernel<<<grid, 128, 0, st>>>(p, keys, perm, Vb, yrank, base_mq, base_v, curve, cmax,
-                                            reinterpret_cast<uint32_t*>(ws + ly.status));
+    curve_eval_kernel<<<grid, 128, 0, st>>>(p, ea);
   }
 }
 

@@ -10,10 +10,23 @@ PEAKS = dict(hbm=6768.8, tensor=1732.7, source="measured")
 def test_sort_pass_work_is_per_launch():
     wl = W.WORKLOADS["C3"]
     work = bench.kernel_work(wl, wl.B_live, "sort_scatter")
-    assert work["bytes"] == wl.units * wl.n * 16  # keys and indices, read and written once
+    # keys and indices read and written once per pass, except the indices of
+    # pass 0 (the token indices themselves): 15 B per key per pass on average
+    assert work["bytes"] == wl.units * wl.n * 15
     r = bench.roofline_for("sort_scatter", work, 0.25, PEAKS)
     assert r["bound"] == "hbm"
     assert abs(r["achieved"] - work["bytes"] / 0.25e-3 / 1e9) < 0.1
+
+
+def test_eval_work_leaves_out_the_last_chunk():
+    """curve_eval's main launch covers every 128-rank chunk but the last, which
+    has its own launch."""
+    wl = W.WORKLOADS["C3"]
+    work = bench.kernel_work(wl, wl.B_live, "curve_eval")
+    assert work["bytes"] == wl.units * (wl.n - 128) * wl.d * 2
+    small = W.WORKLOADS["C1"].with_(n=1000)
+    assert bench.kernel_work(small, small.B_live, "curve_eval")["bytes"] == \
+        small.units * (1000 - 1000 % 128) * small.d * 2
 
 
 def test_decode_work_is_one_step():

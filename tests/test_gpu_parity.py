@@ -34,6 +34,15 @@ CASES = {
                                kind="zipf"),
     "rows768_planted": W.Workload("P7", B=1, L=1, Hq=32, H=2, n=3333, d=128, w=48, keep=(1, 8),
                                   kind="planted"),
+    # head counts that change the allocator's work split: one KV head (three
+    # bisection steps per round), 16 and 32 heads (one step per round, one
+    # warp per head at 32)
+    "mqa_h1": W.Workload("Q1", B=1, L=1, Hq=8, H=1, n=2600, d=128, w=16, keep=(1, 10),
+                         kind="zipf"),
+    "heads16": W.Workload("H16", B=1, L=1, Hq=16, H=16, n=1200, d=128, w=8, keep=(1, 6),
+                          kind="planted"),
+    "heads32": W.Workload("H32", B=1, L=1, Hq=32, H=32, n=700, d=128, w=4, keep=(1, 5),
+                          kind="student_t"),
 }
 
 _cache = {}
