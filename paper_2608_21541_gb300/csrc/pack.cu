@@ -42,14 +42,34 @@ __global__ void __launch_bounds__(128) tail_kernel(
   DF tv{t.x, t.y};
   t = base_k[ci * kD + i];
   DF tk{t.x, t.y};
-  for (int r = b; r < r_end; ++r) {
-    const float a = key_score(ku[r]);
-    const int j = pu[r];
-    const float v = __bfloat162float(Vu[(size_t)j * kD + i]);
-    const float k = __bfloat162float(Ku[(size_t)j * kD + i]);
-    m = df_add_f(m, a);
-    tv = df_add(tv, two_prod(a, v));
-    tk = df_add(tk, two_prod(a, k));
+  // the partial chunk's scores and token indices staged once; then the K and
+  // V values of eight ranks at a time in flight, summed in rank order
+  __shared__ float s_a[kChunk];
+  __shared__ int s_j[kChunk];
+  if (b + i < r_end) {
+    s_a[i] = key_score(ku[b + i]);
+    s_j[i] = pu[b + i];
+  }
+  __syncthreads();
+  for (int r0 = b; r0 < r_end; r0 += 8) {
+    float vv[8], kv[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      vv[e] = kv[e] = 0.f;
+      if (r0 + e < r_end) {
+        const size_t o = (size_t)s_j[r0 + e - b] * kD + i;
+        vv[e] = __bfloat162float(Vu[o]);
+        kv[e] = __bfloat162float(Ku[o]);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      if (r0 + e >= r_end) break;
+      const float a = s_a[r0 + e - b];
+      m = df_add_f(m, a);
+      tv = df_add(tv, two_prod(a, vv[e]));
+      tk = df_add(tk, two_prod(a, kv[e]));
+    }
   }
   DF ks, vs;
   if (m.hi > 0.0f) {
@@ -439,6 +459,7 @@ void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const
     TraceScope ts("select", st);
     select_kernel<<<p.units, 1024, 0, st>>>(p, a, keys, perm, counts, offsets, positions, status);
   }
+
   int ysplit = (p.n + 15) / 16;
   if (ysplit > 64) ysplit = 64;
   {
