@@ -220,6 +220,27 @@ int certkv_compress_host(const certkv_shape* shape, const void* hK, const void* 
                          int32_t chunk, certkv_packed* out, void* workspace,
                          size_t workspace_bytes, void* stream);
 
+/* certkv_compress_host, with the packed cache also copied back to host memory
+ * chunk by chunk (a runtime convenience): as soon as a chunk of (sequence,
+ * layer) pairs is compressed, its slots [bl0 * budget_live, (bl0 + cnt) *
+ * budget_live) of k, v and positions, and its entries of real_counts and
+ * offsets (with the final offset after the last chunk), are copied to
+ * `host_out` on a third stream of the library's own, so that these copies run
+ * while later chunks are copied in and compressed.  `out` (device memory)
+ * receives the same as from certkv_compress_host.  host_out: k, v,
+ * real_counts, offsets and positions are HOST pointers sized as out's
+ * (page-locked memory for asynchronous copies); its other fields are ignored
+ * (the optional device outputs of `out` are not copied back).  The copies
+ * complete on `stream`, like the rest of the call.  Workspace and return
+ * codes as for certkv_compress_host; CERTKV_EINVAL also when host_out or one
+ * of its five pointers is NULL, or when host_out->capacity_slots is below
+ * budget_live * batch * layers. */
+int certkv_compress_host_copyback(const certkv_shape* shape, const void* hK, const void* hV,
+                                  const void* hQ_obs, int64_t budget_live,
+                                  const certkv_params* params, int32_t chunk, certkv_packed* out,
+                                  certkv_packed* host_out, void* workspace,
+                                  size_t workspace_bytes, void* stream);
+
 /* a9: decode attention over the packed cache: for every query head qh of
  * unit u = (b, l, qh / G), out[b][l][qh] = sum_s softmax_s(scale <q, k_s>) v_s
  * over the real_counts[u] (+ 1 tail) slots of segment u.  q, out: bf16

@@ -54,7 +54,7 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_compress_host", "certkv_decode_certified", "certkv_fixed_row_workspace_bytes",
             "certkv_fixed_row_stats", "certkv_coverage_workspace_bytes",
             "certkv_coverage_profile", "certkv_sampled_workspace_bytes",
-            "certkv_sampled_compensation")
+            "certkv_sampled_compensation", "certkv_compress_host_copyback")
 
 _lock = threading.Lock()
 _lib = None
@@ -111,6 +111,8 @@ def load_library(path: Optional[str] = None):
         lib.certkv_host_workspace_bytes.restype = SZ
         lib.certkv_compress_host.argtypes = [sp, P, P, P, I64, pp, I32, kp, P, SZ, P]
         lib.certkv_compress_host.restype = ctypes.c_int
+        lib.certkv_compress_host_copyback.argtypes = [sp, P, P, P, I64, pp, I32, kp, kp, P, SZ, P]
+        lib.certkv_compress_host_copyback.restype = ctypes.c_int
         lib.certkv_decode_certified.argtypes = [sp, P, kp, ctypes.c_float, I32, I32, P, P, P, P,
                                                 SZ, P]
         lib.certkv_decode_certified.restype = ctypes.c_int
@@ -240,6 +242,24 @@ class Packed:
                              _ptr(self.tail_f32), _ptr(self.tail_mass), _ptr(self.cluster_meta),
                              _ptr(self.kept_vmax))
 
+    def host_struct(self) -> certkv_packed:
+        """The struct of a host copy (Packed.empty_host): k, v, offsets,
+        real_counts, positions only."""
+        return certkv_packed(_host_ptr(self.k), _host_ptr(self.v), _host_ptr(self.offsets),
+                             _host_ptr(self.real_counts), _host_ptr(self.positions),
+                             self.k.shape[0], None, None, None, None)
+
+    @staticmethod
+    def empty_host(B: int, L: int, H: int, d: int, B_live: int, pin: bool = True) -> "Packed":
+        """Host (pinned) buffers for the packed cache copied back by
+        certkv_compress_host(..., host_out=...)."""
+        slots, units = B * L * B_live, B * L * H
+        return Packed(k=torch.empty((slots, d), dtype=torch.bfloat16, pin_memory=pin),
+                      v=torch.empty((slots, d), dtype=torch.bfloat16, pin_memory=pin),
+                      offsets=torch.empty(units + 1, dtype=torch.int64, pin_memory=pin),
+                      real_counts=torch.empty(units, dtype=torch.int32, pin_memory=pin),
+                      positions=torch.empty(slots, dtype=torch.int32, pin_memory=pin))
+
     @staticmethod
     def empty(B: int, L: int, H: int, d: int, B_live: int, device, with_tail: bool = False,
               tail_slot: int = 1, clusters: int = 0) -> "Packed":
@@ -339,8 +359,10 @@ def certkv_compress(K, V, Q_obs, budget_live: int, params=None, *, out: Optional
 
 def certkv_compress_host(hK, hV, hQ_obs, budget_live: int, params=None, *, chunk: int = 0,
                          out: Optional[Packed] = None, ws=None, device=None, with_tail: bool = False,
-                         stream=None) -> Packed:
-    """a1-a8 from host tensors, copies overlapped with the compression."""
+                         host_out: Optional[Packed] = None, stream=None) -> Packed:
+    """a1-a8 from host tensors, copies overlapped with the compression; with
+    host_out (Packed.empty_host) the packed cache is also copied back chunk by
+    chunk (certkv_compress_host_copyback)."""
     _bf16(hK, "K"); _bf16(hV, "V"); _bf16(hQ_obs, "Q_obs")
     params = params or certkv_default_params()
     shape = shape_of(hK, hQ_obs)
@@ -352,6 +374,14 @@ def certkv_compress_host(hK, hV, hQ_obs, budget_live: int, params=None, *, chunk
     if ws is None:
         ws = workspace(certkv_host_workspace_bytes(shape, params, chunk), device)
     st = out.struct()
+    if host_out is not None:
+        hst = host_out.host_struct()
+        rc = load_library().certkv_compress_host_copyback(
+            ctypes.byref(shape), _host_ptr(hK), _host_ptr(hV), _host_ptr(hQ_obs), int(budget_live),
+            ctypes.byref(params), int(chunk), ctypes.byref(st), ctypes.byref(hst), _ptr(ws),
+            ws.numel(), _stream(stream))
+        _check(rc, "certkv_compress_host_copyback")
+        return out
     rc = load_library().certkv_compress_host(ctypes.byref(shape), _host_ptr(hK), _host_ptr(hV),
                                              _host_ptr(hQ_obs),
                                              int(budget_live), ctypes.byref(params), int(chunk),

@@ -335,10 +335,13 @@ size_t certkv_host_workspace_bytes(const certkv_shape* shape, const certkv_param
   return hp.total;
 }
 
-int certkv_compress_host(const certkv_shape* shape, const void* hK, const void* hV,
-                         const void* hQ_obs, int64_t budget_live, const certkv_params* params,
-                         int32_t chunk, certkv_packed* out, void* workspace,
-                         size_t workspace_bytes, void* stream) {
+namespace {
+// certkv_compress_host, and with host_out the chunk-by-chunk copy back of the
+// packed cache on a third stream
+int compress_host_impl(const certkv_shape* shape, const void* hK, const void* hV,
+                       const void* hQ_obs, int64_t budget_live, const certkv_params* params,
+                       int32_t chunk, certkv_packed* out, certkv_packed* host_out,
+                       void* workspace, size_t workspace_bytes, void* stream) {
   if (budget_live < 0) return CERTKV_EBUDGET;
   if (chunk < 0) return CERTKV_EINVAL;
   HostPlan hp;
@@ -346,23 +349,38 @@ int certkv_compress_host(const certkv_shape* shape, const void* hK, const void* 
   if (rc) return rc;
   if (!hK || !hV || !hQ_obs) return CERTKV_EINVAL;
   if ((rc = check_packed(hp.full, out))) return rc;
+  if (host_out && (!host_out->k || !host_out->v || !host_out->offsets ||
+                   !host_out->real_counts || !host_out->positions ||
+                   host_out->capacity_slots < (int64_t)hp.full.bl * hp.full.B_live))
+    return CERTKV_EINVAL;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < hp.total) return CERTKV_EWORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   char* ws = reinterpret_cast<char*>(workspace);
   char* stage[2] = {ws + hp.ws_sub, ws + hp.ws_sub + hp.stage};
-  // a private copy stream and its events, released when their work is done
-  cudaStream_t cs = nullptr;
+  // private copy streams (in; back) and their events, released when their
+  // work is done
+  cudaStream_t cs = nullptr, ds = nullptr;
   cudaEvent_t start = nullptr, staged[2] = {nullptr, nullptr}, freed[2] = {nullptr, nullptr};
+  cudaEvent_t packed_ev = nullptr, back_done = nullptr;
   auto release = [&]() {
     for (int i = 0; i < 2; ++i) {
       if (staged[i]) cudaEventDestroy(staged[i]);
       if (freed[i]) cudaEventDestroy(freed[i]);
     }
     if (start) cudaEventDestroy(start);
+    if (packed_ev) cudaEventDestroy(packed_ev);
+    if (back_done) cudaEventDestroy(back_done);
     if (cs) cudaStreamDestroy(cs);
+    if (ds) cudaStreamDestroy(ds);
   };
   if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess ||
       cudaEventCreateWithFlags(&start, cudaEventDisableTiming) != cudaSuccess) {
+    release();
+    return CERTKV_ECUDA;
+  }
+  if (host_out && (cudaStreamCreateWithFlags(&ds, cudaStreamNonBlocking) != cudaSuccess ||
+                   cudaEventCreateWithFlags(&packed_ev, cudaEventDisableTiming) != cudaSuccess ||
+                   cudaEventCreateWithFlags(&back_done, cudaEventDisableTiming) != cudaSuccess)) {
     release();
     return CERTKV_ECUDA;
   }
@@ -412,9 +430,51 @@ int certkv_compress_host(const certkv_shape* shape, const void* hK, const void* 
     launch_score(p, ly, ws, sK, sQ, a, st);
     rc = run_scored(p, ly, ws, sK, sV, a, &o, st);
     if (!rc) rc = cuda_ok(cudaEventRecord(freed[s], st));
+    if (!rc && host_out) {  // this chunk's part of the packed cache back to the host
+      const size_t s0 = (size_t)bl0 * F.B_live, ns = (size_t)cnt * F.B_live;
+      const size_t u0 = (size_t)bl0 * F.H, nu = (size_t)cnt * F.H;
+      const size_t row = (size_t)kD * 2;
+      const bool last = bl0 + cnt == F.bl;
+      rc = cuda_ok(cudaEventRecord(packed_ev, st));
+      if (!rc) rc = cuda_ok(cudaStreamWaitEvent(ds, packed_ev, 0));
+      if (!rc) rc = cuda_ok(cudaMemcpyAsync((char*)host_out->k + s0 * row, (const char*)out->k + s0 * row,
+                                            ns * row, cudaMemcpyDeviceToHost, ds));
+      if (!rc) rc = cuda_ok(cudaMemcpyAsync((char*)host_out->v + s0 * row, (const char*)out->v + s0 * row,
+                                            ns * row, cudaMemcpyDeviceToHost, ds));
+      if (!rc) rc = cuda_ok(cudaMemcpyAsync(host_out->positions + s0, out->positions + s0,
+                                            ns * sizeof(int32_t), cudaMemcpyDeviceToHost, ds));
+      if (!rc) rc = cuda_ok(cudaMemcpyAsync(host_out->real_counts + u0, out->real_counts + u0,
+                                            nu * sizeof(int32_t), cudaMemcpyDeviceToHost, ds));
+      if (!rc) rc = cuda_ok(cudaMemcpyAsync(host_out->offsets + u0, out->offsets + u0,
+                                            (nu + (last ? 1 : 0)) * sizeof(int64_t),
+                                            cudaMemcpyDeviceToHost, ds));
+    }
+  }
+  if (!rc && host_out) {  // the call completes on `stream` with its copies back
+    rc = cuda_ok(cudaEventRecord(back_done, ds));
+    if (!rc) rc = cuda_ok(cudaStreamWaitEvent(st, back_done, 0));
   }
   release();
   return rc;
+}
+}  // namespace
+
+int certkv_compress_host(const certkv_shape* shape, const void* hK, const void* hV,
+                         const void* hQ_obs, int64_t budget_live, const certkv_params* params,
+                         int32_t chunk, certkv_packed* out, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  return compress_host_impl(shape, hK, hV, hQ_obs, budget_live, params, chunk, out, nullptr,
+                            workspace, workspace_bytes, stream);
+}
+
+int certkv_compress_host_copyback(const certkv_shape* shape, const void* hK, const void* hV,
+                                  const void* hQ_obs, int64_t budget_live,
+                                  const certkv_params* params, int32_t chunk, certkv_packed* out,
+                                  certkv_packed* host_out, void* workspace,
+                                  size_t workspace_bytes, void* stream) {
+  if (!host_out) return CERTKV_EINVAL;
+  return compress_host_impl(shape, hK, hV, hQ_obs, budget_live, params, chunk, out, host_out,
+                            workspace, workspace_bytes, stream);
 }
 
 int certkv_compress(const certkv_shape* shape, const void* K, const void* V, const void* Q_obs,

@@ -141,6 +141,31 @@ def test_host_entry_point_validation(lib):
     assert call(ws_bytes=need - 1) == ck.EWORKSPACE
 
 
+def test_host_copyback_validation(lib):
+    s = shape()
+    params = ck.certkv_default_params()
+    need = lib.certkv_host_workspace_bytes(ctypes.byref(s), ctypes.byref(params), 0)
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
+    budget = 2 * s.hkv
+    slots = budget * s.batch * s.layers
+    packed = ck.certkv_packed(fake, fake, fake, fake, fake, 1 << 40, None, None)
+
+    def host(k=fake, cap=slots, pos=fake):
+        return ck.certkv_packed(k, fake, fake, fake, pos, cap, None, None)
+
+    def call(h, ws=256):
+        return lib.certkv_compress_host_copyback(
+            ctypes.byref(s), fake, fake, fake, budget, ctypes.byref(params), 0,
+            ctypes.byref(packed), ctypes.byref(h) if h is not None else None,
+            ctypes.c_void_p(ws) if ws else None, need, None)
+
+    assert call(None) == ck.EINVAL               # no host output
+    assert call(host(k=None)) == ck.EINVAL       # a missing host buffer
+    assert call(host(pos=None)) == ck.EINVAL
+    assert call(host(cap=slots - 1)) == ck.EINVAL  # too few host slots
+    assert call(host(), ws=0) == ck.EWORKSPACE   # the rest as certkv_compress_host
+
+
 def test_coverage_profile_validation(lib):
     s = shape()
     need = lib.certkv_coverage_workspace_bytes(ctypes.byref(s))

@@ -1,6 +1,7 @@
 """certkv_compress_host (host inputs, copies overlapped with the compression)
 gives exactly what certkv_compress gives on the same data, for every chunk
-size, with pinned and with pageable host memory."""
+size, with pinned and with pageable host memory; with a host output the
+packed cache copied back chunk by chunk equals the device one."""
 import pytest
 import torch
 
@@ -53,3 +54,25 @@ def test_host_pipeline_status_and_reuse():
     torch.cuda.synchronize()
     _same(a, b)
     assert ck.certkv_read_status(ws) == 0
+
+
+@pytest.mark.parametrize("chunk", [1, 4, 0])
+def test_host_copyback_equals_device_output(chunk):
+    K, V, Q = W.draw(WL, device="cuda")
+    params = ck.certkv_default_params()
+    ref = _reference(K, V, Q, WL.B_live, params)
+    hK, hV, hQ = K.cpu().pin_memory(), V.cpu().pin_memory(), Q.cpu().pin_memory()
+    host = ck.Packed.empty_host(WL.B, WL.L, WL.H, WL.d, WL.B_live)
+    for t in (host.k, host.v):
+        t.view(torch.int16).fill_(-1)
+    host.positions.fill_(-7)
+    got = ck.certkv_compress_host(hK, hV, hQ, WL.B_live, params, chunk=chunk, with_tail=True,
+                                  host_out=host)
+    torch.cuda.synchronize()  # the copies back complete with the call's stream
+    _same(got, ref)
+    assert torch.equal(host.real_counts, ref.real_counts.cpu())
+    assert torch.equal(host.offsets, ref.offsets.cpu())
+    n = int(ref.offsets[-1])
+    assert torch.equal(host.positions[:n], ref.positions[:n].cpu())
+    assert torch.equal(host.k[:n].view(torch.int16), ref.k[:n].cpu().view(torch.int16))
+    assert torch.equal(host.v[:n].view(torch.int16), ref.v[:n].cpu().view(torch.int16))
