@@ -422,7 +422,8 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
 
 // grid = (ceil(chunks / 4), units), block = 128: warp w of block x takes chunk
 // 4x + w, every chunk but the last (curve_prefix_kernel takes the last ones).
-__global__ void __launch_bounds__(128) curve_eval_kernel(Prob p, EvalArgs ea) {
+__global__ void __launch_bounds__(128, 7)  // seven CTAs per SM: 69 registers, no spills
+curve_eval_kernel(Prob p, EvalArgs ea) {
   __shared__ __align__(16) unsigned char s_ring[4][kEvalRing][kEvalGroupBytes];
   __shared__ float s_a[4][kChunk];
   __shared__ int s_j[4][kChunk];
