@@ -636,7 +636,6 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
         b = bw;
         cur = cw;
       }
-      const int wb = extended ? -1 : wbase;
       if (bw + 1 - wbase >= 64 || extended) {  // refill the winner's window
         if (bw < n - 1) {
           __syncwarp();
@@ -646,7 +645,6 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
           __syncwarp();
         }
       }
-      (void)wb;
     }
     // counts and offsets: segment = b_h real slots (+ 1 tail slot) (+ m cluster summaries)
     const int seg = live ? b + p.tail_slot + p.clusters : 0;
