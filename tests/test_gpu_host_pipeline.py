@@ -76,3 +76,22 @@ def test_host_copyback_equals_device_output(chunk):
     assert torch.equal(host.positions[:n], ref.positions[:n].cpu())
     assert torch.equal(host.k[:n].view(torch.int16), ref.k[:n].cpu().view(torch.int16))
     assert torch.equal(host.v[:n].view(torch.int16), ref.v[:n].cpu().view(torch.int16))
+
+
+def test_host_copyback_with_cluster_summaries():
+    """With clustered tail summaries the device output carries their metadata;
+    the host copy holds the packed slots, counts and offsets, as documented."""
+    K, V, Q = W.draw(WL, device="cuda")
+    params = ck.certkv_default_params(tail_slot=0, tail_clusters=2)
+    ref = ck.certkv_compress(K, V, Q, WL.B_live, params)
+    hK, hV, hQ = K.cpu().pin_memory(), V.cpu().pin_memory(), Q.cpu().pin_memory()
+    host = ck.Packed.empty_host(WL.B, WL.L, WL.H, WL.d, WL.B_live)
+    got = ck.certkv_compress_host(hK, hV, hQ, WL.B_live, params, chunk=2, host_out=host)
+    torch.cuda.synchronize()
+    assert torch.equal(got.cluster_meta, ref.cluster_meta)
+    assert torch.equal(host.offsets, ref.offsets.cpu())
+    assert torch.equal(host.real_counts, ref.real_counts.cpu())
+    n = int(ref.offsets[-1])
+    assert torch.equal(host.positions[:n], ref.positions[:n].cpu())
+    assert torch.equal(host.k[:n].view(torch.int16), ref.k[:n].cpu().view(torch.int16))
+    assert torch.equal(host.v[:n].view(torch.int16), ref.v[:n].cpu().view(torch.int16))
