@@ -46,6 +46,9 @@ def parse():
                     help="time the evaluation instruments and variants (fixed-row and lift "
                          "diagnostics, coverage profile, sampled compensation, clustered "
                          "summaries with the certified decode) instead of the hot path")
+    ap.add_argument("--shard", action="store_true",
+                    help="with several ranks: split ONE job's (sequence, layer) pairs across "
+                         "the ranks (strong scaling) instead of one job per rank (weak)")
     ap.add_argument("--decode-steps", type=int, default=1,
                     help="decode steps per step after the compression, each with fresh queries "
                          "(the C4 configuration decodes 256)")
@@ -171,6 +174,26 @@ def roofline_for(name, work, ms, peaks, traffic=None):
             "peak_source": peaks["source"] + " (copy bandwidth)"}
 
 
+# DRAM bytes (read + write) of the whole compression pass per step, summed over
+# its kernels from one ncu capture of the build as it is now, keyed by
+# workload; null when the pass has changed since the counters were taken.
+MEASURED_PASS_TRAFFIC = {}
+
+
+def compress_roofline(wl, B_live, compress_ms, peaks):
+    """The whole compression pass against the HBM roof: algorithmic bytes =
+    K and V read once + the packed cache written once,
+    B*L*(H*n*2d*2 + B_live*2d*2), over the event-timed compression."""
+    nbytes = wl.B * wl.L * (wl.H * wl.n * wl.d * 2 * 2 + B_live * wl.d * 2 * 2)
+    ach = nbytes / (compress_ms / 1e3) / 1e9
+    return {"kernel": "compress (whole pass, every kernel)", "bound": "hbm",
+            "achieved": round(ach, 1), "peak": peaks["hbm"], "unit": "GB/s",
+            "frac": round(ach / peaks["hbm"], 4),
+            "traffic": MEASURED_PASS_TRAFFIC.get((wl.name, wl.L, wl.B)),
+            "bytes_per_step": nbytes, "ms": round(compress_ms, 4),
+            "peak_source": peaks["source"] + " (copy bandwidth)"}
+
+
 # ------------------------------------------------------------ multi-rank ----
 def max_over_ranks(value: float, world: int) -> float:
     """The maximum of `value` over all ranks (the job's step time)."""
@@ -187,6 +210,46 @@ def max_over_ranks(value: float, world: int) -> float:
 def job_throughput(units_per_rank: int, world: int, ms: float) -> float:
     """Whole-job throughput: every rank processes its own units (weak scaling)."""
     return world * units_per_rank / (ms / 1e3)
+
+
+def shard_range(total: int, world: int, rank: int) -> tuple:
+    """The contiguous share [lo, hi) of a job's `total` (sequence, layer) pairs
+    that `rank` compresses.  The shares of ranks 0..world-1 cover every pair
+    exactly once, in order, and differ in size by at most one."""
+    return total * rank // world, total * (rank + 1) // world
+
+
+def shard_pairs(wl, world: int, rank: int) -> list:
+    """The (sequence, layer) pairs of this rank's share, in job order
+    (pair index = sequence * L + layer)."""
+    lo, hi = shard_range(wl.B * wl.L, world, rank)
+    return [(i // wl.L, i % wl.L) for i in range(lo, hi)]
+
+
+def global_offsets(local_offsets, first_pair: int, B_live: int):
+    """Packed-slot offsets of a shard as they stand in the whole job's packed
+    cache: every (sequence, layer) pair holds exactly B_live slots, so the
+    shard that starts at pair `first_pair` starts at slot first_pair * B_live."""
+    return [int(o) + first_pair * B_live for o in local_offsets]
+
+
+def draw_shard(wl, pairs, seed, device):
+    """K, V, Q of the given (sequence, layer) pairs of the job, stacked as one
+    sequence of len(pairs) layers (pairs are compressed independently); each
+    pair's bytes are those of the whole job's draw."""
+    import torch
+
+    from paper_2608_21541_gb300 import workloads as W
+    cnt = len(pairs)
+    K = torch.empty((1, cnt, wl.H, wl.n, wl.d), dtype=torch.bfloat16, device=device)
+    V = torch.empty_like(K)
+    Q = torch.empty((1, cnt, wl.Hq, wl.w, wl.d), dtype=torch.bfloat16, device=device)
+    for i, (b, l) in enumerate(pairs):
+        k, v, q = W.draw_layer(wl, b, l, seed, device)
+        K[0, i].copy_(k)
+        V[0, i].copy_(v)
+        Q[0, i].copy_(q)
+    return K, V, Q
 
 
 # ----------------------------------------------------------- oracle arms ----
@@ -363,9 +426,19 @@ def run_ours(args, wl, rank, world):
     dev = torch.device("cuda", local)
     peaks = load_peaks()
     B_live = wl.B_live
-    K, V, Q = W.draw(wl, seed=args.seed + rank, device=dev)
+    job = wl
+    sharded = args.shard and world > 1
+    if sharded:
+        # this rank's contiguous share of one job's (sequence, layer) pairs
+        pairs = shard_pairs(job, world, rank)
+        K, V, Q = draw_shard(job, pairs, args.seed, dev)
+        wl = job.with_(B=1, L=len(pairs))
+        qseed = args.seed
+    else:
+        K, V, Q = W.draw(wl, seed=args.seed + rank, device=dev)
+        qseed = args.seed + rank
     nd = max(1, args.decode_steps)
-    qs = [W.draw_decode_queries(wl, i, seed=args.seed + rank, device=dev) for i in range(nd)]
+    qs = [W.draw_decode_queries(wl, i, seed=qseed, device=dev) for i in range(nd)]
     q = qs[0]
     params = ck.certkv_default_params()
     shape = ck.shape_of(K, Q)
@@ -391,71 +464,93 @@ def run_ours(args, wl, rank, world):
             dist.barrier()
 
     clocks = ClockSampler(local)
-    ck.certkv_trace_enable(True)
-    ck.certkv_trace_report()  # clear
     barrier()
     torch.cuda.synchronize()
     clocks.start()
     time.sleep(0.3)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        step()
-    e1.record(stream)
+    # the timed region: no per-launch tracing; one pair of events per step
+    # separates the compression from the decode steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for e_start, e_mid, e_end in ev:
+        e_start.record(stream)
+        ck.certkv_compress(K, V, Q, B_live, params, out=packed, ws=ws, stream=stream)
+        e_mid.record(stream)
+        for qi in qs:
+            ck.certkv_decode_attn(qi, packed, hkv=wl.H, out=out, ws=dws, stream=stream)
+        e_end.record(stream)
     torch.cuda.synchronize()
     barrier()
     clk = clocks.stop()
+    ms_local = ev[0][0].elapsed_time(ev[-1][2]) / args.steps
+    compress_local = sum(a.elapsed_time(b) for a, b, _ in ev) / args.steps
+    ms = max_over_ranks(ms_local, world)
+    compress_ms = max_over_ranks(compress_local, world)
+    if sharded:  # one job split across the ranks: its tokens over the slowest rank
+        value = job.B * job.L * job.n / (ms / 1e3)
+    else:
+        value = job_throughput(wl.B * wl.L * wl.n, world, ms)
+
+    # a separate traced run (CUDA events around every library launch) for the
+    # per-kernel shares; it is not the headline timing
+    trace_steps = max(1, min(args.steps, 3))
+    ck.certkv_trace_enable(True)
+    ck.certkv_trace_report()  # clear
+    for _ in range(trace_steps):
+        step()
+    torch.cuda.synchronize()
     trace = ck.certkv_trace_report()
     ck.certkv_trace_enable(False)
-    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
-    tokens = wl.B * wl.L * wl.n
-    value = job_throughput(tokens, world, ms)
+    traced_ms = sum(v[1] for v in trace.values()) / trace_steps
 
-    # per-kernel shares and the dominant kernel's roofline
+    # per-kernel shares and per-kernel rooflines (traced run)
     kernels = {}
-    launches = 0
+    launches_per_step = 0.0
     total_ms = sum(v[1] for v in trace.values()) or 1.0
     for name, (cnt, tms) in sorted(trace.items(), key=lambda kv: -kv[1][1]):
-        launches += cnt
-        kernels[name] = {"launches_per_step": cnt / args.steps,
-                         "ms_per_step": round(tms / args.steps, 4),
+        launches_per_step += cnt / trace_steps
+        kernels[name] = {"launches_per_step": cnt / trace_steps,
+                         "ms_per_step": round(tms / trace_steps, 4),
                          "share": round(tms / total_ms, 4)}
     roof_all = {}
     for name in kernels:
         work = kernel_work(wl, B_live, name)
         if work:
             per_launch_ms = trace[name][1] / trace[name][0]
-            launches_per_step = trace[name][0] / args.steps
+            lps = trace[name][0] / trace_steps
             roof_all[name] = roofline_for(name, work, per_launch_ms, peaks,
-                                          measured_traffic(name, wl, launches_per_step))
-    dominant = next(iter(kernels))
-    roof = roof_all.get(dominant) or next(iter(roof_all.values()))
+                                          measured_traffic(name, wl, lps))
+    dominant = next((k for k in kernels if k in roof_all), None)
 
-    decode_ms = kernels.get("decode_split", {}).get("ms_per_step", 0) + \
-        kernels.get("decode_merge", {}).get("ms_per_step", 0)
+    decode_ms = ms - compress_ms
     decode_bytes = nd * wl.B * wl.L * B_live * wl.d * 2 * 2  # per step, all decode steps
-    compress_ms = ms - decode_ms
-    roof_bytes = wl.B * wl.L * (wl.H * wl.n * wl.d * 2 * 2 + B_live * wl.d * 2 * 2)
+    roof = compress_roofline(wl, B_live, compress_ms, peaks)
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "strong" if sharded else "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": dict(config_dict(wl, B_live), decode_steps=nd),
+        "config": dict(config_dict(job, B_live), decode_steps=nd,
+                       **({"shard": f"{len(pairs)} of {job.B * job.L} (sequence, layer) pairs "
+                                     f"per rank"} if sharded else {})),
         "compress_ms": compress_ms,
-        "compress_hbm_roofline": {
-            "bytes": roof_bytes, "achieved_GBps": round(roof_bytes / (compress_ms / 1e3) / 1e9, 1),
-            "peak": peaks["hbm"], "frac": round(roof_bytes / (compress_ms / 1e3) / 1e9 /
-                                                peaks["hbm"], 4),
-            "definition": "K+V read + packed cache written, over the compression time"},
-        "decode_GBps": round(decode_bytes / (decode_ms / 1e3) / 1e9, 1) if decode_ms else None,
-        "roofline": roof, "kernels": kernels, "kernel_rooflines": roof_all,
-        "gpu_launches": launches, "device_status": status,
+        "decode_ms": decode_ms,
+        "decode_GBps": round(decode_bytes / (decode_ms / 1e3) / 1e9, 1) if decode_ms > 0 else None,
+        "roofline": roof,
+        "dominant_kernel": roof_all.get(dominant),
+        "kernels": kernels, "kernel_rooflines": roof_all,
+        "traced": {"steps": trace_steps, "ms_per_step": round(traced_ms, 4),
+                   "note": "per-kernel shares from a separate run with CUDA events around "
+                           "every launch; the headline ms_per_step is untraced"},
+        "gpu_launches": int(round(launches_per_step * args.steps)),
+        "device_status": status,
         "clocks": clk,
     }
 
     if not args.no_e2e:
-        line["e2e"] = run_e2e(args, wl, K, V, Q, qs, params, ws, dws, dev, stream, world, B_live)
+        line["e2e"] = run_e2e(args, wl, K, V, Q, qs, params, ws, dws, dev, stream, world, B_live,
+                              job_tokens=job.B * job.L * job.n if sharded else None)
     del K, V, Q
     torch.cuda.empty_cache()
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -470,7 +565,7 @@ def run_ours(args, wl, rank, world):
         print(json.dumps(line), flush=True)
 
 
-def run_e2e(args, wl, K, V, Q, qs, params, ws, dws, dev, stream, world, B_live):
+def run_e2e(args, wl, K, V, Q, qs, params, ws, dws, dev, stream, world, B_live, job_tokens=None):
     """Same metric through the public API with host buffers: pinned host ->
     device copies of the step's inputs, compress, decode, and the packed cache
     and decode output copied back, all inside the timed region.  The packed
@@ -515,10 +610,11 @@ def run_e2e(args, wl, K, V, Q, qs, params, ws, dws, dev, stream, world, B_live):
         step()
     e1.record(stream)
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / steps
+    ms = max_over_ranks(e0.elapsed_time(e1) / steps, world)
     h2d = sum(x.numel() * x.element_size() for x in (hK, hV, hQ, hq))
     d2h = sum(x.numel() * x.element_size() for x in host_out.values())
-    return {"value": world * wl.B * wl.L * wl.n / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
+    tokens = job_tokens if job_tokens is not None else world * wl.B * wl.L * wl.n
+    return {"value": tokens / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
             "steps": steps, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "api": "certkv_compress_host_copyback + certkv_decode_attn, pinned host buffers"}
 

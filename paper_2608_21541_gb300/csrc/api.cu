@@ -134,6 +134,29 @@ Layout make_layout(const Prob& p) {
 
 }  // namespace certkv
 
+namespace certkv {
+
+int decode_prob(const certkv_shape* shape, Prob* p) {
+  int rc = check_shape(shape);
+  if (rc) return rc;
+  certkv_params prm;
+  certkv_default_params(&prm);
+  return make_prob(shape, &prm, -1, p);
+}
+
+int decode_args(const certkv_shape* shape, const void* q, const certkv_packed* packed,
+                float scale, int32_t tail_slot, const void* out, float* sc) {
+  if (!q || !packed || !packed->k || !packed->v || !packed->offsets || !packed->real_counts || !out)
+    return CERTKV_EINVAL;
+  if (((uintptr_t)packed->k | (uintptr_t)packed->v | (uintptr_t)q) % 16 != 0) return CERTKV_EINVAL;
+  if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
+  if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
+  *sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
+  return CERTKV_OK;
+}
+
+}  // namespace certkv
+
 namespace certkv_api {
 
 using namespace certkv;
@@ -500,20 +523,13 @@ int certkv_compress(const certkv_shape* shape, const void* K, const void* V, con
 int certkv_decode_attn(const certkv_shape* shape, const void* q, const certkv_packed* packed,
                        float scale, int32_t tail_slot, void* out, void* workspace,
                        size_t workspace_bytes, void* stream) {
-  int rc = check_shape(shape);
-  if (rc) return rc;
-  if (!q || !packed || !packed->k || !packed->v || !packed->offsets || !packed->real_counts || !out)
-    return CERTKV_EINVAL;
-  if (!aligned(packed->k, 16) || !aligned(packed->v, 16) || !aligned(q, 16)) return CERTKV_EINVAL;
-  if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
-  if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
-  certkv_params prm;
-  certkv_default_params(&prm);
   Prob p;
-  if ((rc = make_prob(shape, &prm, -1, &p))) return rc;
+  int rc = decode_prob(shape, &p);
+  if (rc) return rc;
+  float sc = 0.0f;
+  if ((rc = decode_args(shape, q, packed, scale, tail_slot, out, &sc))) return rc;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < decode_workspace(p))
     return CERTKV_EWORKSPACE;
-  const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (!launch_decode(p, q, packed->k, packed->v, packed->offsets, packed->real_counts, tail_slot,
                      sc, out, reinterpret_cast<char*>(workspace), st))

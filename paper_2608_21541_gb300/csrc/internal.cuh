@@ -6,6 +6,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include "../../include/certkv.h"
+
 namespace certkv {
 
 // One compress/decode call, after host-side validation.
@@ -66,6 +68,17 @@ struct Layout {
 };
 
 Layout make_layout(const Prob& p);
+
+// Validation shared by the decode entry points (certkv_decode_attn and
+// certkv_decode_attn_noalloc), so that both accept exactly the same calls.
+// decode_prob: the shape (as every entry point checks it) -> the problem
+// description of a decode call.  decode_args: query, packed cache and output
+// pointers (non-null, 16-byte aligned), tail_slot in {0, 1}, a finite scale
+// >= 0 -> the effective softmax scale (0 selects 1/sqrt(d)).  Both return
+// CERTKV_OK or CERTKV_EINVAL and launch nothing.
+int decode_prob(const certkv_shape* shape, Prob* p);
+int decode_args(const certkv_shape* shape, const void* q, const certkv_packed* packed,
+                float scale, int32_t tail_slot, const void* out, float* sc);
 
 // ---- launchers (all asynchronous on `st`) --------------------------------
 __global__ void lse_merge_kernel(Prob p, const float2* __restrict__ part, float* __restrict__ lse2);

@@ -31,28 +31,15 @@ extern "C" int certkv_decode_attn_noalloc(const certkv_shape* shape, const void*
                                           const certkv_packed* packed, float scale,
                                           int32_t tail_slot, void* out, void* stream) {
   using namespace certkv;
-  if (!shape || shape->d != 128 || shape->batch < 1 || shape->layers < 1 || shape->hkv < 1 ||
-      shape->hkv > 32 || shape->hq < 1 || shape->hq % shape->hkv != 0)
-    return CERTKV_EINVAL;
-  const int G = shape->hq / shape->hkv;
-  if (G != 1 && G != 2 && G != 4 && G != 8 && G != 16) return CERTKV_EINVAL;
-  if (!q || !packed || !packed->k || !packed->v || !packed->offsets || !packed->real_counts ||
-      !out)
-    return CERTKV_EINVAL;
-  if (((uintptr_t)packed->k | (uintptr_t)packed->v | (uintptr_t)q) % 16 != 0) return CERTKV_EINVAL;
-  if (tail_slot != 0 && tail_slot != 1) return CERTKV_EINVAL;
-  if (!(scale >= 0.0f) || scale > 3.0e38f) return CERTKV_EINVAL;
-
-  Prob p = {};
-  p.B = shape->batch;
-  p.L = shape->layers;
-  p.Hq = shape->hq;
-  p.H = shape->hkv;
-  p.d = shape->d;
-  p.G = G;
-  p.units = p.B * p.L * p.H;
-  p.bl = p.B * p.L;
+  // The same validation as certkv_decode_attn, with the size limit checked
+  // right after the shape: a call that is too large is refused before its
+  // pointers are looked at.
+  Prob p;
+  int rc = decode_prob(shape, &p);
+  if (rc) return rc;
   if (decode_workspace(p) > (size_t)CERTKV_NOALLOC_SCRATCH_BYTES) return CERTKV_ETOOLARGE;
+  float sc = 0.0f;
+  if ((rc = decode_args(shape, q, packed, scale, tail_slot, out, &sc))) return rc;
 
   // Set-up, once per device and with that device current: the device address
   // of the static scratch array.
@@ -68,7 +55,6 @@ extern "C" int certkv_decode_attn_noalloc(const certkv_shape* shape, const void*
     }
     scratch = g_scratch_ptr[dev];
   }
-  const float sc = scale > 0.0f ? scale : 0.08838834764831845f;  // 1/sqrt(128)
   if (!launch_decode(p, q, packed->k, packed->v, packed->offsets, packed->real_counts, tail_slot,
                      sc, out, reinterpret_cast<char*>(scratch),
                      reinterpret_cast<cudaStream_t>(stream)))

@@ -977,6 +977,58 @@ def pin_packed_layout_and_bytes(lib=None):
     assert round(packed / 1e9, 2) == gph["certkv_GB"]
 
 
+# -------------------------------------------------------- bf16 rounding ----
+
+def pin_bf16_rounding(lib=None):
+    """The tail slot is the centroid rounded once to bf16, to nearest with ties
+    to even (reading R-A10).  Pinned against torch's float32 -> bfloat16
+    conversion on every value that is exactly a float32 (an independent
+    round-to-nearest-even implementation), and on hand-made bit patterns: ties
+    at the 8-bit boundary, a value just above a tie that a double -> float32 ->
+    bf16 path would round the wrong way, the carry into the exponent, the
+    subnormal range and its boundary, the largest finite value and overflow."""
+    import torch
+    f = lambda x: oracle.f64_to_bf16_bits(x, lib=lib)
+    rng = np.random.default_rng(21)
+    mant = rng.integers(0, 1 << 23, 4000)
+    expo = rng.integers(-149, 128, 4000)
+    vals = np.concatenate([
+        np.ldexp(1.0 + mant / 2.0 ** 23, expo).astype(np.float32),          # normal and overflow
+        (rng.integers(0, 1 << 23, 1000) * 2.0 ** -149).astype(np.float32),  # float32 subnormals
+        (rng.standard_normal(2000) * 10.0 ** rng.integers(-30, 30, 2000)).astype(np.float32),
+        # exact ties: the low 16 bits of the float32 equal 0x8000
+        ((rng.integers(0x00800000, 0x7F000000, 1000) & ~0xFFFF) | 0x8000).astype(np.uint32).view(np.float32),
+    ])
+    vals = vals[np.isfinite(vals)]
+    want = torch.from_numpy(vals.copy()).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    got = np.array([f(float(x)) for x in vals], np.uint16)
+    bad = np.nonzero(got != want)[0]
+    assert bad.size == 0, [(float(vals[i]), hex(got[i]), hex(want[i])) for i in bad[:5]]
+    cases = [
+        (1.0, 0x3F80), (-1.5, 0xBFC0), (0.0, 0x0000), (-0.0, 0x8000),
+        (1.0 + 2.0 ** -8, 0x3F80),                  # tie between 0x3F80 (even) and 0x3F81
+        (1.0 + 3 * 2.0 ** -8, 0x3F82),              # tie between 0x3F81 and 0x3F82 (even)
+        (1.0 + 2.0 ** -8 + 2.0 ** -40, 0x3F81),     # just above a tie: one rounding step
+        (1.0 + 2.0 ** -8 - 2.0 ** -40, 0x3F80),     # just below it
+        (2.0 - 2.0 ** -8, 0x4000),                  # tie above 0x3FFF: carry into the exponent
+        (2.0 - 2.0 ** -9, 0x4000),
+        (2.0 - 2.0 ** -7, 0x3FFF),
+        (2.0 ** -126, 0x0080),                      # smallest normal
+        (2.0 ** -133, 0x0001),                      # smallest subnormal
+        (2.0 ** -134, 0x0000),                      # half of it: tie to even (zero)
+        (3 * 2.0 ** -134, 0x0002),                  # 1.5 quanta: tie to even (2)
+        (2.0 ** -134 + 2.0 ** -160, 0x0001),        # just above half a quantum
+        (2.0 ** -126 - 2.0 ** -134, 0x0080),        # tie between 0x007F and the smallest normal
+        (127 * 2.0 ** -133, 0x007F),                # largest subnormal
+        ((2.0 - 2.0 ** -7) * 2.0 ** 127, 0x7F7F),   # largest finite
+        ((2.0 - 2.0 ** -8) * 2.0 ** 127, 0x7F80),   # tie above it: overflow to infinity
+        ((2.0 - 2.0 ** -8 - 2.0 ** -30) * 2.0 ** 127, 0x7F7F),
+        (-1e39, 0xFF80), (float("inf"), 0x7F80), (float("-inf"), 0xFF80),
+    ]
+    for x, bits in cases:
+        assert f(x) == bits, (x, hex(f(x)), hex(bits))
+
+
 # ------------------------------------------------------------------ decode --
 
 def pin_decode_textbook(lib=None):

@@ -63,6 +63,12 @@ MUTANTS = {
     "bisection_inverted": ("if (total > B_real) lam_lo = lam; else lam_hi = lam;",
                            "if (total > B_real) lam_hi = lam; else lam_lo = lam;"),
     "kept_not_sorted": ("qsort(kept, (size_t)b, sizeof(int32_t), cmp_int32);", ""),
+    "bf16_truncates": ("double r = nearbyint(ldexp(f, 8));", "double r = floor(ldexp(f, 8));"),
+    "bf16_ties_away_from_zero": ("double r = nearbyint(ldexp(f, 8));",
+                                 "double r = round(ldexp(f, 8));"),
+    "bf16_subnormals_truncate": ("double r = nearbyint(ldexp(ax, 133));",
+                                 "double r = floor(ldexp(ax, 133));"),
+    "bf16_no_exponent_carry": ("if (r == 256.0) { r = 128.0; e += 1; }", ""),
     "decode_drops_tail_slot": ("const int slots = counts[u] + (tail_slot ? 1 : 0);",
                                "const int slots = counts[u];"),
     "wrong_query_group": ("((size_t)bl * g->Hq + (size_t)h * G) * g->w * d",
