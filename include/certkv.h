@@ -76,6 +76,12 @@ extern "C" {
                                          tail slot is the uniform mean instead */
 #define CERTKV_STATUS_TIMEOUT     4u  /* a bounded wait inside a tensor-core
                                          kernel gave up; its outputs are invalid */
+#define CERTKV_STATUS_BOUNDS      8u  /* only in a library built with
+                                         CERTKV_DEBUG: a ragged index or offset
+                                         (a token of the order, a kept position,
+                                         a slot, a radix destination, a budget)
+                                         was outside its extent; the access was
+                                         skipped, the outputs are invalid      */
 
 /* ---- problem description ------------------------------------------------- */
 typedef struct {
@@ -394,6 +400,24 @@ int certkv_coverage_profile(const certkv_shape* shape, const void* q, const void
 int certkv_decode_attn_noalloc(const certkv_shape* shape, const void* q,
                                const certkv_packed* packed, float scale, int32_t tail_slot,
                                void* out, void* stream);
+
+/* Guard words of a compression workspace (a debugging aid with no
+ * counterpart in the paper).  Every region of the workspace that
+ * certkv_workspace_bytes(shape, params) describes is followed by 16 bytes of
+ * padding that no kernel writes.  certkv_workspace_guard_arm fills them with a
+ * fixed pattern (asynchronously, on `stream`); after any number of
+ * certkv_score / certkv_curves / certkv_compress_scored / certkv_compress
+ * calls with the same shape and params on that workspace,
+ * certkv_workspace_guard_check synchronises `stream` and returns how many
+ * guards no longer hold the pattern: 0 means no kernel wrote past the end of
+ * its region.  Both return -1 for an invalid shape, params or workspace (NULL,
+ * misaligned or smaller than certkv_workspace_bytes) or a CUDA error; the
+ * check also writes the count into the status region (it does not change the
+ * status word). */
+int certkv_workspace_guard_arm(const certkv_shape* shape, const certkv_params* params,
+                               void* workspace, size_t workspace_bytes, void* stream);
+int certkv_workspace_guard_check(const certkv_shape* shape, const certkv_params* params,
+                                 void* workspace, size_t workspace_bytes, void* stream);
 
 /* Synchronise `stream`, then return the device status word (CERTKV_STATUS_*
  * bits, 0 = clean) that the last compress call on `workspace` left, or -1 if

@@ -21,6 +21,8 @@ from . import build as _build
 OK, EINVAL, EBUDGET, EWORKSPACE, ECAPACITY, ECUDA, ETOOLARGE = range(7)
 STATUS_NONFINITE = 1
 STATUS_ZERO_TAIL = 2
+STATUS_TIMEOUT = 4
+STATUS_BOUNDS = 8
 STAT_CENTERED, STAT_UNCENTERED, STAT_TAIL_MASS = 0, 1, 2
 
 
@@ -54,7 +56,8 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_compress_host", "certkv_decode_certified", "certkv_fixed_row_workspace_bytes",
             "certkv_fixed_row_stats", "certkv_coverage_workspace_bytes",
             "certkv_coverage_profile", "certkv_sampled_workspace_bytes",
-            "certkv_sampled_compensation", "certkv_compress_host_copyback")
+            "certkv_sampled_compensation", "certkv_compress_host_copyback",
+            "certkv_workspace_guard_arm", "certkv_workspace_guard_check")
 
 _lock = threading.Lock()
 _lib = None
@@ -65,12 +68,14 @@ def library_path() -> str:
 
 
 def load_library(path: Optional[str] = None):
-    """Load libcertkv.so (built by ``build()``); raise if it is missing."""
+    """Load libcertkv.so (built by ``build()``; the environment variable
+    CERTKV_LIBRARY may name another build of it, such as the bounds-checking
+    one); raise if it is missing."""
     global _lib
     with _lock:
         if _lib is not None:
             return _lib
-        path = path or _build.LIB
+        path = path or os.environ.get("CERTKV_LIBRARY") or _build.LIB
         if not os.path.exists(path):
             raise RuntimeError(
                 f"CertKV CUDA library not found at {path}; build it with "
@@ -99,6 +104,10 @@ def load_library(path: Optional[str] = None):
         lib.certkv_decode_attn.restype = ctypes.c_int
         lib.certkv_read_status.argtypes = [P, P]
         lib.certkv_read_status.restype = ctypes.c_int
+        lib.certkv_workspace_guard_arm.argtypes = [sp, pp, P, SZ, P]
+        lib.certkv_workspace_guard_arm.restype = ctypes.c_int
+        lib.certkv_workspace_guard_check.argtypes = [sp, pp, P, SZ, P]
+        lib.certkv_workspace_guard_check.restype = ctypes.c_int
         lib.certkv_strerror.argtypes = [ctypes.c_int]
         lib.certkv_strerror.restype = ctypes.c_char_p
         lib.certkv_trace_enable.argtypes = [ctypes.c_int]
@@ -531,6 +540,29 @@ def certkv_sampled_compensation(q, K, V, packed: Packed, unif, m: int, *, scale:
         _ptr(unif), _ptr(idx), _ptr(stats), _ptr(ws), ws.numel(), _stream(stream))
     _check(rc, "certkv_sampled_compensation")
     return stats, idx
+
+
+def certkv_workspace_guard_arm(ws: torch.Tensor, shape: certkv_shape, params=None,
+                               stream=None) -> None:
+    """Fill the guard words after every region of a compression workspace."""
+    params = params or certkv_default_params()
+    rc = load_library().certkv_workspace_guard_arm(ctypes.byref(shape), ctypes.byref(params),
+                                                   _ptr(ws), ws.numel() * ws.element_size(),
+                                                   _stream(stream))
+    if rc != 0:
+        raise RuntimeError("certkv_workspace_guard_arm failed")
+
+
+def certkv_workspace_guard_check(ws: torch.Tensor, shape: certkv_shape, params=None,
+                                 stream=None) -> int:
+    """Number of guard words that no longer hold their pattern (0: none)."""
+    params = params or certkv_default_params()
+    rc = load_library().certkv_workspace_guard_check(ctypes.byref(shape), ctypes.byref(params),
+                                                     _ptr(ws), ws.numel() * ws.element_size(),
+                                                     _stream(stream))
+    if rc < 0:
+        raise RuntimeError("certkv_workspace_guard_check failed")
+    return rc
 
 
 def certkv_read_status(ws: torch.Tensor, stream=None) -> int:

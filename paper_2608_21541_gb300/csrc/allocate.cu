@@ -655,6 +655,9 @@ __global__ void __launch_bounds__(1024) bisect_repair_kernel(Prob p, const float
       if (lane >= o) incl += y;
     }
     if (live) {
+      // the budget within [b_min, n - 1] and the segments within B_live
+      CERTKV_IN_BOUNDS(b >= p.b_min && b <= p.n - 1, p.status);
+      CERTKV_IN_BOUNDS(incl <= p.B_live, p.status);
       counts[(size_t)bl * H + h] = b;
       offsets[(size_t)bl * H + h] = p.slot_base + (int64_t)bl * p.B_live + (incl - seg);
     }

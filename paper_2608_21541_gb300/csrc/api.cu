@@ -90,10 +90,15 @@ int make_prob(const certkv_shape* s, const certkv_params* q, int64_t budget_live
 
 Layout make_layout(const Prob& p) {
   Layout ly;
+  ly.nguards = 0;
   size_t off = 0;
+  // each region is followed by a 16-byte guard (after its bytes rounded up to
+  // 16) that no kernel writes
   auto take = [&](size_t bytes) {
     size_t o = off;
-    off = align256(off + bytes);
+    const size_t g = o + (bytes + 15) / 16 * 16;
+    if (ly.nguards < Layout::kMaxGuards) ly.guard[ly.nguards++] = g;
+    off = align256(g + 16);
     return o;
   };
   const size_t U = (size_t)p.units, n = (size_t)p.n;
@@ -180,6 +185,32 @@ __global__ void key_init_kernel(Prob p, const float* __restrict__ a, uint32_t* _
   if (bad) raise_status(status, CERTKV_STATUS_NONFINITE);
 }
 
+// The guard words written after every workspace region (a fixed pattern).
+__device__ __constant__ uint32_t kGuard[4] = {0x9E3779B9u, 0x7F4A7C15u, 0xF39CC060u, 0x5CEDC834u};
+struct GuardSet {
+  size_t off[Layout::kMaxGuards];
+  int n;
+};
+GuardSet guard_set(const Layout& ly) {
+  GuardSet g;
+  g.n = ly.nguards;
+  for (int i = 0; i < Layout::kMaxGuards; ++i) g.off[i] = i < ly.nguards ? ly.guard[i] : 0;
+  return g;
+}
+__global__ void guard_arm_kernel(char* ws, GuardSet g) {
+  const int i = threadIdx.x;
+  if (i < g.n)
+    *reinterpret_cast<uint4*>(ws + g.off[i]) = make_uint4(kGuard[0], kGuard[1], kGuard[2], kGuard[3]);
+}
+__global__ void guard_check_kernel(const char* ws, GuardSet g, uint32_t* count) {
+  const int i = threadIdx.x;
+  if (i < g.n) {
+    const uint4 x = *reinterpret_cast<const uint4*>(ws + g.off[i]);
+    if (x.x != kGuard[0] || x.y != kGuard[1] || x.z != kGuard[2] || x.w != kGuard[3])
+      atomicAdd(count, 1u);
+  }
+}
+
 int check_ws(const Prob& p, void* ws, size_t ws_bytes, Layout* ly) {
   *ly = make_layout(p);
   if (!ws || !aligned(ws, 256) || ws_bytes < ly->total) return CERTKV_EWORKSPACE;
@@ -258,6 +289,7 @@ int certkv_score(const certkv_shape* shape, const void* K, const void* Q_obs,
   if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   char* ws = reinterpret_cast<char*>(workspace);
+  p.status = reinterpret_cast<uint32_t*>(ws + ly.status);
   if ((rc = cuda_ok(cudaMemsetAsync(ws + ly.status, 0, 256, st)))) return rc;
   launch_score(p, ly, ws, K, Q_obs, a_out, st);
   return cuda_ok(cudaGetLastError());
@@ -275,6 +307,7 @@ int certkv_curves(const certkv_shape* shape, const void* V, const float* a,
   if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   char* ws = reinterpret_cast<char*>(workspace);
+  p.status = reinterpret_cast<uint32_t*>(ws + ly.status);
   if ((rc = cuda_ok(cudaMemsetAsync(ws + ly.status, 0, 256, st)))) return rc;
   {
     TraceScope ts_("key_init", st);
@@ -298,10 +331,12 @@ int certkv_compress_scored(const certkv_shape* shape, const void* K, const void*
   if (!K || !V || !a) return CERTKV_EINVAL;
   if (!aligned(K, 16) || !aligned(V, 16)) return CERTKV_EINVAL;
   if ((rc = check_packed(p, out))) return rc;
+  p.capacity = out->capacity_slots;
   Layout ly;
   if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   char* ws = reinterpret_cast<char*>(workspace);
+  p.status = reinterpret_cast<uint32_t*>(ws + ly.status);
   if ((rc = cuda_ok(cudaMemsetAsync(ws + ly.status, 0, 256, st)))) return rc;
   {
     TraceScope ts_("key_init", st);
@@ -441,7 +476,9 @@ int compress_host_impl(const certkv_shape* shape, const void* hK, const void* hV
     certkv_shape csub = chunk_shape(shape, cnt);
     if ((rc = make_prob(&csub, params, budget_live, &p))) break;
     p.slot_base = (int64_t)bl0 * F.B_live;
+    p.capacity = out->capacity_slots;
     const Layout ly = make_layout(p);
+    p.status = reinterpret_cast<uint32_t*>(ws + ly.status);
     certkv_packed o = *out;
     o.offsets = out->offsets + (size_t)bl0 * F.H;
     o.real_counts = out->real_counts + (size_t)bl0 * F.H;
@@ -510,10 +547,12 @@ int certkv_compress(const certkv_shape* shape, const void* K, const void* V, con
   if (!K || !V || !Q_obs) return CERTKV_EINVAL;
   if (!aligned(K, 16) || !aligned(V, 16) || !aligned(Q_obs, 16)) return CERTKV_EINVAL;
   if ((rc = check_packed(p, out))) return rc;
+  p.capacity = out->capacity_slots;
   Layout ly;
   if ((rc = check_ws(p, workspace, workspace_bytes, &ly))) return rc;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   char* ws = reinterpret_cast<char*>(workspace);
+  p.status = reinterpret_cast<uint32_t*>(ws + ly.status);
   if ((rc = cuda_ok(cudaMemsetAsync(ws + ly.status, 0, 256, st)))) return rc;
   float* a = reinterpret_cast<float*>(ws + ly.a);
   launch_score(p, ly, ws, K, Q_obs, a, st);
@@ -530,6 +569,7 @@ int certkv_decode_attn(const certkv_shape* shape, const void* q, const certkv_pa
   if ((rc = decode_args(shape, q, packed, scale, tail_slot, out, &sc))) return rc;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < decode_workspace(p))
     return CERTKV_EWORKSPACE;
+  p.capacity = packed->capacity_slots;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (!launch_decode(p, q, packed->k, packed->v, packed->offsets, packed->real_counts, tail_slot,
                      sc, out, reinterpret_cast<char*>(workspace), st))
@@ -556,6 +596,7 @@ int certkv_decode_certified(const certkv_shape* shape, const void* q, const cert
   if ((rc = make_prob(shape, &prm, -1, &p))) return rc;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < decode_workspace(p))
     return CERTKV_EWORKSPACE;
+  p.capacity = packed->capacity_slots;
   const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (!launch_decode_certified(p, q, packed->k, packed->v, packed->offsets,
@@ -675,6 +716,35 @@ int certkv_coverage_profile(const certkv_shape* shape, const void* q, const void
                   abs_counts, top, order, gap, reinterpret_cast<char*>(workspace),
                   reinterpret_cast<cudaStream_t>(stream));
   return cuda_ok(cudaGetLastError());
+}
+
+int certkv_workspace_guard_arm(const certkv_shape* shape, const certkv_params* params,
+                               void* workspace, size_t workspace_bytes, void* stream) {
+  Prob p;
+  if (make_prob(shape, params, -1, &p)) return -1;
+  Layout ly;
+  if (check_ws(p, workspace, workspace_bytes, &ly)) return -1;
+  guard_arm_kernel<<<1, Layout::kMaxGuards, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      reinterpret_cast<char*>(workspace), guard_set(ly));
+  return cudaGetLastError() == cudaSuccess ? 0 : -1;
+}
+
+int certkv_workspace_guard_check(const certkv_shape* shape, const certkv_params* params,
+                                 void* workspace, size_t workspace_bytes, void* stream) {
+  Prob p;
+  if (make_prob(shape, params, -1, &p)) return -1;
+  Layout ly;
+  if (check_ws(p, workspace, workspace_bytes, &ly)) return -1;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* ws = reinterpret_cast<char*>(workspace);
+  uint32_t* count = reinterpret_cast<uint32_t*>(ws + ly.status + 4);  // beside the status word
+  if (cudaMemsetAsync(count, 0, sizeof(uint32_t), st) != cudaSuccess) return -1;
+  guard_check_kernel<<<1, Layout::kMaxGuards, 0, st>>>(ws, guard_set(ly), count);
+  uint32_t v = 0;
+  if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess ||
+      cudaMemcpy(&v, count, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return -1;
+  return (int)v;
 }
 
 int certkv_read_status(const void* workspace, void* stream) {

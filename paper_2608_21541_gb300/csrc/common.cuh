@@ -22,6 +22,22 @@ __device__ __forceinline__ void raise_status(uint32_t* status, uint32_t bit) {
   atomicOr(status, bit);
 }
 
+// ------------------------------------------------------- bounds checks --
+// In a library built with -DCERTKV_DEBUG, CERTKV_IN_BOUNDS(cond, status)
+// evaluates cond and, when it is false, sets CERTKV_STATUS_BOUNDS (4th bit of
+// the status word, if status is not null) and yields false so that the caller
+// skips the access; in the normal build it is the constant true and the
+// condition is not evaluated.
+#ifdef CERTKV_DEBUG
+__device__ __forceinline__ bool in_bounds(bool ok, uint32_t* status) {
+  if (!ok && status) atomicOr(status, 8u);
+  return ok;
+}
+#define CERTKV_IN_BOUNDS(cond, status) (::certkv::in_bounds((cond), (status)))
+#else
+#define CERTKV_IN_BOUNDS(cond, status) (true)
+#endif
+
 // -------------------------------------------------------------- bf16 ------
 __device__ __forceinline__ float bf16lo(uint32_t packed) {
   return __uint_as_float(packed << 16);

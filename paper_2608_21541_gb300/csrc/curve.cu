@@ -121,8 +121,10 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
   for (int e = 0; e < kChunk / 32; ++e) {
     const int r = r0 + e * 32 + lane;
     const bool ok = r < r1;
+    int j = ok ? pu[r] : 0;
+    if (!CERTKV_IN_BOUNDS(j >= 0 && j < n, p.status)) j = 0;
     sa[e * 32 + lane] = ok ? key_score(ku[r]) : 0.f;
-    sj[e * 32 + lane] = ok ? pu[r] : 0;
+    sj[e * 32 + lane] = j;
   }
   __syncwarp();
   const int ngroups = (r1 - r0 + kEvalGroup - 1) / kEvalGroup;  // group g: chunk ranks 8g .. 8g+7
@@ -251,8 +253,10 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
   for (int e = 0; e < kChunk / 32; ++e) {
     const int r = r0 + e * 32 + lane;
     const bool ok = r < r1;
+    int j = ok ? pu[r] : 0;
+    if (!CERTKV_IN_BOUNDS(j >= 0 && j < n, p.status)) j = 0;
     sa[e * 32 + lane] = ok ? key_score(ku[r]) : 0.f;
-    sj[e * 32 + lane] = ok ? pu[r] : 0;
+    sj[e * 32 + lane] = j;
     sy[e * 32 + lane] = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
   }
   __syncwarp();

@@ -164,13 +164,20 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
             !tc::mbar_wait(empty0 + 8 * s, ((k / kDecStages) - 1) & 1, abort_flag))
           break;
         const int t = gt - T[u];
-        const int cnt = min(kDecTile, counts[u] + tail_slot - t * kDecTile);
-        const size_t e0 = (size_t)(offsets[u] + (int64_t)t * kDecTile) * kD;
+        int cnt = min(kDecTile, counts[u] + tail_slot - t * kDecTile);
+        const int64_t s0 = offsets[u] + (int64_t)t * kDecTile;
+        // (debug builds) a tile outside the packed cache is not copied: the
+        // stage completes with no bytes and its outputs are invalid
+        if (!CERTKV_IN_BOUNDS(s0 >= 0 && (p.capacity <= 0 || s0 + cnt <= p.capacity), p.status))
+          cnt = 0;
+        const size_t e0 = (size_t)s0 * kD;
         tc::mbar_expect_tx(full0 + 8 * s, (uint32_t)cnt * 512u);
-        tc::bulk_load(tc::saddr(kst + s * kDecKBytes), pk + e0, (uint32_t)cnt * 256u,
-                      full0 + 8 * s);
-        tc::bulk_load(tc::saddr(vst + s * kDecVBytes), pv + e0, (uint32_t)cnt * 256u,
-                      full0 + 8 * s);
+        if (cnt > 0) {
+          tc::bulk_load(tc::saddr(kst + s * kDecKBytes), pk + e0, (uint32_t)cnt * 256u,
+                        full0 + 8 * s);
+          tc::bulk_load(tc::saddr(vst + s * kDecVBytes), pv + e0, (uint32_t)cnt * 256u,
+                        full0 + 8 * s);
+        }
         issued = k + 1;
       }
       // the last copies must land before the CTA exits

@@ -24,6 +24,8 @@ struct Prob {
   int64_t B_live, B_real;
   int b_min;
   int64_t slot_base;  // packed slot of this problem's first (sequence, layer): offsets are global
+  int64_t capacity;   // packed-cache slots the caller gave (0: not known to the kernels)
+  uint32_t* status;   // the workspace status word (bounds reports of debug builds; may be null)
   // derived launch geometry
   int score_tc;     // 1: tcgen05 scorer (R in {128, 256}); 0: mma.sync scorer
   int score_warps;  // warps per score CTA (16 rows each)
@@ -65,6 +67,10 @@ struct Layout {
   size_t cl_mean;    // float  [U][m][2][d]           stored cluster means
   size_t cl_max;     // float2 [U][m][8 parts]        cluster part radii
   size_t total;
+  // 16-byte guard words after the regions (certkv_workspace_guard_*)
+  static constexpr int kMaxGuards = 32;
+  size_t guard[kMaxGuards];
+  int nguards;
 };
 
 Layout make_layout(const Prob& p);

@@ -40,6 +40,7 @@ extern "C" int certkv_decode_attn_noalloc(const certkv_shape* shape, const void*
   if (decode_workspace(p) > (size_t)CERTKV_NOALLOC_SCRATCH_BYTES) return CERTKV_ETOOLARGE;
   float sc = 0.0f;
   if ((rc = decode_args(shape, q, packed, scale, tail_slot, out, &sc))) return rc;
+  p.capacity = packed->capacity_slots;
 
   // Set-up, once per device and with that device current: the device address
   // of the static scratch array.

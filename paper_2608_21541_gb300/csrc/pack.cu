@@ -29,6 +29,8 @@ __global__ void __launch_bounds__(128) tail_kernel(
   const int u = blockIdx.x, i = threadIdx.x;
   const int n = p.n;
   const int b = counts[u];
+  if (!CERTKV_IN_BOUNDS(b >= 0 && b < n, p.status)) return;
+  if (!CERTKV_IN_BOUNDS(p.capacity <= 0 || offsets[u] + b < p.capacity, p.status)) return;
   const uint32_t* ku = keys + (size_t)u * n;
   const int32_t* pu = perm + (size_t)u * n;
   const __nv_bfloat16* Ku = K + (size_t)u * n * kD;
@@ -47,8 +49,10 @@ __global__ void __launch_bounds__(128) tail_kernel(
   __shared__ float s_a[kChunk];
   __shared__ int s_j[kChunk];
   if (b + i < r_end) {
+    int j = pu[b + i];
+    if (!CERTKV_IN_BOUNDS(j >= 0 && j < n, p.status)) j = 0;
     s_a[i] = key_score(ku[b + i]);
-    s_j[i] = pu[b + i];
+    s_j[i] = j;
   }
   __syncthreads();
   for (int r0 = b; r0 < r_end; r0 += 8) {
@@ -78,7 +82,8 @@ __global__ void __launch_bounds__(128) tail_kernel(
   } else {  // zero tail mass in floating point: uniform mean of the tail
     DF sk = df_make(0.f), sv = df_make(0.f);
     for (int r = b; r < n; ++r) {
-      const int j = pu[r];
+      int j = pu[r];
+      if (!CERTKV_IN_BOUNDS(j >= 0 && j < n, p.status)) j = 0;
       sv = df_add_f(sv, __bfloat162float(Vu[(size_t)j * kD + i]));
       sk = df_add_f(sk, __bfloat162float(Ku[(size_t)j * kD + i]));
     }
@@ -111,6 +116,8 @@ __global__ void __launch_bounds__(1024) select_kernel(Prob p, const float* __res
   const int u = blockIdx.x;
   const int n = p.n;
   const int b = counts[u];
+  if (!CERTKV_IN_BOUNDS(b >= 0 && b < n, p.status)) return;
+  if (!CERTKV_IN_BOUNDS(p.capacity <= 0 || offsets[u] + b <= p.capacity, p.status)) return;
   const uint32_t kt = keys[(size_t)u * n + b];  // first evicted rank
   const int jt = perm[(size_t)u * n + b];
   const float* au = a + (size_t)u * n;
@@ -178,6 +185,9 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloa
   const int u = blockIdx.x;
   const int b = counts[u];
   const int64_t off = offsets[u];
+  if (!CERTKV_IN_BOUNDS(b >= 0 && b < p.n && off >= 0 && (p.capacity <= 0 || off + b <= p.capacity),
+                        p.status))
+    return;
   const uint4* Ku = reinterpret_cast<const uint4*>(K + (size_t)u * p.n * kD);
   const uint4* Vu = reinterpret_cast<const uint4*>(V + (size_t)u * p.n * kD);
   uint4* PK = reinterpret_cast<uint4*>(pk);
@@ -196,6 +206,7 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(Prob p, const __nv_bfloa
     for (int e = 0; e < 4; ++e) {
       const int row = row0 + e * stride;
       j[e] = row < b ? positions[off + row] : -1;
+      if (row < b && !CERTKV_IN_BOUNDS(j[e] >= 0 && j[e] < p.n, p.status)) j[e] = -1;
     }
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
@@ -299,7 +310,8 @@ __global__ void __launch_bounds__(kClusterWarps * 32) cluster_sum_kernel(
     for (int e = 0; e < 4; ++e) {
       const int r = rb + e * kClusterWarps;
       if (r < hi) {
-        const int j = pu[r];
+        int j = pu[r];
+        if (!CERTKV_IN_BOUNDS(j >= 0 && j < n, p.status)) j = 0;
         load_row4(Ku, j, lane, k4[e]);
         load_row4(Vu, j, lane, v4[e]);
       }
@@ -356,6 +368,7 @@ __global__ void __launch_bounds__(256) cluster_mean_kernel(
   const DF mean = cnt > 0 ? df_div(sum, df_make((float)cnt)) : df_make(0.f);
   const uint16_t bits = df_to_bf16(mean.hi, mean.lo);
   const int64_t slot = offsets[u] + b + p.tail_slot + g;
+  if (!CERTKV_IN_BOUNDS(p.capacity <= 0 || (slot >= 0 && slot < p.capacity), p.status)) return;
   reinterpret_cast<uint16_t*>(t == 0 ? pk : pv)[slot * kD + i] = bits;
   means[(((size_t)u * m + g) * 2 + t) * kD + i] = __uint_as_float((uint32_t)bits << 16);
   if (threadIdx.x == 0) positions[slot] = -2 - g;
@@ -386,7 +399,8 @@ __global__ void __launch_bounds__(kClusterWarps * 32) cluster_radius_kernel(
     for (int e = 0; e < 4; ++e) {
       const int r = rb + e * kClusterWarps;
       if (r < hi) {
-        const int j = pu[r];
+        int j = pu[r];
+        if (!CERTKV_IN_BOUNDS(j >= 0 && j < n, p.status)) j = 0;
         load_row4(Ku, j, lane, k4[e]);
         load_row4(Vu, j, lane, v4[e]);
       }

@@ -119,7 +119,8 @@ __global__ void __launch_bounds__(1024) radix_scan_kernel(uint32_t* __restrict__
 template <bool kFirst>  // at most 48 registers: five CTAs per SM to hide the load latency
 __global__ void __launch_bounds__(kSortThreads, 5) radix_scatter_kernel(
     const uint32_t* __restrict__ kin, const int32_t* __restrict__ vin, uint32_t* __restrict__ kout,
-    int32_t* __restrict__ vout, int n, int tiles, int shift, const uint32_t* __restrict__ hist) {
+    int32_t* __restrict__ vout, int n, int tiles, int shift, const uint32_t* __restrict__ hist,
+    uint32_t* status) {
   __shared__ uint32_t wcnt[kWarps][256];
   __shared__ uint32_t gbase[256];
   __shared__ uint32_t tstart[256];
@@ -212,6 +213,7 @@ __global__ void __launch_bounds__(kSortThreads, 5) radix_scatter_kernel(
     const uint32_t k = skey[i];
     const uint32_t d = (k >> shift) & 255u;
     const uint32_t pos = gbase[d] + (uint32_t)i - tstart[d];
+    if (!CERTKV_IN_BOUNDS(pos < (uint32_t)n, status)) continue;
     ko[pos] = k;
     vo[pos] = sval[i];
   }
@@ -242,10 +244,12 @@ void launch_sort(const Prob& p, const Layout& ly, char* ws, const float* /*a*/, 
       TraceScope ts_("sort_scatter", st);
       if (pass == 0)
         radix_scatter_kernel<true><<<grid, kSortThreads, 0, st>>>(kin, vin, kout, vout, p.n,
-                                                                  p.sort_tiles, shift, hist);
+                                                                  p.sort_tiles, shift, hist,
+                                                                  p.status);
       else
         radix_scatter_kernel<false><<<grid, kSortThreads, 0, st>>>(kin, vin, kout, vout, p.n,
-                                                                   p.sort_tiles, shift, hist);
+                                                                   p.sort_tiles, shift, hist,
+                                                                   p.status);
     }
   }
   // after 4 passes the sorted keys / permutation are back in keys0 / vals0

@@ -216,3 +216,26 @@ def test_sampled_compensation_validation(lib):
     assert call(scale=float("nan")) == ck.EINVAL
     assert call(ws=0) == ck.EWORKSPACE
     assert call(ws_bytes=need - 1) == ck.EWORKSPACE
+
+
+def test_workspace_guards_refuse_bad_arguments_on_the_host(lib):
+    """Guard words: an invalid shape or a missing, misaligned or short
+    workspace returns -1 before anything is enqueued."""
+    s, p = shape(), ck.certkv_default_params()
+    need = ck.certkv_workspace_bytes(s, p)
+    assert need > 0
+    for fn in (lib.certkv_workspace_guard_arm, lib.certkv_workspace_guard_check):
+        assert fn(ctypes.byref(s), ctypes.byref(p), None, need, None) == -1
+        assert fn(ctypes.byref(s), ctypes.byref(p), ctypes.c_void_p(256), need - 1, None) == -1
+        assert fn(ctypes.byref(s), ctypes.byref(p), ctypes.c_void_p(16), need, None) == -1
+        assert fn(ctypes.byref(shape(d=64)), ctypes.byref(p), ctypes.c_void_p(256), need, None) == -1
+
+
+def test_bounds_checking_build_compiles_and_exports_the_same_symbols():
+    """The -DCERTKV_DEBUG build (bounds checks on every ragged index) links
+    with the same entry points (compiled here; its GPU test is
+    tests/test_gpu_debug.py)."""
+    path = B.build(debug=True)
+    dbg = ctypes.CDLL(path)
+    for name in declared_functions():
+        assert hasattr(dbg, name), name

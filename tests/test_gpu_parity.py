@@ -57,10 +57,18 @@ def run_case(name, wl=None, params=None, B_live=None, seed=0):
     params = params or ck.certkv_default_params()
     B_live = B_live or wl.B_live
     K, V, Q = W.draw(wl, seed=seed, device=DEV)
-    a = ck.certkv_score(K, Q, params)
-    packed = ck.certkv_compress(K, V, Q, B_live, params, with_tail=True)
-    scored = ck.certkv_compress_scored(K, V, a, B_live, params, hq=wl.Hq, w=wl.w, with_tail=True)
+    # one workspace for the three calls, with its guard words armed: no
+    # kernel may write past the end of a region
+    shape = ck.shape_of(K, Q)
+    ws = ck.workspace(ck.certkv_workspace_bytes(shape, params), DEV)
+    ck.certkv_workspace_guard_arm(ws, shape, params)
+    a = ck.certkv_score(K, Q, params, ws=ws)
+    packed = ck.certkv_compress(K, V, Q, B_live, params, ws=ws, with_tail=True)
+    scored = ck.certkv_compress_scored(K, V, a, B_live, params, hq=wl.Hq, w=wl.w, ws=ws,
+                                       with_tail=True)
     torch.cuda.synchronize()
+    guards = ck.certkv_workspace_guard_check(ws, shape, params)
+    status = ck.certkv_read_status(ws)
     host = dict(K=parity.bits(K), V=parity.bits(V), Q=parity.bits(Q),
                 a=a.cpu().numpy())
     kw = dict(B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, n=wl.n, d=wl.d, w=wl.w, B_live=B_live,
@@ -71,9 +79,19 @@ def run_case(name, wl=None, params=None, B_live=None, seed=0):
     ref_e2e = oracle.compress(host["K"], host["V"], host["Q"], **kw)
     ref_cond = oracle.compress(host["K"], host["V"], None, a_in=host["a"], **kw)
     res = dict(wl=wl, params=params, B_live=B_live, K=K, V=V, Q=Q, a=a, packed=packed,
-               scored=scored, host=host, ref_e2e=ref_e2e, ref_cond=ref_cond)
+               scored=scored, host=host, ref_e2e=ref_e2e, ref_cond=ref_cond, guards=guards,
+               status=status)
     _cache[key] = res
     return res
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+def test_workspace_guards_intact(name):
+    """After certkv_score, certkv_compress and certkv_compress_scored on one
+    workspace, every region's guard words still hold their pattern."""
+    r = run_case(name)
+    assert r["guards"] == 0, f"{r['guards']} workspace guard words overwritten"
+    assert r["status"] == 0, r["status"]
 
 
 @pytest.mark.parametrize("name", sorted(CASES))
