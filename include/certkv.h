@@ -419,6 +419,16 @@ int certkv_workspace_guard_arm(const certkv_shape* shape, const certkv_params* p
 int certkv_workspace_guard_check(const certkv_shape* shape, const certkv_params* params,
                                  void* workspace, size_t workspace_bytes, void* stream);
 
+/* Self-test of the bounded waits the kernels use (a debugging aid with no
+ * counterpart in the paper): one thread waits on an mbarrier that nothing
+ * arrives on, with no copy and no MMA in flight.  The wait must give up after
+ * its poll limit (a few seconds at most) and report a timeout without any
+ * fault.  Synchronises `stream` and returns CERTKV_STATUS_TIMEOUT when it
+ * did; -2 if the wait did not give up as designed; -1 on a CUDA error.  Its
+ * result sits in a small array of the library's own device memory: calls
+ * that overlap on the GPU race on it. */
+int certkv_selftest_bounded_wait(void* stream);
+
 /* Synchronise `stream`, then return the device status word (CERTKV_STATUS_*
  * bits, 0 = clean) that the last compress call on `workspace` left, or -1 if
  * a CUDA call failed.  Host pointer args: none. */

@@ -57,7 +57,8 @@ EXPORTED = ("certkv_default_params", "certkv_live_budget", "certkv_workspace_byt
             "certkv_fixed_row_stats", "certkv_coverage_workspace_bytes",
             "certkv_coverage_profile", "certkv_sampled_workspace_bytes",
             "certkv_sampled_compensation", "certkv_compress_host_copyback",
-            "certkv_workspace_guard_arm", "certkv_workspace_guard_check")
+            "certkv_workspace_guard_arm", "certkv_workspace_guard_check",
+            "certkv_selftest_bounded_wait")
 
 _lock = threading.Lock()
 _lib = None
@@ -108,6 +109,8 @@ def load_library(path: Optional[str] = None):
         lib.certkv_workspace_guard_arm.restype = ctypes.c_int
         lib.certkv_workspace_guard_check.argtypes = [sp, pp, P, SZ, P]
         lib.certkv_workspace_guard_check.restype = ctypes.c_int
+        lib.certkv_selftest_bounded_wait.argtypes = [P]
+        lib.certkv_selftest_bounded_wait.restype = ctypes.c_int
         lib.certkv_strerror.argtypes = [ctypes.c_int]
         lib.certkv_strerror.restype = ctypes.c_char_p
         lib.certkv_trace_enable.argtypes = [ctypes.c_int]

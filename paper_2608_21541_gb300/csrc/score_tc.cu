@@ -468,6 +468,24 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
 
 }  // namespace tc
 
+// Self-test of the bounded wait: one thread waits on an mbarrier that nothing
+// arrives on (no copy and no MMA is issued), so the wait must give up after
+// its poll limit, set the abort flag and report CERTKV_STATUS_TIMEOUT.
+__device__ uint32_t g_selftest_result[2];
+__global__ void selftest_wait_kernel() {
+  uint32_t* result = g_selftest_result;
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(tc::saddr(&bar), 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    const bool done = tc::mbar_wait(tc::saddr(&bar), 0, &abort_flag);
+    result[0] = done ? 0u : tc::kStatusTimeout;
+    result[1] = (uint32_t)abort_flag;
+  }
+}
+
 // --------------------------------------------------------------- host ----
 namespace {
 
@@ -546,3 +564,16 @@ bool launch_score_tc(const Prob& p, const void* K, const void* Q, float2* lse_pa
 }
 
 }  // namespace certkv
+
+extern "C" int certkv_selftest_bounded_wait(void* stream) {
+  using namespace certkv;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t h[2] = {0u, 0u};
+  selftest_wait_kernel<<<1, 32, 0, st>>>();
+  if (cudaGetLastError() != cudaSuccess ||
+      cudaMemcpyFromSymbolAsync(h, g_selftest_result, sizeof h, 0, cudaMemcpyDeviceToHost, st) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return -1;
+  return (h[0] == CERTKV_STATUS_TIMEOUT && h[1] == 1u) ? (int)h[0] : -2;
+}

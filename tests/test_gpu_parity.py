@@ -129,6 +129,15 @@ def test_compress_pass_equals_scored_path(name):
 
 
 @pytest.mark.parametrize("name", sorted(CASES))
+def test_compress_pass_conditioned(name):
+    """certkv_compress itself against the oracle conditioned on the same
+    scores: budgets, positions and real slots bit-exact, tail mass and
+    centroids within 1e-4."""
+    r = run_case(name)
+    parity.check_conditioned(parity.packed_np(r["packed"]), r["ref_cond"], r["wl"].units)
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
 def test_compress_end_to_end(name):
     r = run_case(name)
     got = parity.packed_np(r["packed"])
