@@ -634,6 +634,7 @@ int certkv_fixed_row_stats(const certkv_shape* shape, const void* q, const void*
   if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < fixed_row_workspace(p))
     return CERTKV_EWORKSPACE;
+  p.capacity = packed->capacity_slots;  // its decode runs as certkv_decode_attn does
   const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
   if (!launch_fixed_row(p, q, K, V, scores, packed->offsets, packed->real_counts,
                         packed->positions, packed->k, packed->v, tail_slot, sc, stats,
@@ -667,6 +668,7 @@ int certkv_sampled_compensation(const certkv_shape* shape, const void* q, const 
   if (!(scale >= 0.0f) || !isfinite(scale)) return CERTKV_EINVAL;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < sampled_workspace(p))
     return CERTKV_EWORKSPACE;
+  p.capacity = packed->capacity_slots;
   const float sc = scale > 0.0f ? scale : (float)(1.0 / sqrt((double)shape->d));
   if (!launch_sampled(p, q, K, V, packed->offsets, packed->real_counts, packed->positions, m, unif,
                       idx_out, sc, stats, reinterpret_cast<char*>(workspace),

@@ -361,6 +361,305 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
   __syncthreads();
 }
 
+// ---------------------------------------------------------------------------
+// Tensor-core split kernel for G = 8 and 16 query heads per KV head.  At these
+// group sizes the CUDA-core consumer needs ~4 fp32 FMAs per byte of cache;
+// here both products run as mma.sync m16n8k16 (bf16 in, fp32 accumulate)
+// with the G query heads as the M rows (padded to 16 with zero rows for
+// G = 8): S = Q K^T over 32 slots (4 n-blocks x 8 k-steps), online softmax per
+// row in the log2 domain, then O += P V (2 k-blocks x 16 n-blocks) with P as a
+// bf16 part plus the bf16 rounding of its remainder (fp32-level weights).  The tiles arrive by TMA with 128-byte swizzle (two boxes of
+// 64 dimensions x 32 slots for K and for V), so the ldmatrix reads are free of
+// bank conflicts; rows past the segment (the next segment's, or zeros past
+// the cache) get weight 0.  Work split, records and merge as in
+// decode_split_kernel.
+constexpr int kTcStageBytes = 4 * 4096;  // K and V, two 64-dimension halves each
+template <int G>
+__host__ __device__ constexpr int decode_tc_smem_bytes() {
+  return kDecStages * kTcStageBytes + kDecConsumers * G * kD * 4 + 2 * kDecConsumers * G * 4 +
+         2 * kDecStages * 8 + 16 + 1024;
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+// byte address of (slot, 16-byte chunk c of the 256-byte row) in a tile of 32
+// rows stored as two 128-byte-swizzled halves of 4096 bytes
+__device__ __forceinline__ uint32_t sw_addr(uint32_t tile, int slot, int c) {
+  return tile + (uint32_t)((c >> 3) * 4096 + slot * 128 + (((c & 7) ^ (slot & 7)) << 4));
+}
+
+template <int G>
+__global__ void __launch_bounds__(kDecThreads) decode_split_tc_kernel(
+    const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Prob p,
+    const __nv_bfloat16* __restrict__ q, const int64_t* __restrict__ offsets,
+    const int32_t* __restrict__ counts, const int32_t* __restrict__ T, int tail_slot,
+    float scale_log2, float2* __restrict__ rec_ml, float* __restrict__ rec_acc) {
+  static_assert(G == 8 || G == 16, "the tensor-core decode takes 8 or 16 query heads per KV head");
+  extern __shared__ uint8_t dsm_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
+  // stage s: K halves at + 0 / 4096, V halves at + 8192 / 12288
+  float* wacc = reinterpret_cast<float*>(sm + kDecStages * kTcStageBytes);  // [consumers][G][kD]
+  float* wm = wacc + kDecConsumers * G * kD;                                // [consumers][G]
+  float* wl = wm + kDecConsumers * G;                                       // [consumers][G]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(wl + kDecConsumers * G);     // full, empty
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * kDecStages);
+  const uint32_t full0 = tc::saddr(bars), empty0 = tc::saddr(bars + kDecStages);
+  const uint32_t stage0 = tc::saddr(sm);
+
+  const int units = p.units;
+  const int total = T[units];
+  const int per = (total + (int)gridDim.x - 1) / (int)gridDim.x;
+  const int g0 = min(total, (int)blockIdx.x * per), g1 = min(total, g0 + per);
+  if (g0 >= g1) return;  // uniform over the CTA, before any barrier
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  int lo = 0, hi = units;  // first unit of the range: the last u with T[u] <= g0
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (T[mid] <= g0) lo = mid;
+    else hi = mid;
+  }
+  const int u_first = lo;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kDecStages; ++s) {
+      tc::mbar_init(full0 + 8 * s, 1);
+      tc::mbar_init(empty0 + 8 * s, 1);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+
+  if (warp == 0) {
+    if (lane == 0) {  // producer: tiles g0 .. g1-1 in order, four TMA boxes each
+      int u = u_first, issued = 0;
+      for (int k = 0; k < g1 - g0; ++k) {
+        const int gt = g0 + k;
+        while (T[u + 1] <= gt) ++u;
+        const int s = k % kDecStages;
+        if (k >= kDecStages &&
+            !tc::mbar_wait(empty0 + 8 * s, ((k / kDecStages) - 1) & 1, abort_flag))
+          break;
+        const int t = gt - T[u];
+        const int64_t s0 = offsets[u] + (int64_t)t * kDecTile;
+        const int cnt = min(kDecTile, counts[u] + tail_slot - t * kDecTile);
+        const uint32_t st = stage0 + (uint32_t)(s * kTcStageBytes);
+        tc::mbar_expect_tx(full0 + 8 * s, (uint32_t)kTcStageBytes);
+        // (debug builds) a tile that starts outside the packed cache is not
+        // loaded: the boxes are then read at row 0 and weighted 0
+        const int y = CERTKV_IN_BOUNDS(s0 >= 0 && (p.capacity <= 0 || s0 + cnt <= p.capacity),
+                                       p.status)
+                          ? (int)s0
+                          : 0;
+        tc::tma_load_2d(st, &tmK, 0, y, full0 + 8 * s);
+        tc::tma_load_2d(st + 4096, &tmK, 64, y, full0 + 8 * s);
+        tc::tma_load_2d(st + 8192, &tmV, 0, y, full0 + 8 * s);
+        tc::tma_load_2d(st + 12288, &tmV, 64, y, full0 + 8 * s);
+        issued = k + 1;
+      }
+      // the last copies must land before the CTA exits
+      for (int k = issued > kDecStages ? issued - kDecStages : 0; k < issued; ++k) {
+        volatile int dummy = 0;
+        tc::mbar_wait(full0 + 8 * (k % kDecStages), (k / kDecStages) & 1, &dummy);
+      }
+    }
+  } else {  // consumers: one segment per unit met
+    const int cw = warp - 1, ct = threadIdx.x - 32;
+    const int qr = lane >> 2, qc = lane & 3;  // fragment row (head), column pair
+    // ldmatrix row addresses of this lane: matrix mi = lane / 8, row lane % 8
+    const int mi = lane >> 3, mr = lane & 7;
+    for (int u = u_first; u < units && T[u] < g1; ++u) {
+      const int ka = max(g0, T[u]) - g0, kb = min(g1, T[u + 1]) - g0;
+      if (ka >= kb) continue;  // a unit without tiles (uniform over the consumers)
+      const int bl = u / p.H, h = u - bl * p.H;
+      // Q as the A operand (rows 0..G-1 the group's heads, zero above), 8 k-steps
+      const uint32_t* qg = reinterpret_cast<const uint32_t*>(q + ((size_t)bl * p.Hq + (size_t)h * G) * kD);
+      uint32_t qa[8][4];
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) {
+        const int c0 = (16 * ks + 2 * qc) / 2;  // 32-bit word of dims 16 ks + 2 qc, +1
+        qa[ks][0] = __ldg(qg + qr * (kD / 2) + c0);
+        qa[ks][2] = __ldg(qg + qr * (kD / 2) + c0 + 4);
+        if (G == 16) {
+          qa[ks][1] = __ldg(qg + (qr + 8) * (kD / 2) + c0);
+          qa[ks][3] = __ldg(qg + (qr + 8) * (kD / 2) + c0 + 4);
+        } else {
+          qa[ks][1] = qa[ks][3] = 0u;
+        }
+      }
+      const int slots = counts[u] + tail_slot;
+      float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;  // rows qr, qr + 8
+      float o[16][4];
+#pragma unroll
+      for (int nd = 0; nd < 16; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+      for (int k = ka + ((cw - ka % kDecConsumers) + kDecConsumers) % kDecConsumers; k < kb;
+           k += kDecConsumers) {
+        const int s = k % kDecStages;
+        bool skip = __any_sync(kFull, *abort_flag != 0);
+        if (!skip) skip = !__all_sync(kFull, tc::mbar_wait(full0 + 8 * s, (k / kDecStages) & 1,
+                                                           abort_flag));
+        if (skip) continue;
+        const int t = g0 + k - T[u];
+        const int cnt = min(kDecTile, slots - t * kDecTile);
+        const uint32_t kt = stage0 + (uint32_t)(s * kTcStageBytes), vt = kt + 8192;
+        // S = Q K^T: 4 n-blocks of 8 slots
+        float sc[4][4];
+#pragma unroll
+        for (int nb = 0; nb < 4; ++nb) sc[nb][0] = sc[nb][1] = sc[nb][2] = sc[nb][3] = 0.f;
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks) {
+#pragma unroll
+          for (int np = 0; np < 2; ++np) {  // n-block pair (2 np, 2 np + 1)
+            uint32_t b0, b1, b2, b3;
+            // matrix mi: slots 8 (2 np + mi / 2) + mr, dims 16 ks + 8 (mi & 1)
+            ldsm_x4(sw_addr(kt, 8 * (2 * np + (mi >> 1)) + mr, 2 * ks + (mi & 1)), b0, b1, b2, b3);
+            mma_bf16_16816(sc[2 * np], qa[ks], b0, b1);
+            mma_bf16_16816(sc[2 * np + 1], qa[ks], b2, b3);
+          }
+        }
+        // online softmax (log2 domain) of rows qr and qr + 8 over the tile
+        float tm0 = -INFINITY, tm1 = -INFINITY;
+#pragma unroll
+        for (int nb = 0; nb < 4; ++nb) {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const bool ok = 8 * nb + 2 * qc + e < cnt;
+            sc[nb][e] = ok ? sc[nb][e] * scale_log2 : -INFINITY;
+            sc[nb][2 + e] = ok ? sc[nb][2 + e] * scale_log2 : -INFINITY;
+            tm0 = fmaxf(tm0, sc[nb][e]);
+            tm1 = fmaxf(tm1, sc[nb][2 + e]);
+          }
+        }
+        tm0 = fmaxf(tm0, __shfl_xor_sync(kFull, tm0, 1));
+        tm0 = fmaxf(tm0, __shfl_xor_sync(kFull, tm0, 2));
+        tm1 = fmaxf(tm1, __shfl_xor_sync(kFull, tm1, 1));
+        tm1 = fmaxf(tm1, __shfl_xor_sync(kFull, tm1, 2));
+        const float n0 = fmaxf(m0, tm0), n1 = fmaxf(m1, tm1);
+        const float c0 = exp2f(m0 - n0), c1 = exp2f(m1 - n1);  // both -inf: no slot yet
+        m0 = n0;
+        m1 = n1;
+        // P as the A operand of two k16 blocks, split into a bf16 part and the
+        // bf16 rounding of its remainder (P = ph + pl to ~2^-16 relative), so
+        // that the weights carry fp32 accuracy into the tensor-core products
+        uint32_t ph[2][4], pl[2][4];
+        float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+        for (int nb = 0; nb < 4; ++nb) {
+          const float p0 = n0 > -INFINITY ? exp2f(sc[nb][0] - n0) : 0.f;
+          const float p1 = n0 > -INFINITY ? exp2f(sc[nb][1] - n0) : 0.f;
+          const float p2 = n1 > -INFINITY ? exp2f(sc[nb][2] - n1) : 0.f;
+          const float p3 = n1 > -INFINITY ? exp2f(sc[nb][3] - n1) : 0.f;
+          ps0 += p0 + p1;
+          ps1 += p2 + p3;
+          const uint32_t h01 = pack_bf16(p0, p1), h23 = pack_bf16(p2, p3);
+          const uint32_t l01 = pack_bf16(p0 - bf16lo(h01), p1 - bf16hi(h01));
+          const uint32_t l23 = pack_bf16(p2 - bf16lo(h23), p3 - bf16hi(h23));
+          ph[nb >> 1][(nb & 1) * 2 + 0] = h01;
+          ph[nb >> 1][(nb & 1) * 2 + 1] = h23;
+          pl[nb >> 1][(nb & 1) * 2 + 0] = l01;
+          pl[nb >> 1][(nb & 1) * 2 + 1] = l23;
+        }
+        l0 = l0 * (n0 > -INFINITY ? c0 : 1.f) + ps0;
+        l1 = l1 * (n1 > -INFINITY ? c1 : 1.f) + ps1;
+        const float r0 = n0 > -INFINITY ? c0 : 1.f, r1 = n1 > -INFINITY ? c1 : 1.f;
+#pragma unroll
+        for (int nd = 0; nd < 16; ++nd) {
+          o[nd][0] *= r0;
+          o[nd][1] *= r0;
+          o[nd][2] *= r1;
+          o[nd][3] *= r1;
+        }
+        // O += P V: k16 blocks of slots, n-block pairs of dimensions
+#pragma unroll
+        for (int kb2 = 0; kb2 < 2; ++kb2) {
+#pragma unroll
+          for (int np = 0; np < 8; ++np) {
+            uint32_t b0, b1, b2, b3;
+            // matrix mi: slots 16 kb2 + 8 (mi & 1) + mr, dims 8 (2 np + mi / 2)
+            ldsm_x4_t(sw_addr(vt, 16 * kb2 + 8 * (mi & 1) + mr, 2 * np + (mi >> 1)), b0, b1, b2,
+                      b3);
+            mma_bf16_16816(o[2 * np], ph[kb2], b0, b1);
+            mma_bf16_16816(o[2 * np + 1], ph[kb2], b2, b3);
+            mma_bf16_16816(o[2 * np], pl[kb2], b0, b1);
+            mma_bf16_16816(o[2 * np + 1], pl[kb2], b2, b3);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(empty0 + 8 * s);
+      }
+      // the row sums over the quad, then this warp's record slices
+      l0 += __shfl_xor_sync(kFull, l0, 1);
+      l0 += __shfl_xor_sync(kFull, l0, 2);
+      l1 += __shfl_xor_sync(kFull, l1, 1);
+      l1 += __shfl_xor_sync(kFull, l1, 2);
+      if (qc == 0) {
+        wm[cw * G + qr] = m0;
+        wl[cw * G + qr] = l0;
+        if (G == 16) {
+          wm[cw * G + qr + 8] = m1;
+          wl[cw * G + qr + 8] = l1;
+        }
+      }
+#pragma unroll
+      for (int nd = 0; nd < 16; ++nd) {
+        const int d = 8 * nd + 2 * qc;
+        *reinterpret_cast<float2*>(&wacc[(cw * G + qr) * kD + d]) = make_float2(o[nd][0], o[nd][1]);
+        if (G == 16)
+          *reinterpret_cast<float2*>(&wacc[(cw * G + qr + 8) * kD + d]) =
+              make_float2(o[nd][2], o[nd][3]);
+      }
+      consumers_sync();
+      const bool failed = *abort_flag != 0;
+      const size_t rec = (size_t)blockIdx.x + u;
+      for (int idx = ct; idx < G * kD; idx += kDecConsumers * 32) {
+        const int g = idx / kD, i = idx - g * kD;
+        float M = -INFINITY;
+#pragma unroll
+        for (int wi = 0; wi < kDecConsumers; ++wi) M = fmaxf(M, wm[wi * G + g]);
+        float L = 0.f, A = 0.f;
+#pragma unroll
+        for (int wi = 0; wi < kDecConsumers; ++wi) {
+          if (wm[wi * G + g] > -INFINITY) {
+            const float f = exp2f(wm[wi * G + g] - M);
+            L += wl[wi * G + g] * f;
+            A += wacc[(wi * G + g) * kD + i] * f;
+          }
+        }
+        if (failed) {
+          M = 0.f;
+          L = A = __int_as_float(0x7fc00000);
+        }
+        rec_acc[(rec * G + g) * kD + i] = A;
+        if (i == 0) rec_ml[rec * G + g] = make_float2(M, L);
+      }
+      consumers_sync();  // wm / wl / wacc are reused by the next unit
+    }
+  }
+  __syncthreads();
+}
+
 // The records of unit u, merged for query head g of its group (log2 domain):
 // returns the running maximum and sum and this thread's dimension of the sum.
 __device__ __forceinline__ void merge_records(const int32_t* __restrict__ T, int units, int nb,
@@ -535,6 +834,45 @@ int launch_split(const Prob& p, const __nv_bfloat16* q, const __nv_bfloat16* pk,
   return nb;
 }
 
+template <int G>
+int split_tc_blocks() {
+  static int cached[kDecMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
+  if (dev < kDecMaxDevices && cached[dev] > 0) return cached[dev];
+  int sms = 0, per_sm = 0;
+  if (cudaFuncSetAttribute(decode_split_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           decode_tc_smem_bytes<G>()) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_split_tc_kernel<G>,
+                                                    kDecThreads, decode_tc_smem_bytes<G>()) !=
+          cudaSuccess ||
+      per_sm < 1 || sms < 1)
+    return 0;
+  const int nb = sms * per_sm < kDecMaxBlocks ? sms * per_sm : kDecMaxBlocks;
+  if (dev < kDecMaxDevices) cached[dev] = nb;
+  return nb;
+}
+
+// the tensor-core split kernel (G = 8, 16); 0 if it cannot run (no tensor
+// maps for the packed cache, or no occupancy)
+template <int G>
+int launch_split_tc(const Prob& p, const __nv_bfloat16* q, const void* pk, const void* pv,
+                    const int64_t* offsets, const int32_t* counts, const int32_t* T, int tail_slot,
+                    float sl2, float2* ml, float* acc, cudaStream_t st) {
+  if (p.capacity <= 0) return 0;
+  CUtensorMap mk, mv;
+  if (!make_row_map(&mk, pk, (uint64_t)p.capacity, kDecTile) ||
+      !make_row_map(&mv, pv, (uint64_t)p.capacity, kDecTile))
+    return 0;
+  const int nb = split_tc_blocks<G>();
+  if (nb < 1) return 0;
+  TraceScope ts_("decode_split", st);
+  decode_split_tc_kernel<G><<<nb, kDecThreads, decode_tc_smem_bytes<G>(), st>>>(
+      mk, mv, p, q, offsets, counts, T, tail_slot, sl2, ml, acc);
+  return nb;
+}
+
 // plan + split kernels; returns the number of split CTAs (0: nothing launched)
 int run_splits(const Prob& p, const void* q, const void* pk, const void* pv,
                const int64_t* offsets, const int32_t* counts, int tail_slot, float scale,
@@ -555,8 +893,14 @@ int run_splits(const Prob& p, const void* q, const void* pk, const void* pv,
     case 1: return launch_split<1>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
     case 2: return launch_split<2>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
     case 4: return launch_split<4>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
-    case 8: return launch_split<8>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
-    case 16: return launch_split<16>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    case 8: {
+      const int nb = launch_split_tc<8>(p, qb, pk, pv, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+      return nb > 0 ? nb : launch_split<8>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    }
+    case 16: {
+      const int nb = launch_split_tc<16>(p, qb, pk, pv, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+      return nb > 0 ? nb : launch_split<16>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    }
     default: return 0;
   }
 }
