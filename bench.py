@@ -146,9 +146,9 @@ def kernel_work(wl, B_live, name):
 
 
 # DRAM bytes (read + write) per unit from one ncu capture of the kernel as it
-# is now (dram__bytes_read.sum + dram__bytes_write.sum over a 16-unit launch,
-# profiles/curve_agg_eval_c3_2layers.md), scaled by the units of a launch.
-# A kernel that changes after its capture must lose its entry here.
+# is now (dram__bytes_read.sum + dram__bytes_write.sum over a 16-unit launch of
+# the 2-layer C3 case), scaled by the units of a launch.  A kernel that changes
+# after its capture must lose its entry here.
 MEASURED_TRAFFIC_PER_UNIT = {"curve_agg": (1.090560e9 + 33.102336e6) / 16}
 
 
@@ -174,10 +174,20 @@ def roofline_for(name, work, ms, peaks, traffic=None):
             "peak_source": peaks["source"] + " (copy bandwidth)"}
 
 
-# DRAM bytes (read + write) of the whole compression pass per step, summed over
-# its kernels from one ncu capture of the build as it is now, keyed by
-# workload; null when the pass has changed since the counters were taken.
-MEASURED_PASS_TRAFFIC = {}
+# DRAM bytes (read + write) of the whole compression pass per unit (one KV
+# head of one layer), summed over every compression kernel of one ncu capture
+# of the 2-layer C3 case (16 units, 131072 tokens each; each layer's K and V
+# are 4x the L2, so the traffic grows in proportion to the units), keyed by
+# workload.  A workload without an entry, or a pass changed since the
+# counters were taken, reports null.
+MEASURED_PASS_TRAFFIC_PER_UNIT = {"C3": (3054909099 + 131264341) / 16}
+
+
+def measured_pass_traffic(wl):
+    per_unit = MEASURED_PASS_TRAFFIC_PER_UNIT.get(wl.name)
+    if per_unit is None or wl.n != 131072:
+        return None
+    return round(per_unit * wl.units)
 
 
 def compress_roofline(wl, B_live, compress_ms, peaks):
@@ -189,7 +199,7 @@ def compress_roofline(wl, B_live, compress_ms, peaks):
     return {"kernel": "compress (whole pass, every kernel)", "bound": "hbm",
             "achieved": round(ach, 1), "peak": peaks["hbm"], "unit": "GB/s",
             "frac": round(ach / peaks["hbm"], 4),
-            "traffic": MEASURED_PASS_TRAFFIC.get((wl.name, wl.L, wl.B)),
+            "traffic": measured_pass_traffic(wl),
             "bytes_per_step": nbytes, "ms": round(compress_ms, 4),
             "peak_source": peaks["source"] + " (copy bandwidth)"}
 

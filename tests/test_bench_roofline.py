@@ -43,3 +43,16 @@ def test_score_passes_are_tensor_bound_at_full_size():
     assert work["flops"] == 2.0 * wl.G * wl.w * wl.d * wl.n * wl.units
     r = bench.roofline_for("score_pass1", work, 1.8, PEAKS)
     assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
+
+
+def test_pass_traffic_scales_with_units():
+    """The whole-pass DRAM traffic was counted on 16 units (2 layers x 8 KV
+    heads) and is reported for a launch of any number of 131072-token units;
+    other workloads report none."""
+    wl = W.WORKLOADS["C3"]
+    full = bench.measured_pass_traffic(wl)
+    two = bench.measured_pass_traffic(wl.with_(L=2))
+    assert abs(full - 16 * two) <= 16
+    assert bench.compress_roofline(wl, wl.B_live, 10.0, PEAKS)["traffic"] == full
+    assert bench.measured_pass_traffic(W.WORKLOADS["C1"]) is None
+    assert bench.measured_pass_traffic(wl.with_(n=4096)) is None
