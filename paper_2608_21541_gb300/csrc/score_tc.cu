@@ -13,8 +13,9 @@
 //   warp 1      TMEM allocation and the single MMA-issuing thread
 //               (tcgen05.mma kind::f16, bf16 x bf16 -> fp32 in TMEM, two
 //               accumulator buffers so MMA and epilogue overlap);
-//   warps 2..17 epilogue: two groups of 8 warps, group g reads the
-//               accumulator buffer g (tiles of parity g): tcgen05.ld, exp2,
+//   warps 2..17 epilogue: warp (q, cq) reads TMEM lane quadrant q and the
+//               64-column quarter cq of every tile's accumulator buffer
+//               (tcgen05.ld), releases the buffer, then does the exp2 and the
 //               reductions.
 // Every mbarrier wait is bounded; a timeout sets an abort flag and the status
 // word, every role then drains and the CTA frees its TMEM before returning.
