@@ -33,13 +33,18 @@ namespace tc {
 #ifndef CERTKV_TC_STAGES
 #define CERTKV_TC_STAGES 4
 #endif
+#ifndef CERTKV_TC_STAGES1
+#define CERTKV_TC_STAGES1 3
+#endif
 constexpr int kEpiWarps = 16;  // warp (q, cq): TMEM lane quadrant q, 64-column quarter cq
 constexpr int kThreads = (2 + kEpiWarps) * 32;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kStatusTimeout = CERTKV_STATUS_TIMEOUT;
 
-// Shared-memory plan of one pass: Q rows staged once, a ring of K tiles.
-template <int QROWS, int TKEYS, int STAGES>
+// Shared-memory plan of one pass: Q rows staged once, a ring of K tiles, then
+// MISC bytes: the barriers (256 B), the TMEM slot and abort flag (256 B) and
+// any per-pass scratch.
+template <int QROWS, int TKEYS, int STAGES, int MISC>
 struct Cfg {
   static constexpr int kQRows = QROWS;
   static constexpr int kTileKeys = TKEYS;
@@ -47,12 +52,16 @@ struct Cfg {
   static constexpr int kQBytes = QROWS * 128 * 2;        // two 128-B-wide halves
   static constexpr int kStageBytes = TKEYS * 128 * 2;    // one K tile, two halves
   static constexpr int kBarOff = kQBytes + STAGES * kStageBytes;
-  static constexpr int kSmemBytes = kBarOff + 8192 + 1024;  // + misc + alignment slack
+  static constexpr int kSmemBytes = kBarOff + MISC + 1024;  // + alignment slack
+  static_assert(kSmemBytes <= 232448, "over the 227 KB of shared memory a CTA can have");
 };
-// pass 1: one 128-row half of Q per CTA, 256-key tiles (M128 x N256 MMAs)
-using Pass1 = Cfg<128, 256, 2>;
-// pass 2: all (<= 256) rows of Q, 128-key tiles (M128 x N<=256 MMAs)
-using Pass2 = Cfg<256, 128, CERTKV_TC_STAGES>;
+// pass 1: one 128-row half of Q per CTA, 256-key tiles (M128 x N256 MMAs),
+// three stages so that each tile's copy has two tile periods to land; the
+// final (max, sum) merge reuses the Q region once every MMA has completed
+using Pass1 = Cfg<128, 256, CERTKV_TC_STAGES1, 512>;
+// pass 2: all (<= 256) rows of Q, 128-key tiles (M128 x N<=256 MMAs); the
+// rows' log-sum-exp values (1 KB) after the barriers
+using Pass2 = Cfg<256, 128, CERTKV_TC_STAGES, 512 + 1024>;
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
 // 128 B, groups of 8 rows 1024 B apart.
@@ -73,13 +82,6 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
          ((uint32_t)(M >> 4) << 24);
 }
 
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
-                                          uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
-}
 __device__ __forceinline__ void umma_commit(uint32_t mbar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                    mbar)
@@ -160,10 +162,11 @@ struct Shared {
   __device__ volatile int* abort_flag() const {
     return reinterpret_cast<volatile int*>(base + C::kBarOff + 260);
   }
-  // misc region: lse[256] (pass 2) or the partial (max, sum) of 4 x 128 rows (pass 1)
+  // lse[256] of pass 2 after the barriers; the partial (max, sum) of 4 x 128
+  // rows of pass 1 in the Q region (written only after the last MMA)
   __device__ float* lse() const { return reinterpret_cast<float*>(base + C::kBarOff + 512); }
-  __device__ float* pm() const { return reinterpret_cast<float*>(base + C::kBarOff + 512); }
-  __device__ float* pl() const { return reinterpret_cast<float*>(base + C::kBarOff + 2560); }
+  __device__ float* pm() const { return reinterpret_cast<float*>(base); }
+  __device__ float* pl() const { return reinterpret_cast<float*>(base + 2048); }
 };
 
 template <class C>
@@ -246,25 +249,59 @@ __device__ __forceinline__ void produce(const Shared<C>& sh, const CUtensorMap* 
   mbar_wait(sh.qfull(), 0, &dummy);
 }
 
+// The 8 k-steps of one tile as back-to-back MMAs into d: a and b are the
+// descriptors of the operands' first k-step; k-step ks starts (ks & 3) * 32
+// bytes into the 128-byte swizzled rows of half ks >> 2, which lies ha (hb)
+// descriptor units after the first half.  A descriptor's address field is
+// the byte address / 16 in its low 14 bits, and no operand reaches 256 KB,
+// so the offsets are plain additions.
+template <uint32_t ha, uint32_t hb>
+__device__ __forceinline__ void umma_tile(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc) {
+#define CERTKV_A(ks) (a + (uint64_t)(((ks) >> 2) * ha + ((ks) & 3) * 2))
+#define CERTKV_B(ks) (b + (uint64_t)(((ks) >> 2) * hb + ((ks) & 3) * 2))
+  asm volatile(
+      "{\n .reg .pred p0, p1;\n setp.ne.b32 p0, %17, %17;\n setp.eq.b32 p1, %17, %17;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %18, p0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %3, %4, %18, p1;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %5, %6, %18, p1;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %7, %8, %18, p1;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %9, %10, %18, p1;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %11, %12, %18, p1;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %13, %14, %18, p1;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %15, %16, %18, p1;\n}\n" ::"r"(d),
+      "l"(CERTKV_A(0)), "l"(CERTKV_B(0)), "l"(CERTKV_A(1)), "l"(CERTKV_B(1)), "l"(CERTKV_A(2)),
+      "l"(CERTKV_B(2)), "l"(CERTKV_A(3)), "l"(CERTKV_B(3)), "l"(CERTKV_A(4)), "l"(CERTKV_B(4)),
+      "l"(CERTKV_A(5)), "l"(CERTKV_B(5)), "l"(CERTKV_A(6)), "l"(CERTKV_B(6)), "l"(CERTKV_A(7)),
+      "l"(CERTKV_B(7)), "r"(0u), "r"(idesc));
+#undef CERTKV_A
+#undef CERTKV_B
+}
+
 // MMA issuer: for each tile, 8 k-steps of one M128 x N MMA into buffer t & 1.
-// `a_of(kh, koff)` / `b_of(stage, kh, koff)` give the operand smem addresses.
-template <class C, class AOf, class BOf>
+// kKeysA: the K tile is the A operand (pass 2), else Q is (pass 1).  The
+// descriptors are formed once; each tile only adds its stage's offset, so
+// the issuing thread (which shares its SM sub-partition with four epilogue
+// warps) spends few instructions per tile.
+template <class C, bool kKeysA>
 __device__ __forceinline__ void issue_mmas(const Shared<C>& sh, uint32_t tmem, uint32_t idesc,
-                                           int ntiles, AOf a_of, BOf b_of) {
+                                           int ntiles) {
   volatile int* ab = sh.abort_flag();
   bool ok = mbar_wait(sh.qfull(), 0, ab);
   tc_fence_after();
+  const uint64_t dq = sw128_desc(sh.q());
+  const uint64_t dk0 = sw128_desc(sh.kst(0));
+  constexpr uint32_t kHalfQ = (uint32_t)(C::kQBytes / 2) >> 4;
+  constexpr uint32_t kHalfK = (uint32_t)(C::kStageBytes / 2) >> 4;
+  constexpr uint32_t kStep = (uint32_t)C::kStageBytes >> 4;
   for (int t = 0; ok && t < ntiles; ++t) {
     const int s = t % C::kStages, b = t & 1;
     if (!mbar_wait(sh.full(s), (t / C::kStages) & 1, ab)) break;
     if (t >= 2 && !mbar_wait(sh.acce(b), ((t >> 1) - 1) & 1, ab)) break;
     tc_fence_after();
     const uint32_t d = tmem + (uint32_t)(b * 256);
-#pragma unroll
-    for (int ks = 0; ks < 8; ++ks) {
-      const uint32_t kh = ks >> 2, koff = (ks & 3) * 32;
-      umma_bf16(d, sw128_desc(a_of(s, kh, koff)), sw128_desc(b_of(s, kh, koff)), idesc, ks > 0);
-    }
+    const uint64_t dk = dk0 + (uint64_t)((uint32_t)s * kStep);
+    if (kKeysA) umma_tile<kHalfK, kHalfQ>(d, dk, dq, idesc);
+    else umma_tile<kHalfQ, kHalfK>(d, dq, dk, idesc);
     umma_commit(sh.empty(s));
     umma_commit(sh.accf(b));
   }
@@ -300,12 +337,7 @@ __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_consta
     if (lane == 0) produce<C>(sh, &tmK, &tmQ, u * R + half * 128, 128, (long)u * n + j_begin, ntiles);
   } else if (warp == 1) {
     if (lane == 0)
-      issue_mmas<C>(
-          sh, tmem, idesc_bf16(128, C::kTileKeys), ntiles,
-          [&](int, uint32_t kh, uint32_t koff) { return sh.q() + kh * (C::kQBytes / 2) + koff; },
-          [&](int s, uint32_t kh, uint32_t koff) {
-            return sh.kst(s) + kh * (C::kStageBytes / 2) + koff;
-          });
+      issue_mmas<C, false>(sh, tmem, idesc_bf16(128, C::kTileKeys), ntiles);
   } else {
     // every warp takes every tile: warp (q, cq) owns rows q*32.. of the half
     // (its TMEM lane quadrant) and keys cq*64 .. cq*64+63 of each 256-key tile.
@@ -410,12 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1) colsum_tc_kernel(const __grid_con
     if (lane == 0) produce<C>(sh, &tmK, &tmQ, u * R + rg0, RG, (long)u * n + j_begin, ntiles);
   } else if (warp == 1) {
     if (lane == 0)
-      issue_mmas<C>(
-          sh, tmem, idesc_bf16(C::kTileKeys, RG), ntiles,
-          [&](int s, uint32_t kh, uint32_t koff) {
-            return sh.kst(s) + kh * (C::kStageBytes / 2) + koff;
-          },
-          [&](int, uint32_t kh, uint32_t koff) { return sh.q() + kh * (C::kQBytes / 2) + koff; });
+      issue_mmas<C, true>(sh, tmem, idesc_bf16(C::kTileKeys, RG), ntiles);
   } else {
     // every warp takes every tile: warp (q, cq) owns keys q*32.. of the tile
     // (its TMEM lane quadrant) and rows rg0 + cq*64 .. +63, summed into row
