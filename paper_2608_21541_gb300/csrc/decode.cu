@@ -362,11 +362,12 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_kernel(
 }
 
 // ---------------------------------------------------------------------------
-// Tensor-core split kernel for G = 8 and 16 query heads per KV head.  At these
-// group sizes the CUDA-core consumer needs ~4 fp32 FMAs per byte of cache;
-// here both products run as mma.sync m16n8k16 (bf16 in, fp32 accumulate)
-// with the G query heads as the M rows (padded to 16 with zero rows for
-// G = 8): S = Q K^T over 32 slots (4 n-blocks x 8 k-steps), online softmax per
+// Tensor-core split kernel for G = 4, 8 and 16 query heads per KV head.  At
+// G = 8 the CUDA-core consumer needs ~4 fp32 FMAs per byte of cache; here both
+// products run as mma.sync m16n8k16 (bf16 in, fp32 accumulate) with the G
+// query heads as the M rows (padded to 16 with zero rows for G = 4 and 8;
+// the padded rows' results are dropped): S = Q K^T over 32 slots (4 n-blocks
+// x 8 k-steps), online softmax per
 // row in the log2 domain, then O += P V (2 k-blocks x 16 n-blocks) with P as a
 // bf16 part plus the bf16 rounding of its remainder (fp32-level weights).  The tiles arrive by TMA with 128-byte swizzle (two boxes of
 // 64 dimensions x 32 slots for K and for V), so the ldmatrix reads are free of
@@ -416,7 +417,9 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_tc_kernel(
     const __nv_bfloat16* __restrict__ q, const int64_t* __restrict__ offsets,
     const int32_t* __restrict__ counts, const int32_t* __restrict__ T, int tail_slot,
     float scale_log2, float2* __restrict__ rec_ml, float* __restrict__ rec_acc) {
-  static_assert(G == 8 || G == 16, "the tensor-core decode takes 8 or 16 query heads per KV head");
+  static_assert(G == 4 || G == 8 || G == 16,
+                "the tensor-core decode takes 4, 8 or 16 query heads per KV head");
+  constexpr bool kPadded = G < 8;  // rows G..7 of the first fragment row block are zero
   extern __shared__ uint8_t dsm_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)dsm_raw + 1023) & ~(uintptr_t)1023);
   // stage s: K halves at + 0 / 4096, V halves at + 8192 / 12288
@@ -500,8 +503,9 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_tc_kernel(
 #pragma unroll
       for (int ks = 0; ks < 8; ++ks) {
         const int c0 = (16 * ks + 2 * qc) / 2;  // 32-bit word of dims 16 ks + 2 qc, +1
-        qa[ks][0] = __ldg(qg + qr * (kD / 2) + c0);
-        qa[ks][2] = __ldg(qg + qr * (kD / 2) + c0 + 4);
+        const bool row = !kPadded || qr < G;
+        qa[ks][0] = row ? __ldg(qg + qr * (kD / 2) + c0) : 0u;
+        qa[ks][2] = row ? __ldg(qg + qr * (kD / 2) + c0 + 4) : 0u;
         if (G == 16) {
           qa[ks][1] = __ldg(qg + (qr + 8) * (kD / 2) + c0);
           qa[ks][3] = __ldg(qg + (qr + 8) * (kD / 2) + c0 + 4);
@@ -614,7 +618,8 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_tc_kernel(
       l0 += __shfl_xor_sync(kFull, l0, 2);
       l1 += __shfl_xor_sync(kFull, l1, 1);
       l1 += __shfl_xor_sync(kFull, l1, 2);
-      if (qc == 0) {
+      const bool own_row = !kPadded || qr < G;  // padded rows are not the group's heads
+      if (qc == 0 && own_row) {
         wm[cw * G + qr] = m0;
         wl[cw * G + qr] = l0;
         if (G == 16) {
@@ -625,7 +630,8 @@ __global__ void __launch_bounds__(kDecThreads) decode_split_tc_kernel(
 #pragma unroll
       for (int nd = 0; nd < 16; ++nd) {
         const int d = 8 * nd + 2 * qc;
-        *reinterpret_cast<float2*>(&wacc[(cw * G + qr) * kD + d]) = make_float2(o[nd][0], o[nd][1]);
+        if (own_row)
+          *reinterpret_cast<float2*>(&wacc[(cw * G + qr) * kD + d]) = make_float2(o[nd][0], o[nd][1]);
         if (G == 16)
           *reinterpret_cast<float2*>(&wacc[(cw * G + qr + 8) * kD + d]) =
               make_float2(o[nd][2], o[nd][3]);
@@ -892,7 +898,10 @@ int run_splits(const Prob& p, const void* q, const void* pk, const void* pv,
   switch (p.G) {
     case 1: return launch_split<1>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
     case 2: return launch_split<2>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
-    case 4: return launch_split<4>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    case 4: {
+      const int nb = launch_split_tc<4>(p, qb, pk, pv, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+      return nb > 0 ? nb : launch_split<4>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
+    }
     case 8: {
       const int nb = launch_split_tc<8>(p, qb, pk, pv, offsets, counts, T, tail_slot, sl2, ml, acc, st);
       return nb > 0 ? nb : launch_split<8>(p, qb, kb, vb, offsets, counts, T, tail_slot, sl2, ml, acc, st);
