@@ -7,8 +7,13 @@ Tolerances (stated once, used by every parity test):
     when the oracle starts from the GPU's own fp32 scores (conditioned mode);
   * from raw inputs (end-to-end mode) a budget may differ only as a certified
     near-tie of the allocation objective (relative gap <= 1e-6 under the
-    oracle's curves), and a kept set may differ only by tokens whose score
-    lies within 1e-6 relative of the cut;
+    oracle's curves), or where the order itself has a near-tie: scores that
+    differ by less than 1e-6 relative in float64 can be equal in fp32, whose
+    order (ties to the lower index) is then an equally valid order of the
+    float64 scores; there the GPU's order must be a descending order of the
+    float64 scores up to such near-ties, and the conditioned check certifies
+    its budgets on that order.  A kept set may differ only by tokens whose
+    score lies within 1e-6 relative of the cut;
   * decode outputs (bf16): 2e-2 maximum absolute error plus half a bf16 ulp
     of the reference value (the output is a bf16 number: rounding the exact
     result to bf16 alone moves it by up to half an ulp, 2^-5 at |o| = 8).
@@ -22,6 +27,7 @@ import oracle
 RTOL_MASS = 1e-4
 CUT_RTOL = 1e-6
 OBJ_RTOL = 1e-6
+ORDER_RTOL = 1e-6
 DECODE_ATOL = 2e-2
 
 
@@ -97,10 +103,29 @@ def check_conditioned(got: dict, ref: dict, units: int, tail_slot: int = 1):
     return worst
 
 
+def gpu_order(a_gpu_u: np.ndarray) -> np.ndarray:
+    """The order the CUDA path sorts into: its fp32 scores descending, equal
+    values by lower index."""
+    idx = np.arange(a_gpu_u.shape[0])
+    return np.lexsort((idx, -np.asarray(a_gpu_u, np.float64)))
+
+
+def order_near_tie(perm_gpu: np.ndarray, perm_ref: np.ndarray, a_ref_u: np.ndarray) -> bool:
+    """True when the two orders differ and the first is nevertheless a
+    descending order of the float64 scores up to near-ties (each adjacent pair
+    out of float64 order within ORDER_RTOL relative)."""
+    if np.array_equal(perm_gpu, perm_ref):
+        return False
+    s = a_ref_u[perm_gpu]
+    drop = s[1:] - s[:-1]  # > 0 where the GPU order rises in float64
+    return bool((drop <= ORDER_RTOL * np.maximum(np.abs(s[1:]), 1e-300)).all())
+
+
 def check_end_to_end(got: dict, ref: dict, a_gpu: np.ndarray, H: int):
     """Budgets equal or certified near-ties; kept sets equal up to near-cut swaps.
 
-    Returns the number of certified near-tie budget differences."""
+    Returns the number of certified near-tie budget differences (of the
+    objective or of the order)."""
     counts, offsets, pos = got["counts"], got["offsets"], got["positions"]
     units = counts.shape[0]
     near_ties = 0
@@ -112,7 +137,14 @@ def check_end_to_end(got: dict, ref: dict, a_gpu: np.ndarray, H: int):
             obj_ref = sum(cur[h, ref["counts"][bl * H + h]] for h in range(H))
             gap = abs(obj_gpu - obj_ref) / max(abs(obj_ref), 1e-300)
             assert counts[sl].sum() == ref["counts"][sl].sum()
-            assert gap <= OBJ_RTOL, f"budget mismatch in (seq,layer) {bl}: gap {gap:.3e}"
+            if gap > OBJ_RTOL:
+                heads = range(bl * H, (bl + 1) * H)
+                ties = [order_near_tie(gpu_order(a_gpu[u]), ref["perm"][u], ref["a"][u])
+                        for u in heads]
+                valid = all(np.array_equal(gpu_order(a_gpu[u]), ref["perm"][u]) or t
+                            for u, t in zip(heads, ties))
+                assert any(ties) and valid, \
+                    f"budget mismatch in (seq,layer) {bl}: gap {gap:.3e} with no order near-tie"
             near_ties += 1
     for u in range(units):
         o, c = int(offsets[u]), int(counts[u])

@@ -1,0 +1,81 @@
+"""Tiny shapes against the float64 oracle, through the C ABI: contexts of 2 to
+64 tokens with 1 to 4 KV heads and every group size, so that every sort tile,
+dispersion chunk, hull segment and decode tile is ragged or nearly empty and
+the allocator's bracket is a handful of tokens.  Conditioned mode bit-exact,
+end to end up to certified near-ties, decode within its tolerance; and the
+whole pass bit-identical over ten repeats on a case with several tiles."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import parity
+from paper_2608_21541_gb300 import certkv as ck
+from paper_2608_21541_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+# (n, KV heads H, group size G): contexts from the smallest the method admits
+# (n = 2, window 1) up to a half-filled dispersion chunk
+SHAPES = [(2, 1, 1), (2, 4, 2), (3, 2, 4), (4, 1, 8), (5, 2, 2), (7, 3, 2), (9, 1, 16),
+          (16, 2, 1), (16, 4, 4), (33, 1, 2), (33, 2, 8), (64, 3, 4), (64, 4, 1)]
+
+
+def _case(n, H, G, kind="zipf"):
+    w = min(n - 1, 1 + n % 5)
+    # planted keys of distinct strengths (the Zipf recipe): identical planted
+    # rows side by side, as a 64-token context of the plain recipe has, give
+    # exactly equal scores whose order the float64 oracle breaks by index and
+    # the fp32 path by rounding, and both orders are correct
+    wl = W.Workload(f"tiny{n}_{H}_{G}", B=1, L=2, Hq=H * G, H=H, n=n, d=128, w=w,
+                    keep=(1, 3), kind=kind, description="tiny shape")
+    B_live = H * min(n, max(2, n // 3))
+    return wl, B_live
+
+
+@pytest.mark.parametrize("n,H,G,kind", [s + ("zipf",) for s in SHAPES] + [(64, 4, 1, "planted")])
+def test_tiny_shapes_match_oracle(n, H, G, kind):
+    """The last case has identical planted keys side by side, so some scores
+    tie exactly in float64: it exercises the order near-tie rule."""
+    wl, B_live = _case(n, H, G, kind)
+    params = ck.certkv_default_params()
+    K, V, Q = W.draw(wl, device=DEV)
+    a = ck.certkv_score(K, Q, params)
+    packed = ck.certkv_compress(K, V, Q, B_live, params, with_tail=True)
+    scored = ck.certkv_compress_scored(K, V, a, B_live, params, hq=wl.Hq, w=wl.w, with_tail=True)
+    host = dict(K=parity.bits(K), V=parity.bits(V), Q=parity.bits(Q), a=a.cpu().numpy())
+    kw = dict(B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, n=n, d=wl.d, w=wl.w, B_live=B_live)
+    ref_e2e = oracle.compress(host["K"], host["V"], host["Q"], **kw)
+    ref_cond = oracle.compress(host["K"], host["V"], None, a_in=host["a"], **kw)
+    parity.check_scores(host["a"], ref_e2e["a"])
+    parity.check_conditioned(parity.packed_np(scored), ref_cond, wl.units)
+    got = parity.packed_np(packed)
+    parity.check_end_to_end(got, ref_e2e, host["a"], H)
+    assert got["counts"].reshape(-1, H).sum(1).tolist() == [B_live - H] * (wl.B * wl.L)
+    q = W.draw_decode_queries(wl, 0, device=DEV)
+    out = ck.certkv_decode_attn(q, packed, hkv=H)
+    ref = oracle.decode(parity.bits(q), got["pk"], got["pv"], got["offsets"], got["counts"],
+                        B=wl.B, L=wl.L, Hq=wl.Hq, H=H, d=wl.d)
+    parity.check_decode(out, ref)
+
+
+def test_ten_repeats_bit_identical():
+    """Every output of the compression and of a decode step is bit-identical
+    over ten calls (no atomics decide an order or a sum)."""
+    wl = W.Workload("R", B=1, L=2, Hq=8, H=2, n=9000, d=128, w=64, keep=(1, 10),
+                    kind="zipf", description="repeat case")
+    K, V, Q = W.draw(wl, device=DEV)
+    q = W.draw_decode_queries(wl, 0, device=DEV)
+    first = None
+    for _ in range(10):
+        packed = ck.certkv_compress(K, V, Q, wl.B_live, with_tail=True)
+        got = parity.packed_np(packed)
+        out = ck.certkv_decode_attn(q, packed, hkv=wl.H)
+        got["out"] = out.view(-1).view(torch.int16).cpu().numpy()
+        if first is None:
+            first = got
+            continue
+        for k in first:
+            np.testing.assert_array_equal(first[k], got[k], err_msg=k)
