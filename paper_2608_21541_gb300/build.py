@@ -8,6 +8,7 @@ from __future__ import annotations
 
 import glob
 import os
+import shutil
 import subprocess
 from concurrent.futures import ThreadPoolExecutor
 
@@ -52,11 +53,15 @@ def build(force: bool = False, verbose: bool = False, extra_flags=(), debug: boo
         extra_flags = (*extra_flags, "-DCERTKV_DEBUG")
     if not force and not _stale(lib):
         return lib
-    os.makedirs(out_dir, exist_ok=True)
+    # objects go to a directory of this process, so that processes that build
+    # at the same time (the ranks of a multi-GPU run) never link each other's
+    # half-written objects; the library itself is replaced atomically
+    obj_dir = os.path.join(out_dir, f"obj{os.getpid()}")
+    os.makedirs(obj_dir, exist_ok=True)
     srcs = _sources()
 
     def compile_one(src):
-        obj = os.path.join(out_dir, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(obj_dir, os.path.basename(src)[:-3] + ".o")
         cmd = [NVCC, *FLAGS, *extra_flags, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -72,6 +77,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=(), debug: boo
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")
     os.replace(tmp, lib)
+    shutil.rmtree(obj_dir, ignore_errors=True)
     return lib
 
 
