@@ -122,7 +122,8 @@ class ClockSampler:
 
 # -------------------------------------------------------------- roofline ----
 def kernel_work(wl, B_live, name):
-    """Algorithmic bytes and flops per launch of a kernel."""
+    """Algorithmic bytes and flops per launch of a kernel: the bytes each must
+    read and write once, or the tensor flops of a score pass."""
     U = wl.units
     n, d, R = wl.n, wl.d, wl.G * wl.w
     kbytes = U * n * d * 2
