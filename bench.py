@@ -40,6 +40,9 @@ def parse():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="time direct library calls instead of the replay of one CUDA graph "
+                         "that captured them")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: compress this many layers instead of the workload's")
     ap.add_argument("--rows", action="store_true",
@@ -480,15 +483,34 @@ def run_ours(args, wl, rank, world):
     clocks.start()
     time.sleep(0.3)
     # the timed region: no per-launch tracing; one pair of events per step
-    # separates the compression from the decode steps
+    # separates the compression from the decode steps.  By default the step's
+    # library calls (the same launches with the same arguments) were captured
+    # once into two CUDA graphs, which each step replays.
+    def compress_call(st):
+        ck.certkv_compress(K, V, Q, B_live, params, out=packed, ws=ws, stream=st)
+
+    def decode_calls(st):
+        for qi in qs:
+            ck.certkv_decode_attn(qi, packed, hkv=wl.H, out=out, ws=dws, stream=st)
+
+    if args.no_graph:
+        run_compress = lambda: compress_call(stream)
+        run_decode = lambda: decode_calls(stream)
+    else:
+        g_compress, g_decode = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_compress):
+            compress_call(torch.cuda.current_stream())
+        with torch.cuda.graph(g_decode):
+            decode_calls(torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        run_compress, run_decode = g_compress.replay, g_decode.replay
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     for e_start, e_mid, e_end in ev:
         e_start.record(stream)
-        ck.certkv_compress(K, V, Q, B_live, params, out=packed, ws=ws, stream=stream)
+        run_compress()
         e_mid.record(stream)
-        for qi in qs:
-            ck.certkv_decode_attn(qi, packed, hkv=wl.H, out=out, ws=dws, stream=stream)
+        run_decode()
         e_end.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -543,6 +565,9 @@ def run_ours(args, wl, rank, world):
         "scaling": "strong" if sharded else "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": dict(config_dict(job, B_live), decode_steps=nd,
+                       launch=("direct library calls" if args.no_graph else
+                               "one step's library calls captured once as CUDA graphs "
+                               "(compression, decode), replayed each step"),
                        **({"shard": f"{len(pairs)} of {job.B * job.L} (sequence, layer) pairs "
                                      f"per rank"} if sharded else {})),
         "compress_ms": compress_ms,
