@@ -396,18 +396,22 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
     }
     const DF Mt = df_add_same_sign(base_m, sm);
     const DF Qt = df_add_same_sign(base_q, sq);
-    DF c;
+    DF c, arg = df_make(0.f);
     if (p.statistic == 2) {
       c = Mt;
     } else if (p.statistic == 1) {
-      c = df_sqrt_newton(df_mul(Mt, Qt));
+      arg = df_mul(Mt, Qt);
+      c = df_sqrt_newton(arg);
     } else {
       const DF W2 = df_add(wb2, xt);
-      c = df_sqrt_newton(df_add(df_mul(Mt, Qt), df_neg(W2)));
+      arg = df_add(df_mul(Mt, Qt), df_neg(W2));
+      c = df_sqrt_newton(arg);
     }
     if (ok) {
       curve[(size_t)u * n + r] = make_float2(c.hi, c.lo);
-      if (!(c.hi <= 3.0e38f)) bad = true;
+      // a non-finite value (the square root maps a NaN argument, such as
+      // inf - inf from an infinite value row, to 0, so test the argument too)
+      if (!(c.hi <= 3.0e38f) || arg.hi != arg.hi) bad = true;
       unsigned long long k = df_order_key(c);
       best = k > best ? k : best;
     }

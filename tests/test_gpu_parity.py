@@ -219,6 +219,24 @@ def test_deterministic():
         np.testing.assert_array_equal(p1[k], p2[k], err_msg=k)
 
 
+@pytest.mark.parametrize("where", ["K_nan", "V_nan", "V_inf", "Q_inf"])
+def test_status_word_nonfinite_inputs(where):
+    """A NaN or an infinity in K, V or the observation queries raises
+    CERTKV_STATUS_NONFINITE (the call returns normally), and the next call
+    with finite inputs on the same workspace reports a clean status again."""
+    wl = CASES["small_ragged"]
+    K, V, Q = W.draw(wl, device=DEV)
+    shape = ck.shape_of(K, Q)
+    ws = ck.workspace(ck.certkv_workspace_bytes(shape), K.device)
+    bad = {"K": K.clone(), "V": V.clone(), "Q": Q.clone()}
+    name, kind = where.split("_")
+    bad[name].view(-1)[1234] = float("nan") if kind == "nan" else float("inf")
+    ck.certkv_compress(bad["K"], bad["V"], bad["Q"], wl.B_live, ws=ws)
+    assert ck.certkv_read_status(ws) & ck.STATUS_NONFINITE
+    ck.certkv_compress(K, V, Q, wl.B_live, ws=ws)
+    assert ck.certkv_read_status(ws) == 0
+
+
 def test_status_word():
     wl = CASES["small_ragged"]
     K, V, Q = W.draw(wl, device=DEV)
