@@ -79,3 +79,63 @@ def test_ten_repeats_bit_identical():
             continue
         for k in first:
             np.testing.assert_array_equal(first[k], got[k], err_msg=k)
+
+
+@pytest.mark.parametrize("case", ["K_zero", "V_zero", "KV_zero", "V_rows_equal"])
+def test_degenerate_inputs(case):
+    """The method's degenerate inputs, against the oracle: all keys zero (every
+    logit 0, so the scores tie except for the pooling edges and the protected
+    window), all values zero (every curve c(b) = 0, so the allocator's ties
+    decide every budget: smallest b, then the lowest head in the repair), both,
+    and identical value rows (the centred dispersion is exactly 0)."""
+    wl = W.Workload("D", B=1, L=2, Hq=8, H=2, n=3000, d=128, w=20, keep=(1, 10),
+                    kind="planted", description="degenerate inputs")
+    K, V, Q = W.draw(wl, device=DEV)
+    if "K" in case:
+        K.zero_()
+    if case in ("V_zero", "KV_zero"):
+        V.zero_()
+    if case == "V_rows_equal":
+        V.copy_(V[:, :, :, :1, :].expand_as(V))
+    params = ck.certkv_default_params()
+    a = ck.certkv_score(K, Q, params)
+    packed = ck.certkv_compress(K, V, Q, wl.B_live, params, with_tail=True)
+    scored = ck.certkv_compress_scored(K, V, a, wl.B_live, params, hq=wl.Hq, w=wl.w, with_tail=True)
+    host = dict(K=parity.bits(K), V=parity.bits(V), Q=parity.bits(Q), a=a.cpu().numpy())
+    kw = dict(B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, n=wl.n, d=wl.d, w=wl.w, B_live=wl.B_live)
+    ref_e2e = oracle.compress(host["K"], host["V"], host["Q"], **kw)
+    ref_cond = oracle.compress(host["K"], host["V"], None, a_in=host["a"], **kw)
+    parity.check_scores(host["a"], ref_e2e["a"])
+    got = parity.packed_np(packed)
+    if case != "V_rows_equal":
+        parity.check_conditioned(parity.packed_np(scored), ref_cond, wl.units)
+        parity.check_end_to_end(got, ref_e2e, host["a"], wl.H)
+    else:
+        # m Q - ||W||^2 is zero in exact arithmetic for every b: each side's
+        # curve is its own rounding of 0, and the budgets follow that
+        # rounding.  The path's c^2 carries the fp32 rounding of its in-chunk
+        # terms 2<W_base, P> + ||P||^2 (at most m^2 ||v||^2 = m Q here, a few
+        # units of 2^-24 relative over a 128-rank chunk): within 16 2^-24 m Q,
+        # so c within sqrt(2^-20 m Q) absolutely.  What is unique is checked:
+        # the curve within that bound, the budget sums, the kept tokens as the
+        # top of the path's own order for its own budgets, and the packed rows.
+        perm, c = ck.certkv_curves(V, a, params, hq=wl.Hq, w=wl.w)
+        perm, c = perm.cpu().numpy(), c.cpu().numpy()
+        v = oracle.bf16_bits_to_f64(host["V"].reshape(wl.units, wl.n, wl.d)[:, 0])
+        for u in range(wl.units):
+            m = np.cumsum(ref_cond["a"][u][ref_cond["perm"][u]][::-1])[::-1]
+            bound = np.sqrt(2.0 ** -20) * m * np.linalg.norm(v[u]) + 1e-30
+            ratio = float((np.abs(c[u] - ref_cond["c"][u]) / bound).max())
+            assert ratio <= 1.0, f"curve beyond its bound (unit {u}): {ratio:.3f} of it"
+            o, b = int(got["offsets"][u]), int(got["counts"][u])
+            want = np.sort(perm[u][:b])
+            np.testing.assert_array_equal(got["positions"][o:o + b], want)
+            rows = host["V"].reshape(wl.units, wl.n, wl.d)[u][want]
+            assert (got["pv"][o:o + b] == rows).all()
+        B_real = wl.B_live - wl.H
+        assert (got["counts"].reshape(-1, wl.H).sum(1) == B_real).all()
+    q = W.draw_decode_queries(wl, 0, device=DEV)
+    out = ck.certkv_decode_attn(q, packed, hkv=wl.H)
+    ref = oracle.decode(parity.bits(q), got["pk"], got["pv"], got["offsets"], got["counts"],
+                        B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, d=wl.d)
+    parity.check_decode(out, ref)
