@@ -94,3 +94,16 @@ def test_c5_full_budget_sweep():
         wl = base.with_(keep=keep)
         _run(wl, wl.B_live, samples=[(0, 0), (0, 79)], e2e_scores=[(0, 79)], decode_steps=1,
              inputs=inputs)
+
+
+def test_context_of_2_20_tokens():
+    """A 1048576-token context (one layer, 8 KV heads, 32 query heads, budget
+    1/10), beyond the benchmark configurations: 512 sort tiles, 8192
+    dispersion chunks and 4096 hull segments per head; at about ten hull
+    candidates per group of eight segments (as at 131072 tokens) a layer has
+    some 40 k candidates, more than the 12288 the allocator stages in shared
+    memory, so its global-memory path runs.  Conditioned mode bit-exact on the
+    layer, decode within its tolerance."""
+    wl = W.Workload("L20", B=1, L=1, Hq=32, H=8, n=1 << 20, d=128, w=64, keep=(1, 10),
+                    kind="zipf", description="2^20-token context")
+    _run(wl, wl.B_live, samples=[(0, 0)], decode_steps=1)
