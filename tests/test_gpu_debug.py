@@ -25,6 +25,9 @@ CASES = [
     ("heads32", (1, 1, 32, 32, 700, 4, (1, 5), "student_t"), {}),
     ("clusters", (1, 2, 8, 2, 2300, 16, (1, 8), "planted"), {"tail_clusters": 3}),
     ("no_tail_slot", (1, 1, 8, 2, 1800, 16, (1, 8), "zipf"), {"tail_slot": 0}),
+    ("n2", (1, 2, 8, 4, 2, 1, (1, 1), "zipf"), {}),       # the smallest context
+    ("n3_g16", (1, 1, 16, 1, 3, 2, (2, 3), "zipf"), {}),
+    ("n64_h3", (2, 1, 12, 3, 64, 4, (1, 3), "planted"), {}),
 ]
 
 
