@@ -284,8 +284,10 @@ __global__ void __launch_bounds__(128) fixed_row_merge_kernel(
   const int bl = u / p.H, h = u - bl * p.H;
   const size_t qi = (size_t)bl * p.Hq + (size_t)h * G + g;
   const float oh = __bfloat162float(ohat[qi * kD + i]);
-  const float vbt = pS < 1.f ? uu / (1.f - pS) : 0.f;
-  const float f = os + (1.f - pS) * (vbt - os) - o;
+  // the tail mass is pT (computed from the tail's own sum), not 1 - pS, which
+  // loses it to cancellation when the kept tokens hold almost all the mass
+  const float vbt = pT > 0.f ? uu / pT : 0.f;
+  const float f = os + pT * (vbt - os) - o;
   const float nO = block_sum_128(o * o, red);
   const float eS = block_sum_128((os - o) * (os - o), red);
   const float nu = block_sum_128(uu * uu, red);
@@ -331,8 +333,9 @@ __global__ void __launch_bounds__(128) fixed_row_merge_kernel(
       a2 += fabsf(e * invLA - qstar * r);  // |A_j - q r_j|
     }
     d1 = block_sum_128(a1, red);
-    // on S the lifted row is Ahat = A * Z / Zhat, so sum_S |A - Ahat| = |p_S - (1 - q)|
-    d2 = fabsf(pS - (1.f - qstar)) + block_sum_128(a2, red);
+    // on S the lifted row is Ahat = A * Z / Zhat, so sum_S |A - Ahat| =
+    // |p_S - (1 - q)| = |q - p_T|
+    d2 = fabsf(qstar - pT) + block_sum_128(a2, red);
   }
   if (i == 0) {
     float* st = stats + qi * CERTKV_FIXED_ROW_STATS;
@@ -340,7 +343,7 @@ __global__ void __launch_bounds__(128) fixed_row_merge_kernel(
     st[1] = sqrtf(nO);
     st[2] = sqrtf(eS);
     st[3] = sqrtf(nu);
-    st[4] = 2.f * vm * (1.f - pS);
+    st[4] = 2.f * vm * pT;
     st[5] = sqrtf(eh);
     st[6] = vm;
     st[7] = sqrtf(res);
@@ -539,7 +542,9 @@ __global__ void __launch_bounds__(kSampThreads) sampled_kernel(
     }
     for (int s2 = 0; s2 < kDiagSplits; ++s2) sq += part_tm[((size_t)u * kDiagSplits + s2) * kSvStride + kD];
     const double s2v = N > 0 ? (sq - sv2 / N) / ((double)kD * N) : 0.0;
-    const double pSd = (double)sc.y / (double)LA, omp2 = (1.0 - pSd) * (1.0 - pSd);
+    // 1 - p_S as the tail's own mass (no cancellation when p_S is near 1)
+    const double pSd = (double)sc.y / (double)LA, pTd = (double)sc.z / (double)LA;
+    const double omp2 = pTd * pTd;
     const double QT = wq[0] / ((double)LA * (double)LA);
     const double imb = omp2 > 0.0 ? QT / omp2 : 0.0;
     const double mse_w = kD * s2v * omp2 / m * (1.0 - imb);

@@ -21,6 +21,11 @@ CASES = {
                              kind="planted"),
     "zipf_g8": W.Workload("Z", B=1, L=1, Hq=16, H=2, n=5000, d=128, w=32, keep=(1, 5),
                           kind="zipf"),
+    # tiny contexts: every tile of the instrument ragged; tails of 20 tokens or more
+    "tiny33_g16": W.Workload("T33", B=1, L=2, Hq=16, H=1, n=33, d=128, w=3, keep=(1, 3),
+                             kind="zipf"),
+    "tiny64_h3": W.Workload("T64", B=1, L=1, Hq=12, H=3, n=64, d=128, w=4, keep=(1, 4),
+                            kind="zipf"),
 }
 NF = len(ck.FIXED_ROW_FIELDS)
 
