@@ -776,17 +776,20 @@ __global__ void __launch_bounds__(128) decode_certified_merge_kernel(
   }
   out[qi * kD + i] = __float2bfloat16_rn(num / Z);
   if (i == 0) {
-    float DZ = 0.f, DN = 0.f, vmax = kept_vmax[u];
+    // a few scalars per query head, in float64: e^r (e^r - 1) overflows fp32
+    // from r = 44 on, which a strong key in a cluster reaches with a unit
+    // query; the bound is stored as fp32 (+inf when it exceeds its range)
+    double DZ = 0.0, DN = 0.0, vmax = kept_vmax[u];
     for (int c = 0; c < m; ++c) {
       if (!(s_lam[c] > -INFINITY)) continue;
-      const float zg = exp2f(s_lam[c] - M);
-      const float er = expf(s_r[c]);
-      DZ += (er - 1.f) * er * zg;
-      DN += er * zg * ((er - 1.f) * s_vn[c] + s_rho[c]);
-      vmax = fmaxf(vmax, s_vn[c] + s_rho[c]);
+      const double zg = exp2((double)(s_lam[c] - M));
+      const double er = exp((double)s_r[c]);
+      DZ += (er - 1.0) * er * zg;
+      DN += er * zg * ((er - 1.0) * s_vn[c] + s_rho[c]);
+      vmax = fmax(vmax, (double)(s_vn[c] + s_rho[c]));
     }
-    bound[qi] = 3.f / Z * (DN + vmax * DZ);
-    certified[qi] = DZ <= Z / 3.f ? 1 : 0;
+    bound[qi] = (float)(3.0 / Z * (DN + vmax * DZ));
+    certified[qi] = DZ <= Z / 3.0 ? 1 : 0;
   }
 }
 

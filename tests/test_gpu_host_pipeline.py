@@ -95,3 +95,18 @@ def test_host_copyback_with_cluster_summaries():
     assert torch.equal(host.positions[:n], ref.positions[:n].cpu())
     assert torch.equal(host.k[:n].view(torch.int16), ref.k[:n].cpu().view(torch.int16))
     assert torch.equal(host.v[:n].view(torch.int16), ref.v[:n].cpu().view(torch.int16))
+
+
+@pytest.mark.parametrize("chunk", [1, 2, 0])
+def test_host_pipeline_tiny_contexts(chunk):
+    """The host-input pipeline on 5 (sequence, layer) pairs of 17-token
+    contexts with 3 KV heads: chunks of one pair, of two (the last one short)
+    and the automatic size all equal one device call bit for bit."""
+    wl = W.Workload("T17", B=1, L=5, Hq=12, H=3, n=17, d=128, w=2, keep=(1, 3), kind="zipf")
+    K, V, Q = W.draw(wl, device="cuda")
+    params = ck.certkv_default_params()
+    ref = _reference(K, V, Q, wl.B_live, params)
+    got = ck.certkv_compress_host(K.cpu().pin_memory(), V.cpu().pin_memory(), Q.cpu().pin_memory(),
+                                  wl.B_live, params, chunk=chunk, with_tail=True)
+    torch.cuda.synchronize()
+    _same(got, ref)
