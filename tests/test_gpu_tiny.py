@@ -139,3 +139,33 @@ def test_degenerate_inputs(case):
     ref = oracle.decode(parity.bits(q), got["pk"], got["pv"], got["offsets"], got["counts"],
                         B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, d=wl.d)
     parity.check_decode(out, ref)
+
+
+@pytest.mark.parametrize("gain", [4.0, 16.0])
+def test_large_logits(gain):
+    """Keys scaled up by 4 and 16 (logit spreads of hundreds of nats, most of a
+    row's softmax probabilities below fp32's normal range): the scores, column
+    sums of many rows, stay within the 1e-4 tolerance (measured 2.8e-6 and
+    1.8e-5; the smallest score at gain 16 is ~1e-19, inside fp32's range);
+    conditioned mode bit-exact, end to end within the contract, decode within
+    its tolerance."""
+    wl = W.Workload("G", B=1, L=2, Hq=8, H=2, n=3000, d=128, w=20, keep=(1, 10),
+                    kind="zipf", description="large logits")
+    K, V, Q = W.draw(wl, device="cuda")
+    K = (K.float() * gain).to(torch.bfloat16)
+    params = ck.certkv_default_params()
+    a = ck.certkv_score(K, Q, params)
+    packed = ck.certkv_compress(K, V, Q, wl.B_live, params, with_tail=True)
+    host = dict(K=parity.bits(K), V=parity.bits(V), Q=parity.bits(Q), a=a.cpu().numpy())
+    kw = dict(B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, n=wl.n, d=wl.d, w=wl.w, B_live=wl.B_live)
+    ref_cond = oracle.compress(host["K"], host["V"], None, a_in=host["a"], **kw)
+    ref_e2e = oracle.compress(host["K"], host["V"], host["Q"], **kw)
+    got = parity.packed_np(packed)
+    parity.check_conditioned(got, ref_cond, wl.units)
+    parity.check_scores(host["a"], ref_e2e["a"])
+    parity.check_end_to_end(got, ref_e2e, host["a"], wl.H)
+    q = W.draw_decode_queries(wl, 0, device=DEV)
+    out = ck.certkv_decode_attn(q, packed, hkv=wl.H)
+    ref = oracle.decode(parity.bits(q), got["pk"], got["pv"], got["offsets"], got["counts"],
+                        B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, d=wl.d)
+    parity.check_decode(out, ref)
