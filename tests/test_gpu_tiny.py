@@ -169,3 +169,29 @@ def test_large_logits(gain):
     ref = oracle.decode(parity.bits(q), got["pk"], got["pv"], got["offsets"], got["counts"],
                         B=wl.B, L=wl.L, Hq=wl.Hq, H=wl.H, d=wl.d)
     parity.check_decode(out, ref)
+
+
+def test_budget_sweep():
+    """Twelve live budgets from the smallest (one real token per head) to the
+    largest (every head keeps n - 1 real tokens), odd ones included, on one
+    case: every regime of the allocator (the floor b_min, short and long
+    repairs, the budget ends) bit-exact in conditioned mode and within the
+    contract end to end."""
+    wl = W.Workload("BS", B=1, L=2, Hq=8, H=4, n=500, d=128, w=12, keep=(1, 10),
+                    kind="zipf", description="budget sweep")
+    K, V, Q = W.draw(wl, device=DEV)
+    params = ck.certkv_default_params()
+    a = ck.certkv_score(K, Q, params)
+    host = dict(K=parity.bits(K), V=parity.bits(V), Q=parity.bits(Q), a=a.cpu().numpy())
+    H, n = wl.H, wl.n
+    budgets = sorted({2 * H, 2 * H + 1, 2 * H + 3, 3 * H, 37, 101, 250, 499, 1001, 1500,
+                      H * n - 5, H * n})
+    for B_live in budgets:
+        kw = dict(B=wl.B, L=wl.L, Hq=wl.Hq, H=H, n=n, d=wl.d, w=wl.w, B_live=B_live)
+        packed = ck.certkv_compress(K, V, Q, B_live, params, with_tail=True)
+        got = parity.packed_np(packed)
+        ref_cond = oracle.compress(host["K"], host["V"], None, a_in=host["a"], **kw)
+        parity.check_conditioned(got, ref_cond, wl.units)
+        ref_e2e = oracle.compress(host["K"], host["V"], host["Q"], **kw)
+        parity.check_end_to_end(got, ref_e2e, host["a"], H)
+        assert (got["counts"].reshape(-1, H).sum(1) == B_live - H).all(), B_live
