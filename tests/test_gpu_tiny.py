@@ -195,3 +195,45 @@ def test_budget_sweep():
         ref_e2e = oracle.compress(host["K"], host["V"], host["Q"], **kw)
         parity.check_end_to_end(got, ref_e2e, host["a"], H)
         assert (got["counts"].reshape(-1, H).sum(1) == B_live - H).all(), B_live
+
+
+TINY_VARIANTS = {
+    "uncentered": dict(statistic=1),
+    "tail_mass": dict(statistic=2),
+    "no_tail_slot": dict(tail_slot=0),
+    "no_bisection": dict(bisect_steps=0),
+    "alpha0": dict(alpha_num=0, alpha_den=1),
+    "alpha1": dict(alpha_num=1, alpha_den=1),
+    "pool1_no_protect": dict(pool_kernel=1, protect_window=0),
+    "pool255": dict(pool_kernel=255),          # wider than the whole context
+    "allocator_uniform": dict(allocator=1),
+    "allocator_greedy": dict(allocator=2),
+}
+
+
+@pytest.mark.parametrize("var", sorted(TINY_VARIANTS))
+@pytest.mark.parametrize("n,H,G", [(9, 2, 2), (40, 3, 4)])
+def test_tiny_parameter_variants(var, n, H, G):
+    """Every parameter variant on tiny contexts (a pooling window wider than
+    the context, the safeguard at 0 and 1, no bisection, the ablation
+    allocators): conditioned mode bit-exact, decode within its tolerance."""
+    wl, B_live = _case(n, H, G)
+    params = ck.certkv_default_params(**TINY_VARIANTS[var])
+    K, V, Q = W.draw(wl, device=DEV)
+    a = ck.certkv_score(K, Q, params)
+    packed = ck.certkv_compress_scored(K, V, a, B_live, params, hq=wl.Hq, w=wl.w, with_tail=True)
+    host = dict(K=parity.bits(K), V=parity.bits(V), Q=parity.bits(Q), a=a.cpu().numpy())
+    kw = dict(B=wl.B, L=wl.L, Hq=wl.Hq, H=H, n=n, d=wl.d, w=wl.w, B_live=B_live,
+              scale=params.scale, pool=params.pool_kernel, protect=params.protect_window,
+              alpha_num=params.alpha_num, alpha_den=params.alpha_den, T=params.bisect_steps,
+              statistic=params.statistic, tail_slot=params.tail_slot, allocator=params.allocator)
+    ref_e2e = oracle.compress(host["K"], host["V"], host["Q"], **kw)
+    ref_cond = oracle.compress(host["K"], host["V"], None, a_in=host["a"], **kw)
+    parity.check_scores(host["a"], ref_e2e["a"])
+    got = parity.packed_np(packed)
+    parity.check_conditioned(got, ref_cond, wl.units, tail_slot=params.tail_slot)
+    q = W.draw_decode_queries(wl, 0, device=DEV)
+    out = ck.certkv_decode_attn(q, packed, hkv=H)
+    ref = oracle.decode(parity.bits(q), got["pk"], got["pv"], got["offsets"], got["counts"],
+                        B=wl.B, L=wl.L, Hq=wl.Hq, H=H, d=wl.d, tail_slot=params.tail_slot)
+    parity.check_decode(out, ref)
