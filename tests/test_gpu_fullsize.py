@@ -107,3 +107,13 @@ def test_context_of_2_20_tokens():
     wl = W.Workload("L20", B=1, L=1, Hq=32, H=8, n=1 << 20, d=128, w=64, keep=(1, 10),
                     kind="zipf", description="2^20-token context")
     _run(wl, wl.B_live, samples=[(0, 0)], decode_steps=1)
+
+
+def test_context_of_2_24_tokens():
+    """The largest context the C ABI accepts: 16777216 tokens for 2 KV heads
+    (4 query heads, budget 1/10; K and V 17 GB).  Byte offsets within a head
+    reach 2^32 and the packed cache holds 3.4 M slots: conditioned mode
+    bit-exact, decode within its tolerance."""
+    wl = W.Workload("L24", B=1, L=1, Hq=4, H=2, n=1 << 24, d=128, w=32, keep=(1, 10),
+                    kind="zipf", description="2^24-token context")
+    _run(wl, wl.B_live, samples=[(0, 0)], decode_steps=1)
