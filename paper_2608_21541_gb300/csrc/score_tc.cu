@@ -111,6 +111,14 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// max(a, b, c) in one instruction (sm_100 family); like fmaxf, a NaN operand
+// is ignored.
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 // Hardware base-2 exponential (MUFU), flush-to-zero, relative error ~2^-22.
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -360,12 +368,14 @@ __global__ void __launch_bounds__(kThreads, 1) lse_tc_kernel(const __grid_consta
       const int jc = j_begin + t * C::kTileKeys + cq * 64;
       const bool interior = (jc + 64 <= j_end) && (jc + 63 <= n - p.w);
       if (interior) {
+        // the tile's maximum with three-input maxima (exact, as fmaxf)
         float mx0 = v[0], mx1 = v[1];
 #pragma unroll
-        for (int i = 2; i < 64; i += 2) {
-          mx0 = fmaxf(mx0, v[i]);
-          mx1 = fmaxf(mx1, v[i + 1]);
+        for (int i = 2; i < 62; i += 4) {
+          mx0 = fmax3(mx0, v[i], v[i + 1]);
+          mx1 = fmax3(mx1, v[i + 2], v[i + 3]);
         }
+        mx0 = fmax3(mx0, v[62], v[63]);
         const float nm = fmaxf(m, fmaxf(mx0, mx1) * sl2);  // sl2 > 0: max commutes with scaling
         // the scale-and-subtract and the accumulation two-wide (f32x2), each
         // element into acc[i & 7] in order as a one-wide loop would add it
