@@ -263,7 +263,7 @@ __global__ void __launch_bounds__(256) score_pool_kernel(Prob p, const float* __
                                                          float* __restrict__ s_pool,
                                                          float4* __restrict__ fin_part,
                                                          uint32_t* status) {
-  extern __shared__ float s_win[];  // s over [j0 - half, j1 + half)
+  extern __shared__ __align__(16) float s_win[];  // s over [lo, lo + window), lo <= j0 - half
   __shared__ float red_max[8];
   __shared__ DF red_sum[8];
   const int slice = blockIdx.x, u = blockIdx.y;
@@ -271,10 +271,54 @@ __global__ void __launch_bounds__(256) score_pool_kernel(Prob p, const float* __
   const int j0 = slice * kFinSpan, j1 = min(n, j0 + kFinSpan);
   const float invR = 1.0f / (float)p.R;
   const float invPool = 1.0f / (float)p.pool;
-  const int lo = j0 - half, cnt = (j1 + half) - lo;
-  // the row-block partials summed in row-block order; four window positions
-  // per thread and iteration, so that their loads are in flight together
+  // the row-block partials summed in row-block order
   const float* sb = s_part + (size_t)u * p.row_blocks * n;
+  int lo = j0 - half, cnt = (j1 + half) - lo;
+  if ((n & 3) == 0) {
+    // rows of s_part 16-byte aligned: the window widened to whole float4s
+    // ([lo, lo + cnt) rounded out to multiples of 4; j0 is one), each float4
+    // either wholly inside [0, n) or wholly outside; two float4s per thread
+    // and iteration with four row blocks unrolled, so that eight 16-byte loads
+    // are in flight together
+    lo = -(((half - j0) + 3) >> 2) * 4;  // floor to a multiple of 4 of j0 - half
+    if (j0 - half >= 0) lo = (j0 - half) & ~3;
+    const int hi = (j1 + half + 3) & ~3;
+    const int nv = (hi - lo) >> 2;
+    const float4* sb4 = reinterpret_cast<const float4*>(sb);
+    const int rs4 = n >> 2;  // row stride in float4s
+    for (int t0 = threadIdx.x; t0 < nv; t0 += 2 * blockDim.x) {
+      float4 s[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
+      int i4[2];
+      bool in[2];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int t = t0 + e * (int)blockDim.x;
+        i4[e] = (lo >> 2) + t;
+        in[e] = t < nv && i4[e] >= 0 && i4[e] < rs4;
+      }
+#pragma unroll 4
+      for (int rb = 0; rb < p.row_blocks; ++rb) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const float4 x = in[e] ? sb4[(size_t)rb * rs4 + i4[e]] : make_float4(0.f, 0.f, 0.f, 0.f);
+          s[e].x += x.x;
+          s[e].y += x.y;
+          s[e].z += x.z;
+          s[e].w += x.w;
+        }
+      }
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int t = t0 + e * (int)blockDim.x;
+        if (t < nv)
+          reinterpret_cast<float4*>(s_win)[t] =
+              make_float4(s[e].x * invR, s[e].y * invR, s[e].z * invR, s[e].w * invR);
+      }
+    }
+    cnt = 0;  // the scalar loop below has nothing left to do
+  }
+  // four window positions per thread and iteration, so that their loads are
+  // in flight together
   for (int t0 = threadIdx.x; t0 < cnt; t0 += 4 * blockDim.x) {
     float s[4] = {0.f, 0.f, 0.f, 0.f};
     for (int rb = 0; rb < p.row_blocks; ++rb) {
@@ -418,7 +462,8 @@ void launch_score(const Prob& p, const Layout& ly, char* ws, const void* K, cons
   uint32_t* status = reinterpret_cast<uint32_t*>(ws + ly.status);
   {
     TraceScope ts_("score_pool", st);
-    const size_t fsmem = (size_t)(kFinSpan + p.pool) * sizeof(float);
+    // the window [j0 - half, j1 + half), widened by up to 3 keys on each side
+    const size_t fsmem = (size_t)(kFinSpan + p.pool + 8) * sizeof(float);
     score_pool_kernel<<<fgrid, 256, fsmem, st>>>(p, s_part, s_pool, fin_part, status);
   }
   {
