@@ -640,17 +640,22 @@ def run_e2e(args, wl, K, V, Q, qs, params, ws, dws, dev, stream, world, B_live, 
     step()
     torch.cuda.synchronize()
     steps = max(1, min(args.steps, 5))
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(steps):
+    # one event per step boundary: the mean over the steps is the value; the
+    # per-step times show the host link's spread (the same copy has taken
+    # from 82 to 200 ms on one box)
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    evs[0].record(stream)
+    for i in range(steps):
         step()
-    e1.record(stream)
+        evs[i + 1].record(stream)
     torch.cuda.synchronize()
-    ms = max_over_ranks(e0.elapsed_time(e1) / steps, world)
+    per_step = [evs[i].elapsed_time(evs[i + 1]) for i in range(steps)]
+    ms = max_over_ranks(evs[0].elapsed_time(evs[-1]) / steps, world)
     h2d = sum(x.numel() * x.element_size() for x in (hK, hV, hQ, hq))
     d2h = sum(x.numel() * x.element_size() for x in host_out.values())
     tokens = job_tokens if job_tokens is not None else world * wl.B * wl.L * wl.n
     return {"value": tokens / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
+            "per_step_ms": [round(t, 2) for t in per_step],
             "steps": steps, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "api": "certkv_compress_host_copyback + certkv_decode_attn, pinned host buffers"}
 
