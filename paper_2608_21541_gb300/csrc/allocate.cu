@@ -120,14 +120,18 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   // so), with the sheared values of eight consecutive points evaluated ahead
   // (their curve loads in flight together)
   // and kept on the thread-private stack next to b (as its offset in the
-  // segment), so that a pop needs no reload.  Each test takes the largest
-  // error bound of the points seen so far, at least that of its own three
-  // points: the filter can only keep more.
+  // segment), so that a pop needs no curve reload.  The top two entries are
+  // also held in registers (xa, ya: entry top - 2; xb, yb: entry top - 1):
+  // a point that pops nothing reads no stack memory, and a pop reloads one
+  // entry.  Each test takes the largest error bound of the points seen so
+  // far, at least that of its own three points: the filter can only keep more.
   static_assert(kHullSeg <= 256, "segment offsets are stored in one byte");
   uint8_t st[kHullSeg];
   float sty[kHullSeg];
   float dmax = 0.f;
   int top = 0;
+  int xa = 0, xb = 0;
+  float ya = 0.f, yb = 0.f;
   const int count = b1 - b0;
   for (int i0 = 0; i0 < count; i0 += 8) {
     float yv[8], dv[8];
@@ -139,12 +143,22 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
       if (i0 + k >= count) break;
       const int i = i0 + k;
       dmax = fmaxf(dmax, dv[k]);
-      while (top >= 2 && clearly_above(st[top - 2], sty[top - 2], st[top - 1], sty[top - 1], i,
-                                       yv[k], dmax))
+      while (top >= 2 && clearly_above(xa, ya, xb, yb, i, yv[k], dmax)) {
         --top;
+        xb = xa;
+        yb = ya;
+        if (top >= 2) {
+          xa = st[top - 2];
+          ya = sty[top - 2];
+        }
+      }
       st[top] = (uint8_t)i;
       sty[top] = yv[k];
       ++top;
+      xa = xb;
+      ya = yb;
+      xb = i;
+      yb = yv[k];
     }
   }
   for (int i = 0; i < top; ++i) out[i] = b0 + st[i];
