@@ -103,7 +103,11 @@ __device__ __forceinline__ DF df_from_double(double x) {
 
 }  // namespace
 
-// grid = (ceil(hull_segs / 128), units), one thread per segment.
+// Stack slots per hull_seg thread held in shared memory (8 B each).
+constexpr int kHullWin = 16;
+
+// grid = (ceil(hull_segs / 128), units), block = 128 (the window's thread
+// dimension), one thread per segment.
 __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __restrict__ curve,
                                                        int32_t* __restrict__ cand,
                                                        int32_t* __restrict__ ncand) {
@@ -118,18 +122,26 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   const Shear sh = make_shear(cu, b0, b1 - 1);
   // tolerant monotone chain (a point is dropped only when clearly_above says
   // so), with the sheared values of eight consecutive points evaluated ahead
-  // (their curve loads in flight together)
-  // and kept on the thread-private stack next to b (as its offset in the
-  // segment), so that a pop needs no curve reload.  The top two entries are
-  // also held in registers (xa, ya: entry top - 2; xb, yb: entry top - 1):
-  // a point that pops nothing reads no stack memory, and a pop reloads one
-  // entry.  Each test takes the largest error bound of the points seen so
-  // far, at least that of its own three points: the filter can only keep more.
+  // (their curve loads in flight together) and kept on the thread-private
+  // stack next to b (as its offset in the segment), so that a pop needs no
+  // curve reload.  The top two entries are held in registers (xa, ya: entry
+  // top - 2; xb, yb: entry top - 1), so a point that pops nothing reads no
+  // stack memory.  Entries [spill, top) live in a window of kHullWin slots per
+  // thread in shared memory (slot = entry mod kHullWin, one bank per lane
+  // whatever the entries the lanes touch); older entries [0, spill) move to
+  // the local arrays when the window is full (the stack stays within 18
+  // entries on C3-shaped curves, so that is rare).  Each test takes the
+  // largest error bound of the points seen so far, at least that of its own
+  // three points: the filter can only keep more.
   static_assert(kHullSeg <= 256, "segment offsets are stored in one byte");
+  static_assert((kHullWin & (kHullWin - 1)) == 0 && kHullWin >= 2, "window slots by mask");
+  __shared__ int win_b[kHullWin][128];
+  __shared__ float win_y[kHullWin][128];
+  const int tid = threadIdx.x;
   uint8_t st[kHullSeg];
   float sty[kHullSeg];
   float dmax = 0.f;
-  int top = 0;
+  int top = 0, spill = 0;
   int xa = 0, xb = 0;
   float ya = 0.f, yb = 0.f;
   const int count = b1 - b0;
@@ -145,15 +157,27 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
       dmax = fmaxf(dmax, dv[k]);
       while (top >= 2 && clearly_above(xa, ya, xb, yb, i, yv[k], dmax)) {
         --top;
+        if (top < spill) spill = top;
         xb = xa;
         yb = ya;
         if (top >= 2) {
-          xa = st[top - 2];
-          ya = sty[top - 2];
+          const int e = top - 2;
+          if (e >= spill) {
+            xa = win_b[e & (kHullWin - 1)][tid];
+            ya = win_y[e & (kHullWin - 1)][tid];
+          } else {
+            xa = st[e];
+            ya = sty[e];
+          }
         }
       }
-      st[top] = (uint8_t)i;
-      sty[top] = yv[k];
+      if (top - spill == kHullWin) {  // window full: its oldest entry to local memory
+        st[spill] = (uint8_t)win_b[spill & (kHullWin - 1)][tid];
+        sty[spill] = win_y[spill & (kHullWin - 1)][tid];
+        ++spill;
+      }
+      win_b[top & (kHullWin - 1)][tid] = i;
+      win_y[top & (kHullWin - 1)][tid] = yv[k];
       ++top;
       xa = xb;
       ya = yb;
@@ -161,7 +185,7 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
       yb = yv[k];
     }
   }
-  for (int i = 0; i < top; ++i) out[i] = b0 + st[i];
+  for (int e = 0; e < top; ++e) out[e] = b0 + (e < spill ? (int)st[e] : win_b[e & (kHullWin - 1)][tid]);
   ncand[(size_t)u * ncand_stride(p) + seg] = top;
 }
 
