@@ -57,7 +57,11 @@ struct Shear {
   int b0;
   DF c0, slope;
   __device__ __forceinline__ void at(int b, float& y, float& dy) const {
-    const DF cb = curve_df(cu, b);
+    at_value(b, cu[b], y, dy);
+  }
+  // the same for a curve value c(b) already loaded
+  __device__ __forceinline__ void at_value(int b, float2 v, float& y, float& dy) const {
+    const DF cb{v.x, v.y};
     const DF line = df_add(c0, df_mul_f(slope, (float)(b - b0)));
     y = df_add(cb, df_neg(line)).hi;
     dy = 9.094947e-13f * fmaxf(fabsf(cb.hi), fabsf(line.hi));
@@ -145,11 +149,19 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   int xa = 0, xb = 0;
   float ya = 0.f, yb = 0.f;
   const int count = b1 - b0;
+  // the curve values of the next eight points are loaded while the chain
+  // takes the current eight
+  float2 nxt[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) nxt[k] = k < count ? cu[b0 + k] : make_float2(0.f, 0.f);
   for (int i0 = 0; i0 < count; i0 += 8) {
     float yv[8], dv[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k)
-      if (i0 + k < count) sh.at(b0 + i0 + k, yv[k], dv[k]);
+      if (i0 + k < count) sh.at_value(b0 + i0 + k, nxt[k], yv[k], dv[k]);
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      nxt[k] = i0 + 8 + k < count ? cu[b0 + i0 + 8 + k] : make_float2(0.f, 0.f);
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       if (i0 + k >= count) break;

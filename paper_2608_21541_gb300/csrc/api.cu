@@ -120,7 +120,6 @@ Layout make_layout(const Prob& p) {
   ly.agg_k = take(U * p.chunks * kD * sizeof(float));
   ly.base_mq = take(U * p.chunks * sizeof(float4));
   ly.base_v = take(U * p.chunks * kD * sizeof(float2));
-  ly.base_k = take(U * p.chunks * kD * sizeof(float2));
   ly.curve = take(U * n * sizeof(float2));
   ly.cmax = take(U * sizeof(unsigned long long));
   ly.cand = take(U * n * sizeof(int32_t));

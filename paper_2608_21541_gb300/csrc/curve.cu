@@ -443,21 +443,20 @@ curve_eval_kernel(Prob p, EvalArgs ea) {
                     s_y[warp]);
 }
 
-// grid = (units, (need_k ? 2 : 1) + 1), block = 160: exclusive suffix sums
-// over chunks in double-float, folded from the last chunk down in chunk order.
-// Threads 0..127 take one dimension of the V sums (blockIdx.y = 0) or of the K
-// sums (blockIdx.y = 1), with the next kPrefixBlock chunks' loads in flight
-// while the current ones are folded; warp 4 of the V block takes the scalar
-// sums m and Q, one chunk per lane per round.  In the last y slice, warp 0
-// evaluates the unit's last chunk of ranks instead (its W_base, m and Q bases
-// are zero, so it needs none of these sums), in double-float, alongside.
+// grid = (units, 2), block = 160: exclusive suffix sums over chunks in
+// double-float, folded from the last chunk down in chunk order.  In
+// blockIdx.y = 0, threads 0..127 take one dimension of the V sums, with the
+// next kPrefixBlock chunks' loads in flight while the current ones are
+// folded, and warp 4 the scalar sums m and Q, one chunk per lane per round.
+// In blockIdx.y = 1, warp 0 evaluates the unit's last chunk of ranks instead
+// (its W_base, m and Q bases are zero, so it needs none of these sums), in
+// double-float, alongside.  The K sums are needed at one chunk per unit only
+// (the tail slot's), so the tail kernel folds them itself.
 constexpr int kPrefixBlock = 32;
 __global__ void __launch_bounds__(160) curve_prefix_kernel(Prob p, const float4* __restrict__ agg_mq,
                                                            const float* __restrict__ agg_v,
-                                                           const float* __restrict__ agg_k,
                                                            float4* __restrict__ base_mq,
                                                            float2* __restrict__ base_v,
-                                                           float2* __restrict__ base_k,
                                                            EvalArgs ea) {
   const int u = blockIdx.x;
   if (blockIdx.y == gridDim.y - 1) {
@@ -471,7 +470,6 @@ __global__ void __launch_bounds__(160) curve_prefix_kernel(Prob p, const float4*
   const int chunks = p.chunks;
   const size_t c0 = (size_t)u * chunks;
   if (threadIdx.x >= kD) {
-    if (blockIdx.y != 0) return;
     const int lane = threadIdx.x & 31;
     DF rm = df_make(0.f), rq = df_make(0.f);
     float4 nxt = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -490,8 +488,8 @@ __global__ void __launch_bounds__(160) curve_prefix_kernel(Prob p, const float4*
     return;
   }
   const int i = threadIdx.x;
-  const float* src = (blockIdx.y == 0 ? agg_v : agg_k) + c0 * kD + i;
-  float2* dst = (blockIdx.y == 0 ? base_v : base_k) + c0 * kD + i;
+  const float* src = agg_v + c0 * kD + i;
+  float2* dst = base_v + c0 * kD + i;
   DF r = df_make(0.f);
   float nxt[kPrefixBlock];
 #pragma unroll
@@ -548,7 +546,6 @@ void launch_curves(const Prob& p, const Layout& ly, char* ws, const void* K, con
   float2* yrank = reinterpret_cast<float2*>(ws + ly.yrank);
   float4* base_mq = reinterpret_cast<float4*>(ws + ly.base_mq);
   float2* base_v = reinterpret_cast<float2*>(ws + ly.base_v);
-  float2* base_k = reinterpret_cast<float2*>(ws + ly.base_k);
   float2* curve = reinterpret_cast<float2*>(ws + ly.curve);
   unsigned long long* cmax = reinterpret_cast<unsigned long long*>(ws + ly.cmax);
   dim3 grid((p.chunks + 3) / 4, p.units);
@@ -571,8 +568,7 @@ void launch_curves(const Prob& p, const Layout& ly, char* ws, const void* K, con
                     curve,   cmax,  reinterpret_cast<uint32_t*>(ws + ly.status)};
   {
     TraceScope ts_("curve_prefix", st);
-    curve_prefix_kernel<<<dim3(p.units, (need_k ? 2 : 1) + 1), 160, 0, st>>>(
-        p, agg_mq, agg_v, agg_k, base_mq, base_v, base_k, ea);
+    curve_prefix_kernel<<<dim3(p.units, 2), 160, 0, st>>>(p, agg_mq, agg_v, base_mq, base_v, ea);
   }
   {
     TraceScope ts_("curve_eval", st);

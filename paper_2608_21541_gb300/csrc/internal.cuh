@@ -58,7 +58,6 @@ struct Layout {
   size_t agg_k;      // float  [U][chunks][d]
   size_t base_mq;    // float4 [U][chunks]  suffix after the chunk
   size_t base_v;     // float2 [U][chunks][d]
-  size_t base_k;     // float2 [U][chunks][d]
   size_t curve;      // float2 [U][n]  c(b) as hi + lo
   size_t cmax;       // uint64 [U]     order key of max_b c(b)
   size_t cand;       // int32  [U][n]  allocator candidates

@@ -4,6 +4,9 @@
 //           b_h..n-1 (§4: the key and value centroids of the evicted suffix
 //           under r_j = a_j / m), from the chunk suffix sums plus the partial
 //           chunk, in double-float; rounded once to bf16 into the last slot.
+//           The V and m suffix sums come from the curve's prefix kernel; the
+//           K ones, needed at this one chunk only, are folded here from the
+//           chunk sums in the same order (last chunk down).
 //   select  top-b_h real tokens = ranks 0..b_h-1; emitted in ascending
 //           position by comparing each token's sort key with the first
 //           evicted one (a threshold) and compacting in position order.
@@ -22,7 +25,7 @@ __global__ void __launch_bounds__(128) tail_kernel(
     Prob p, const uint32_t* __restrict__ keys, const int32_t* __restrict__ perm,
     const __nv_bfloat16* __restrict__ K, const __nv_bfloat16* __restrict__ V,
     const float4* __restrict__ base_mq, const float2* __restrict__ base_v,
-    const float2* __restrict__ base_k, const int32_t* __restrict__ counts,
+    const float* __restrict__ agg_k, const int32_t* __restrict__ counts,
     const int64_t* __restrict__ offsets, __nv_bfloat16* __restrict__ pk,
     __nv_bfloat16* __restrict__ pv, int32_t* __restrict__ positions, float* __restrict__ tail_f32,
     double* __restrict__ tail_mass, uint32_t* status) {
@@ -42,8 +45,30 @@ __global__ void __launch_bounds__(128) tail_kernel(
   DF m{bmq.x, bmq.y};
   float2 t = base_v[ci * kD + i];
   DF tv{t.x, t.y};
-  t = base_k[ci * kD + i];
-  DF tk{t.x, t.y};
+  // the K sums over the chunks after chunk kb, folded from the last chunk
+  // down; the next 32 chunks' loads are in flight while 32 are folded
+  DF tk = df_make(0.f);
+  {
+    const float* src = agg_k + (size_t)u * p.chunks * kD + i;
+    float nxt[32];
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+      const int c = p.chunks - 1 - e;
+      nxt[e] = c > kb ? src[(size_t)c * kD] : 0.f;
+    }
+    for (int top = p.chunks - 1; top > kb; top -= 32) {
+      float x[32];
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        x[e] = nxt[e];
+        const int c = top - 32 - e;
+        nxt[e] = c > kb ? src[(size_t)c * kD] : 0.f;
+      }
+#pragma unroll
+      for (int e = 0; e < 32; ++e)
+        if (top - e > kb) tk = df_add_f(tk, x[e]);
+    }
+  }
   // the partial chunk's scores and token indices staged once; then the K and
   // V values of eight ranks at a time in flight, summed in rank order
   __shared__ float s_a[kChunk];
@@ -512,7 +537,7 @@ void launch_pack(const Prob& p, const Layout& ly, char* ws, const void* K, const
     tail_kernel<<<p.units, 128, 0, st>>>(
         p, keys, perm, Kb, Vb, reinterpret_cast<const float4*>(ws + ly.base_mq),
         reinterpret_cast<const float2*>(ws + ly.base_v),
-        reinterpret_cast<const float2*>(ws + ly.base_k), counts, offsets, PK, PV, positions,
+        reinterpret_cast<const float*>(ws + ly.agg_k), counts, offsets, PK, PV, positions,
         tail_f32, tail_mass, status);
   }
 }
