@@ -40,7 +40,7 @@ __device__ __forceinline__ bool in_bounds(bool ok, uint32_t* status) {
 
 // -------------------------------------------------------------- bf16 ------
 __device__ __forceinline__ float bf16lo(uint32_t packed) {
-  return __uint_as_float(packed << 16);
+  return __uint_as_float(packed * 65536u);  // the shift by 16 as a multiply (FMA pipe)
 }
 __device__ __forceinline__ float bf16hi(uint32_t packed) {
   return __uint_as_float(packed & 0xffff0000u);

@@ -323,16 +323,31 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
       float2 P01 = make_float2(P[0], P[1]), P23 = make_float2(P[2], P[3]);
       const float2 W01 = make_float2(wb2x[0], wb2x[1]), W23 = make_float2(wb2x[2], wb2x[3]);
       float xg[8];
+      if (cnt >= 8) {  // a whole group (every group but a partial chunk's): no per-rank tests
+        const float4 alo = *reinterpret_cast<const float4*>(sa + rl);
+        const float4 ahi = *reinterpret_cast<const float4*>(sa + rl + 4);
+        const float as8[8] = {alo.x, alo.y, alo.z, alo.w, ahi.x, ahi.y, ahi.z, ahi.w};
 #pragma unroll
-      for (int t = 7; t >= 0; --t) {
-        const float as = sa[rl + t];
-        uint2 raw = make_uint2(0u, 0u);
-        if (t < cnt) raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
-        const float2 a2 = make_float2(as, as);
-        P01 = ffma2(a2, make_float2(bf16lo(raw.x), bf16hi(raw.x)), P01);
-        P23 = ffma2(a2, make_float2(bf16lo(raw.y), bf16hi(raw.y)), P23);
-        const float2 acc = ffma2(fadd2(W23, P23), P23, fmul2(fadd2(W01, P01), P01));
-        xg[t] = (t < cnt) ? acc.x + acc.y : 0.f;
+        for (int t = 7; t >= 0; --t) {
+          const uint2 raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
+          const float2 a2 = make_float2(as8[t], as8[t]);
+          P01 = ffma2(a2, make_float2(bf16lo(raw.x), bf16hi(raw.x)), P01);
+          P23 = ffma2(a2, make_float2(bf16lo(raw.y), bf16hi(raw.y)), P23);
+          const float2 acc = ffma2(fadd2(W23, P23), P23, fmul2(fadd2(W01, P01), P01));
+          xg[t] = acc.x + acc.y;
+        }
+      } else {
+#pragma unroll
+        for (int t = 7; t >= 0; --t) {
+          const float as = sa[rl + t];
+          uint2 raw = make_uint2(0u, 0u);
+          if (t < cnt) raw = *reinterpret_cast<const uint2*>(rows + t * (kD * 2) + lane * 8);
+          const float2 a2 = make_float2(as, as);
+          P01 = ffma2(a2, make_float2(bf16lo(raw.x), bf16hi(raw.x)), P01);
+          P23 = ffma2(a2, make_float2(bf16lo(raw.y), bf16hi(raw.y)), P23);
+          const float2 acc = ffma2(fadd2(W23, P23), P23, fmul2(fadd2(W01, P01), P01));
+          xg[t] = (t < cnt) ? acc.x + acc.y : 0.f;
+        }
       }
       P[0] = P01.x;
       P[1] = P01.y;
@@ -433,7 +448,7 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
 __global__ void __launch_bounds__(128, 7)  // seven CTAs per SM: 69 registers, no spills
 curve_eval_kernel(Prob p, EvalArgs ea) {
   __shared__ __align__(16) unsigned char s_ring[4][kEvalRing][kEvalGroupBytes];
-  __shared__ float s_a[4][kChunk];
+  __shared__ __align__(16) float s_a[4][kChunk];  // read as float4 by whole groups
   __shared__ int s_j[4][kChunk];
   __shared__ float2 s_y[4][kChunk];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -461,7 +476,7 @@ __global__ void __launch_bounds__(160) curve_prefix_kernel(Prob p, const float4*
   const int u = blockIdx.x;
   if (blockIdx.y == gridDim.y - 1) {
     __shared__ __align__(16) unsigned char l_ring[kEvalRing][kEvalGroupBytes];
-    __shared__ float l_a[kChunk];
+    __shared__ __align__(16) float l_a[kChunk];
     __shared__ int l_j[kChunk];
     __shared__ float2 l_y[kChunk];
     if (threadIdx.x < 32) eval_chunk<true>(p, ea, p.chunks - 1, u, threadIdx.x, l_ring[0], l_a, l_j, l_y);
