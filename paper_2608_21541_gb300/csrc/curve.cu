@@ -263,6 +263,7 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
   const int nb = (r1 - r0 + 31) / 32;
   const int ngroups = nb * 4;  // group g: ranks r0 + 32*(nb-1-g/4) + 24 - 8*(g%4) + 0..7
   // lane l copies 16-byte piece (l & 15) of rows (l >> 4) + 2k, k = 0..3
+  const bool full = r1 - r0 == kChunk;  // every chunk but a partial last one
   auto stage = [&](int g) {
     if (g < ngroups) {
       const int rl = 32 * (nb - 1 - g / 4) + 24 - 8 * (g % 4);  // first rank of the group, chunk-local
@@ -270,7 +271,7 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         const int t = (lane >> 4) + 2 * k;
-        if (r0 + rl + t < r1)
+        if (full || r0 + rl + t < r1)
           cp_async16(dst + t * (kD * 2) + (lane & 15) * 16,
                      Vu + (size_t)sj[rl + t] * (kD * 2) + (lane & 15) * 16);
       }
