@@ -11,7 +11,7 @@ namespace certkv {
 constexpr int kD = 128;          // head dimension supported by the kernels
 constexpr int kChunk = 128;      // ranks per dispersion chunk (one warp)
 constexpr int kHullSeg = 256;    // curve points per hull-filter thread
-constexpr int kGroupSegs = 8;    // hull-filter segments per group
+constexpr int kGroupSegs = 4;    // hull-filter segments per group
 constexpr int kSortTile = 2048;  // keys per radix-sort tile
 constexpr int kSortThreads = 256;
 constexpr uint32_t kFull = 0xffffffffu;
