@@ -201,11 +201,13 @@ __global__ void __launch_bounds__(128) hull_seg_kernel(Prob p, const float2* __r
   ncand[(size_t)u * ncand_stride(p) + seg] = top;
 }
 
-// grid = (ceil(groups / 128), units), one thread per group of segments.  The
+// grid = (ceil(groups / 128), units), block = 128 (the window's thread
+// dimension), one thread per group of segments.  The
 // tolerant chain over the segment survivors in order, eight points at a time:
 // their b, then their sheared values, each batch of loads in flight together.
 // The stack is the group's own candidate list (it never overtakes the read
-// position); a pop reloads the sheared value of the new top.  Each test takes
+// position); a pop below the shared-memory window reloads the new top and
+// recomputes its sheared value.  Each test takes
 // the largest error bound seen so far (the filter can only keep more).
 __global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* __restrict__ curve,
                                                          int32_t* __restrict__ cand,
@@ -222,7 +224,13 @@ __global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* _
   const int b1 = min(n, p.b_min + s1 * kHullSeg) - 1;
   const Shear sh = make_shear(cu, b0, b1);
   int32_t* st = cl + (size_t)s0 * kHullSeg;
-  int top = 0;
+  // entries [spill, top) also in a window of kHullWin slots per thread in
+  // shared memory with their sheared values (one bank per lane), so that a
+  // pop within it reads neither the list nor the curve again
+  __shared__ int win_b[kHullWin][128];
+  __shared__ float win_y[kHullWin][128];
+  const int tid = threadIdx.x;
+  int top = 0, spill = 0;
   int xa = 0, xb = 0;
   float ya = 0.f, yb = 0.f, dmax = 0.f;
   for (int s = s0; s < s1; ++s) {
@@ -243,14 +251,24 @@ __global__ void __launch_bounds__(128) hull_group_kernel(Prob p, const float2* _
         dmax = fmaxf(dmax, dv[k]);
         while (top >= 2 && clearly_above(xa, ya, xb, yb, b, yv[k], dmax)) {
           --top;
+          if (top < spill) spill = top;
           xb = xa;
           yb = ya;
           if (top >= 2) {
-            xa = st[top - 2];
-            float d;
-            sh.at(xa, ya, d);
+            const int e = top - 2;
+            if (e >= spill) {
+              xa = win_b[e & (kHullWin - 1)][tid];
+              ya = win_y[e & (kHullWin - 1)][tid];
+            } else {
+              xa = st[e];
+              float d;
+              sh.at(xa, ya, d);
+            }
           }
         }
+        if (top - spill == kHullWin) ++spill;  // the oldest window entry stays in the list only
+        win_b[top & (kHullWin - 1)][tid] = b;
+        win_y[top & (kHullWin - 1)][tid] = yv[k];
         st[top++] = b;  // top <= the points read so far: never past the read position
         xa = xb;
         ya = yb;

@@ -129,7 +129,7 @@ __global__ void __launch_bounds__(128) tail_kernel(
 }
 
 // grid = units, block = 1024: positions of the kept tokens in ascending order.
-__global__ void __launch_bounds__(1024) select_kernel(Prob p, const float* __restrict__ a,
+__global__ void __launch_bounds__(1024, 2) select_kernel(Prob p, const float* __restrict__ a,
                                                       const uint32_t* __restrict__ keys,
                                                       const int32_t* __restrict__ perm,
                                                       const int32_t* __restrict__ counts,
@@ -151,6 +151,13 @@ __global__ void __launch_bounds__(1024) select_kernel(Prob p, const float* __res
   constexpr int kPer = 4;
   if (threadIdx.x == 0) carry = 0;
   __syncthreads();
+  // the next round's scores are loaded while this round is ranked
+  float x[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) {
+    const int j = threadIdx.x * kPer + e;
+    x[e] = j < n ? au[j] : 0.f;
+  }
   for (int base = 0; base < n; base += blockDim.x * kPer) {
     int j0 = base + threadIdx.x * kPer;
     bool kept[kPer];
@@ -160,11 +167,16 @@ __global__ void __launch_bounds__(1024) select_kernel(Prob p, const float* __res
       int j = j0 + e;
       bool k = false;
       if (j < n) {
-        uint32_t kj = score_key(au[j]);
+        uint32_t kj = score_key(x[e]);
         k = (kj < kt) || (kj == kt && j < jt);
       }
       kept[e] = k;
       cnt += k;
+    }
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) {
+      const int j = j0 + blockDim.x * kPer + e;
+      x[e] = j < n ? au[j] : 0.f;
     }
     int incl = cnt;
 #pragma unroll
