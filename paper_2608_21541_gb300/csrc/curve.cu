@@ -214,7 +214,9 @@ __global__ void __launch_bounds__(128) curve_agg_kernel(Prob p, const uint32_t* 
 // One warp evaluates chunk `chunk` of unit u.  The V rows of the chunk are
 // staged in groups of 8 ranks (descending) through the warp's ring in shared
 // memory (ring_w, kEvalRing groups), kEvalAhead groups ahead of the
-// evaluation; sa, sj, sy hold the chunk's scores, token indices and ||v||^2.
+// evaluation; sa, sj hold the chunk's scores and token indices.  Each lane
+// loads the ||v||^2 of its rank of a 32-rank batch into a register at the
+// batch's first group; it is used at the batch's end.
 // kLast: the unit's last chunk (W_base = 0), in double-float.
 struct EvalArgs {
   const uint32_t* keys;
@@ -229,8 +231,7 @@ struct EvalArgs {
 };
 template <bool kLast>
 __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, int chunk, int u,
-                                           int lane, unsigned char* ring_w, float* sa, int* sj,
-                                           float2* sy) {
+                                           int lane, unsigned char* ring_w, float* sa, int* sj) {
   const uint32_t* __restrict__ keys = ea.keys;
   const int32_t* __restrict__ perm = ea.perm;
   const __nv_bfloat16* __restrict__ V = ea.V;
@@ -257,7 +258,6 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
     if (!CERTKV_IN_BOUNDS(j >= 0 && j < n, p.status)) j = 0;
     sa[e * 32 + lane] = ok ? key_score(ku[r]) : 0.f;
     sj[e * 32 + lane] = j;
-    sy[e * 32 + lane] = ok ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
   }
   __syncwarp();
   const int nb = (r1 - r0 + 31) / 32;
@@ -310,12 +310,17 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
   bool bad = false;
   DF xt = df_make(0.f);  // lane r: ||W_base + P(b)||^2 - ||W_base||^2 for rank r of the batch
   DF yt = df_make(0.f);  // lane r: ||v||^2 of rank r of the batch (last chunk only)
+  float2 yv = make_float2(0.f, 0.f);  // lane r: ||v||^2 of rank r of the batch (as staged)
   for (int g = 0; g < ngroups; ++g) {
     stage(g + kEvalAhead);
-    asm volatile("cp.async.wait_group %0;" ::"n"(kEvalAhead) : "memory");
-    __syncwarp();
     const int bi = nb - 1 - g / 4;
     const int s0 = 24 - 8 * (g % 4);
+    if (!exact && s0 == 24) {  // the batch's first group: its ranks' ||v||^2, used at its end
+      const int r = r0 + 32 * bi + lane;
+      yv = r < r1 ? yrank[(size_t)u * n + r] : make_float2(0.f, 0.f);
+    }
+    asm volatile("cp.async.wait_group %0;" ::"n"(kEvalAhead) : "memory");
+    __syncwarp();
     const int rl = 32 * bi + s0;
     const int cnt = r1 - (r0 + rl);  // rows of the group that exist (may exceed 8)
     const unsigned char* rows = ring_w + (g % kEvalRing) * kEvalGroupBytes;
@@ -396,7 +401,6 @@ __device__ __forceinline__ void eval_chunk(const Prob& p, const EvalArgs& ea, in
     const int r = r0 + 32 * bi + lane;
     const bool ok = r < r1;
     const float at = sa[32 * bi + lane];
-    const float2 yv = sy[32 * bi + lane];
     // in-batch inclusive suffix sums over lanes >= t (a and a||v||^2 are
     // non-negative: same-sign double-float additions)
     DF sm = df_make(at);
@@ -451,12 +455,10 @@ curve_eval_kernel(Prob p, EvalArgs ea) {
   __shared__ __align__(16) unsigned char s_ring[4][kEvalRing][kEvalGroupBytes];
   __shared__ __align__(16) float s_a[4][kChunk];  // read as float4 by whole groups
   __shared__ int s_j[4][kChunk];
-  __shared__ float2 s_y[4][kChunk];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int chunk = blockIdx.x * 4 + warp;
   if (chunk >= p.chunks - 1) return;
-  eval_chunk<false>(p, ea, chunk, blockIdx.y, lane, s_ring[warp][0], s_a[warp], s_j[warp],
-                    s_y[warp]);
+  eval_chunk<false>(p, ea, chunk, blockIdx.y, lane, s_ring[warp][0], s_a[warp], s_j[warp]);
 }
 
 // grid = (units, 2), block = 160: exclusive suffix sums over chunks in
@@ -479,8 +481,7 @@ __global__ void __launch_bounds__(160) curve_prefix_kernel(Prob p, const float4*
     __shared__ __align__(16) unsigned char l_ring[kEvalRing][kEvalGroupBytes];
     __shared__ __align__(16) float l_a[kChunk];
     __shared__ int l_j[kChunk];
-    __shared__ float2 l_y[kChunk];
-    if (threadIdx.x < 32) eval_chunk<true>(p, ea, p.chunks - 1, u, threadIdx.x, l_ring[0], l_a, l_j, l_y);
+    if (threadIdx.x < 32) eval_chunk<true>(p, ea, p.chunks - 1, u, threadIdx.x, l_ring[0], l_a, l_j);
     return;
   }
   const int chunks = p.chunks;
