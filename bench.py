@@ -184,7 +184,7 @@ def roofline_for(name, work, ms, peaks, traffic=None):
 # are 4x the L2, so the traffic grows in proportion to the units), keyed by
 # workload.  A workload without an entry, or a pass changed since the
 # counters were taken, reports null.
-MEASURED_PASS_TRAFFIC_PER_UNIT = {"C3": (3054506496 + 131641088) / 16}
+MEASURED_PASS_TRAFFIC_PER_UNIT = {"C3": (3054573909 + 131305899) / 16}
 
 
 def measured_pass_traffic(wl):
