@@ -345,6 +345,15 @@ __global__ void __launch_bounds__(256) score_pool_kernel(Prob p, const float* __
     if (j < nw) {
       if (p.pool == 1) {
         v = s_win[j - lo];
+      } else if (p.pool == 5 && j >= 2 && j + 2 < nw) {  // the default width, window inside
+        const float* w5 = s_win + (j - 2 - lo);          // the same additions, in order
+        float acc = 0.f;
+        acc += w5[0];
+        acc += w5[1];
+        acc += w5[2];
+        acc += w5[3];
+        acc += w5[4];
+        v = acc * invPool;
       } else {
         float acc = 0.f;
         for (int i = j - half; i <= j + half; ++i)
