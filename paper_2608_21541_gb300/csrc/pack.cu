@@ -70,7 +70,7 @@ __global__ void __launch_bounds__(128) tail_kernel(
     }
   }
   // the partial chunk's scores and token indices staged once; then the K and
-  // V values of eight ranks at a time in flight, summed in rank order
+  // V values of sixteen ranks at a time in flight, summed in rank order
   __shared__ float s_a[kChunk];
   __shared__ int s_j[kChunk];
   if (b + i < r_end) {
@@ -80,10 +80,10 @@ __global__ void __launch_bounds__(128) tail_kernel(
     s_j[i] = j;
   }
   __syncthreads();
-  for (int r0 = b; r0 < r_end; r0 += 8) {
-    float vv[8], kv[8];
+  for (int r0 = b; r0 < r_end; r0 += 16) {
+    float vv[16], kv[16];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
+    for (int e = 0; e < 16; ++e) {
       vv[e] = kv[e] = 0.f;
       if (r0 + e < r_end) {
         const size_t o = (size_t)s_j[r0 + e - b] * kD + i;
@@ -92,7 +92,7 @@ __global__ void __launch_bounds__(128) tail_kernel(
       }
     }
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
+    for (int e = 0; e < 16; ++e) {
       if (r0 + e >= r_end) break;
       const float a = s_a[r0 + e - b];
       m = df_add_f(m, a);
