@@ -136,8 +136,11 @@ __global__ void __launch_bounds__(1024, 2) select_kernel(Prob p, const float* __
                                                       const int64_t* __restrict__ offsets,
                                                       int32_t* __restrict__ positions,
                                                       uint32_t* status) {
-  __shared__ int warp_tot[32];
-  __shared__ int carry;
+  // per-warp totals, double-buffered by round: a round's buffer is rewritten
+  // two rounds later, after two more barriers, so two barriers per round
+  // suffice; every thread keeps the same running offset `carry`
+  __shared__ int warp_tot2[2][32];
+  int carry = 0;
   const int u = blockIdx.x;
   const int n = p.n;
   const int b = counts[u];
@@ -149,8 +152,6 @@ __global__ void __launch_bounds__(1024, 2) select_kernel(Prob p, const float* __
   int32_t* out = positions + offsets[u];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   constexpr int kPer = 4;
-  if (threadIdx.x == 0) carry = 0;
-  __syncthreads();
   // the next round's scores are loaded while this round is ranked
   float x[kPer];
 #pragma unroll
@@ -158,7 +159,8 @@ __global__ void __launch_bounds__(1024, 2) select_kernel(Prob p, const float* __
     const int j = threadIdx.x * kPer + e;
     x[e] = j < n ? au[j] : 0.f;
   }
-  for (int base = 0; base < n; base += blockDim.x * kPer) {
+  for (int base = 0, round = 0; base < n; base += blockDim.x * kPer, ++round) {
+    int* warp_tot = warp_tot2[round & 1];
     int j0 = base + threadIdx.x * kPer;
     bool kept[kPer];
     int cnt = 0;
@@ -203,9 +205,7 @@ __global__ void __launch_bounds__(1024, 2) select_kernel(Prob p, const float* __
         if (pos < b) out[pos] = j0 + e;
         ++pos;
       }
-    __syncthreads();
-    if (threadIdx.x == 0) carry += warp_tot[(blockDim.x >> 5) - 1];
-    __syncthreads();
+    carry += warp_tot[(blockDim.x >> 5) - 1];
   }
   if (threadIdx.x == 0 && carry != b) raise_status(status, 1u);
 }
